@@ -1,0 +1,786 @@
+/*
+ * Tsubame per-step logit path -- CPU ORACLE.
+ *
+ * TEST INFRASTRUCTURE ONLY. This is a plain, slow, single-threaded reference of what the
+ * plan / replay / verify path computes, written from the paper (Tsubame: Tree Replay for
+ * Diffusion-Based Speculative Decoding) and the works it cites for the sampling and
+ * verification rules. Only the test suite, the smoke check and the benchmark's CPU-baseline
+ * leg may load it. It shares no code, header, helper or constant table with the CUDA
+ * library; both sides follow the same written contract (counter layout, tie rules).
+ *
+ * Arithmetic: a logit z (bf16 or fp32) is widened exactly to fp32 and multiplied once by
+ * invT = fp32(1/T) in fp32, x = fp32(z) * invT (one IEEE rounding, identical on every
+ * machine). Everything after that is fp64 with libm, in the order the algorithm states.
+ * Build with -ffp-contract=off so no multiply-add is fused behind our back.
+ *
+ * Every decision taken from floating point (a heap pop, a Gumbel selection, an acceptance
+ * test) also reports whether it was a near tie, so the tests can exempt exactly those
+ * decisions where a correct fp32 implementation may legitimately decide differently.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORC_CHUNK 256 /* fixed chunk of the hierarchical replay sampler (contract) */
+
+/* Purposes of the counter-based random stream (contract). */
+enum {
+    PURPOSE_REPLAY_CHUNK = 0, /* node = parent, draw = chunk index        */
+    PURPOSE_REPLAY_ELEM = 1,  /* node = parent, draw = token id           */
+    PURPOSE_ACCEPT = 2,       /* node = child being tested, draw = 0      */
+    PURPOSE_FINAL = 3,        /* node = where the final token is drawn, draw = token id */
+    PURPOSE_BLOCK_ETA = 4     /* node = chain position i, draw = 0         */
+};
+
+/* Uniform-space half-width of a near tie (the parity contract's 1e-6 band). */
+static const double U_BAND = 1e-6;
+
+/* ------------------------------------------------------------------------------------ */
+/* Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3",
+ * SC 2011, Sec. 3.2). Ten rounds of the 4x32 S-box; the key is bumped by the Weyl
+ * constants between rounds.                                                              */
+void orc_philox4x32_10(const uint32_t ctr_in[4], const uint32_t key_in[2], uint32_t out[4])
+{
+    uint32_t c0 = ctr_in[0], c1 = ctr_in[1], c2 = ctr_in[2], c3 = ctr_in[3];
+    uint32_t k0 = key_in[0], k1 = key_in[1];
+    for (int round = 0; round < 10; ++round) {
+        if (round > 0) {
+            k0 += 0x9E3779B9u;
+            k1 += 0xBB67AE85u;
+        }
+        uint64_t prod0 = (uint64_t)0xD2511F53u * (uint64_t)c0;
+        uint64_t prod1 = (uint64_t)0xCD9E8D57u * (uint64_t)c2;
+        uint32_t hi0 = (uint32_t)(prod0 >> 32), lo0 = (uint32_t)prod0;
+        uint32_t hi1 = (uint32_t)(prod1 >> 32), lo1 = (uint32_t)prod1;
+        uint32_t n0 = hi1 ^ c1 ^ k0;
+        uint32_t n2 = hi0 ^ c3 ^ k1;
+        c0 = n0;
+        c1 = lo1;
+        c2 = n2;
+        c3 = lo0;
+    }
+    out[0] = c0;
+    out[1] = c1;
+    out[2] = c2;
+    out[3] = c3;
+}
+
+/* The uniform of one draw: counter {draw/4, node, batch, purpose}, key {seed lo, seed hi},
+ * word draw%4; U = (top 24 bits + 1/2) * 2^-24, which lies in (0,1) and is exact in fp32. */
+double orc_uniform(uint64_t seed, int32_t purpose, int32_t batch, int32_t node, int32_t draw)
+{
+    uint32_t ctr[4] = {(uint32_t)draw >> 2, (uint32_t)node, (uint32_t)batch, (uint32_t)purpose};
+    uint32_t key[2] = {(uint32_t)seed, (uint32_t)(seed >> 32)};
+    uint32_t w[4];
+    orc_philox4x32_10(ctr, key, w);
+    uint32_t bits = w[(uint32_t)draw & 3u] >> 8;
+    return ((double)bits + 0.5) * (1.0 / 16777216.0);
+}
+
+/* Standard Gumbel by inversion, G(U) = -log(-log U). */
+static double gumbel_of(double u) { return -log(-log(u)); }
+
+/* dG/dU: how fast a Gumbel key moves per unit of its uniform (used to turn key margins
+ * into uniform-space margins). */
+static double gumbel_slope(double u) { return 1.0 / (u * -log(u)); }
+
+/* ------------------------------------------------------------------------------------ */
+/* Logit tensors: element (b, r, v) sits at data[b*batch_stride + r*row_stride + v].      */
+typedef struct {
+    const void *data;
+    int32_t dtype; /* 0 = fp32, 1 = bf16 (raw 16-bit patterns) */
+    int32_t B, R, V;
+    int64_t batch_stride, row_stride;
+} orc_logits;
+
+/* x_v = fp32(z_v) * invT for one row, widened to double (exactly). */
+static void read_row(const orc_logits *t, int b, int r, float invT, double *x)
+{
+    const int64_t base = (int64_t)b * t->batch_stride + (int64_t)r * t->row_stride;
+    for (int v = 0; v < t->V; ++v) {
+        float z;
+        if (t->dtype == 1) {
+            uint32_t bits = (uint32_t)((const uint16_t *)t->data)[base + v] << 16;
+            memcpy(&z, &bits, sizeof z);
+        } else {
+            z = ((const float *)t->data)[base + v];
+        }
+        float xf = z * invT;
+        x[v] = (double)xf;
+    }
+}
+
+/* log sum_v exp(x_v), shifted by the maximum (plain definition of the softmax normaliser). */
+static double logsumexp(const double *x, int n)
+{
+    double m = -INFINITY;
+    for (int v = 0; v < n; ++v)
+        if (x[v] > m) m = x[v];
+    double s = 0.0;
+    for (int v = 0; v < n; ++v) s += exp(x[v] - m);
+    return m + log(s);
+}
+
+/* softmax into out[], fp64 */
+static void softmax(const double *x, int n, double *out)
+{
+    double lse = logsumexp(x, n);
+    for (int v = 0; v < n; ++v) out[v] = exp(x[v] - lse);
+}
+
+/* (x desc, id asc): does (xa, a) come before (xb, b)? */
+static int before_xv(double xa, int a, double xb, int b) { return xa > xb || (xa == xb && a < b); }
+
+/* Top-K of a row by (x desc, id asc): K rounds of "best element after the previous one". */
+static void topk_row(const double *x, int V, int K, int32_t *ids, double *xs)
+{
+    double px = INFINITY;
+    int pid = -1;
+    for (int k = 0; k < K; ++k) {
+        int best = -1;
+        for (int v = 0; v < V; ++v) {
+            int after_prev = (x[v] < px) || (x[v] == px && v > pid);
+            if (!after_prev) continue;
+            if (best < 0 || before_xv(x[v], v, x[best], best)) best = v;
+        }
+        ids[k] = best;
+        xs[k] = x[best];
+        px = x[best];
+        pid = best;
+    }
+}
+
+/* Row statistics of step a1: max, log-normaliser, top-K, chunk log-masses.
+ * Exposed for the tests (row_lse/topk pins).                                             */
+int orc_row_stats(const orc_logits *rows, float temperature, int32_t K, double *row_max, double *row_lse,
+                  int32_t *topk_id, float *topk_x, double *chunk_lse)
+{
+    if (!rows || !(temperature > 0.0f) || K < 1 || K > rows->V) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = rows->V, C = (V + ORC_CHUNK - 1) / ORC_CHUNK;
+    double *x = (double *)malloc(sizeof(double) * V);
+    double *xs = (double *)malloc(sizeof(double) * K);
+    if (!x || !xs) { free(x); free(xs); return -3; }
+    for (int b = 0; b < rows->B; ++b)
+        for (int r = 0; r < rows->R; ++r) {
+            const int64_t row = (int64_t)b * rows->R + r;
+            read_row(rows, b, r, invT, x);
+            double m = -INFINITY;
+            for (int v = 0; v < V; ++v)
+                if (x[v] > m) m = x[v];
+            if (row_max) row_max[row] = m;
+            if (row_lse) row_lse[row] = logsumexp(x, V);
+            if (topk_id || topk_x) {
+                int32_t ids[64];
+                topk_row(x, V, K, ids, xs);
+                for (int k = 0; k < K; ++k) {
+                    if (topk_id) topk_id[row * K + k] = ids[k];
+                    if (topk_x) topk_x[row * K + k] = (float)xs[k];
+                }
+            }
+            if (chunk_lse)
+                for (int c = 0; c < C; ++c) {
+                    int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+                    chunk_lse[row * C + c] = logsumexp(x + lo, hi - lo);
+                }
+        }
+    free(x);
+    free(xs);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* PLAN (first pass, Sec. 3.1; max-heap expansion of DDTree as described in Sec. 2.2 and
+ * App. B.3): best-first expansion by cumulative draft path log-probability under a node
+ * budget. Node 0 is the root; nodes 1..N are numbered in pop order.
+ *
+ * Path score of a node at depth d reached through ranks (r_1..r_d):
+ *     score = sum_j log q_j(y_j) = (sum_j x_{j, r_j}) - (sum_{j<=d} LSE_j)
+ * held as the exact fp64 sum Sx of the x's plus the depth; key = Sx - CL[d] with
+ * CL[d] = LSE_1 + ... + LSE_d. Candidates pop in the order
+ *     (key desc, depth asc, Sx desc, parent asc, rank asc),
+ * a total order in which same-depth candidates compare through Sx exactly.               */
+typedef struct {
+    double key, sx;
+    int depth, parent, rank;
+} cand;
+
+static int cand_before(const cand *a, const cand *b)
+{
+    if (a->key != b->key) return a->key > b->key;
+    if (a->depth != b->depth) return a->depth < b->depth;
+    if (a->sx != b->sx) return a->sx > b->sx;
+    if (a->parent != b->parent) return a->parent < b->parent;
+    return a->rank < b->rank;
+}
+
+/* Maximum node count a (K, L) tree can hold besides the root: K + K^2 + ... + K^L. */
+static int64_t max_nodes(int K, int L)
+{
+    int64_t total = 0, level = 1;
+    for (int d = 1; d <= L; ++d) {
+        level *= K;
+        total += level;
+        if (total > (int64_t)1 << 40) return total;
+    }
+    return total;
+}
+
+int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L,
+             int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
+             int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+{
+    if (!draft || N < 1 || K < 1 || L < 1 || K > 64 || K > draft->V || draft->R < L) return -1;
+    if (!(temperature > 0.0f)) return -1;
+    if ((int64_t)N > max_nodes(K, L)) return -2;
+    const float invT = 1.0f / temperature;
+    const int V = draft->V, NN = N + 1;
+    double *x = (double *)malloc(sizeof(double) * V);
+    double *lse = (double *)malloc(sizeof(double) * L);
+    double *CL = (double *)malloc(sizeof(double) * (L + 1));
+    int32_t *tid = (int32_t *)malloc(sizeof(int32_t) * L * K);
+    double *tx = (double *)malloc(sizeof(double) * L * K);
+    double *sxn = (double *)malloc(sizeof(double) * NN);
+    cand *front = (cand *)malloc(sizeof(cand) * (2 * (size_t)NN + 2));
+    int32_t *nchild = (int32_t *)malloc(sizeof(int32_t) * NN);
+    if (!x || !lse || !CL || !tid || !tx || !sxn || !front || !nchild) return -3;
+
+    for (int b = 0; b < draft->B; ++b) {
+        int32_t *par = parent + (int64_t)b * NN, *dep = depth + (int64_t)b * NN;
+        int32_t *rk = rank + (int64_t)b * NN, *tok = plan_token + (int64_t)b * NN;
+        double *sc = score + (int64_t)b * NN;
+        /* per-depth candidate pools: top-K of draft row d (tokens of depth d+1) */
+        for (int d = 0; d < L; ++d) {
+            read_row(draft, b, d, invT, x);
+            lse[d] = logsumexp(x, V);
+            topk_row(x, V, K, tid + d * K, tx + d * K);
+        }
+        CL[0] = 0.0;
+        for (int d = 1; d <= L; ++d) CL[d] = CL[d - 1] + lse[d - 1];
+
+        par[0] = -1; dep[0] = 0; rk[0] = -1; tok[0] = -1; sc[0] = 0.0; sxn[0] = 0.0;
+        int nf = 0;
+        front[nf].sx = tx[0];
+        front[nf].depth = 1;
+        front[nf].parent = 0;
+        front[nf].rank = 0;
+        front[nf].key = front[nf].sx - CL[1];
+        ++nf;
+        uint8_t ex = 0;
+        double mm = INFINITY;
+        for (int i = 1; i <= N; ++i) {
+            if (nf == 0) return -4; /* cannot happen when N <= max_nodes */
+            int best = 0;
+            for (int f = 1; f < nf; ++f)
+                if (cand_before(&front[f], &front[best])) best = f;
+            /* Near-tie check: only keys of different depths depend on the log-normalisers;
+             * same-depth order is decided exactly through Sx. */
+            for (int f = 0; f < nf; ++f) {
+                if (f == best || front[f].depth == front[best].depth) continue;
+                double margin = front[best].key - front[f].key;
+                if (margin < mm) mm = margin;
+                if (margin < key_eps * (1.0 + fabs(front[best].key))) ex = 1;
+            }
+            cand c = front[best];
+            front[best] = front[--nf];
+            par[i] = c.parent;
+            dep[i] = c.depth;
+            rk[i] = c.rank;
+            tok[i] = tid[(c.depth - 1) * K + c.rank];
+            sc[i] = c.key;
+            sxn[i] = c.sx;
+            if (c.rank + 1 < K) { /* next sibling */
+                cand s;
+                s.depth = c.depth;
+                s.parent = c.parent;
+                s.rank = c.rank + 1;
+                s.sx = sxn[c.parent] + tx[(c.depth - 1) * K + c.rank + 1];
+                s.key = s.sx - CL[s.depth];
+                front[nf++] = s;
+            }
+            if (c.depth < L) { /* first child */
+                cand f;
+                f.depth = c.depth + 1;
+                f.parent = i;
+                f.rank = 0;
+                f.sx = sxn[i] + tx[c.depth * K + 0];
+                f.key = f.sx - CL[f.depth];
+                front[nf++] = f;
+            }
+        }
+        if (exempt) exempt[b] = ex;
+        if (min_margin) min_margin[b] = mm;
+        /* child lists (CSR) in slot (= rank = pop) order */
+        int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        for (int u = 0; u < NN; ++u) nchild[u] = 0;
+        for (int i = 1; i <= N; ++i) nchild[par[i]]++;
+        off[0] = 0;
+        for (int u = 0; u < NN; ++u) off[u + 1] = off[u] + nchild[u];
+        for (int u = 0; u < NN; ++u) nchild[u] = 0;
+        for (int i = 1; i <= N; ++i) ids[off[par[i]] + nchild[par[i]]++] = i;
+    }
+    free(x); free(lse); free(CL); free(tid); free(tx); free(sxn); free(front); free(nchild);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* REPLAY (second pass, Sec. 3.2, Eq. replay-distribution; WoR as defined in App. A).
+ * For each parent u with m_u children, draw m_u tokens without replacement from
+ * q_u = softmax(x_row(u)); the j-th draw fills child slot j.
+ *
+ * WoR draws are the top-m_u of the Gumbel keys x_v + G_v (Gumbel-top-k: Vieira 2014;
+ * Kool, van Hoof & Welling 2019). The keys are built top-down (Maddison, Tarlow & Minka
+ * 2014, A* sampling; Kool et al. 2019, App. B): chunk keys K_c ~ Gumbel(A_c) with
+ * A_c = log sum_{v in c} exp(x_v); inside each of the top-m_u chunks, fresh element keys
+ * g_v ~ Gumbel(x_v) are shifted to the law conditional on their maximum being K_c,
+ *     k_v = -log(exp(-K_c) - exp(-Z_c) + exp(-g_v)),   Z_c = max_{v in c} g_v,
+ * which leaves the joint law of all keys that of flat Gumbel-top-k.                       */
+
+/* stable form of the conditional shift (Kool et al. 2019, App. B) */
+static double shift_key(double T, double Z, double g)
+{
+    double u = T - g + log1p(-exp(g - Z));
+    double sp = (u > 0 ? u : 0.0) + log1p(exp(-fabs(u)));
+    return T - sp;
+}
+
+typedef struct {
+    double k;  /* key */
+    int v;     /* token id */
+    double sens; /* max |d key / d uniform| over the uniforms the key depends on */
+} elem_key;
+
+static int elem_before(const elem_key *a, const elem_key *b) { return a->k > b->k || (a->k == b->k && a->v < b->v); }
+
+/* Sort the first n entries so the first `take` are the best in order (selection sort). */
+static void partial_sort(elem_key *e, int n, int take)
+{
+    for (int i = 0; i < take && i < n; ++i) {
+        int best = i;
+        for (int j = i + 1; j < n; ++j)
+            if (elem_before(&e[j], &e[best])) best = j;
+        elem_key t = e[i];
+        e[i] = e[best];
+        e[best] = t;
+    }
+}
+
+/* Is the decision "a before b" a near tie in uniform space? */
+static int near_tie(const elem_key *a, const elem_key *b)
+{
+    double dk = a->k - b->k;
+    double s = a->sens > b->sens ? a->sens : b->sens;
+    return dk < U_BAND * s;
+}
+
+static int replay_row_index(const int32_t *qrow_of_node, const int32_t *depth, int64_t idx) { return qrow_of_node ? qrow_of_node[idx] : depth[idx]; }
+
+int orc_replay(const orc_logits *q, float temperature, const int32_t *qrow_of_node, int32_t N,
+               const int32_t *depth, const int32_t *child_off, const int32_t *child_ids, uint64_t seed,
+               int32_t *token, uint8_t *exempt_node)
+{
+    if (!q || N < 0 || !(temperature > 0.0f)) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = q->V, C = (V + ORC_CHUNK - 1) / ORC_CHUNK, NN = N + 1;
+    double *x = (double *)malloc(sizeof(double) * V);
+    elem_key *ck = (elem_key *)malloc(sizeof(elem_key) * C);
+    double *A = (double *)malloc(sizeof(double) * C);
+    elem_key *ek = (elem_key *)malloc(sizeof(elem_key) * (size_t)V);
+    if (!x || !ck || !A || !ek) return -3;
+    for (int b = 0; b < q->B; ++b) {
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        token[(int64_t)b * NN + 0] = -1;
+        for (int u = 0; u < NN; ++u) {
+            if (exempt_node) exempt_node[(int64_t)b * NN + u] = 0;
+            const int m = off[u + 1] - off[u];
+            if (m == 0) continue;
+            const int r = replay_row_index(qrow_of_node, depth, (int64_t)b * NN + u);
+            if (r < 0 || r >= q->R) return -5;
+            read_row(q, b, r, invT, x);
+            /* 1. chunk log-masses and chunk keys */
+            for (int c = 0; c < C; ++c) {
+                int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+                A[c] = logsumexp(x + lo, hi - lo);
+                double uc = orc_uniform(seed, PURPOSE_REPLAY_CHUNK, b, u, c);
+                ck[c].k = A[c] + gumbel_of(uc);
+                ck[c].v = c;
+                ck[c].sens = gumbel_slope(uc);
+            }
+            /* 2. the top-m chunks by (K desc, c asc) */
+            const int msel = m < C ? m : C;
+            partial_sort(ck, C, msel + 1 < C ? msel + 1 : C);
+            uint8_t ex = 0;
+            if (C > msel && near_tie(&ck[msel - 1], &ck[msel])) ex = 1;
+            /* 3. element keys inside the selected chunks, shifted to max K_c */
+            int ne = 0;
+            for (int s = 0; s < msel; ++s) {
+                const int c = ck[s].v;
+                const double Tc = ck[s].k;
+                const double uc_slope = ck[s].sens;
+                int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+                int first = ne;
+                double Z = -INFINITY;
+                int jmax = -1;
+                double umax = 0.5;
+                for (int v = lo; v < hi; ++v) {
+                    double uv = orc_uniform(seed, PURPOSE_REPLAY_ELEM, b, u, v);
+                    double g = x[v] + gumbel_of(uv);
+                    ek[ne].k = g; /* raw key for now */
+                    ek[ne].v = v;
+                    ek[ne].sens = gumbel_slope(uv);
+                    if (g > Z) { Z = g; jmax = ne; umax = uv; }
+                    ++ne;
+                }
+                for (int e = first; e < ne; ++e) {
+                    if (e == jmax) {
+                        ek[e].k = Tc;
+                        ek[e].sens = uc_slope;
+                    } else {
+                        double g = ek[e].k;
+                        double k = shift_key(Tc, Z, g);
+                        /* sensitivities through g (own uniform), T (chunk uniform), Z (max's uniform) */
+                        double s_own = ek[e].sens * exp(k - g);
+                        double s_T = uc_slope * exp(k - Tc);
+                        double s_Z = gumbel_slope(umax) * exp(k - Z);
+                        double s = s_own > s_T ? s_own : s_T;
+                        if (s_Z > s) s = s_Z;
+                        ek[e].k = k;
+                        ek[e].sens = s;
+                    }
+                }
+            }
+            /* 4. the top-m keys over the selected chunks are the ordered WoR draws */
+            partial_sort(ek, ne, m + 1 < ne ? m + 1 : ne);
+            for (int j = 0; j < m; ++j) {
+                if (j + 1 < ne && near_tie(&ek[j], &ek[j + 1])) ex = 1;
+                token[(int64_t)b * NN + ids[off[u] + j]] = ek[j].v;
+            }
+            if (exempt_node) exempt_node[(int64_t)b * NN + u] = ex;
+        }
+    }
+    free(x); free(ck); free(A); free(ek);
+    return 0;
+}
+
+/* Flat Gumbel-top-m over the whole row (independent cross-check of the law only). */
+int orc_replay_flat(const orc_logits *q, float temperature, const int32_t *qrow_of_node, int32_t N,
+                    const int32_t *depth, const int32_t *child_off, const int32_t *child_ids, uint64_t seed,
+                    int32_t *token)
+{
+    if (!q || N < 0 || !(temperature > 0.0f)) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = q->V, NN = N + 1;
+    double *x = (double *)malloc(sizeof(double) * V);
+    elem_key *ek = (elem_key *)malloc(sizeof(elem_key) * (size_t)V);
+    if (!x || !ek) return -3;
+    for (int b = 0; b < q->B; ++b) {
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        token[(int64_t)b * NN] = -1;
+        for (int u = 0; u < NN; ++u) {
+            const int m = off[u + 1] - off[u];
+            if (m == 0) continue;
+            const int r = replay_row_index(qrow_of_node, depth, (int64_t)b * NN + u);
+            if (r < 0 || r >= q->R) return -5;
+            read_row(q, b, r, invT, x);
+            for (int v = 0; v < V; ++v) {
+                ek[v].k = x[v] + gumbel_of(orc_uniform(seed, PURPOSE_REPLAY_ELEM, b, u, v));
+                ek[v].v = v;
+                ek[v].sens = 0;
+            }
+            partial_sort(ek, V, m);
+            for (int j = 0; j < m; ++j) token[(int64_t)b * NN + ids[off[u] + j]] = ek[j].v;
+        }
+    }
+    free(x); free(ek);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* VERIFY: recursive rejection sampling for WoR candidates down the tree (Sec. 2.3 Eq.
+ * rs-overlap for one candidate; App. A for the WoR variant used by Sequoia / EAGLE / RSD).
+ * At a node with target law P, draft law Q and children y_1..y_m (in slot order):
+ *   slot i: q' = Q(y_i)/t (t = draft mass not yet drawn), p' = P(y_i);
+ *           accept iff U_i * q' < p'  (probability min(1, p'/q'));
+ *           on reject: R(v) = max(P(v) - Q(v)/t [v not drawn], 0), P <- R / sum R,
+ *                      y_i joins the drawn set, t <- t - Q(y_i).
+ * If a child is accepted its token is emitted and the walk continues there; if all are
+ * rejected the final token is drawn from the last residual R; at a leaf the bonus token
+ * is drawn from the node's target row. Losslessness: Prop. 1.                          */
+
+static double draft_ratio(double qv, double t) { return (qv > 0.0 && t > 0.0) ? qv / t : 0.0; }
+
+/* One rejection step: unnormalised residual R and its mass. */
+static double rrs_residual(int V, const double *P, const double *Q, double t, const uint8_t *drawn, double *R)
+{
+    double Z = 0.0;
+    for (int v = 0; v < V; ++v) {
+        double qv = drawn[v] ? 0.0 : draft_ratio(Q[v], t);
+        double r = P[v] - qv;
+        R[v] = r > 0.0 ? r : 0.0;
+        Z += R[v];
+    }
+    return Z;
+}
+
+/* Gumbel-max over log w(v) (w >= 0, entries with w = 0 excluded) with the FINAL stream of
+ * (b, node); reports whether the winner and the runner-up are a near tie.               */
+static int gumbel_argmax_logw(const double *w, int V, uint64_t seed, int b, int node, uint8_t *ex)
+{
+    int best = -1, second = -1;
+    double kb = -INFINITY, ks = -INFINITY, sb = 0, ss = 0;
+    for (int v = 0; v < V; ++v) {
+        if (!(w[v] > 0.0)) continue;
+        double u = orc_uniform(seed, PURPOSE_FINAL, b, node, v);
+        double k = log(w[v]) + gumbel_of(u);
+        if (best < 0 || k > kb) {
+            second = best; ks = kb; ss = sb;
+            best = v; kb = k; sb = gumbel_slope(u);
+        } else if (second < 0 || k > ks) {
+            second = v; ks = k; ss = gumbel_slope(u);
+        }
+    }
+    if (second >= 0 && ex) {
+        double s = sb > ss ? sb : ss;
+        if (kb - ks < U_BAND * s) *ex = 1;
+    }
+    return best;
+}
+
+/* Gumbel-max over logits x (the bonus token) */
+static int gumbel_argmax_logits(const double *x, int V, uint64_t seed, int b, int node, uint8_t *ex)
+{
+    int best = -1, second = -1;
+    double kb = -INFINITY, ks = -INFINITY, sb = 0, ss = 0;
+    for (int v = 0; v < V; ++v) {
+        double u = orc_uniform(seed, PURPOSE_FINAL, b, node, v);
+        double k = x[v] + gumbel_of(u);
+        if (best < 0 || k > kb) {
+            second = best; ks = kb; ss = sb;
+            best = v; kb = k; sb = gumbel_slope(u);
+        } else if (second < 0 || k > ks) {
+            second = v; ks = k; ss = gumbel_slope(u);
+        }
+    }
+    if (second >= 0 && ex) {
+        double s = sb > ss ? sb : ss;
+        if (kb - ks < U_BAND * s) *ex = 1;
+    }
+    return best;
+}
+
+/* Exact law of one node's verification for a fixed ordered child tuple (for the
+ * enumeration pins): acc[i] = P(accept slot i | slots before it rejected), and the law of
+ * the final token when every slot is rejected. Uses the same update as the sampler.    */
+int orc_rrs_node_law(int32_t V, const double *P_in, const double *Q, int32_t m, const int32_t *y, double *acc,
+                     double *final_law)
+{
+    double *P = (double *)malloc(sizeof(double) * V), *R = (double *)malloc(sizeof(double) * V);
+    uint8_t *drawn = (uint8_t *)calloc(V, 1);
+    if (!P || !R || !drawn) return -3;
+    memcpy(P, P_in, sizeof(double) * V);
+    double t = 1.0;
+    int degenerate = 0;
+    for (int i = 0; i < m; ++i) acc[i] = 0.0;
+    for (int i = 0; i < m; ++i) {
+        double qp = draft_ratio(Q[y[i]], t), pp = P[y[i]];
+        acc[i] = qp > 0.0 ? (pp / qp < 1.0 ? pp / qp : 1.0) : (pp > 0.0 ? 1.0 : 0.0);
+        double Z = rrs_residual(V, P, Q, t, drawn, R);
+        if (!(Z > 0.0)) {
+            /* no residual mass: fine when this slot cannot be rejected (later slots and the
+             * final law are then unreachable), degenerate otherwise */
+            if (acc[i] < 1.0 - 1e-12) degenerate = 1; /* beyond rounding */
+            for (int v = 0; v < V; ++v) P[v] = 0.0;
+            break;
+        }
+        for (int v = 0; v < V; ++v) P[v] = R[v] / Z;
+        drawn[y[i]] = 1;
+        t -= Q[y[i]];
+    }
+    /* after the last rejection P holds R_m / Z_m */
+    for (int v = 0; v < V; ++v) final_law[v] = P[v];
+    free(P); free(R); free(drawn);
+    return degenerate;
+}
+
+int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperature, const int32_t *qrow_of_node,
+                   int32_t N, int32_t L, const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
+                   const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len,
+                   uint8_t *exempt)
+{
+    if (!target || !q || N < 0 || L < 1 || !(temperature > 0.0f) || target->V != q->V || target->R < N + 1) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = target->V, NN = N + 1;
+    double *xt = (double *)malloc(sizeof(double) * V), *xq = (double *)malloc(sizeof(double) * V);
+    double *P = (double *)malloc(sizeof(double) * V), *Q = (double *)malloc(sizeof(double) * V);
+    double *R = (double *)malloc(sizeof(double) * V);
+    uint8_t *drawn = (uint8_t *)malloc(V);
+    if (!xt || !xq || !P || !Q || !R || !drawn) return -3;
+    for (int b = 0; b < target->B; ++b) {
+        const int64_t nb = (int64_t)b * NN;
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        int32_t *otok = out_tokens + (int64_t)b * (L + 1), *onode = out_nodes + (int64_t)b * L;
+        for (int k = 0; k <= L; ++k) otok[k] = -1;
+        for (int k = 0; k < L; ++k) onode[k] = -1;
+        uint8_t ex = 0;
+        int u = 0, nacc = 0, final_tok = -1;
+        for (int step = 0; step <= L; ++step) { /* depth grows by one per accepted node */
+            const int m = off[u + 1] - off[u];
+            read_row(target, b, u, invT, xt);
+            if (m == 0) { /* leaf: bonus token from the node's target row */
+                final_tok = gumbel_argmax_logits(xt, V, seed, b, u, &ex);
+                break;
+            }
+            const int r = replay_row_index(qrow_of_node, depth, nb + u);
+            if (r < 0 || r >= q->R) return -5;
+            read_row(q, b, r, invT, xq);
+            softmax(xt, V, P);
+            softmax(xq, V, Q);
+            memset(drawn, 0, V);
+            double t = 1.0;
+            int accepted = -1;
+            for (int i = 0; i < m; ++i) {
+                const int c = ids[off[u] + i];
+                const int y = token[nb + c];
+                if (y < 0 || y >= V) return -6;
+                double qp = draft_ratio(Q[y], t), pp = P[y];
+                double U = orc_uniform(seed, PURPOSE_ACCEPT, b, c, 0);
+                if (qp > 0.0 && fabs(U - pp / qp) < U_BAND) ex = 1;
+                if (U * qp < pp) { accepted = c; break; }
+                double Z = rrs_residual(V, P, Q, t, drawn, R);
+                if (!(Z > 0.0)) { /* underflow only: draw from the current target law */
+                    final_tok = gumbel_argmax_logw(P, V, seed, b, u, &ex);
+                    break;
+                }
+                if (i == m - 1) { /* every slot rejected: draw from the last residual */
+                    final_tok = gumbel_argmax_logw(R, V, seed, b, u, &ex);
+                    break;
+                }
+                for (int v = 0; v < V; ++v) P[v] = R[v] / Z;
+                drawn[y] = 1;
+                t -= Q[y];
+            }
+            if (accepted < 0) break;
+            otok[nacc] = token[nb + accepted];
+            onode[nacc] = accepted;
+            ++nacc;
+            u = accepted;
+        }
+        otok[nacc] = final_tok;
+        out_len[b] = nacc + 1;
+        if (exempt) exempt[b] = ex;
+    }
+    free(xt); free(xq); free(P); free(Q); free(R); free(drawn);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* BLOCK VERIFICATION of a sampled chain X_1..X_g (Sun et al. 2025, cited in Sec. 1,
+ * Table 2 and App. A). With Mb_i = target law after prefix X^i (i = 0..g) and
+ * Ms_i = draft law of the next token after X^i (i = 0..g-1):
+ *   w_0 = 1, w_i = min(w_{i-1} Mb_{i-1}(X_i) / Ms_{i-1}(X_i), 1);
+ *   h_i = S_i / (S_i + 1 - w_i) with S_i = sum_x max(w_i Mb_i(x) - Ms_i(x), 0) (i < g),
+ *         h_i = 1 when the denominator is 0;  h_g = w_g;
+ *   tau = max{ i in 1..g : eta_i <= h_i }, 0 if none;
+ *   final token ~ Mb_g if tau = g, else ~ max(w_tau Mb_tau - Ms_tau, 0) (normalised).
+ * Emits X_1..X_tau and the final token.                                                  */
+static void blockv_weights(int g, int V, const double *Mb, const double *Ms, const int32_t *X, double *w, double *h,
+                           double *resid /* [g*V] unnormalised, may be NULL */)
+{
+    w[0] = 1.0;
+    for (int i = 1; i <= g; ++i) {
+        double num = Mb[(int64_t)(i - 1) * V + X[i - 1]], den = Ms[(int64_t)(i - 1) * V + X[i - 1]];
+        double ratio = den > 0.0 ? w[i - 1] * num / den : 1.0;
+        w[i] = ratio < 1.0 ? ratio : 1.0;
+    }
+    for (int i = 0; i < g; ++i) {
+        double S = 0.0;
+        for (int v = 0; v < V; ++v) {
+            double r = w[i] * Mb[(int64_t)i * V + v] - Ms[(int64_t)i * V + v];
+            r = r > 0.0 ? r : 0.0;
+            if (resid) resid[(int64_t)i * V + v] = r;
+            S += r;
+        }
+        double den = S + 1.0 - w[i];
+        h[i] = den > 0.0 ? S / den : 1.0;
+    }
+    h[g] = w[g];
+}
+
+/* Exact pieces of the block-verification law for one chain (for the enumeration pins). */
+int orc_blockv_law(int32_t g, int32_t V, const double *Mb, const double *Ms, const int32_t *X, double *w, double *h,
+                   double *resid)
+{
+    blockv_weights(g, V, Mb, Ms, X, w, h, resid);
+    return 0;
+}
+
+int orc_verify_block(const orc_logits *target, const orc_logits *q, float temperature, const int32_t *qrow_of_node,
+                     int32_t N, int32_t L, const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
+                     const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len,
+                     uint8_t *exempt, int32_t *tau_out)
+{
+    if (!target || !q || N < 1 || N > L || !(temperature > 0.0f) || target->V != q->V || target->R < N + 1) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = target->V, NN = N + 1, g = N;
+    double *x = (double *)malloc(sizeof(double) * V);
+    double *Mb = (double *)malloc(sizeof(double) * (size_t)(g + 1) * V);
+    double *Ms = (double *)malloc(sizeof(double) * (size_t)g * V);
+    double *resid = (double *)malloc(sizeof(double) * (size_t)g * V);
+    double *w = (double *)malloc(sizeof(double) * (g + 1)), *h = (double *)malloc(sizeof(double) * (g + 1));
+    int32_t *X = (int32_t *)malloc(sizeof(int32_t) * g);
+    if (!x || !Mb || !Ms || !resid || !w || !h || !X) return -3;
+    for (int b = 0; b < target->B; ++b) {
+        const int64_t nb = (int64_t)b * NN;
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        /* the tree must be the chain 0 -> 1 -> ... -> g */
+        for (int i = 0; i <= g; ++i) {
+            int want = i < g ? 1 : 0;
+            if (off[i + 1] - off[i] != want || (want && ids[off[i]] != i + 1)) return -7;
+        }
+        for (int i = 0; i <= g; ++i) {
+            read_row(target, b, i, invT, x);
+            softmax(x, V, Mb + (int64_t)i * V);
+        }
+        for (int i = 0; i < g; ++i) {
+            const int r = replay_row_index(qrow_of_node, depth, nb + i);
+            if (r < 0 || r >= q->R) return -5;
+            read_row(q, b, r, invT, x);
+            softmax(x, V, Ms + (int64_t)i * V);
+            X[i] = token[nb + i + 1];
+            if (X[i] < 0 || X[i] >= V) return -6;
+        }
+        blockv_weights(g, V, Mb, Ms, X, w, h, resid);
+        uint8_t ex = 0;
+        int tau = 0;
+        for (int i = 1; i <= g; ++i)
+            if (orc_uniform(seed, PURPOSE_BLOCK_ETA, b, i, 0) <= h[i]) tau = i;
+        for (int i = (tau > 1 ? tau : 1); i <= g; ++i) /* decisions that could move tau */
+            if (fabs(orc_uniform(seed, PURPOSE_BLOCK_ETA, b, i, 0) - h[i]) < U_BAND) ex = 1;
+        int final_tok;
+        if (tau == g) {
+            read_row(target, b, g, invT, x);
+            final_tok = gumbel_argmax_logits(x, V, seed, b, g, &ex);
+        } else {
+            double S = 0.0;
+            for (int v = 0; v < V; ++v) S += resid[(int64_t)tau * V + v];
+            if (S > 0.0)
+                final_tok = gumbel_argmax_logw(resid + (int64_t)tau * V, V, seed, b, tau, &ex);
+            else /* cannot carry mass in exact arithmetic; draw from the target law there */
+                final_tok = gumbel_argmax_logw(Mb + (int64_t)tau * V, V, seed, b, tau, &ex);
+        }
+        int32_t *otok = out_tokens + (int64_t)b * (L + 1), *onode = out_nodes + (int64_t)b * L;
+        for (int k = 0; k <= L; ++k) otok[k] = -1;
+        for (int k = 0; k < L; ++k) onode[k] = -1;
+        for (int i = 1; i <= tau; ++i) {
+            otok[i - 1] = X[i - 1];
+            onode[i - 1] = i;
+        }
+        otok[tau] = final_tok;
+        out_len[b] = tau + 1;
+        if (exempt) exempt[b] = ex;
+        if (tau_out) tau_out[b] = tau;
+    }
+    free(x); free(Mb); free(Ms); free(resid); free(w); free(h); free(X);
+    return 0;
+}
