@@ -1,0 +1,464 @@
+#!/usr/bin/env python3
+"""Benchmark of the per-step logit path (plan + replay + verify) on one GB300 per rank.
+
+Workload (batched serving): B=16 trees, V=151,936, draft block L=16, N=64 planned nodes,
+top-k 8, T=1, bf16 logits; target rows [16, 65, V] = the node's depth row + N(0, 0.7^2).
+A step = tsb_row_stats + tsb_plan + tsb_replay + tsb_verify on one batch (4 kernel launches).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tsb|reference]
+
+Prints one JSON line (rank 0). ``value`` is the mean device time per step in microseconds
+(lower is better), timed with CUDA events over exactly K steps after W warm-up steps, with
+the inputs resident in HBM. Inputs rotate over several independent sets whose per-step
+footprint together exceeds the L2 several times, so no step finds its rows in L2 from an
+earlier step. ``e2e`` repeats the measurement through the same C ABI with host (pinned)
+inputs: every step copies its draft and target rows to the device and its outputs back.
+``--impl reference`` times the CPU oracle on the same workload (one tree per step, scaled to
+the batch), rank 0 only.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+WORKLOAD = dict(name="batched", B=16, V=151936, L=16, N=64, K=8, T=1.0, dtype="bf16", target_noise=0.7)
+METRIC = "plan+replay+verify us/step and HBM GB/s (% of GB300 peak), V=151,936, N=64"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_HBM_GBS = 6800.0
+NOMINAL_HBM_GBS = 8000.0
+L2_BYTES = 129 * 1024 * 1024
+KERNELS = ("tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify")
+KERNEL_SOURCES = {"tsb_row_stats": "k_row_stats.cu", "tsb_plan": "k_plan.cu", "tsb_replay": "k_replay.cu",
+                  "tsb_verify": "k_verify.cu"}
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=None)
+    ap.add_argument("--impl", choices=("tsb", "reference"), default="tsb")
+    ap.add_argument("--sets", type=int, default=8, help="independent input sets rotated across steps")
+    ap.add_argument("--e2e-steps", type=int, default=40)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--workload", default="batched", choices=("batched", "batched128k"))
+    args = ap.parse_args()
+    if args.steps is None:
+        args.steps = 2000 if args.impl == "tsb" else 8
+    if args.warmup is None:
+        args.warmup = 20 if args.impl == "tsb" else 1
+    if args.warmup < 3 and args.impl == "tsb":
+        args.warmup = 3
+    return args
+
+
+def workload(args):
+    w = dict(WORKLOAD)
+    if args.workload == "batched128k":
+        w.update(name="batched128k", V=128256)
+    return w
+
+
+def config_of(w, extra=None):
+    cfg = {"workload": f"batched serving: B={w['B']}, V={w['V']}, L={w['L']}, N={w['N']}, K={w['K']}, "
+                       f"T={w['T']}, {w['dtype']} logits, target = depth row + N(0,{w['target_noise']}^2)",
+           "B": w["B"], "V": w["V"], "L": w["L"], "N": w["N"], "K": w["K"], "temperature": w["T"]}
+    if extra:
+        cfg.update(extra)
+    return cfg
+
+
+def measured_peak_hbm():
+    try:
+        with open(PEAKS_FILE) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def source_hash(name):
+    with open(os.path.join(ROOT, "paper_2609_33652_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic(kernel, workload_name):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current
+    source of that kernel (profiles/ncu_traffic.txt lines: kernel workload src_hash bytes)."""
+    path = os.path.join(ROOT, "profiles", "ncu_traffic.txt")
+    if not os.path.exists(path):
+        return None
+    want = source_hash(KERNEL_SOURCES[kernel])
+    with open(path) as f:
+        for line in f:
+            p = line.split()
+            if len(p) >= 4 and not line.startswith("#") and p[0] == kernel and p[1] == workload_name and p[2] == want:
+                return float(p[3])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason sampling while the timed region runs."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            time.sleep(0.15)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.06)
+            self.proc.terminate()
+            try:
+                out, _ = self.proc.communicate(timeout=5)
+            except Exception:
+                self.proc.kill()
+                out = ""
+            self.lines = [ln for ln in out.splitlines() if ln.strip()]
+
+    def summary(self):
+        sm, smax, reasons = [], [], set()
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        for ln in self.lines:
+            p = [x.strip() for x in ln.split(",")]
+            if len(p) < 9:
+                continue
+            try:
+                sm.append(float(p[1]))
+                smax.append(float(p[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, p[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------------------
+def build_sets(w, S, device, rank):
+    import torch
+
+    from paper_2609_33652_gb300 import synth, tsb
+
+    sets = []
+    for s in range(S):
+        seed = 1003 + 100 * s + 10000 * rank
+        draft = synth.draft_logits(w["B"], w["L"], w["V"], "planted", w["dtype"], seed, device=device)
+        buf = tsb.TsbBuffers.allocate(w["B"], w["L"], w["N"], w["K"], w["V"], w["T"], device=device)
+        tsb.tsb_row_stats(draft, w["T"], buf.stats, buf.ws)
+        tsb.tsb_plan(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+        target = synth.rows_from_depth(draft, buf.tree["depth"], w["target_noise"], seed + 1)
+        torch.cuda.synchronize()
+        if tsb.tsb_device_status(buf.ws) != 0:
+            raise RuntimeError("device status set while preparing inputs")
+        sets.append(dict(draft=draft, target=target, buf=buf,
+                         child_off=buf.tree["child_off"].cpu().numpy()))
+    return sets
+
+
+def algorithmic_bytes(w, sets, out_len, out_nodes):
+    """Per step: draft rows once (B*L*V*s) + target rows of the visited nodes; plus the q rows
+    the verifier stages (visited nodes with children), reported separately."""
+    es = 2 if w["dtype"] == "bf16" else 4
+    row = w["V"] * es
+    K = out_len.shape[0]
+    S = len(sets)
+    visited = out_len.sum(axis=1).astype(np.int64)  # root + accepted nodes per tree
+    staged_q = np.zeros(K, dtype=np.int64)
+    for k in range(K):
+        off = sets[k % S]["child_off"]
+        for b in range(out_len.shape[1]):
+            n = int(out_len[k, b])
+            nodes = [0] + [int(x) for x in out_nodes[k, b, :n - 1]]
+            staged_q[k] += sum(1 for u in nodes if off[b, u + 1] > off[b, u])
+    draft_bytes = w["B"] * w["L"] * row
+    return draft_bytes, visited * row, staged_q * row, visited
+
+
+def run_tsb(args):
+    import torch
+
+    from paper_2609_33652_gb300 import tsb
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    device = torch.device("cuda", local)
+    torch.cuda.set_device(device)
+    w = workload(args)
+    from paper_2609_33652_gb300 import build as libbuild
+
+    libbuild.build()
+    tsb.load()
+    S = args.sets
+    sets = build_sets(w, S, device, rank)
+    K, W = args.steps, args.warmup
+    B, L = w["B"], w["L"]
+    out_tokens = torch.empty(K, B, L + 1, dtype=torch.int32, device=device)
+    out_nodes = torch.empty(K, B, L, dtype=torch.int32, device=device)
+    out_len = torch.empty(K, B, dtype=torch.int32, device=device)
+
+    def prepared(k, seed, tgt_slot=True):
+        st = sets[k % S]
+        if tgt_slot:
+            return tsb.PreparedStep(st["buf"], st["draft"], st["target"], seed, out_tokens=out_tokens[k],
+                                    out_nodes=out_nodes[k], out_len=out_len[k])
+        return tsb.PreparedStep(st["buf"], st["draft"], st["target"], seed)
+
+    warm = [prepared(k, 900_000 + k, tgt_slot=False) for k in range(W)]
+    steps = [prepared(k, 1 + k + 1_000_000 * rank) for k in range(K)]
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(K)]
+    for p in warm:
+        p.run()
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(local) as clocks:
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+        start.record()
+        for k in range(K):
+            steps[k].run(events[k])
+        end.record()
+        torch.cuda.synchronize()
+        if dist is not None:
+            dist.barrier()
+    total_ms = start.elapsed_time(end)
+    if dist is not None:
+        t = torch.tensor([total_ms], device=device, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    for st in sets:
+        if tsb.tsb_device_status(st["buf"].ws) != 0:
+            raise RuntimeError("device status bits set during the timed region")
+    per_kernel = {n: [] for n in KERNELS}
+    for k in range(K):
+        for i, n in enumerate(KERNELS):
+            per_kernel[n].append(events[k][i].elapsed_time(events[k][i + 1]) * 1e3)
+    kern_us = {n: statistics.mean(v) for n, v in per_kernel.items()}
+    us_step = total_ms * 1e3 / K
+
+    h_len = out_len.cpu().numpy()
+    h_nodes = out_nodes.cpu().numpy()
+    draft_bytes, target_bytes, q_bytes, visited = algorithmic_bytes(w, sets, h_len, h_nodes)
+    step_bytes = draft_bytes + float(target_bytes.mean())
+    hbm_gbs = step_bytes / (us_step * 1e-6) / 1e9
+    peak, peak_kind = measured_peak_hbm()
+
+    # roofline of the dominant kernel (largest share of the step)
+    dom = max(kern_us, key=kern_us.get)
+    C = (w["V"] + 255) // 256
+    es = 2 if w["dtype"] == "bf16" else 4
+    kernel_bytes = {
+        "tsb_row_stats": B * L * w["V"] * es + B * L * C * 8,
+        "tsb_verify": float(target_bytes.mean()),
+        "tsb_plan": B * L * C * 8,
+        "tsb_replay": B * w["N"] * (C * 8),
+    }
+    achieved = kernel_bytes[dom] / (kern_us[dom] * 1e-6) / 1e9
+    roofline = {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+                "frac": round(achieved / peak, 4), "peak_source": f"{peak_kind} (MEASURED_PEAKS hbm_gbs copy)",
+                "traffic": profiled_traffic(dom, w["name"]),
+                "bytes_per_launch": float(kernel_bytes[dom])}
+    per_kernel_gbs = {n: round(kernel_bytes[n] / (kern_us[n] * 1e-6) / 1e9, 1) for n in KERNELS}
+
+    # end to end through the C ABI with pinned host buffers
+    e2e = run_e2e(args, w, sets, device) if args.e2e_steps > 0 else None
+
+    cpu = None
+    if rank == 0 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(w, sets, seconds=12.0)
+
+    rows_per_s = world * (B * L + float(visited.mean())) / (us_step * 1e-6)
+    line = {
+        "metric": METRIC, "value": round(us_step, 3), "unit": "us/step", "n_gpus": world, "steps": K, "warmup": W,
+        "ms_per_step": round(us_step / 1e3, 6), "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
+        "dtype": w["dtype"], "data": "synthetic (seeded; shapes and value distributions of the batched serving "
+                                     "workload; no datasets or model weights)",
+        "config": config_of(w, {"parallelism": f"replicas x{world}" if world > 1 else "single GPU",
+                                "l2": f"{S} input sets rotated (per-step footprint {step_bytes / 1e6:.0f} MB, "
+                                      f"{S * step_bytes / L2_BYTES:.1f}x L2)",
+                                "launch": "eager C-ABI calls, inputs resident in HBM"}),
+        "hbm_gbs": round(hbm_gbs, 1), "hbm_frac_of_measured": round(hbm_gbs / peak, 4),
+        "hbm_frac_of_nominal_8tbs": round(hbm_gbs / NOMINAL_HBM_GBS, 4),
+        "algorithmic_bytes_per_step": round(step_bytes), "rows_per_s": round(rows_per_s, 1),
+        "mean_emitted_len": round(float(h_len.mean()), 4),
+        "per_kernel_us": {n: round(v, 3) for n, v in kern_us.items()},
+        "per_kernel_gbs": per_kernel_gbs,
+        "roofline": roofline,
+        "gpu_launches": 4 * K,
+        "clocks": clocks.summary(),
+        "e2e": e2e,
+        "cpu_baseline": cpu,
+    }
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+def run_e2e(args, w, sets, device):
+    import torch
+
+    from paper_2609_33652_gb300 import tsb
+
+    S = len(sets)
+    E = args.e2e_steps
+    h_draft = [st["draft"].cpu().pin_memory() for st in sets]
+    h_target = [st["target"].cpu().pin_memory() for st in sets]
+    d_draft = torch.empty_like(sets[0]["draft"])
+    d_target = torch.empty_like(sets[0]["target"])
+    bufs = [st["buf"] for st in sets]
+    B, L = w["B"], w["L"]
+    h_tok = torch.empty(B, L + 1, dtype=torch.int32).pin_memory()
+    h_len = torch.empty(B, dtype=torch.int32).pin_memory()
+    preps = [tsb.PreparedStep(bufs[k % S], d_draft, d_target, 5_000_000 + k) for k in range(E + 3)]
+
+    def one(k):
+        d_draft.copy_(h_draft[k % S], non_blocking=True)
+        d_target.copy_(h_target[k % S], non_blocking=True)
+        preps[k].run()
+        h_tok.copy_(bufs[k % S].out_tokens, non_blocking=True)
+        h_len.copy_(bufs[k % S].out_len, non_blocking=True)
+
+    for k in range(3):
+        one(k)
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record()
+    for k in range(3, 3 + E):
+        one(k)
+    b.record()
+    torch.cuda.synchronize()
+    us = a.elapsed_time(b) * 1e3 / E
+    es = sets[0]["draft"].element_size()
+    h2d = (sets[0]["draft"].numel() + sets[0]["target"].numel()) * es
+    d2h = h_tok.numel() * 4 + h_len.numel() * 4
+    return {"value": round(us, 3), "unit": "us/step", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
+            "steps": E}
+
+
+# ---------------------------------------------------------------------------------------
+def oracle_tree_step(w, draft_h, seed):
+    """The CPU oracle on one tree: plan, replay, then verify against target rows built (by the
+    shared input generator) from the oracle's own plan."""
+    import torch
+
+    import oracle
+    from paper_2609_33652_gb300 import synth
+
+    t0 = time.perf_counter()
+    ref = oracle.plan(draft_h, w["T"], w["N"], w["K"], w["L"])
+    tok, _ = oracle.replay(draft_h, w["T"], ref, seed)
+    t1 = time.perf_counter()
+    dt = torch.from_numpy(draft_h.view(np.int16)).view(torch.bfloat16) if draft_h.dtype == np.uint16 else \
+        torch.from_numpy(draft_h)
+    target = synth.to_host(synth.rows_from_depth(dt, torch.from_numpy(ref["depth"]), w["target_noise"], seed + 7))
+    t2 = time.perf_counter()
+    out = oracle.verify_rrs(target, draft_h, w["T"], ref, tok, seed, w["L"])
+    t3 = time.perf_counter()
+    return (t1 - t0) + (t3 - t2), out
+
+
+def cpu_baseline(w, sets, seconds=12.0):
+    import oracle
+    from paper_2609_33652_gb300 import synth
+
+    oracle.build()
+    times = []
+    k = 0
+    t_start = time.perf_counter()
+    while time.perf_counter() - t_start < seconds or k < 1:
+        st = sets[k % len(sets)]
+        b = k % w["B"]
+        h = synth.to_host(st["draft"][b:b + 1])
+        t, _ = oracle_tree_step(w, h, 100 + k)
+        times.append(t)
+        k += 1
+    per_tree = statistics.mean(times)
+    return {"value": round(per_tree * w["B"] * 1e6, 1), "unit": "us/step", "cores": 1, "kind": "oracle",
+            "sample": f"{k} single trees of the workload (plan + replay + verify, one thread), "
+                      f"mean per tree x B={w['B']}"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    from paper_2609_33652_gb300 import synth
+
+    w = workload(args)
+    K, W = args.steps, args.warmup
+    import torch
+
+    drafts = [synth.draft_logits(w["B"], w["L"], w["V"], "planted", w["dtype"], 1003 + 100 * s, device="cpu")
+              for s in range(2)]
+
+    def sample(k):
+        h = synth.to_host(drafts[k % 2][(k // 2) % w["B"]:(k // 2) % w["B"] + 1])
+        return oracle_tree_step(w, h, 10 + k)[0]
+
+    for k in range(W):
+        sample(k)
+    t_one = sample(W)
+    budget = 150.0
+    run_k = K if K * t_one <= budget else max(3, int(budget / t_one))
+    times = [sample(W + 1 + k) for k in range(run_k)]
+    us = statistics.mean(times) * w["B"] * 1e6
+    sample_txt = (f"one tree of B={w['B']} per step (plan + replay + verify, one thread), scaled by B; "
+                  f"{run_k} of the {K} requested steps run to stay within {budget:.0f} s")
+    line = {"impl": "reference", "metric": METRIC, "value": round(us, 1), "unit": "us/step", "n_gpus": args.gpus,
+            "steps": K, "steps_run": run_k, "warmup": W, "ms_per_step": round(us / 1e3, 4), "higher_is_better": False,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config_of(w),
+            "cpu_baseline": {"value": round(us, 1), "unit": "us/step", "cores": 1, "kind": "oracle",
+                             "sample": sample_txt},
+            "e2e": {"value": round(us, 1), "unit": "us/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    del torch
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_tsb(args)
+
+
+if __name__ == "__main__":
+    main()

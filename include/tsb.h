@@ -1,0 +1,179 @@
+/*
+ * tsb.h -- C ABI of libtsb, a GB300 (sm_103a) library for the per-step logit path of
+ * Tsubame's two-pass tree speculative decoding (Weng, Hu & Yairi, "Tsubame: Tree Replay for
+ * Diffusion-Based Speculative Decoding").
+ *
+ * One decoding step on B independent trees:
+ *
+ *   tsb_row_stats   draft rows            -> chunk statistics (max, sum of exp)
+ *   tsb_plan        draft rows + stats    -> frozen topology T (first pass, Sec. 3.1)
+ *   tsb_replay      q rows + stats + T    -> one fresh token per node (second pass, Sec. 3.2)
+ *   tsb_verify      target rows + q rows + T + tokens -> accepted path and final token
+ *                   (recursive rejection sampling, Sec. 2.3 and App. A; or block verification
+ *                   of a sampled chain, Sun et al. 2025 as cited in Sec. 1 and App. A)
+ *
+ * Conventions
+ *   - Every tensor pointer is a DEVICE pointer owned by the caller. The library never
+ *     allocates, frees or synchronises; the only call that waits is tsb_device_status.
+ *   - Calls are asynchronous on the given stream (NULL = legacy default stream).
+ *   - Host validation runs before anything is launched; on any error status nothing has
+ *     been launched and no output was touched.
+ *   - Problems that only the device can see (non-finite logits, an index out of range in a
+ *     caller-supplied array) set bits in a sticky status word kept in the caller's workspace;
+ *     tsb_device_status reads and clears it. Outputs of a call that set a bit are undefined.
+ *   - Functions keep no global state and are safe to call from several host threads on
+ *     different workspaces.
+ *   - Logits: element (b, r, v) is at data[b*batch_stride + r*row_stride + v], in elements.
+ *     batch_stride may be 0 (every tree shares the same rows). Every row must start on a
+ *     16-byte boundary (data, batch_stride*elem_size and row_stride*elem_size multiples of 16).
+ *     Values must be finite. A logit z is used as x = fp32(z) * fp32(1/T), one fp32 multiply.
+ *   - Randomness is Philox4x32-10 (Salmon et al., SC 2011) with key {seed lo32, seed hi32} and
+ *     counter {draw/4, node, batch, purpose}, word draw%4, uniform U = (w>>8 + 1/2) * 2^-24.
+ *     Every draw is keyed by what it is, so results do not depend on launch geometry.
+ */
+#ifndef TSB_H
+#define TSB_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *tsb_stream; /* the same type as cudaStream_t */
+
+typedef enum {
+    TSB_OK = 0,
+    TSB_ERR_ARG = 1,       /* NULL pointer, bad enum, non-positive or non-finite temperature */
+    TSB_ERR_SHAPE = 2,     /* sizes out of range or inconsistent between arguments */
+    TSB_ERR_DTYPE = 3,     /* logits dtype not TSB_F32 / TSB_BF16 */
+    TSB_ERR_ALIGN = 4,     /* a row does not start on a 16-byte boundary */
+    TSB_ERR_WORKSPACE = 5, /* workspace or stats buffer too small or misaligned */
+    TSB_ERR_CUDA = 6,      /* a CUDA runtime call or kernel launch failed */
+    TSB_ERR_DEVICE = 7     /* tsb_device_status found device-side status bits set */
+} tsb_status;
+
+/* Device status bits (sticky, in the workspace). */
+#define TSB_DEV_NONFINITE 0x1u /* a logit was NaN or infinite after the temperature multiply */
+#define TSB_DEV_BAD_INDEX 0x2u /* a token, row index or child index was out of range */
+#define TSB_DEV_BAD_TREE 0x4u  /* tree arrays inconsistent (e.g. block verification on a non-chain) */
+
+typedef enum { TSB_F32 = 0, TSB_BF16 = 1 } tsb_dtype;
+
+typedef enum {
+    TSB_VERIFY_RRS = 0,  /* recursive rejection sampling, WoR candidates, any topology */
+    TSB_VERIFY_BLOCK = 1 /* block verification; the topology must be the chain 0->1->...->N */
+} tsb_verify_mode;
+
+/* Limits (validated). */
+#define TSB_CHUNK 256 /* fixed chunk of the chunk statistics and of the replay sampler */
+#define TSB_MAX_K 32
+#define TSB_MAX_L 64
+#define TSB_MAX_N 1024
+#define TSB_MAX_B 65535
+#define TSB_MAX_V 409600 /* the verifier keeps one target and one q row slice per CTA in shared memory */
+
+typedef struct {
+    const void *data;     /* device pointer */
+    int32_t dtype;        /* tsb_dtype */
+    int32_t B, R, V;      /* trees, rows per tree, vocabulary */
+    int64_t batch_stride; /* elements between trees (0 = shared rows) */
+    int64_t row_stride;   /* elements between rows, >= V */
+} tsb_logits;
+
+typedef struct {
+    int32_t B;         /* trees in the batch, 1..TSB_MAX_B */
+    int32_t L;         /* draft block length = depth cap, 1..TSB_MAX_L */
+    int32_t N;         /* planned nodes besides the root, 1..TSB_MAX_N, N <= K + K^2 + ... + K^L */
+    int32_t K;         /* candidates per draft row = maximum children per node, 1..TSB_MAX_K, K <= V */
+    int32_t V;         /* vocabulary, 1..TSB_MAX_V */
+    float temperature; /* T > 0 and finite; applied to draft, q and target rows alike */
+} tsb_cfg;
+
+/* Frozen topology, device arrays. Node 0 is the root; nodes 1..N are numbered in the order
+ * the first pass pops them, so parent[i] < i. The children of u, in slot (rank) order, are
+ * child_ids[child_off[u] .. child_off[u+1]). */
+typedef struct {
+    int32_t *parent;     /* [B, N+1], parent[0] = -1 */
+    int32_t *depth;      /* [B, N+1], depth[0] = 0 */
+    int32_t *rank;       /* [B, N+1], slot among siblings; rank[0] = -1 */
+    int32_t *plan_token; /* [B, N+1], first-pass token (discarded by replay); -1 at the root */
+    float *score;        /* [B, N+1], draft path log-probability; 0 at the root */
+    int32_t *child_off;  /* [B, N+2] */
+    int32_t *child_ids;  /* [B, N] */
+} tsb_tree;
+
+/* Library version, major*10000 + minor*100 + patch. */
+int32_t tsb_version(void);
+
+/* Human-readable name of a status. Never NULL. */
+const char *tsb_status_str(tsb_status status);
+
+/* Bytes of the chunk-statistics buffer for B*R rows of V logits: one (max, sum exp) float
+ * pair per chunk of TSB_CHUNK logits, [B][R][ceil(V/TSB_CHUNK)]. 0 if the sizes are invalid. */
+size_t tsb_stats_bytes(int32_t B, int32_t R, int32_t V);
+
+/* Bytes of the workspace for a configuration: a status word plus per-(tree, node) scalars
+ * used by block verification, 256 + B*(N+1)*32. The workspace must be 256-byte aligned;
+ * tsb_row_stats needs only the first 256 bytes. 0 if the configuration is invalid. */
+size_t tsb_workspace_bytes(const tsb_cfg *cfg);
+
+/* Zero the workspace's status word on the stream. Call once before first use. */
+tsb_status tsb_workspace_init(void *ws, size_t ws_bytes, tsb_stream stream);
+
+/* Waits for the stream, then returns the device status bits in *bits and clears them.
+ * Returns TSB_OK if no bit was set, TSB_ERR_DEVICE if some were, TSB_ERR_CUDA if the CUDA
+ * context reported an error. */
+tsb_status tsb_device_status(void *ws, tsb_stream stream, uint32_t *bits);
+
+/* Chunk statistics of every row (the streaming pass over the logits): for chunk
+ * c = [c*TSB_CHUNK, min(V, (c+1)*TSB_CHUNK)) of row (b, r) it writes
+ * stats[(b*R + r)*C + c] = { m_c = max x_v, s_c = sum exp(x_v - m_c) }, x = fp32(z)*fp32(1/T).
+ * They give every row's log-normaliser, the per-position candidate pools of the first pass
+ * (Sec. 3.1) and the chunk log-masses of the replay sampler. stats: float2-aligned device
+ * buffer of tsb_stats_bytes(B, R, V). */
+tsb_status tsb_row_stats(const tsb_logits *rows, float temperature, void *stats, size_t stats_bytes, void *ws,
+                         size_t ws_bytes, tsb_stream stream);
+
+/* First pass (Sec. 3.1, App. B.3): per draft row d the top-K tokens by (x desc, id asc),
+ * then best-first (max-heap) expansion by cumulative draft path log-probability, popping N
+ * nodes. Candidates pop in the order (path log-probability desc, depth asc, sum of x desc,
+ * parent asc, rank asc); a node at depth d takes its token from draft row d-1; a node at
+ * depth L gets no children. draft: [B, >=L, V]; draft_stats: tsb_row_stats of the same rows
+ * and temperature. Writes every array of *out. */
+tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats, size_t stats_bytes,
+                    const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
+
+/* Second pass (Sec. 3.2, Eq. replay-distribution; WoR as in App. A): for every parent u
+ * with m_u children, draws m_u tokens without replacement from q_u = softmax(x of row
+ * qrow(u)) and writes the j-th draw to child slot j: token[b, child_ids[child_off[u]+j]].
+ * token[b, 0] = -1. qrows: [B, Rq, V] with its stats (same temperature); qrow_of_node:
+ * [B, N+1] row index per node, or NULL for per-depth rows (qrow(u) = depth[u]). The draws
+ * are the top-m_u Gumbel keys, built top-down over chunks of TSB_CHUNK tokens. */
+tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,
+                      const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
+                      size_t ws_bytes, tsb_stream stream);
+
+/* Verification on the frozen topology with the replayed tokens (Prop. 1).
+ * TSB_VERIFY_RRS: from the root, test the children in slot order, accept child i iff
+ *   U * q'(y_i) < p'(y_i) with q' the draft law renormalised over tokens not yet drawn and
+ *   p' the current residual target law; on rejection p' <- max(p' - q', 0) normalised over
+ *   the full vocabulary. An accepted child is emitted and the walk continues there; when all
+ *   children are rejected the final token is drawn from the last residual; at a leaf the
+ *   bonus token is drawn from the node's target row.
+ * TSB_VERIFY_BLOCK: block verification of the chain 0->1->...->N (requires N <= L).
+ * target: [B, N+1, V], row u = target logits after the path to node u. qrows / qstats /
+ * qrow_of_node as in tsb_replay. Outputs: out_tokens [B, L+1] (accepted tokens then the
+ * final token, -1 after), out_nodes [B, L] (accepted node ids, -1 after), out_len [B]
+ * (number of emitted tokens = accepted + 1). */
+tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target, const tsb_logits *qrows,
+                      const void *qstats, size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree,
+                      const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
+                      int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* TSB_H */

@@ -1,0 +1,183 @@
+// Second pass (Sec. 3.2, Eq. replay-distribution; sampling without replacement, App. A).
+//
+// For every parent u with m_u children, the m_u ordered draws without replacement from
+// q_u = softmax(x_row(u)) are the top-m_u Gumbel keys x_v + G_v (Gumbel-top-k). The keys are
+// built top-down (Maddison et al. 2014; Kool et al. 2019, App. B):
+//   1. chunk keys K_c = A_c + G(U[chunk c]) with A_c = m_c + log s_c from the chunk
+//      statistics; keep the top-m_u chunks by (K_c desc, c asc);
+//   2. inside each kept chunk, element keys g_v = x_v + G(U[token v]) are shifted to the law
+//      conditional on their maximum Z_c being K_c:
+//        k_v = K_c - softplus(K_c - g_v + log1p(-exp(g_v - Z_c))),  k_argmax = K_c;
+//   3. the top-m_u keys by (k desc, v asc) over the kept chunks are the draws; draw j fills
+//      child slot j.
+// Every token outside the kept chunks is below m_u distinct chunk maxima, so it can never
+// be among the top m_u: the joint law is exactly that of flat Gumbel-top-k over V tokens,
+// at ceil(V/256) + m_u*256 draws per parent instead of V.
+//
+// One warp per (tree, node); nodes without children return at once.
+#include "tsb_device.cuh"
+#include "tsb_launch.h"
+
+namespace tsb {
+namespace {
+
+constexpr int kWarps = 8;
+
+struct ReplayArgs {
+    const void *q;
+    int64_t bstride, rstride;
+    int R, V, C;
+    const float2 *stats;
+    const int32_t *qrow_of_node, *depth, *child_off, *child_ids;
+    int B, N;
+    float invT;
+    uint64_t seed;
+    int32_t *token;
+    uint32_t *status;
+};
+
+// Gumbel key conditioned on the chunk maximum (stable form).
+__device__ __forceinline__ float shifted_key(float T, float Z, float g) {
+    const float u = T - g + log1pf(-expf(g - Z));
+    const float sp = fmaxf(u, 0.f) + log1pf(expf(-fabsf(u)));
+    return T - sp;
+}
+
+template <int KCAP, typename T>
+__global__ void __launch_bounds__(kWarps * 32) k_replay(ReplayArgs a) {
+    __shared__ uint64_t sel_all[kWarps][KCAP];
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int NN = a.N + 1;
+    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
+    if (gw >= (int64_t)a.B * NN) return;
+    const int b = (int)(gw / NN), u = (int)(gw - (int64_t)b * NN);
+    if (u == 0 && lane == 0) a.token[(int64_t)b * NN] = -1;
+    const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+    const int o = off[u], m = off[u + 1] - o;
+    if (m <= 0) return;
+    if (m > KCAP || o < 0 || o + m > a.N) {
+        if (lane == 0) raise_status(a.status, kDevBadTree);
+        return;
+    }
+    const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
+    const int32_t *kids = a.child_ids + (int64_t)b * a.N + o;
+    if (r < 0 || r >= a.R) {
+        if (lane == 0) raise_status(a.status, kDevBadIndex);
+        return;
+    }
+    const float2 *st = a.stats + ((int64_t)b * a.R + r) * a.C;
+    const T *row = static_cast<const T *>(a.q) + (int64_t)b * a.bstride + (int64_t)r * a.rstride;
+    const uint32_t ub = (uint32_t)b, un = (uint32_t)u;
+
+    // 1. chunk keys; lane handles chunks 4j..4j+3 so one Philox block serves four draws
+    TopList<KCAP> cl;
+    cl.clear();
+    for (int c4 = lane * 4; c4 < a.C; c4 += 128) {
+        const Words4 w = draw_block(a.seed, kReplayChunk, ub, un, (uint32_t)(c4 >> 2));
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const int c = c4 + i;
+            if (c < a.C) {
+                const float2 s = st[c];
+                const float Kc = (s.x + logf(s.y)) + gumbel_of(w.w[i]);
+                cl.insert(pack_key(Kc, (uint32_t)c));
+            }
+        }
+    }
+    const int msel = min(m, a.C);
+    uint64_t *sel = sel_all[warp];
+    for (int j = 0; j < msel; ++j) {
+        const uint64_t best = warp_max_u64(cl.k[0]);
+        if (lane == 0) sel[j] = best;
+        if (cl.k[0] == best) cl.pop_front();
+    }
+    __syncwarp();
+
+    // 2. element keys inside the kept chunks, shifted to their chunk key
+    TopList<KCAP> el;
+    el.clear();
+    for (int s = 0; s < msel; ++s) {
+        const uint64_t kk = sel[s];
+        const int c = (int)key_id(kk);
+        const float Tc = key_value(kk);
+        const int v0 = c * kChunk + lane * 8;
+        float x[8];
+        Logit<T>::load8(row, v0, a.V, x);
+        const Words4 w0 = draw_block(a.seed, kReplayElem, ub, un, (uint32_t)(v0 >> 2));
+        const Words4 w1 = draw_block(a.seed, kReplayElem, ub, un, (uint32_t)(v0 >> 2) + 1u);
+        float g[8];
+        uint64_t zk = 0;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            g[i] = -INFINITY;
+            if (v0 + i < a.V) {
+                const uint32_t wi = i < 4 ? w0.w[i] : w1.w[i - 4];
+                g[i] = __fadd_rn(__fmul_rn(x[i], a.invT), gumbel_of(wi));
+                const uint64_t k = pack_key(g[i], (uint32_t)(v0 + i));
+                zk = k > zk ? k : zk;
+            }
+        }
+        zk = warp_max_u64(zk);
+        const float Z = key_value(zk);
+        const uint32_t jmax = key_id(zk);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+            if (v0 + i >= a.V) continue;
+            const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_key(Tc, Z, g[i]);
+            el.insert(pack_key(k, (uint32_t)(v0 + i)));
+        }
+    }
+    // 3. the top-m keys are the ordered draws
+    int32_t *tok = a.token + (int64_t)b * NN;
+    for (int j = 0; j < m; ++j) {
+        const uint64_t best = warp_max_u64(el.k[0]);
+        if (lane == 0) {
+            const int child = kids[j];
+            if (child > 0 && child < NN)
+                tok[child] = (int32_t)key_id(best);
+            else
+                raise_status(a.status, kDevBadTree);
+        }
+        if (el.k[0] == best) el.pop_front();
+    }
+}
+
+template <int KCAP, typename T>
+cudaError_t launch_replay_t(const ReplayArgs &a, cudaStream_t s) {
+    const int64_t warps = (int64_t)a.B * (a.N + 1);
+    const int64_t blocks = (warps + kWarps - 1) / kWarps;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    k_replay<KCAP, T><<<(unsigned)blocks, kWarps * 32, 0, s>>>(a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
+                          int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token, uint32_t *status,
+                          cudaStream_t s) {
+    ReplayArgs a;
+    a.q = q.data;
+    a.bstride = q.batch_stride;
+    a.rstride = q.row_stride;
+    a.R = q.R;
+    a.V = q.V;
+    a.C = num_chunks(q.V);
+    a.stats = qstats;
+    a.qrow_of_node = qrow_of_node;
+    a.depth = tree.depth;
+    a.child_off = tree.child_off;
+    a.child_ids = tree.child_ids;
+    a.B = B;
+    a.N = N;
+    a.invT = invT;
+    a.seed = seed;
+    a.token = token;
+    a.status = status;
+    // sibling groups have at most K members: a list of 8 covers K <= 8
+    if (q.dtype == 1)
+        return K <= 8 ? launch_replay_t<8, __nv_bfloat16>(a, s) : launch_replay_t<32, __nv_bfloat16>(a, s);
+    return K <= 8 ? launch_replay_t<8, float>(a, s) : launch_replay_t<32, float>(a, s);
+}
+
+}  // namespace tsb

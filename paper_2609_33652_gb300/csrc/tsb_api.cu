@@ -1,0 +1,218 @@
+// C ABI of libtsb (include/tsb.h): argument validation, workspace layout and kernel
+// launches on the caller's stream. Nothing is launched unless every check passes.
+#include <math.h>
+#include <stdint.h>
+
+#include "../../include/tsb.h"
+#include "tsb_launch.h"
+
+namespace {
+
+constexpr size_t kStatusBytes = 256;  // status word region at the start of the workspace
+constexpr size_t kBvRowBytes = 32;    // per (tree, chain position) scalars of block verification
+
+bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+
+int64_t max_nodes(int K, int L) {
+    int64_t total = 0, level = 1;
+    for (int d = 1; d <= L; ++d) {
+        level *= K;
+        total += level;
+        if (total > (int64_t)1 << 40) break;
+    }
+    return total;
+}
+
+tsb_status check_cfg(const tsb_cfg *c) {
+    if (!c) return TSB_ERR_ARG;
+    if (!(c->temperature > 0.0f) || !isfinite(c->temperature)) return TSB_ERR_ARG;
+    if (c->B < 1 || c->B > TSB_MAX_B || c->L < 1 || c->L > TSB_MAX_L || c->K < 1 || c->K > TSB_MAX_K ||
+        c->N < 1 || c->N > TSB_MAX_N || c->V < 1 || c->V > TSB_MAX_V || c->K > c->V)
+        return TSB_ERR_SHAPE;
+    if ((int64_t)c->N > max_nodes(c->K, c->L)) return TSB_ERR_SHAPE;
+    return TSB_OK;
+}
+
+// rows must hold at least B trees x R rows x V logits, 16-byte aligned rows
+tsb_status check_logits(const tsb_logits *t, int B, int R_min, int V) {
+    if (!t || !t->data) return TSB_ERR_ARG;
+    if (t->dtype != TSB_F32 && t->dtype != TSB_BF16) return TSB_ERR_DTYPE;
+    if (t->B != B || t->V != V || t->R < R_min || t->R < 1 || t->row_stride < t->V || t->batch_stride < 0)
+        return TSB_ERR_SHAPE;
+    const int64_t es = t->dtype == TSB_BF16 ? 2 : 4;
+    if (!aligned(t->data, 16) || (t->row_stride * es) % 16 != 0 || (t->batch_stride * es) % 16 != 0)
+        return TSB_ERR_ALIGN;
+    return TSB_OK;
+}
+
+tsb::RowsDesc rows_of(const tsb_logits *t) {
+    tsb::RowsDesc r;
+    r.data = t->data;
+    r.dtype = t->dtype;
+    r.B = t->B;
+    r.R = t->R;
+    r.V = t->V;
+    r.batch_stride = t->batch_stride;
+    r.row_stride = t->row_stride;
+    return r;
+}
+
+tsb::TreeDesc tree_of(const tsb_tree *t) {
+    tsb::TreeDesc d;
+    d.parent = t->parent;
+    d.depth = t->depth;
+    d.rank = t->rank;
+    d.plan_token = t->plan_token;
+    d.score = t->score;
+    d.child_off = t->child_off;
+    d.child_ids = t->child_ids;
+    return d;
+}
+
+size_t ws_bytes_for(const tsb_cfg *c) { return kStatusBytes + (size_t)c->B * ((size_t)c->N + 1) * kBvRowBytes; }
+
+tsb_status check_ws(void *ws, size_t ws_bytes, size_t need) {
+    if (!ws) return TSB_ERR_ARG;
+    if (!aligned(ws, 256) || ws_bytes < need) return TSB_ERR_WORKSPACE;
+    return TSB_OK;
+}
+
+tsb_status check_stats(const void *stats, size_t bytes, int B, int R, int V) {
+    if (!stats) return TSB_ERR_ARG;
+    if (!aligned(stats, 16) || bytes < tsb_stats_bytes(B, R, V)) return TSB_ERR_WORKSPACE;
+    return TSB_OK;
+}
+
+tsb_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TSB_OK : TSB_ERR_CUDA; }
+
+float inv_temperature(float T) { return 1.0f / T; }
+
+}  // namespace
+
+extern "C" {
+
+int32_t tsb_version(void) { return 100; }
+
+const char *tsb_status_str(tsb_status s) {
+    switch (s) {
+        case TSB_OK: return "ok";
+        case TSB_ERR_ARG: return "invalid argument";
+        case TSB_ERR_SHAPE: return "shape out of range or inconsistent";
+        case TSB_ERR_DTYPE: return "unsupported dtype";
+        case TSB_ERR_ALIGN: return "row not 16-byte aligned";
+        case TSB_ERR_WORKSPACE: return "workspace or stats buffer too small or misaligned";
+        case TSB_ERR_CUDA: return "CUDA error";
+        case TSB_ERR_DEVICE: return "device status bits set";
+    }
+    return "unknown status";
+}
+
+size_t tsb_stats_bytes(int32_t B, int32_t R, int32_t V) {
+    if (B < 1 || R < 1 || V < 1 || V > TSB_MAX_V) return 0;
+    return (size_t)B * (size_t)R * (size_t)tsb::num_chunks(V) * sizeof(float2);
+}
+
+size_t tsb_workspace_bytes(const tsb_cfg *cfg) {
+    if (!cfg || check_cfg(cfg) != TSB_OK) return 0;
+    return ws_bytes_for(cfg);
+}
+
+tsb_status tsb_workspace_init(void *ws, size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_ws(ws, ws_bytes, kStatusBytes);
+    if (st != TSB_OK) return st;
+    return cuda_status(cudaMemsetAsync(ws, 0, sizeof(uint32_t), (cudaStream_t)stream));
+}
+
+tsb_status tsb_device_status(void *ws, tsb_stream stream, uint32_t *bits) {
+    if (!ws || !bits) return TSB_ERR_ARG;
+    uint32_t host = 0;
+    cudaError_t e = cudaMemcpyAsync(&host, ws, sizeof host, cudaMemcpyDeviceToHost, (cudaStream_t)stream);
+    if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e == cudaSuccess && host) {
+        e = cudaMemsetAsync(ws, 0, sizeof(uint32_t), (cudaStream_t)stream);
+        if (e == cudaSuccess) e = cudaStreamSynchronize((cudaStream_t)stream);
+    }
+    *bits = host;
+    if (e != cudaSuccess) return TSB_ERR_CUDA;
+    return host ? TSB_ERR_DEVICE : TSB_OK;
+}
+
+tsb_status tsb_row_stats(const tsb_logits *rows, float temperature, void *stats, size_t stats_bytes, void *ws,
+                         size_t ws_bytes, tsb_stream stream) {
+    if (!rows) return TSB_ERR_ARG;
+    if (!(temperature > 0.0f) || !isfinite(temperature)) return TSB_ERR_ARG;
+    if (rows->B < 1 || rows->B > TSB_MAX_B || rows->V < 1 || rows->V > TSB_MAX_V) return TSB_ERR_SHAPE;
+    tsb_status st = check_logits(rows, rows->B, 1, rows->V);
+    if (st == TSB_OK) st = check_stats(stats, stats_bytes, rows->B, rows->R, rows->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, kStatusBytes);
+    if (st != TSB_OK) return st;
+    return cuda_status(tsb::launch_row_stats(rows_of(rows), inv_temperature(temperature),
+                                             static_cast<float2 *>(stats), static_cast<uint32_t *>(ws),
+                                             (cudaStream_t)stream));
+}
+
+tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats, size_t stats_bytes,
+                    const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_logits(draft, cfg->B, cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(draft_stats, stats_bytes, cfg->B, draft->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!out || !out->parent || !out->depth || !out->rank || !out->plan_token || !out->score || !out->child_off ||
+        !out->child_ids)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_plan(rows_of(draft), static_cast<const float2 *>(draft_stats), cfg->L, cfg->N,
+                                        cfg->K, inv_temperature(cfg->temperature), tree_of(out),
+                                        static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+}
+
+tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,
+                      const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
+                      size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(qstats, stats_bytes, cfg->B, qrows->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!tree || !tree->child_off || !tree->child_ids || (!qrow_of_node && !tree->depth) || !token)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_replay(rows_of(qrows), static_cast<const float2 *>(qstats), qrow_of_node, cfg->B,
+                                          cfg->N, cfg->K, tree_of(tree), inv_temperature(cfg->temperature), seed,
+                                          token, static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+}
+
+tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target, const tsb_logits *qrows,
+                      const void *qstats, size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree,
+                      const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
+                      int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    if (mode != TSB_VERIFY_RRS && mode != TSB_VERIFY_BLOCK) return TSB_ERR_ARG;
+    if (mode == TSB_VERIFY_BLOCK && cfg->N > cfg->L) return TSB_ERR_SHAPE;
+    st = check_logits(target, cfg->B, cfg->N + 1, cfg->V);
+    if (st == TSB_OK) st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
+    if (st == TSB_OK && target->dtype != qrows->dtype) st = TSB_ERR_DTYPE;
+    if (st == TSB_OK) st = check_stats(qstats, stats_bytes, cfg->B, qrows->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!tree || !tree->child_off || !tree->child_ids || (!qrow_of_node && !tree->depth) || !token ||
+        !out_tokens || !out_nodes || !out_len)
+        return TSB_ERR_ARG;
+    const float invT = inv_temperature(cfg->temperature);
+    cudaError_t e;
+    if (mode == TSB_VERIFY_RRS)
+        e = tsb::launch_verify_rrs(rows_of(target), rows_of(qrows), static_cast<const float2 *>(qstats),
+                                   qrow_of_node, cfg->B, cfg->N, cfg->L, tree_of(tree), token, invT, seed,
+                                   out_tokens, out_nodes, out_len, static_cast<uint32_t *>(ws),
+                                   (cudaStream_t)stream);
+    else
+        e = tsb::launch_verify_block(rows_of(target), rows_of(qrows), static_cast<const float2 *>(qstats),
+                                     qrow_of_node, cfg->B, cfg->N, cfg->L, tree_of(tree), token, invT, seed,
+                                     out_tokens, out_nodes, out_len, static_cast<uint32_t *>(ws),
+                                     (cudaStream_t)stream);
+    return cuda_status(e);
+}
+
+}  // extern "C"

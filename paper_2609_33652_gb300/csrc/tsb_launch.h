@@ -1,0 +1,44 @@
+// Host-side launchers of the libtsb kernels (internal; the public ABI is include/tsb.h).
+// Arguments are validated by the ABI layer before any of these is called.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace tsb {
+
+struct RowsDesc {
+    const void *data;
+    int dtype;  // 0 fp32, 1 bf16
+    int B, R, V;
+    int64_t batch_stride, row_stride;
+};
+
+struct TreeDesc {
+    int32_t *parent, *depth, *rank, *plan_token;
+    float *score;
+    int32_t *child_off, *child_ids;
+};
+
+inline int num_chunks(int V) { return (V + 255) / 256; }
+
+cudaError_t launch_row_stats(const RowsDesc &rows, float invT, float2 *stats, uint32_t *status, cudaStream_t s);
+
+cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
+                        const TreeDesc &tree, uint32_t *status, cudaStream_t s);
+
+cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
+                          int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token, uint32_t *status,
+                          cudaStream_t s);
+
+cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
+                              const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
+                              const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                              int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s);
+
+cudaError_t launch_verify_block(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
+                                const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
+                                const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                                int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s);
+
+}  // namespace tsb

@@ -50,8 +50,17 @@ def _gen(seed: int, device) -> torch.Generator:
     return g
 
 
+def _padded(V: int) -> int:
+    """Row length rounded up to 8 elements, so every row starts on a 16-byte boundary."""
+    return (V + 7) // 8 * 8
+
+
 def draft_logits(B: int, L: int, V: int, kind: str, dtype: str, seed: int, device="cpu") -> torch.Tensor:
-    """Per-depth draft logits [B, L, V] in ``dtype`` ("f32" or "bf16")."""
+    """Per-depth draft logits [B, L, V] in ``dtype`` ("f32" or "bf16"); rows are padded to a
+    multiple of 8 elements (the returned tensor is a view when V is not)."""
+    Vp = _padded(V)
+    if Vp != V:
+        return draft_logits(B, L, Vp, kind, dtype, seed, device)[..., :V]
     g = _gen(seed, device)
     if kind == "normal2":
         z = 2.0 * torch.randn(B, L, V, generator=g, device=device, dtype=torch.float32)
@@ -80,7 +89,10 @@ def rows_from_depth(draft: torch.Tensor, depth: torch.Tensor, noise_std: float, 
     base = torch.gather(draft.to(torch.float32), 1, idx.unsqueeze(-1).expand(B, NN, V))
     g = _gen(seed, draft.device)
     noise = torch.randn(B, NN, V, generator=g, device=draft.device, dtype=torch.float32)
-    return (base + noise_std * noise).to(draft.dtype).contiguous()
+    rows = (base + noise_std * noise).to(draft.dtype)
+    out = torch.empty(B, NN, _padded(V), dtype=draft.dtype, device=draft.device)[..., :V]
+    out.copy_(rows)
+    return out
 
 
 def to_host(t: torch.Tensor) -> np.ndarray:

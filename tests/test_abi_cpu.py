@@ -1,0 +1,133 @@
+"""The C ABI library builds, loads and exports every function include/tsb.h declares; host
+validation rejects bad arguments before any CUDA call (no GPU needed: the pointers below are
+fake device addresses that validation never dereferences)."""
+import ctypes
+import math
+import os
+import re
+
+import pytest
+
+from paper_2609_33652_gb300 import build as libbuild
+from paper_2609_33652_gb300 import tsb
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "tsb.h")
+
+OK, ARG, SHAPE, DTYPE, ALIGN, WS = 0, 1, 2, 3, 4, 5
+FAKE = 0x7F00_0000_0000  # 256-aligned fake device address
+
+
+@pytest.fixture(scope="module")
+def lib():
+    libbuild.build()
+    return tsb.load()
+
+
+def _declared():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(tsb_\w+)\s*\(", text)))
+
+
+def test_exports_every_declared_function(lib):
+    names = _declared()
+    assert set(names) == set(tsb.EXPORTS)
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_host_queries(lib):
+    assert tsb.tsb_version() >= 100
+    for s in range(8):
+        assert tsb.tsb_status_str(s)
+    assert tsb.tsb_status_str(99) == "unknown status"
+    assert tsb.tsb_stats_bytes(2, 3, 151936) == 2 * 3 * 594 * 8
+    assert tsb.tsb_stats_bytes(1, 1, 257) == 2 * 8
+    assert tsb.tsb_stats_bytes(0, 1, 10) == 0
+    cfg = tsb.make_cfg(16, 16, 64, 8, 151936, 1.0)
+    assert tsb.tsb_workspace_bytes(cfg) == 256 + 16 * 65 * 32
+    assert tsb.tsb_workspace_bytes(tsb.make_cfg(1, 2, 7, 2, 8, 1.0)) == 0  # N above K + K^2
+
+
+def _logits(B, R, V, dtype=0, data=FAKE, bstride=None, rstride=None):
+    rs = V if rstride is None else rstride
+    return tsb.Logits(data, dtype, B, R, V, R * rs if bstride is None else bstride, rs)
+
+
+def _tree():
+    return tsb.Tree(*([FAKE] * 7))
+
+
+def _plan(lib, cfg, draft, stats_bytes=1 << 30, ws_bytes=1 << 30, ws=FAKE, tree=None):
+    t = tree if tree is not None else _tree()
+    return lib.tsb_plan(ctypes.byref(cfg) if cfg is not None else None, ctypes.byref(draft), FAKE, stats_bytes,
+                        ctypes.byref(t), ws, ws_bytes, None)
+
+
+def test_plan_validation(lib):
+    good = tsb.make_cfg(4, 16, 64, 8, 1024, 1.0)
+    d = _logits(4, 16, 1024)
+    assert _plan(lib, None, d) == ARG
+    for T in (0.0, -1.0, math.nan, math.inf):
+        assert _plan(lib, tsb.make_cfg(4, 16, 64, 8, 1024, T), d) == ARG
+    assert _plan(lib, tsb.make_cfg(4, 16, 64, 33, 1024, 1.0), d) == SHAPE  # K > 32
+    assert _plan(lib, tsb.make_cfg(4, 16, 64, 8, 4, 1.0), _logits(4, 16, 4)) == SHAPE  # K > V
+    assert _plan(lib, tsb.make_cfg(4, 2, 7, 2, 1024, 1.0), _logits(4, 2, 1024)) == SHAPE  # N > K + K^2
+    assert _plan(lib, tsb.make_cfg(4, 65, 64, 8, 1024, 1.0), _logits(4, 65, 1024)) == SHAPE  # L > 64
+    assert _plan(lib, tsb.make_cfg(4, 16, 1025, 8, 1024, 1.0), d) == SHAPE  # N > 1024
+    assert _plan(lib, tsb.make_cfg(0, 16, 64, 8, 1024, 1.0), _logits(0, 16, 1024)) == SHAPE
+    assert _plan(lib, good, _logits(4, 15, 1024)) == SHAPE  # fewer draft rows than L
+    assert _plan(lib, good, _logits(5, 16, 1024)) == SHAPE  # batch mismatch
+    assert _plan(lib, good, _logits(4, 16, 1024, dtype=2)) == DTYPE
+    assert _plan(lib, good, _logits(4, 16, 1024, data=FAKE + 4)) == ALIGN
+    assert _plan(lib, good, _logits(4, 16, 1024, rstride=1026)) == ALIGN  # 1026 * 4 bytes
+    assert _plan(lib, good, _logits(4, 16, 1024, dtype=1, rstride=1028)) == ALIGN  # 1028 * 2 bytes
+    assert _plan(lib, good, _logits(4, 16, 1024, rstride=1000)) == SHAPE  # row stride < V
+    assert _plan(lib, good, d, stats_bytes=4 * 16 * 4 * 8 - 8) == WS
+    assert _plan(lib, good, d, ws_bytes=255) == WS
+    assert _plan(lib, good, d, ws=FAKE + 8) == WS
+    assert _plan(lib, good, d, ws=None) == ARG
+    t = _tree()
+    t.child_ids = None
+    assert _plan(lib, good, d, tree=t) == ARG
+    # broadcast rows (batch stride 0) are accepted by validation
+    cfg1 = tsb.make_cfg(4, 2, 6, 2, 8, 1.0)
+    assert lib.tsb_workspace_bytes(ctypes.byref(cfg1)) == 256 + 4 * 7 * 32
+
+
+def test_replay_verify_validation(lib):
+    cfg = tsb.make_cfg(2, 4, 8, 4, 64, 1.0)
+    q = _logits(2, 4, 64)
+    t = _tree()
+
+    def replay(cfg=cfg, q=q, qrow=None, token=FAKE):
+        return lib.tsb_replay(ctypes.byref(cfg), ctypes.byref(q), FAKE, 1 << 30, qrow, ctypes.byref(t), 1, token,
+                              FAKE, 1 << 30, None)
+
+    assert replay(token=None) == ARG
+    assert replay(q=_logits(2, 3, 64)) == SHAPE  # per-depth rows need L rows
+    assert replay(q=_logits(2, 3, 64), qrow=FAKE) != SHAPE  # per-node rows: any row count (validated on device)
+
+    def verify(mode=0, target=None, q=q, cfg=cfg, out=FAKE):
+        tg = target if target is not None else _logits(2, 9, 64)
+        return lib.tsb_verify(ctypes.byref(cfg), mode, ctypes.byref(tg), ctypes.byref(q), FAKE, 1 << 30, None,
+                              ctypes.byref(t), FAKE, 1, out, FAKE, FAKE, FAKE, 1 << 30, None)
+
+    assert verify(mode=2) == ARG
+    assert verify(target=_logits(2, 8, 64)) == SHAPE  # needs N+1 target rows
+    assert verify(target=_logits(2, 9, 64, dtype=1)) == DTYPE  # target / q dtypes differ
+    assert verify(out=None) == ARG
+    assert verify(mode=1, cfg=tsb.make_cfg(2, 4, 5, 4, 64, 1.0)) == SHAPE  # block: chain longer than L
+
+
+def test_workspace_and_status_validation(lib):
+    assert lib.tsb_workspace_init(None, 256, None) == ARG
+    assert lib.tsb_workspace_init(FAKE, 100, None) == WS
+    bits = ctypes.c_uint32(0)
+    assert lib.tsb_device_status(None, None, ctypes.byref(bits)) == ARG
+    assert lib.tsb_row_stats(None, 1.0, FAKE, 1 << 20, FAKE, 256, None) == ARG
+    rows = _logits(1, 2, 300)
+    assert lib.tsb_row_stats(ctypes.byref(rows), 0.0, FAKE, 1 << 20, FAKE, 256, None) == ARG
+    assert lib.tsb_row_stats(ctypes.byref(rows), 1.0, FAKE, 2 * 2 * 8 - 1, FAKE, 256, None) == WS
+    assert lib.tsb_row_stats(ctypes.byref(_logits(1, 2, 409601)), 1.0, FAKE, 1 << 30, FAKE, 256, None) == SHAPE

@@ -1,0 +1,219 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on identical seeded
+inputs, for every workload shape, plus edge cases, losslessness and device status bits."""
+import numpy as np
+import pytest
+import torch
+
+import helpers
+import oracle
+from gpu_harness import check_status, gpu_plan, run_step
+from paper_2609_33652_gb300 import synth, tsb
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2609_33652_gb300 import build
+
+    build.build()
+    oracle.build()
+    tsb.load()
+
+
+DEV = "cuda"
+
+
+def _draft(B, L, V, kind, dtype, seed):
+    return synth.draft_logits(B, L, V, kind, dtype, seed, device=DEV)
+
+
+def _assert_mostly_compared(rep, min_frac=0.9):
+    for stage in ("plan", "replay", "verify"):
+        tot = rep.compared[stage] + rep.skipped[stage]
+        if tot:
+            assert rep.compared[stage] >= min_frac * tot, rep
+
+
+# --------------------------------------------------------------------------------------
+@pytest.mark.parametrize("B,R,V,dtype,T", [(3, 4, 32, "f32", 1.0), (2, 3, 1000, "bf16", 1.0),
+                                           (2, 2, 1001, "f32", 0.6), (2, 3, 151936, "bf16", 1.0),
+                                           (1, 2, 128256, "f32", 0.6)])
+def test_row_stats(B, R, V, dtype, T):
+    rows = _draft(B, R, V, "planted" if V > 100 else "normal2", dtype, 1)
+    stats = torch.empty(tsb.tsb_stats_bytes(B, R, V) // 4, dtype=torch.float32, device=DEV)
+    ws = torch.zeros(256, dtype=torch.uint8, device=DEV)
+    tsb.tsb_row_stats(rows, T, stats, ws)
+    assert tsb.tsb_device_status(ws) == 0
+    C = (V + 255) // 256
+    st = stats.view(B, R, C, 2).cpu().numpy().astype(np.float64)
+    h = synth.to_host(rows.contiguous())
+    ref = oracle.row_stats(h, T)
+    x = (h.astype(np.float32) if h.dtype == np.float32 else (h.astype(np.uint32) << 16).view(np.float32))
+    x = x * np.float32(np.float32(1.0) / np.float32(T))
+    for c in range(C):
+        np.testing.assert_array_equal(st[:, :, c, 0], x[:, :, c * 256:(c + 1) * 256].max(axis=2))
+    np.testing.assert_allclose(st[..., 0] + np.log(st[..., 1]), ref["chunk_lse"], rtol=1e-6, atol=2e-6)
+
+
+@pytest.mark.parametrize("seed", [1, 2])
+def test_step_tiny(seed):
+    w = synth.WORKLOADS["tiny"]
+    draft = _draft(256, w["L"], w["V"], "normal2", "f32", 1000 + seed)
+    rep, buf, _ = run_step(draft, w["L"], w["N"], w["K"], w["T"], seed=seed, target_noise=1.0)
+    _assert_mostly_compared(rep, 0.98)
+
+
+def test_step_single_stream():
+    w = synth.WORKLOADS["single"]
+    draft = _draft(4, w["L"], w["V"], "planted", "bf16", 1001)
+    rep, _, _ = run_step(draft, w["L"], w["N"], w["K"], w["T"], seed=11, target_noise=w["target_noise"])
+    _assert_mostly_compared(rep, 0.74)
+
+
+@pytest.mark.parametrize("V", [151936, 128256])
+def test_step_batched(V):
+    w = synth.WORKLOADS["batched"]
+    draft = _draft(w["B"], w["L"], V, "planted", "bf16", 1003)
+    rep, _, gout = run_step(draft, w["L"], w["N"], w["K"], w["T"], seed=5, target_noise=w["target_noise"])
+    _assert_mostly_compared(rep, 0.85)
+    assert (gout["len"] >= 1).all()
+
+
+@pytest.mark.parametrize("T", [0.6, 1.0])
+def test_step_corrected_per_node_rows(T):
+    w = synth.WORKLOADS["corrected"]
+    B = 4
+    draft = _draft(B, w["L"], w["V"], "planted", "bf16", 1002)
+    buf = gpu_plan(draft, w["L"], w["N"], w["K"], T)
+    qrows = synth.rows_from_depth(draft, buf.tree["depth"], w["per_node_noise"], seed=3000)
+    qidx = torch.arange(w["N"] + 1, dtype=torch.int32, device=DEV).repeat(B, 1).contiguous()
+    rep, _, _ = run_step(draft, w["L"], w["N"], w["K"], T, seed=9, target_noise=w["target_noise"], qrows=qrows,
+                         qrow_of_node=qidx)
+    _assert_mostly_compared(rep, 0.74)
+
+
+@pytest.mark.parametrize("N,dtype", [(16, "bf16"), (256, "f32")])
+def test_step_sweep_sampled(N, dtype):
+    """Full-size batch (B=64); the oracle checks a sample of trees one by one."""
+    w = synth.WORKLOADS["sweep"]
+    draft = _draft(64, w["L"], w["V"], "planted", dtype, 1004)
+    rep, _, _ = run_step(draft, w["L"], N, w["K"], w["T"], seed=3, target_noise=w["target_noise"],
+                         trees=[0, 21, 42, 63])
+    _assert_mostly_compared(rep, 0.74)
+
+
+def test_block_verification_chain():
+    """Sampled chain (plan with K=1, replay = one draw per node) verified by block
+    verification, on the batched workload's draft rows."""
+    w = synth.WORKLOADS["batched"]
+    g = 16
+    draft = _draft(w["B"], w["L"], 151936, "planted", "bf16", 1003)
+    rep, buf, gout = run_step(draft, w["L"], g, 1, w["T"], seed=21, target_noise=w["target_noise"],
+                              mode=tsb.TSB_VERIFY_BLOCK)
+    _assert_mostly_compared(rep, 0.85)
+    assert (gout["len"] >= 1).all() and (gout["len"] <= g + 1).all()
+
+
+def test_block_verification_tiny_many():
+    w = synth.WORKLOADS["tiny"]
+    draft = _draft(300, w["L"], w["V"], "normal2", "f32", 1010)
+    rep, _, _ = run_step(draft, w["L"], w["L"], 1, 1.0, seed=4, target_noise=1.0, mode=tsb.TSB_VERIFY_BLOCK)
+    _assert_mostly_compared(rep, 0.98)
+
+
+# --------------------------------------------------------------------------------------
+# edge cases
+def test_edges_chain_full_tree_ragged():
+    # K = 1 (chain of length min(N, L))
+    draft = _draft(8, 6, 1000, "normal3", "f32", 7)
+    run_step(draft, 6, 6, 1, 1.0, seed=1, target_noise=0.7)
+    # N = full capacity of a K=2, L=3 tree
+    draft = _draft(8, 3, 640, "normal3", "bf16", 8)
+    run_step(draft, 3, 14, 2, 1.0, seed=2, target_noise=0.7)
+    # V not a multiple of 8 (scalar tail), V below one chunk, K = V
+    run_step(_draft(8, 4, 1001, "normal3", "f32", 9), 4, 20, 4, 0.8, seed=3, target_noise=0.7)
+    run_step(_draft(8, 4, 1001, "normal3", "bf16", 9), 4, 20, 4, 0.8, seed=3, target_noise=0.7)
+    run_step(_draft(8, 3, 5, "normal2", "f32", 10), 3, 12, 5, 1.0, seed=4, target_noise=1.0)
+    # N = 1, L = 1
+    run_step(_draft(8, 1, 300, "normal3", "bf16", 11), 1, 1, 1, 1.0, seed=5, target_noise=0.7)
+    # K = 32 (largest candidate list)
+    run_step(_draft(4, 4, 4096, "normal3", "bf16", 12), 4, 200, 32, 1.0, seed=6, target_noise=0.7)
+
+
+def test_edges_broadcast_rows():
+    """Every tree shares the same draft rows (batch stride 0): identical topology, different
+    draws per tree."""
+    w = synth.WORKLOADS["tiny"]
+    base = _draft(1, w["L"], 512, "normal3", "f32", 13)
+    draft = base.expand(64, -1, -1)
+    rep, buf, _ = run_step(draft, w["L"], w["N"], w["K"], 1.0, seed=8, target_noise=0.7)
+    p = buf.tree["parent"].cpu().numpy()
+    assert (p == p[0]).all()
+    tok = buf.token.cpu().numpy()
+    assert len({tuple(t) for t in tok}) > 1
+
+
+def test_determinism_and_launch_independence():
+    w = synth.WORKLOADS["tiny"]
+    draft = _draft(32, w["L"], 2000, "normal3", "bf16", 14)
+    _, _, g1 = run_step(draft, w["L"], 30, 4, 1.0, seed=9, target_noise=0.7)
+    _, _, g2 = run_step(draft, w["L"], 30, 4, 1.0, seed=9, target_noise=0.7)
+    for k in g1:
+        assert np.array_equal(g1[k], g2[k])
+
+
+# --------------------------------------------------------------------------------------
+def test_losslessness_on_gpu():
+    """1e5 trees share the tiny workload's draft rows; targets are functions of the token
+    path. The first emitted token must follow the root target law (chi-square), and the GPU
+    outputs must equal the oracle's on every non-exempt tree."""
+    w = synth.WORKLOADS["tiny"]
+    B, L, N, K, V, T = 100_000, w["L"], w["N"], w["K"], w["V"], w["T"]
+    base1 = _draft(1, L, V, "normal2", "f32", 1000)
+    draft = base1.expand(B, -1, -1)
+    buf = gpu_plan(draft, L, N, K, T)
+    seed = 31
+    tsb.tsb_replay(buf.cfg, draft, buf.stats, None, buf.tree, seed, buf.token, buf.ws)
+    check_status(buf)
+    tree = {k: v.cpu().numpy() for k, v in buf.tree.items()}
+    tok = buf.token.cpu().numpy()
+    base = synth.to_host(base1)[0]
+    target_h = synth.path_keyed_rows(base, tree["parent"], tree["depth"], tok, 1.0, seed=77)
+    target = torch.from_numpy(target_h).to(DEV)
+    tsb.tsb_verify(buf.cfg, tsb.TSB_VERIFY_RRS, target, draft, buf.stats, None, buf.tree, buf.token, seed,
+                   buf.out_tokens, buf.out_nodes, buf.out_len, buf.ws)
+    check_status(buf)
+    first = buf.out_tokens[:, 0].cpu().numpy()
+    p_root = helpers.softmax64(synth.path_keyed_row(base, [], 1.0, 77))
+    assert helpers.chi2_pvalue(np.bincount(first, minlength=V), p_root) > 1e-4
+    # oracle on the same inputs (its own plan, replay and path-keyed targets)
+    h_draft = np.ascontiguousarray(np.broadcast_to(base[None], (B, L, V)))
+    ref = oracle.plan(h_draft, T, N, K, L)
+    for k in ("parent", "child_ids"):
+        assert np.array_equal(ref[k], tree[k])
+    rtok, rex = oracle.replay(h_draft, T, ref, seed)
+    rt = synth.path_keyed_rows(base, ref["parent"], ref["depth"], rtok, 1.0, seed=77)
+    rout = oracle.verify_rrs(rt, h_draft, T, ref, rtok, seed, L)
+    ok = ~rex.any(axis=1)
+    assert np.array_equal(tok[ok], rtok[ok])
+    ok &= ~rout["exempt"]
+    assert ok.mean() > 0.995
+    assert np.array_equal(buf.out_len.cpu().numpy()[ok], rout["len"][ok])
+    assert np.array_equal(buf.out_tokens.cpu().numpy()[ok], rout["tokens"][ok])
+
+
+def test_device_status_bits():
+    draft = _draft(2, 3, 512, "normal3", "f32", 15).clone()
+    draft[1, 2, 100] = float("nan")
+    buf = gpu_plan(draft, 3, 10, 3, 1.0)
+    assert tsb.tsb_device_status(buf.ws) & tsb.TSB_DEV_NONFINITE
+    assert tsb.tsb_device_status(buf.ws) == 0  # cleared by the read
+    draft = _draft(2, 3, 512, "normal3", "f32", 16)
+    buf = gpu_plan(draft, 3, 10, 3, 1.0)
+    check_status(buf)
+    bad = torch.full((2, 11), 7, dtype=torch.int32, device=DEV)  # row 7 of a 3-row tensor
+    tsb.tsb_replay(buf.cfg, draft, buf.stats, bad, buf.tree, 1, buf.token, buf.ws)
+    assert tsb.tsb_device_status(buf.ws) & tsb.TSB_DEV_BAD_INDEX
