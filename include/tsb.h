@@ -71,7 +71,7 @@ typedef enum {
 #define TSB_MAX_K 32
 #define TSB_MAX_L 64
 #define TSB_MAX_N 1024
-#define TSB_MAX_B 65535
+#define TSB_MAX_B 1048576
 #define TSB_MAX_V 409600 /* the verifier keeps one target and one q row slice per CTA in shared memory */
 
 typedef struct {
@@ -114,9 +114,10 @@ const char *tsb_status_str(tsb_status status);
  * pair per chunk of TSB_CHUNK logits, [B][R][ceil(V/TSB_CHUNK)]. 0 if the sizes are invalid. */
 size_t tsb_stats_bytes(int32_t B, int32_t R, int32_t V);
 
-/* Bytes of the workspace for a configuration: a status word plus per-(tree, node) scalars
- * used by block verification, 256 + B*(N+1)*32. The workspace must be 256-byte aligned;
- * tsb_row_stats needs only the first 256 bytes. 0 if the configuration is invalid. */
+/* Bytes of the workspace for a configuration: a status word (256 bytes), per-(tree, node)
+ * scalars of block verification (B*(N+1)*32) and the first pass's per-draft-row results
+ * (B*L*(8 + 8*K)). The workspace must be 256-byte aligned; tsb_row_stats needs only the first
+ * 256 bytes. 0 if the configuration is invalid. */
 size_t tsb_workspace_bytes(const tsb_cfg *cfg);
 
 /* Zero the workspace's status word on the stream. Call once before first use. */

@@ -38,7 +38,8 @@ _LIB_PATH = os.path.join(_HERE, "liboracle.so")
 _lib = None
 
 CHUNK = 256
-PURPOSE_REPLAY_CHUNK, PURPOSE_REPLAY_ELEM, PURPOSE_ACCEPT, PURPOSE_FINAL, PURPOSE_BLOCK_ETA = 0, 1, 2, 3, 4
+(PURPOSE_REPLAY_CHUNK, PURPOSE_REPLAY_ELEM, PURPOSE_ACCEPT, PURPOSE_FINAL, PURPOSE_BLOCK_ETA,
+ PURPOSE_FINAL_CHUNK) = 0, 1, 2, 3, 4, 5
 
 
 def build_command(out=_LIB_PATH):
@@ -78,13 +79,14 @@ def _load():
         "orc_uniform": (ctypes.c_double, [ctypes.c_uint64, _I, _I, _I, _I]),
         "orc_row_stats": (_I, [_P, ctypes.c_float, _I, _P, _P, _P, _P, _P]),
         "orc_plan": (_I, [_P, ctypes.c_float, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, ctypes.c_double, _P, _P]),
-        "orc_replay": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, ctypes.c_uint64, _P, _P]),
-        "orc_replay_flat": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, ctypes.c_uint64, _P]),
+        "orc_replay": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, ctypes.c_uint64, _P, _P, _P]),
+        "orc_replay_flat": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, ctypes.c_uint64, _P, _P]),
         "orc_rrs_node_law": (_I, [_I, _P, _P, _I, _P, _P, _P]),
-        "orc_verify_rrs": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P]),
+        "orc_verify_rrs": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P,
+                                _P]),
         "orc_blockv_law": (_I, [_I, _I, _P, _P, _P, _P, _P, _P]),
         "orc_verify_block": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P,
-                                  _P, _P]),
+                                  _P, _P, _P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -182,9 +184,12 @@ def _tree_ptrs(tree):
     return (_i32(tree["depth"]), _i32(tree["child_off"]), _i32(tree["child_ids"]))
 
 
-def replay(q: np.ndarray, temperature: float, tree, seed: int, qrow_of_node=None, flat: bool = False):
-    """Tokens [B, N+1] (root -1) and, for the hierarchical sampler, a per-parent near-tie flag."""
+def replay(q: np.ndarray, temperature: float, tree, seed: int, qrow_of_node=None, flat: bool = False,
+           batch_ids=None):
+    """Tokens [B, N+1] (root -1) and, for the hierarchical sampler, a per-parent near-tie flag.
+    ``batch_ids`` gives the Philox batch index of each tree (default 0..B-1)."""
     lib = _load()
+    bids = _i32(batch_ids)
     B = q.shape[0]
     NN = tree["depth"].shape[1]
     d, keep = _logits(q)
@@ -193,17 +198,18 @@ def replay(q: np.ndarray, temperature: float, tree, seed: int, qrow_of_node=None
     token = np.zeros(B * NN, dtype=np.int32)
     if flat:
         _check(lib.orc_replay_flat(ctypes.byref(d), temperature, _ptr(qr), NN - 1, _ptr(depth), _ptr(off), _ptr(ids),
-                                   int(seed), _ptr(token)), "replay_flat")
+                                   int(seed), _ptr(bids), _ptr(token)), "replay_flat")
         return token.reshape(B, NN)
     exempt = np.zeros(B * NN, dtype=np.uint8)
     _check(lib.orc_replay(ctypes.byref(d), temperature, _ptr(qr), NN - 1, _ptr(depth), _ptr(off), _ptr(ids),
-                          int(seed), _ptr(token), _ptr(exempt)), "replay")
+                          int(seed), _ptr(bids), _ptr(token), _ptr(exempt)), "replay")
     return token.reshape(B, NN), exempt.reshape(B, NN).astype(bool)
 
 
 def verify_rrs(target: np.ndarray, q: np.ndarray, temperature: float, tree, token, seed: int, L: int,
-               qrow_of_node=None):
+               qrow_of_node=None, batch_ids=None):
     lib = _load()
+    bids = _i32(batch_ids)
     B = target.shape[0]
     NN = tree["depth"].shape[1]
     dt, keep_t = _logits(target)
@@ -216,14 +222,15 @@ def verify_rrs(target: np.ndarray, q: np.ndarray, temperature: float, tree, toke
     olen = np.zeros(B, dtype=np.int32)
     ex = np.zeros(B, dtype=np.uint8)
     _check(lib.orc_verify_rrs(ctypes.byref(dt), ctypes.byref(dq), temperature, _ptr(qr), NN - 1, L, _ptr(depth),
-                              _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(otok), _ptr(onode), _ptr(olen),
-                              _ptr(ex)), "verify_rrs")
+                              _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(bids), _ptr(otok), _ptr(onode),
+                              _ptr(olen), _ptr(ex)), "verify_rrs")
     return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool)}
 
 
 def verify_block(target: np.ndarray, q: np.ndarray, temperature: float, tree, token, seed: int, L: int,
-                 qrow_of_node=None):
+                 qrow_of_node=None, batch_ids=None):
     lib = _load()
+    bids = _i32(batch_ids)
     B = target.shape[0]
     NN = tree["depth"].shape[1]
     dt, keep_t = _logits(target)
@@ -237,8 +244,8 @@ def verify_block(target: np.ndarray, q: np.ndarray, temperature: float, tree, to
     ex = np.zeros(B, dtype=np.uint8)
     tau = np.zeros(B, dtype=np.int32)
     _check(lib.orc_verify_block(ctypes.byref(dt), ctypes.byref(dq), temperature, _ptr(qr), NN - 1, L, _ptr(depth),
-                                _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(otok), _ptr(onode), _ptr(olen),
-                                _ptr(ex), _ptr(tau)), "verify_block")
+                                _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(bids), _ptr(otok), _ptr(onode),
+                                _ptr(olen), _ptr(ex), _ptr(tau)), "verify_block")
     return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool),
             "tau": tau}
 

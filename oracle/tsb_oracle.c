@@ -30,11 +30,16 @@ enum {
     PURPOSE_REPLAY_ELEM = 1,  /* node = parent, draw = token id           */
     PURPOSE_ACCEPT = 2,       /* node = child being tested, draw = 0      */
     PURPOSE_FINAL = 3,        /* node = where the final token is drawn, draw = token id */
-    PURPOSE_BLOCK_ETA = 4     /* node = chain position i, draw = 0         */
+    PURPOSE_BLOCK_ETA = 4,    /* node = chain position i, draw = 0         */
+    PURPOSE_FINAL_CHUNK = 5   /* node = where the final token is drawn, draw = chunk index */
 };
 
-/* Uniform-space half-width of a near tie (the parity contract's 1e-6 band). */
+/* Near ties. A decision taken from floating point is flagged when a uniform that decides it
+ * lies within U_BAND of the value that would flip it (the parity contract's 1e-6 band), or
+ * when the compared keys differ by less than KEY_BAND relative (fp32 key rounding on the
+ * device side, a few ulp). */
 static const double U_BAND = 1e-6;
+static const double KEY_BAND = 1e-6;
 
 /* ------------------------------------------------------------------------------------ */
 /* Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3",
@@ -367,18 +372,26 @@ static void partial_sort(elem_key *e, int n, int take)
 }
 
 /* Is the decision "a before b" a near tie in uniform space? */
+static int near_tie_keys(double ka, double kb, double sens)
+{
+    double dk = ka - kb;
+    double mag = fabs(ka) > 1.0 ? fabs(ka) : 1.0;
+    return dk < U_BAND * sens || dk < KEY_BAND * mag;
+}
+
 static int near_tie(const elem_key *a, const elem_key *b)
 {
-    double dk = a->k - b->k;
-    double s = a->sens > b->sens ? a->sens : b->sens;
-    return dk < U_BAND * s;
+    return near_tie_keys(a->k, b->k, a->sens > b->sens ? a->sens : b->sens);
 }
+
+/* The Philox batch index of local tree b (callers may pass a sample of a larger batch). */
+static int batch_of(const int32_t *batch_ids, int b) { return batch_ids ? batch_ids[b] : b; }
 
 static int replay_row_index(const int32_t *qrow_of_node, const int32_t *depth, int64_t idx) { return qrow_of_node ? qrow_of_node[idx] : depth[idx]; }
 
 int orc_replay(const orc_logits *q, float temperature, const int32_t *qrow_of_node, int32_t N,
                const int32_t *depth, const int32_t *child_off, const int32_t *child_ids, uint64_t seed,
-               int32_t *token, uint8_t *exempt_node)
+               const int32_t *batch_ids, int32_t *token, uint8_t *exempt_node)
 {
     if (!q || N < 0 || !(temperature > 0.0f)) return -1;
     const float invT = 1.0f / temperature;
@@ -402,7 +415,7 @@ int orc_replay(const orc_logits *q, float temperature, const int32_t *qrow_of_no
             for (int c = 0; c < C; ++c) {
                 int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
                 A[c] = logsumexp(x + lo, hi - lo);
-                double uc = orc_uniform(seed, PURPOSE_REPLAY_CHUNK, b, u, c);
+                double uc = orc_uniform(seed, PURPOSE_REPLAY_CHUNK, batch_of(batch_ids, b), u, c);
                 ck[c].k = A[c] + gumbel_of(uc);
                 ck[c].v = c;
                 ck[c].sens = gumbel_slope(uc);
@@ -424,7 +437,7 @@ int orc_replay(const orc_logits *q, float temperature, const int32_t *qrow_of_no
                 int jmax = -1;
                 double umax = 0.5;
                 for (int v = lo; v < hi; ++v) {
-                    double uv = orc_uniform(seed, PURPOSE_REPLAY_ELEM, b, u, v);
+                    double uv = orc_uniform(seed, PURPOSE_REPLAY_ELEM, batch_of(batch_ids, b), u, v);
                     double g = x[v] + gumbel_of(uv);
                     ek[ne].k = g; /* raw key for now */
                     ek[ne].v = v;
@@ -466,7 +479,7 @@ int orc_replay(const orc_logits *q, float temperature, const int32_t *qrow_of_no
 /* Flat Gumbel-top-m over the whole row (independent cross-check of the law only). */
 int orc_replay_flat(const orc_logits *q, float temperature, const int32_t *qrow_of_node, int32_t N,
                     const int32_t *depth, const int32_t *child_off, const int32_t *child_ids, uint64_t seed,
-                    int32_t *token)
+                    const int32_t *batch_ids, int32_t *token)
 {
     if (!q || N < 0 || !(temperature > 0.0f)) return -1;
     const float invT = 1.0f / temperature;
@@ -484,7 +497,7 @@ int orc_replay_flat(const orc_logits *q, float temperature, const int32_t *qrow_
             if (r < 0 || r >= q->R) return -5;
             read_row(q, b, r, invT, x);
             for (int v = 0; v < V; ++v) {
-                ek[v].k = x[v] + gumbel_of(orc_uniform(seed, PURPOSE_REPLAY_ELEM, b, u, v));
+                ek[v].k = x[v] + gumbel_of(orc_uniform(seed, PURPOSE_REPLAY_ELEM, batch_of(batch_ids, b), u, v));
                 ek[v].v = v;
                 ek[v].sens = 0;
             }
@@ -506,7 +519,9 @@ int orc_replay_flat(const orc_logits *q, float temperature, const int32_t *qrow_
  *                      y_i joins the drawn set, t <- t - Q(y_i).
  * If a child is accepted its token is emitted and the walk continues there; if all are
  * rejected the final token is drawn from the last residual R; at a leaf the bonus token
- * is drawn from the node's target row. Losslessness: Prop. 1.                          */
+ * is drawn from the node's target row. Losslessness: Prop. 1. A residual with no mass after
+ * a rejection cannot occur in exact arithmetic (a rejection needs p' < q', so some token has
+ * p > q); should rounding produce one, the final token is drawn from the node's target row. */
 
 static double draft_ratio(double qv, double t) { return (qv > 0.0 && t > 0.0) ? qv / t : 0.0; }
 
@@ -523,49 +538,55 @@ static double rrs_residual(int V, const double *P, const double *Q, double t, co
     return Z;
 }
 
-/* Gumbel-max over log w(v) (w >= 0, entries with w = 0 excluded) with the FINAL stream of
- * (b, node); reports whether the winner and the runner-up are a near tie.               */
-static int gumbel_argmax_logw(const double *w, int V, uint64_t seed, int b, int node, uint8_t *ex)
+/* Final-token draw from the law proportional to w (w >= 0), two-level Gumbel-max:
+ *   chunk keys  K_c = log(sum_{v in c} w_v) + G(U[FINAL_CHUNK, node, c]) over chunks of
+ *               ORC_CHUNK tokens with positive mass; the best chunk c* by (K desc, c asc);
+ *   token       argmax_{v in c*, w_v > 0} log w_v + G(U[FINAL, node, v]) by (key desc, v asc).
+ * P(c*) = mass(c)/total and, independently, P(v | c*) = w_v / mass(c*), so the token has law
+ * w / total exactly (the m = 1 case of the hierarchical sampler of the replay pass).
+ * With logits = 1 the input holds log-weights (x_v), as for a bonus token from a target row. */
+static int sample_final(const double *w, int logits, int V, uint64_t seed, int bid, int node, uint8_t *ex)
 {
-    int best = -1, second = -1;
-    double kb = -INFINITY, ks = -INFINITY, sb = 0, ss = 0;
-    for (int v = 0; v < V; ++v) {
-        if (!(w[v] > 0.0)) continue;
-        double u = orc_uniform(seed, PURPOSE_FINAL, b, node, v);
-        double k = log(w[v]) + gumbel_of(u);
-        if (best < 0 || k > kb) {
-            second = best; ks = kb; ss = sb;
-            best = v; kb = k; sb = gumbel_slope(u);
-        } else if (second < 0 || k > ks) {
-            second = v; ks = k; ss = gumbel_slope(u);
+    const int C = (V + ORC_CHUNK - 1) / ORC_CHUNK;
+    int bc = -1;
+    double kb = -INFINITY, ks = -INFINITY, sb = 0.0, ss = 0.0;
+    for (int c = 0; c < C; ++c) {
+        int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+        double A;
+        if (logits) {
+            A = logsumexp(w + lo, hi - lo);
+        } else {
+            double m = 0.0;
+            for (int v = lo; v < hi; ++v) m += w[v];
+            if (!(m > 0.0)) continue;
+            A = log(m);
+        }
+        double u = orc_uniform(seed, PURPOSE_FINAL_CHUNK, bid, node, c);
+        double k = A + gumbel_of(u);
+        if (bc < 0 || k > kb) {
+            ks = kb; ss = sb;
+            bc = c; kb = k; sb = gumbel_slope(u);
+        } else if (k > ks) {
+            ks = k; ss = gumbel_slope(u);
         }
     }
-    if (second >= 0 && ex) {
-        double s = sb > ss ? sb : ss;
-        if (kb - ks < U_BAND * s) *ex = 1;
-    }
-    return best;
-}
-
-/* Gumbel-max over logits x (the bonus token) */
-static int gumbel_argmax_logits(const double *x, int V, uint64_t seed, int b, int node, uint8_t *ex)
-{
-    int best = -1, second = -1;
-    double kb = -INFINITY, ks = -INFINITY, sb = 0, ss = 0;
-    for (int v = 0; v < V; ++v) {
-        double u = orc_uniform(seed, PURPOSE_FINAL, b, node, v);
-        double k = x[v] + gumbel_of(u);
-        if (best < 0 || k > kb) {
-            second = best; ks = kb; ss = sb;
-            best = v; kb = k; sb = gumbel_slope(u);
-        } else if (second < 0 || k > ks) {
-            second = v; ks = k; ss = gumbel_slope(u);
+    if (bc < 0) return -1;
+    if (ex && ks > -INFINITY && near_tie_keys(kb, ks, sb > ss ? sb : ss)) *ex = 1;
+    int lo = bc * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+    int best = -1;
+    double eb = -INFINITY, es = -INFINITY, tb = 0.0, ts = 0.0;
+    for (int v = lo; v < hi; ++v) {
+        if (!logits && !(w[v] > 0.0)) continue;
+        double u = orc_uniform(seed, PURPOSE_FINAL, bid, node, v);
+        double k = (logits ? w[v] : log(w[v])) + gumbel_of(u);
+        if (best < 0 || k > eb) {
+            es = eb; ts = tb;
+            best = v; eb = k; tb = gumbel_slope(u);
+        } else if (k > es) {
+            es = k; ts = gumbel_slope(u);
         }
     }
-    if (second >= 0 && ex) {
-        double s = sb > ss ? sb : ss;
-        if (kb - ks < U_BAND * s) *ex = 1;
-    }
+    if (ex && es > -INFINITY && near_tie_keys(eb, es, tb > ts ? tb : ts)) *ex = 1;
     return best;
 }
 
@@ -605,8 +626,8 @@ int orc_rrs_node_law(int32_t V, const double *P_in, const double *Q, int32_t m, 
 
 int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperature, const int32_t *qrow_of_node,
                    int32_t N, int32_t L, const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
-                   const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len,
-                   uint8_t *exempt)
+                   const int32_t *token, uint64_t seed, const int32_t *batch_ids, int32_t *out_tokens,
+                   int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
 {
     if (!target || !q || N < 0 || L < 1 || !(temperature > 0.0f) || target->V != q->V || target->R < N + 1) return -1;
     const float invT = 1.0f / temperature;
@@ -618,6 +639,7 @@ int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperat
     if (!xt || !xq || !P || !Q || !R || !drawn) return -3;
     for (int b = 0; b < target->B; ++b) {
         const int64_t nb = (int64_t)b * NN;
+        const int bid = batch_of(batch_ids, b);
         const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
         int32_t *otok = out_tokens + (int64_t)b * (L + 1), *onode = out_nodes + (int64_t)b * L;
         for (int k = 0; k <= L; ++k) otok[k] = -1;
@@ -628,7 +650,7 @@ int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperat
             const int m = off[u + 1] - off[u];
             read_row(target, b, u, invT, xt);
             if (m == 0) { /* leaf: bonus token from the node's target row */
-                final_tok = gumbel_argmax_logits(xt, V, seed, b, u, &ex);
+                final_tok = sample_final(xt, 1, V, seed, bid, u, &ex);
                 break;
             }
             const int r = replay_row_index(qrow_of_node, depth, nb + u);
@@ -644,16 +666,16 @@ int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperat
                 const int y = token[nb + c];
                 if (y < 0 || y >= V) return -6;
                 double qp = draft_ratio(Q[y], t), pp = P[y];
-                double U = orc_uniform(seed, PURPOSE_ACCEPT, b, c, 0);
+                double U = orc_uniform(seed, PURPOSE_ACCEPT, bid, c, 0);
                 if (qp > 0.0 && fabs(U - pp / qp) < U_BAND) ex = 1;
                 if (U * qp < pp) { accepted = c; break; }
                 double Z = rrs_residual(V, P, Q, t, drawn, R);
-                if (!(Z > 0.0)) { /* underflow only: draw from the current target law */
-                    final_tok = gumbel_argmax_logw(P, V, seed, b, u, &ex);
+                if (!(Z > 0.0)) { /* no residual mass (rounding only): draw from the node's target row */
+                    final_tok = sample_final(xt, 1, V, seed, bid, u, &ex);
                     break;
                 }
                 if (i == m - 1) { /* every slot rejected: draw from the last residual */
-                    final_tok = gumbel_argmax_logw(R, V, seed, b, u, &ex);
+                    final_tok = sample_final(R, 0, V, seed, bid, u, &ex);
                     break;
                 }
                 for (int v = 0; v < V; ++v) P[v] = R[v] / Z;
@@ -717,8 +739,8 @@ int orc_blockv_law(int32_t g, int32_t V, const double *Mb, const double *Ms, con
 
 int orc_verify_block(const orc_logits *target, const orc_logits *q, float temperature, const int32_t *qrow_of_node,
                      int32_t N, int32_t L, const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
-                     const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len,
-                     uint8_t *exempt, int32_t *tau_out)
+                     const int32_t *token, uint64_t seed, const int32_t *batch_ids, int32_t *out_tokens,
+                     int32_t *out_nodes, int32_t *out_len, uint8_t *exempt, int32_t *tau_out)
 {
     if (!target || !q || N < 1 || N > L || !(temperature > 0.0f) || target->V != q->V || target->R < N + 1) return -1;
     const float invT = 1.0f / temperature;
@@ -751,23 +773,26 @@ int orc_verify_block(const orc_logits *target, const orc_logits *q, float temper
             if (X[i] < 0 || X[i] >= V) return -6;
         }
         blockv_weights(g, V, Mb, Ms, X, w, h, resid);
+        const int bid = batch_of(batch_ids, b);
         uint8_t ex = 0;
         int tau = 0;
         for (int i = 1; i <= g; ++i)
-            if (orc_uniform(seed, PURPOSE_BLOCK_ETA, b, i, 0) <= h[i]) tau = i;
+            if (orc_uniform(seed, PURPOSE_BLOCK_ETA, bid, i, 0) <= h[i]) tau = i;
         for (int i = (tau > 1 ? tau : 1); i <= g; ++i) /* decisions that could move tau */
-            if (fabs(orc_uniform(seed, PURPOSE_BLOCK_ETA, b, i, 0) - h[i]) < U_BAND) ex = 1;
+            if (fabs(orc_uniform(seed, PURPOSE_BLOCK_ETA, bid, i, 0) - h[i]) < U_BAND) ex = 1;
         int final_tok;
         if (tau == g) {
             read_row(target, b, g, invT, x);
-            final_tok = gumbel_argmax_logits(x, V, seed, b, g, &ex);
+            final_tok = sample_final(x, 1, V, seed, bid, g, &ex);
         } else {
             double S = 0.0;
             for (int v = 0; v < V; ++v) S += resid[(int64_t)tau * V + v];
             if (S > 0.0)
-                final_tok = gumbel_argmax_logw(resid + (int64_t)tau * V, V, seed, b, tau, &ex);
-            else /* cannot carry mass in exact arithmetic; draw from the target law there */
-                final_tok = gumbel_argmax_logw(Mb + (int64_t)tau * V, V, seed, b, tau, &ex);
+                final_tok = sample_final(resid + (int64_t)tau * V, 0, V, seed, bid, tau, &ex);
+            else { /* cannot carry mass in exact arithmetic; draw from the target row there */
+                read_row(target, b, tau, invT, x);
+                final_tok = sample_final(x, 1, V, seed, bid, tau, &ex);
+            }
         }
         int32_t *otok = out_tokens + (int64_t)b * (L + 1), *onode = out_nodes + (int64_t)b * L;
         for (int k = 0; k <= L; ++k) otok[k] = -1;

@@ -300,8 +300,8 @@ __global__ void __launch_bounds__(kThreads) k_bv_final(BvArgs a) {
     __syncthreads();
     const int tau = tau_sh;
     const float wt = wtau_sh;
-    // final token: residual at tau (or the target row g, or the target row tau when the
-    // residual carries no mass)
+    // final token, two-level Gumbel-max over chunks of 256 tokens: from the residual at tau,
+    // or from the target row (tau = g, or a residual without mass)
     const BvRow &rw = a.rows[(int64_t)b * NN + tau];
     const bool from_target = tau == g || !(rw.S > 0.0);
     float th, tl, qh, ql;
@@ -309,34 +309,78 @@ __global__ void __launch_bounds__(kThreads) k_bv_final(BvArgs a) {
     split(tau < g ? rw.lse_q : 0.0, qh, ql);
     const T *trow = trow_ptr<T>(a, b, tau);
     const T *qrow = tau < g ? qrow_ptr<T>(a, b, qrow_index(a, b, tau)) : trow;
-    unsigned long long best = 0ull;
-    float xt[8], xq[8];
-    const int groups = (a.V + 7) >> 3;
-    if (ok_sh)
-        for (int gg = threadIdx.x; gg < groups; gg += kThreads) {
-            const int v0 = 8 * gg;
-            Logit<T>::load8(trow, v0, a.V, xt);
-            if (!from_target) Logit<T>::load8(qrow, v0, a.V, xq);
-            const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)tau, (uint32_t)(v0 >> 2));
-            const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)tau, (uint32_t)(v0 >> 2) + 1u);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    // 8 consecutive tokens from v0: log-weights x*invT (target row) or weights r >= 0 (residual);
+    // tokens past V get -inf / 0
+    auto vals8 = [&](int v0, float out[8]) {
+        float xt[8], xq[8];
+        Logit<T>::load8(trow, v0, a.V, xt);
+        if (!from_target) Logit<T>::load8(qrow, v0, a.V, xq);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                if (v0 + k >= a.V) break;
-                const float G = gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4]);
-                float key;
-                if (from_target) {
-                    key = __fadd_rn(__fmul_rn(xt[k], a.invT), G);
-                } else {
-                    const float p = prob_of(xt[k], a.invT, th, tl), q = prob_of(xq[k], a.invT, qh, ql);
-                    const float r = fmaxf(__fsub_rn(__fmul_rn(wt, p), q), 0.f);
-                    if (!(r > 0.f)) continue;
-                    key = __fadd_rn(logf(r), G);
-                }
-                const unsigned long long pk = pack_key(key, (uint32_t)(v0 + k));
+        for (int k = 0; k < 8; ++k) {
+            if (v0 + k >= a.V) {
+                out[k] = from_target ? -INFINITY : 0.f;
+            } else if (from_target) {
+                out[k] = __fmul_rn(xt[k], a.invT);
+            } else {
+                const float p = prob_of(xt[k], a.invT, th, tl), q = prob_of(xq[k], a.invT, qh, ql);
+                out[k] = fmaxf(__fsub_rn(__fmul_rn(wt, p), q), 0.f);
+            }
+        }
+    };
+    unsigned long long best = 0ull;
+    if (ok_sh)
+        for (int c = warp; c < a.C; c += kWarps) {
+            float v[8];
+            vals8(c * kChunk + lane * 8, v);
+            float A = -INFINITY;
+            if (from_target) {  // chunk log-mass = log-sum-exp of the logits
+                float mx = -INFINITY;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) mx = fmaxf(mx, v[k]);
+                mx = warp_max(mx);
+                float s = 0.f;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) s += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
+                s = warp_sum(s);
+                A = __fadd_rn(mx, logf(s));
+            } else {  // chunk mass = sum of the residual weights
+                float s = 0.f;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) s += v[k];
+                s = warp_sum(s);
+                if (s > 0.f) A = logf(s);
+            }
+            if (lane == 0 && A != -INFINITY) {
+                const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)tau, (uint32_t)c);
+                const unsigned long long pk = pack_key(__fadd_rn(A, gumbel_of(w)), (uint32_t)c);
                 best = pk > best ? pk : best;
             }
         }
     best = block_argmax(sh, best);
+    unsigned long long tokk = 0ull;
+    if (best != 0ull && warp == 0) {
+        const int v0 = (int)key_id(best) * kChunk + lane * 8;
+        float v[8];
+        vals8(v0, v);
+        const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)tau, (uint32_t)(v0 >> 2));
+        const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)tau, (uint32_t)(v0 >> 2) + 1u);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+            if (v0 + k >= a.V) break;
+            float l;
+            if (from_target) {
+                l = v[k];
+            } else {
+                if (!(v[k] > 0.f)) continue;
+                l = logf(v[k]);
+            }
+            const float key = __fadd_rn(l, gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4]));
+            const unsigned long long pk = pack_key(key, (uint32_t)(v0 + k));
+            tokk = pk > tokk ? pk : tokk;
+        }
+    }
+    tokk = block_argmax(sh, tokk);
     if (threadIdx.x == 0) {
         int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
         int32_t *onode = a.out_nodes + (int64_t)b * a.L;
@@ -347,7 +391,7 @@ __global__ void __launch_bounds__(kThreads) k_bv_final(BvArgs a) {
             otok[i - 1] = a.token[(int64_t)b * NN + i];
             onode[i - 1] = i;
         }
-        otok[t] = ok_sh ? (int32_t)key_id(best) : -1;
+        otok[t] = (ok_sh && tokk != 0ull) ? (int32_t)key_id(tokk) : -1;
         a.out_len[b] = ok_sh ? t + 1 : 0;
     }
 }

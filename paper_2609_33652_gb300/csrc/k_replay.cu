@@ -14,7 +14,9 @@
 // be among the top m_u: the joint law is exactly that of flat Gumbel-top-k over V tokens,
 // at ceil(V/256) + m_u*256 draws per parent instead of V.
 //
-// One warp per (tree, node); nodes without children return at once.
+// One CTA of 8 warps per (tree, node); nodes without children return at once. Chunk keys are
+// spread over the CTA (four chunks per thread share one Philox block), each warp then takes
+// one kept chunk, and per-warp candidate lists are merged in shared memory.
 #include "tsb_device.cuh"
 #include "tsb_launch.h"
 
@@ -22,6 +24,7 @@ namespace tsb {
 namespace {
 
 constexpr int kWarps = 8;
+constexpr int kThreads = kWarps * 32;
 
 struct ReplayArgs {
     const void *q;
@@ -43,111 +46,135 @@ __device__ __forceinline__ float shifted_key(float T, float Z, float g) {
     return T - sp;
 }
 
+// Merge per-warp lists: each warp writes its top n keys to cand[warp][0..n).
+template <int CAP>
+__device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t *dst) {
+    const int lane = threadIdx.x & 31;
+    for (int j = 0; j < n; ++j) {
+        const uint64_t best = warp_max_u64(list.k[0]);
+        if (lane == 0) dst[j] = best;
+        if (best != 0ull && list.k[0] == best) list.pop_front();
+    }
+}
+
+// Warp 0: the top n keys of cand[0..kWarps)[0..n) into out[0..n).
+template <int CAP>
+__device__ __forceinline__ void merge_warps(const uint64_t (*cand)[CAP], int n, uint64_t *out) {
+    const int lane = threadIdx.x & 31;
+    TopList<CAP> t;
+    t.clear();
+    for (int e = lane; e < kWarps * n; e += 32) t.insert(cand[e / n][e % n]);
+    warp_top_to(t, n, out);
+}
+
 template <int KCAP, typename T>
-__global__ void __launch_bounds__(kWarps * 32) k_replay(ReplayArgs a) {
-    __shared__ uint64_t sel_all[kWarps][KCAP];
+__global__ void __launch_bounds__(kThreads) k_replay(ReplayArgs a) {
+    __shared__ uint64_t cand[kWarps][KCAP];
+    __shared__ uint64_t sel[KCAP];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int NN = a.N + 1;
-    const int64_t gw = (int64_t)blockIdx.x * kWarps + warp;
-    if (gw >= (int64_t)a.B * NN) return;
-    const int b = (int)(gw / NN), u = (int)(gw - (int64_t)b * NN);
-    if (u == 0 && lane == 0) a.token[(int64_t)b * NN] = -1;
+    const int b = blockIdx.x / NN, u = blockIdx.x - (blockIdx.x / NN) * NN;
+    if (u == 0 && threadIdx.x == 0) a.token[(int64_t)b * NN] = -1;
     const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
     const int o = off[u], m = off[u + 1] - o;
-    if (m <= 0) return;
+    if (m <= 0) return;  // uniform over the CTA
     if (m > KCAP || o < 0 || o + m > a.N) {
-        if (lane == 0) raise_status(a.status, kDevBadTree);
+        if (threadIdx.x == 0) raise_status(a.status, kDevBadTree);
         return;
     }
     const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
-    const int32_t *kids = a.child_ids + (int64_t)b * a.N + o;
     if (r < 0 || r >= a.R) {
-        if (lane == 0) raise_status(a.status, kDevBadIndex);
+        if (threadIdx.x == 0) raise_status(a.status, kDevBadIndex);
         return;
     }
+    const int32_t *kids = a.child_ids + (int64_t)b * a.N + o;
     const float2 *st = a.stats + ((int64_t)b * a.R + r) * a.C;
     const T *row = static_cast<const T *>(a.q) + (int64_t)b * a.bstride + (int64_t)r * a.rstride;
     const uint32_t ub = (uint32_t)b, un = (uint32_t)u;
-
-    // 1. chunk keys; lane handles chunks 4j..4j+3 so one Philox block serves four draws
-    TopList<KCAP> cl;
-    cl.clear();
-    for (int c4 = lane * 4; c4 < a.C; c4 += 128) {
-        const Words4 w = draw_block(a.seed, kReplayChunk, ub, un, (uint32_t)(c4 >> 2));
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const int c = c4 + i;
-            if (c < a.C) {
-                const float2 s = st[c];
-                const float Kc = (s.x + logf(s.y)) + gumbel_of(w.w[i]);
-                cl.insert(pack_key(Kc, (uint32_t)c));
-            }
-        }
-    }
     const int msel = min(m, a.C);
-    uint64_t *sel = sel_all[warp];
-    for (int j = 0; j < msel; ++j) {
-        const uint64_t best = warp_max_u64(cl.k[0]);
-        if (lane == 0) sel[j] = best;
-        if (cl.k[0] == best) cl.pop_front();
-    }
-    __syncwarp();
 
-    // 2. element keys inside the kept chunks, shifted to their chunk key
-    TopList<KCAP> el;
-    el.clear();
-    for (int s = 0; s < msel; ++s) {
-        const uint64_t kk = sel[s];
-        const int c = (int)key_id(kk);
-        const float Tc = key_value(kk);
-        const int v0 = c * kChunk + lane * 8;
-        float x[8];
-        Logit<T>::load8(row, v0, a.V, x);
-        const Words4 w0 = draw_block(a.seed, kReplayElem, ub, un, (uint32_t)(v0 >> 2));
-        const Words4 w1 = draw_block(a.seed, kReplayElem, ub, un, (uint32_t)(v0 >> 2) + 1u);
-        float g[8];
-        uint64_t zk = 0;
+    // 1. chunk keys: thread t takes chunks 4t..4t+3 (+1024k), one Philox block each
+    {
+        TopList<KCAP> cl;
+        cl.clear();
+        for (int c4 = threadIdx.x * 4; c4 < a.C; c4 += 4 * kThreads) {
+            const Words4 w = draw_block(a.seed, kReplayChunk, ub, un, (uint32_t)(c4 >> 2));
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            g[i] = -INFINITY;
-            if (v0 + i < a.V) {
-                const uint32_t wi = i < 4 ? w0.w[i] : w1.w[i - 4];
-                g[i] = __fadd_rn(__fmul_rn(x[i], a.invT), gumbel_of(wi));
-                const uint64_t k = pack_key(g[i], (uint32_t)(v0 + i));
-                zk = k > zk ? k : zk;
+            for (int i = 0; i < 4; ++i) {
+                const int c = c4 + i;
+                if (c < a.C) {
+                    const float2 s = st[c];
+                    const float Kc = (s.x + logf(s.y)) + gumbel_of(w.w[i]);
+                    cl.insert(pack_key(Kc, (uint32_t)c));
+                }
             }
         }
-        zk = warp_max_u64(zk);
-        const float Z = key_value(zk);
-        const uint32_t jmax = key_id(zk);
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            if (v0 + i >= a.V) continue;
-            const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_key(Tc, Z, g[i]);
-            el.insert(pack_key(k, (uint32_t)(v0 + i)));
-        }
+        warp_top_to(cl, msel, cand[warp]);
     }
-    // 3. the top-m keys are the ordered draws
-    int32_t *tok = a.token + (int64_t)b * NN;
-    for (int j = 0; j < m; ++j) {
-        const uint64_t best = warp_max_u64(el.k[0]);
-        if (lane == 0) {
-            const int child = kids[j];
+    __syncthreads();
+    if (warp == 0) merge_warps<KCAP>(cand, msel, sel);
+    __syncthreads();
+
+    // 2. element keys of each kept chunk (one warp per chunk), shifted to the chunk key
+    {
+        TopList<KCAP> el;
+        el.clear();
+        for (int s = warp; s < msel; s += kWarps) {
+            const uint64_t kk = sel[s];
+            const int c = (int)key_id(kk);
+            const float Tc = key_value(kk);
+            const int v0 = c * kChunk + lane * 8;
+            float x[8];
+            Logit<T>::load8(row, v0, a.V, x);
+            const Words4 w0 = draw_block(a.seed, kReplayElem, ub, un, (uint32_t)(v0 >> 2));
+            const Words4 w1 = draw_block(a.seed, kReplayElem, ub, un, (uint32_t)(v0 >> 2) + 1u);
+            float g[8];
+            uint64_t zk = 0;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                g[i] = -INFINITY;
+                if (v0 + i < a.V) {
+                    const uint32_t wi = i < 4 ? w0.w[i] : w1.w[i - 4];
+                    g[i] = __fadd_rn(__fmul_rn(x[i], a.invT), gumbel_of(wi));
+                    const uint64_t k = pack_key(g[i], (uint32_t)(v0 + i));
+                    zk = k > zk ? k : zk;
+                }
+            }
+            zk = warp_max_u64(zk);
+            const float Z = key_value(zk);
+            const uint32_t jmax = key_id(zk);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+                if (v0 + i >= a.V) continue;
+                const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_key(Tc, Z, g[i]);
+                el.insert(pack_key(k, (uint32_t)(v0 + i)));
+            }
+        }
+        __syncthreads();  // the chunk lists in cand[] are no longer needed
+        warp_top_to(el, m, cand[warp]);
+    }
+    __syncthreads();
+
+    // 3. the top-m keys are the ordered draws; draw j fills child slot j
+    if (warp == 0) {
+        merge_warps<KCAP>(cand, m, sel);
+        __syncwarp();
+        int32_t *tok = a.token + (int64_t)b * NN;
+        if (lane < m) {
+            const int child = kids[lane];
             if (child > 0 && child < NN)
-                tok[child] = (int32_t)key_id(best);
+                tok[child] = (int32_t)key_id(sel[lane]);
             else
                 raise_status(a.status, kDevBadTree);
         }
-        if (el.k[0] == best) el.pop_front();
     }
 }
 
 template <int KCAP, typename T>
 cudaError_t launch_replay_t(const ReplayArgs &a, cudaStream_t s) {
-    const int64_t warps = (int64_t)a.B * (a.N + 1);
-    const int64_t blocks = (warps + kWarps - 1) / kWarps;
+    const int64_t blocks = (int64_t)a.B * (a.N + 1);
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    k_replay<KCAP, T><<<(unsigned)blocks, kWarps * 32, 0, s>>>(a);
+    k_replay<KCAP, T><<<(unsigned)blocks, kThreads, 0, s>>>(a);
     return cudaGetLastError();
 }
 

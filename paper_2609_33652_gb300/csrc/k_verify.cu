@@ -1,23 +1,27 @@
 // Tree verification by recursive rejection sampling for WoR candidates (Sec. 2.3 Eq.
 // rs-overlap; App. A), lossless on the frozen topology (Prop. 1).
 //
-// One thread-block cluster per tree; CTA r of the cluster owns the vocabulary slice
-// [r*slice, (r+1)*slice) and keeps that slice of the current node's target row and q row in
-// shared memory, so every pass after the first reads shared memory, not L2/HBM. Scalars
-// (log-normalisers, residual masses, argmax keys) are combined across the cluster through
-// distributed shared memory: each CTA publishes its partial, the cluster barrier orders the
-// writes, and every CTA combines all partials in rank order, so all CTAs hold bitwise
-// identical values and take identical decisions.
+// One thread-block cluster per tree. CTA r of the cluster owns the chunk-aligned vocabulary
+// slice [r*slice, (r+1)*slice) and keeps that slice of the current node in shared memory as
+// fp32: P holds the target logits, later the current residual; Q holds the normalised draft
+// law once it is needed. Scalars (log-normalisers, residual masses, argmax keys) are combined
+// across the cluster through distributed shared memory: each CTA publishes its partial, the
+// cluster barrier orders the writes, and every CTA combines all partials in rank order, so
+// all CTAs hold bitwise identical values and take identical decisions.
 //
-// Walk at node u with children y_1..y_m (slot order), P = softmax(target row u),
-// Q = softmax(q row of u), t = 1:
-//   slot i: p' = P_i(y_i), q' = Q(y_i)/t_i; accept iff U * q' < p';
-//           on reject R(v) = max(P_i(v) - Q(v)/t_i, 0), Z = sum R, P_{i+1} = R / Z,
-//           t_{i+1} = t_i - Q(y_i). A rejected token has P_{i+1} = 0 from then on, so the
-//           explicit exclusion of drawn tokens from Q is implied by the residual.
-//   P_i(v) is recomputed per element from P_0(v), Q(v) and the stored (t_j, Z_j), j < i.
-// All children rejected -> final token = argmax_v log R(v) + G(U_v); leaf -> bonus token =
-// argmax_v x_v + G(U_v); Z = 0 (underflow only) -> argmax_v log P_i(v) + G(U_v).
+// Walk at node u with children y_1..y_m (slot order), P0 = softmax(target row u),
+// Q = softmax(q row of u), t_0 = 1:
+//   slot i: p' = p_i(y_i), q' = Q(y_i)/t_i; accept iff U * q' < p';
+//           on reject R_{i+1}(v) = max(p_i(v) - Q(v)/t_i, 0), Z_{i+1} = sum R_{i+1},
+//           p_{i+1} = R_{i+1}/Z_{i+1}, t_{i+1} = t_i - Q(y_i).
+//   A rejected token has p_{i+1} = 0 from then on, which is exactly the exclusion of drawn
+//   tokens from the renormalised draft law. Each pass is O(1) per element: P keeps R_i and
+//   p_i(v) = P[v] / Z_i; the point value p_i(y) repeats the same fp32 operations from P0(y).
+// Per node: one staging pass (the target log-normaliser is accumulated while staging); the
+// q row is staged by the first rejection pass only, so a node whose first child is accepted
+// reads one row. Final tokens (all children rejected: from R_m; leaf: bonus from the target
+// row) are drawn with the two-level Gumbel-max of the contract: chunk keys
+// log(chunk mass) + G over chunks of 256 tokens, then the best token of the winning chunk.
 #include <cooperative_groups.h>
 
 #include "tsb_device.cuh"
@@ -65,18 +69,17 @@ struct Scratch {
 
 __device__ __forceinline__ float qratio(float q, float t) { return (q > 0.f && t > 0.f) ? __fdiv_rn(q, t) : 0.f; }
 
-// P_i(v) from P_0(v), Q(v) and the first i rejections.
-__device__ __forceinline__ float resid_chain(float p, float q, const float *zs, const float *ts, int i) {
+// exp(x - LSE) with LSE = hi + lo; x = fp32(z) * invT
+__device__ __forceinline__ float prob_of(float x, float hi, float lo) { return expf(__fsub_rn(__fsub_rn(x, hi), lo)); }
+
+// p_i(y) from P0(y), Q(y): the same fp32 operations the element passes perform.
+__device__ __forceinline__ float point_residual(float p0, float q, const float *zs, const float *ts, int i) {
+    float p = p0;
     for (int j = 0; j < i; ++j) {
-        p = fmaxf(__fsub_rn(p, qratio(q, ts[j])), 0.f);
-        p = __fdiv_rn(p, zs[j]);
+        const float r = fmaxf(__fsub_rn(p, qratio(q, ts[j])), 0.f);
+        p = __fdiv_rn(r, zs[j]);
     }
     return p;
-}
-
-// exp(x*invT - LSE) with LSE = hi + lo
-__device__ __forceinline__ float prob_of(float z, float invT, float hi, float lo) {
-    return expf(__fsub_rn(__fsub_rn(__fmul_rn(z, invT), hi), lo));
 }
 
 // One cluster-wide reduction of (max, sum-exp) x2, a plain sum and an argmax key.
@@ -146,6 +149,7 @@ __device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &clu
         o.s2 = S2;
         o.z = Z;
         o.key = Kx;
+        o.hi1 = o.lo1 = o.hi2 = o.lo2 = 0.f;
         if (S1 > 0.0) {
             const double l1 = (double)M1 + log(S1);
             o.hi1 = (float)l1;
@@ -161,82 +165,148 @@ __device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &clu
     par ^= 1;
 }
 
-// Copy this CTA's slice of a row into shared memory.
-template <typename T>
-__device__ __forceinline__ void stage(const T *row, T *dst, int lo, int n, int V) {
-    const int groups = (n + 7) >> 3;
-    for (int g = threadIdx.x; g < groups; g += kThreads) {
-        const int v0 = lo + 8 * g;
-        if (v0 + 8 <= V) {
-            if (sizeof(T) == 2) {
-                reinterpret_cast<uint4 *>(dst)[g] = __ldg(reinterpret_cast<const uint4 *>(row + v0));
-            } else {
-                const float4 *src = reinterpret_cast<const float4 *>(row + v0);
-                reinterpret_cast<float4 *>(dst)[2 * g] = __ldg(src);
-                reinterpret_cast<float4 *>(dst)[2 * g + 1] = __ldg(src + 1);
+// Per-thread online (max, sum of exp(x - max)) accumulation.
+struct OnlineLse {
+    float m = -INFINITY;
+    KahanF s;
+    __device__ __forceinline__ void add(float x) {
+        if (x > m) {
+            if (m != -INFINITY) {
+                const float scale = fast_exp2(__fmul_rn(__fsub_rn(m, x), kLog2e));
+                s.s = __fmul_rn(s.s, scale);
+                s.c = __fmul_rn(s.c, scale);
             }
+            m = x;
+            s.add(1.0f);
         } else {
-            for (int i = 0; i < 8; ++i)
-                if (v0 + i < V) dst[8 * g + i] = row[v0 + i];
+            s.add(fast_exp2(__fmul_rn(__fsub_rn(x, m), kLog2e)));
         }
     }
-}
+};
 
 template <typename T>
-__device__ __forceinline__ float as_f32(T v);
-template <>
-__device__ __forceinline__ float as_f32<float>(float v) {
-    return v;
-}
-template <>
-__device__ __forceinline__ float as_f32<__nv_bfloat16>(__nv_bfloat16 v) {
-    return __uint_as_float((uint32_t)__bfloat16_as_ushort(v) << 16);
-}
+struct Walk {
+    const VerifyArgs &a;
+    Scratch &sh;
+    const cg::cluster_group &cluster;
+    float *P, *Qs;
+    int &par;
+    int b, lo, n, crank;
 
-enum PassKind { kBonus = 0, kResidualArgmax = 1, kTargetArgmax = 2 };
+    __device__ int groups() const { return (n + 7) >> 3; }
 
-// Gumbel-max over this CTA's slice; returns the thread's best packed key.
-// kind = kBonus: keys x_v + G; otherwise keys log w(v) + G with w = R_{i+1} (residual after
-// rejecting slot i, unnormalised) or w = P_i (current target law).
-template <typename T>
-__device__ unsigned long long gumbel_pass(const VerifyArgs &a, const T *xt_s, const T *xq_s, int lo, int n, int b,
-                                          int node, int kind, int i, float t_i, float lt_hi, float lt_lo,
-                                          float lq_hi, float lq_lo, const float *zs, const float *ts) {
-    unsigned long long best = 0ull;
-    const int groups = (n + 7) >> 3;
-    for (int g = threadIdx.x; g < groups; g += kThreads) {
-        const int v0 = lo + 8 * g;
-        const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
-        const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2) + 1u);
+    // Stage x = fp32(z) * invT of this CTA's target slice into P; optionally accumulate the
+    // target row's log-normaliser.
+    __device__ void stage_target(const T *row, OnlineLse *lse) {
+        for (int g = threadIdx.x; g < groups(); g += kThreads) {
+            float x[8];
+            Logit<T>::load8(row, lo + 8 * g, a.V, x);
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int v = v0 + k;
-            if (v >= a.V) break;
-            const float G = gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4]);
-            const float zt = as_f32(xt_s[8 * g + k]);
-            float key;
-            if (kind == kBonus) {
-                key = __fadd_rn(__fmul_rn(zt, a.invT), G);
-            } else {
-                const float P0 = prob_of(zt, a.invT, lt_hi, lt_lo);
-                const float Q = prob_of(as_f32(xq_s[8 * g + k]), a.invT, lq_hi, lq_lo);
-                float w = resid_chain(P0, Q, zs, ts, i);
-                if (kind == kResidualArgmax) w = fmaxf(__fsub_rn(w, qratio(Q, t_i)), 0.f);
-                if (!(w > 0.f)) continue;
-                key = __fadd_rn(logf(w), G);
+            for (int k = 0; k < 8; ++k) {
+                const bool in = lo + 8 * g + k < a.V;
+                const float xv = in ? __fmul_rn(x[k], a.invT) : -INFINITY;
+                P[8 * g + k] = xv;
+                if (lse && in) lse->add(xv);
             }
-            const unsigned long long pk = pack_key(key, (uint32_t)v);
-            best = pk > best ? pk : best;
         }
     }
-    return best;
-}
+
+    // argmax over the winning chunk of lw + G (warp 0 of the owner CTA computes it).
+    template <typename LW>
+    __device__ int element_argmax(int node, int c, LW lw) {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        unsigned long long best = 0ull;
+        const int i0c = c * kChunk - lo;  // chunk start in this CTA's slice
+        if (warp == 0 && i0c >= 0 && i0c < n) {
+            const int i0 = i0c + lane * 8, v0 = lo + i0;
+            const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
+            const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2) + 1u);
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                if (i0 + k >= n) break;
+                const float l = lw(i0 + k, v0 + k);
+                if (l == -INFINITY) continue;
+                const float key = __fadd_rn(l, gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4]));
+                const unsigned long long pk = pack_key(key, (uint32_t)(v0 + k));
+                best = pk > best ? pk : best;
+            }
+        }
+        reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, best);
+        return sh.res.key == 0ull ? -1 : (int)key_id(sh.res.key);
+    }
+
+    // Two-level draw from log-weights lw(smem index, token) (-inf = no mass); chunk masses
+    // are log-sum-exp of the log-weights.
+    template <typename LW>
+    __device__ int draw_logits(int node, LW lw) {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        const int nch = (n + kChunk - 1) / kChunk;
+        unsigned long long best = 0ull;
+        for (int cl = warp; cl < nch; cl += kWarps) {
+            const int i0 = cl * kChunk + lane * 8;
+            float v[8];
+            float mx = -INFINITY;
+#pragma unroll
+            for (int k = 0; k < 8; ++k) {
+                v[k] = (i0 + k < n) ? lw(i0 + k, lo + i0 + k) : -INFINITY;
+                mx = fmaxf(mx, v[k]);
+            }
+            mx = warp_max(mx);
+            float s = 0.f;
+            if (mx != -INFINITY) {
+#pragma unroll
+                for (int k = 0; k < 8; ++k) s += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
+            }
+            s = warp_sum(s);
+            if (lane == 0 && mx != -INFINITY) {
+                const int c = (lo >> 8) + cl;
+                const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
+                const float key = __fadd_rn(__fadd_rn(mx, logf(s)), gumbel_of(w));
+                const unsigned long long pk = pack_key(key, (uint32_t)c);
+                best = pk > best ? pk : best;
+            }
+        }
+        reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, best);
+        if (sh.res.key == 0ull) return -1;
+        return element_argmax(node, (int)key_id(sh.res.key), lw);
+    }
+
+    // Two-level draw from non-negative weights wf(smem index, token); chunk mass = sum w.
+    template <typename WF>
+    __device__ int draw_weights(int node, WF wf) {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        const int nch = (n + kChunk - 1) / kChunk;
+        unsigned long long best = 0ull;
+        for (int cl = warp; cl < nch; cl += kWarps) {
+            const int i0 = cl * kChunk + lane * 8;
+            float s = 0.f;
+#pragma unroll
+            for (int k = 0; k < 8; ++k)
+                if (i0 + k < n) s += wf(i0 + k, lo + i0 + k);
+            s = warp_sum(s);
+            if (lane == 0 && s > 0.f) {
+                const int c = (lo >> 8) + cl;
+                const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
+                const float key = __fadd_rn(logf(s), gumbel_of(w));
+                const unsigned long long pk = pack_key(key, (uint32_t)c);
+                best = pk > best ? pk : best;
+            }
+        }
+        reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, best);
+        if (sh.res.key == 0ull) return -1;
+        auto lw = [&](int i, int v) {
+            const float w = wf(i, v);
+            return w > 0.f ? logf(w) : -INFINITY;
+        };
+        return element_argmax(node, (int)key_id(sh.res.key), lw);
+    }
+};
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
-    extern __shared__ __align__(16) unsigned char dyn[];
-    T *xt_s = reinterpret_cast<T *>(dyn);
-    T *xq_s = xt_s + a.slice;
+    extern __shared__ __align__(16) float dyn[];
+    float *P = dyn;
+    float *Qs = dyn + a.slice;
     __shared__ Scratch sh;
 
     cg::cluster_group cluster = cg::this_cluster();
@@ -248,6 +318,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     const int n = max(0, min(a.V - lo, a.slice));
     const bool writer = crank == 0 && threadIdx.x == 0;
     int par = 0;
+    Walk<T> W{a, sh, cluster, P, Qs, par, b, lo, n, crank};
+    const int groups = W.groups();
 
     const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
     const int32_t *kids = a.child_ids + (int64_t)b * a.N;
@@ -266,90 +338,103 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             break;
         }
         const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
-        const T *qrow = nullptr;
-        int r = -1;
-        if (m > 0) {
-            r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
-            if (r < 0 || r >= a.q_R) {
-                bad = true;
-                break;
-            }
-            qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
-        }
         __syncthreads();
-        stage<T>(trow, xt_s, lo, n, a.V);
-        if (m > 0) stage<T>(qrow, xq_s, lo, n, a.V);
-        __syncthreads();
-
         if (m == 0) {  // leaf: bonus token from the node's target row
-            const unsigned long long k =
-                gumbel_pass<T>(a, xt_s, xq_s, lo, n, b, u, kBonus, 0, 0.f, 0.f, 0.f, 0.f, 0.f, sh.zs, sh.ts);
-            reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, k);
-            final_tok = (int)key_id(sh.res.key);
+            W.stage_target(trow, nullptr);
+            __syncthreads();
+            final_tok = W.draw_logits(u, [&](int i, int) { return P[i]; });
             break;
         }
+        const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
+        if (r < 0 || r >= a.q_R) {
+            bad = true;
+            break;
+        }
+        const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
 
-        // log-normalisers: target row from the staged slice, q row from its chunk statistics
-        float m1 = -INFINITY, m2 = -INFINITY;
-        const int groups = (n + 7) >> 3;
-        for (int g = threadIdx.x; g < groups; g += kThreads)
-            for (int k = 0; k < 8 && lo + 8 * g + k < a.V; ++k)
-                m1 = fmaxf(m1, __fmul_rn(as_f32(xt_s[8 * g + k]), a.invT));
-        KahanF s1;
-        if (m1 != -INFINITY)
-            for (int g = threadIdx.x; g < groups; g += kThreads)
-                for (int k = 0; k < 8 && lo + 8 * g + k < a.V; ++k)
-                    s1.add(expf(__fsub_rn(__fmul_rn(as_f32(xt_s[8 * g + k]), a.invT), m1)));
+        // staging pass with the target log-normaliser; q row log-normaliser from its chunk stats
+        OnlineLse lt;
+        W.stage_target(trow, &lt);
         const float2 *st = a.qstats + ((int64_t)b * a.q_R + r) * a.C;
+        float m2 = -INFINITY;
         for (int c = crank * kThreads + threadIdx.x; c < a.C; c += CS * kThreads) m2 = fmaxf(m2, st[c].x);
         KahanF s2;
         if (m2 != -INFINITY)
             for (int c = crank * kThreads + threadIdx.x; c < a.C; c += CS * kThreads)
                 s2.add(st[c].y * expf(st[c].x - m2));
-        reduce_round(sh, par, cluster, m1, s1.value(), m2, s2.value(), 0.0, 0ull);
+        reduce_round(sh, par, cluster, lt.m, lt.s.value(), m2, s2.value(), 0.0, 0ull);
         const float lt_hi = sh.res.hi1, lt_lo = sh.res.lo1, lq_hi = sh.res.hi2, lq_lo = sh.res.lo2;
 
         double t = 1.0;
         int accepted = -1;
         for (int i = 0; i < m; ++i) {
-            const int c = kids[i];
+            const int c = kids[o + i];
             const int y = (c >= 1 && c <= a.N) ? tok[c] : -1;
             if (y < 0 || y >= a.V) {
                 bad = true;
                 break;
             }
             const float t_i = (float)t;
-            const float P0 = prob_of(Logit<T>::load1(trow, y), a.invT, lt_hi, lt_lo);
-            const float Qy = prob_of(Logit<T>::load1(qrow, y), a.invT, lq_hi, lq_lo);
-            const float pp = resid_chain(P0, Qy, sh.zs, sh.ts, i);
+            const float P0y = prob_of(__fmul_rn(Logit<T>::load1(trow, y), a.invT), lt_hi, lt_lo);
+            const float Qy = prob_of(__fmul_rn(Logit<T>::load1(qrow, y), a.invT), lq_hi, lq_lo);
+            const float pp = point_residual(P0y, Qy, sh.zs, sh.ts, i);
             const float qp = qratio(Qy, t_i);
             const float U = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
             if (__fmul_rn(U, qp) < pp) {
                 accepted = c;
                 break;
             }
-            if (i == m - 1) {  // every slot rejected: final token from the last residual
-                const unsigned long long k = gumbel_pass<T>(a, xt_s, xq_s, lo, n, b, u, kResidualArgmax, i, t_i,
-                                                            lt_hi, lt_lo, lq_hi, lq_lo, sh.zs, sh.ts);
-                reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, k);
-                final_tok = (int)key_id(sh.res.key);
+            // p_i(v) of the element at smem index j
+            const float zprev = i > 0 ? sh.zs[i - 1] : 1.f;
+            auto p_of = [&](int j) { return i == 0 ? prob_of(P[j], lt_hi, lt_lo) : __fdiv_rn(P[j], zprev); };
+            if (i == m - 1) {  // every slot rejected: final token from R_m = max(p_i - Q/t_i, 0)
+                if (i == 0) {  // the q slice was never staged: stage it (normalised) now
+                    for (int g = threadIdx.x; g < groups; g += kThreads) {
+                        float x[8];
+                        Logit<T>::load8(qrow, lo + 8 * g, a.V, x);
+#pragma unroll
+                        for (int k = 0; k < 8; ++k) Qs[8 * g + k] = prob_of(__fmul_rn(x[k], a.invT), lq_hi, lq_lo);
+                    }
+                    __syncthreads();
+                }
+                final_tok = W.draw_weights(u, [&](int j, int) {
+                    return fmaxf(__fsub_rn(p_of(j), qratio(Qs[j], t_i)), 0.f);
+                });
+                if (final_tok < 0) {  // no residual mass (rounding only): the node's target row
+                    __syncthreads();
+                    W.stage_target(trow, nullptr);
+                    __syncthreads();
+                    final_tok = W.draw_logits(u, [&](int j, int) { return P[j]; });
+                }
                 break;
             }
-            // residual mass after rejecting slot i
-            KahanF zloc;
-            for (int g = threadIdx.x; g < groups; g += kThreads)
-                for (int k = 0; k < 8 && lo + 8 * g + k < a.V; ++k) {
-                    const float P0v = prob_of(as_f32(xt_s[8 * g + k]), a.invT, lt_hi, lt_lo);
-                    const float Qv = prob_of(as_f32(xq_s[8 * g + k]), a.invT, lq_hi, lq_lo);
-                    zloc.add(fmaxf(__fsub_rn(resid_chain(P0v, Qv, sh.zs, sh.ts, i), qratio(Qv, t_i)), 0.f));
+            // residual pass (the first one also stages the normalised q slice)
+            KahanF zl;
+            for (int g = threadIdx.x; g < groups; g += kThreads) {
+                float xq[8];
+                if (i == 0) Logit<T>::load8(qrow, lo + 8 * g, a.V, xq);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) {
+                    const int j = 8 * g + k;
+                    if (lo + j >= a.V) break;
+                    float qv;
+                    if (i == 0) {
+                        qv = prob_of(__fmul_rn(xq[k], a.invT), lq_hi, lq_lo);
+                        Qs[j] = qv;
+                    } else {
+                        qv = Qs[j];
+                    }
+                    const float rr = fmaxf(__fsub_rn(p_of(j), qratio(qv, t_i)), 0.f);
+                    P[j] = rr;
+                    zl.add(rr);
                 }
-            reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, zloc.value(), 0ull);
+            }
+            reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, zl.value(), 0ull);
             const double Z = sh.res.z;
-            if (!(Z > 0.0)) {  // underflow only: draw from the current target law
-                const unsigned long long k = gumbel_pass<T>(a, xt_s, xq_s, lo, n, b, u, kTargetArgmax, i, t_i,
-                                                            lt_hi, lt_lo, lq_hi, lq_lo, sh.zs, sh.ts);
-                reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, k);
-                final_tok = (int)key_id(sh.res.key);
+            if (!(Z > 0.0)) {  // no residual mass (rounding only): the node's target row
+                W.stage_target(trow, nullptr);
+                __syncthreads();
+                final_tok = W.draw_logits(u, [&](int j, int) { return P[j]; });
                 break;
             }
             if (threadIdx.x == 0) {
@@ -381,17 +466,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
-int pick_cluster(int V, int elem_bytes, int *slice_out, size_t *smem_out) {
+constexpr size_t kSmemLimit = 210 * 1024;
+
+// Cluster size and chunk-aligned slice for a vocabulary: enough CTAs to spread a row, and
+// the two fp32 slices must fit in shared memory.
+int pick_cluster(int V, int *slice_out, size_t *smem_out) {
     int cs = V >= 32768 ? 8 : V >= 8192 ? 4 : V >= 2048 ? 2 : 1;
     for (;;) {
         int slice = (V + cs - 1) / cs;
-        slice = (slice + 7) & ~7;
-        const size_t smem = 2 * (size_t)slice * elem_bytes;
-        if (smem <= 200 * 1024 || cs == 16) {
+        slice = (slice + kChunk - 1) / kChunk * kChunk;
+        const size_t smem = 2 * (size_t)slice * sizeof(float);
+        if (smem <= kSmemLimit) {
             *slice_out = slice;
             *smem_out = smem;
-            return smem <= 200 * 1024 ? cs : -1;
+            return cs;
         }
+        if (cs == 16) return -1;
         cs *= 2;
     }
 }
@@ -400,7 +490,7 @@ template <typename T>
 cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     int slice = 0;
     size_t smem = 0;
-    const int cs = pick_cluster(a.V, (int)sizeof(T), &slice, &smem);
+    const int cs = pick_cluster(a.V, &slice, &smem);
     if (cs < 0) return cudaErrorInvalidValue;
     a.slice = slice;
     cudaError_t e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -8,8 +8,7 @@
 
 namespace {
 
-constexpr size_t kStatusBytes = 256;  // status word region at the start of the workspace
-constexpr size_t kBvRowBytes = 32;    // per (tree, chain position) scalars of block verification
+constexpr size_t kStatusBytes = tsb::kWsStatusBytes;  // status word region at the start of the workspace
 
 bool aligned(const void *p, size_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
@@ -69,7 +68,7 @@ tsb::TreeDesc tree_of(const tsb_tree *t) {
     return d;
 }
 
-size_t ws_bytes_for(const tsb_cfg *c) { return kStatusBytes + (size_t)c->B * ((size_t)c->N + 1) * kBvRowBytes; }
+size_t ws_bytes_for(const tsb_cfg *c) { return tsb::workspace_bytes(c->B, c->N, c->L, c->K); }
 
 tsb_status check_ws(void *ws, size_t ws_bytes, size_t need) {
     if (!ws) return TSB_ERR_ARG;
@@ -163,8 +162,8 @@ tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *dra
         !out->child_ids)
         return TSB_ERR_ARG;
     return cuda_status(tsb::launch_plan(rows_of(draft), static_cast<const float2 *>(draft_stats), cfg->L, cfg->N,
-                                        cfg->K, inv_temperature(cfg->temperature), tree_of(out),
-                                        static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+                                        cfg->K, inv_temperature(cfg->temperature), tree_of(out), ws,
+                                        (cudaStream_t)stream));
 }
 
 tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,

@@ -12,7 +12,7 @@ constexpr int kChunk = 256;   // logits per chunk (chunk statistics, replay samp
 constexpr int kMaxK = 32;
 constexpr unsigned kFull = 0xffffffffu;
 
-enum Purpose : uint32_t { kReplayChunk = 0, kReplayElem = 1, kAccept = 2, kFinal = 3, kBlockEta = 4 };
+enum Purpose : uint32_t { kReplayChunk = 0, kReplayElem = 1, kAccept = 2, kFinal = 3, kBlockEta = 4, kFinalChunk = 5 };
 
 constexpr uint32_t kDevNonFinite = 1u, kDevBadIndex = 2u, kDevBadTree = 4u;
 

@@ -22,10 +22,30 @@ struct TreeDesc {
 
 inline int num_chunks(int V) { return (V + 255) / 256; }
 
+// Workspace layout (caller-owned, 256-byte aligned):
+//   [0, 256)                       sticky status word
+//   B*(N+1) x 32 bytes             per-(tree, chain position) scalars of block verification
+//   B*L doubles, B*L*K floats,     per-draft-row log-normaliser and top-K (x, id) of the
+//   B*L*K int32                    first pass
+constexpr size_t kWsStatusBytes = 256;
+constexpr size_t kWsBvRowBytes = 32;
+
+inline size_t workspace_bytes(int B, int N, int L, int K) {
+    return kWsStatusBytes + (size_t)B * ((size_t)N + 1) * kWsBvRowBytes + (size_t)B * L * sizeof(double) +
+           (size_t)B * L * K * (sizeof(float) + sizeof(int32_t));
+}
+
+struct PlanScratch {
+    double *lse;
+    float *topk_x;
+    int32_t *topk_id;
+};
+PlanScratch plan_scratch(void *ws, int B, int N, int L, int K);
+
 cudaError_t launch_row_stats(const RowsDesc &rows, float invT, float2 *stats, uint32_t *status, cudaStream_t s);
 
 cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
-                        const TreeDesc &tree, uint32_t *status, cudaStream_t s);
+                        const TreeDesc &tree, void *ws, cudaStream_t s);
 
 cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
                           int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token, uint32_t *status,

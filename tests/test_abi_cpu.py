@@ -46,7 +46,7 @@ def test_host_queries(lib):
     assert tsb.tsb_stats_bytes(1, 1, 257) == 2 * 8
     assert tsb.tsb_stats_bytes(0, 1, 10) == 0
     cfg = tsb.make_cfg(16, 16, 64, 8, 151936, 1.0)
-    assert tsb.tsb_workspace_bytes(cfg) == 256 + 16 * 65 * 32
+    assert tsb.tsb_workspace_bytes(cfg) == 256 + 16 * 65 * 32 + 16 * 16 * (8 + 8 * 8)
     assert tsb.tsb_workspace_bytes(tsb.make_cfg(1, 2, 7, 2, 8, 1.0)) == 0  # N above K + K^2
 
 
@@ -93,7 +93,7 @@ def test_plan_validation(lib):
     assert _plan(lib, good, d, tree=t) == ARG
     # broadcast rows (batch stride 0) are accepted by validation
     cfg1 = tsb.make_cfg(4, 2, 6, 2, 8, 1.0)
-    assert lib.tsb_workspace_bytes(ctypes.byref(cfg1)) == 256 + 4 * 7 * 32
+    assert lib.tsb_workspace_bytes(ctypes.byref(cfg1)) == 256 + 4 * 7 * 32 + 4 * 2 * (8 + 8 * 2)
 
 
 def test_replay_verify_validation(lib):

@@ -150,3 +150,32 @@ def test_verify_outputs_padding(orc):
         assert 1 <= n <= L + 1
         assert np.all(out["tokens"][b, n:] == -1)
         assert np.all(out["nodes"][b, n - 1:] == -1)
+
+
+def test_final_token_law_across_chunks(orc):
+    """V = 1000 spans four chunks (the last ragged), so the final token's two-level draw (chunk,
+    then token inside it) is exercised both for the residual after rejections and for the
+    bonus token at a leaf. Draft and target laws differ strongly, so every child is often
+    rejected. First emitted token vs the root target law; second vs the child's target law."""
+    B, V, m = 30_000, 1000, 3
+    rng = np.random.default_rng(31)
+    zq = rng.standard_normal((1, V)).astype(np.float32)
+    zq[0, [5, 400, 990]] += np.float32(6.0)
+    zt = rng.standard_normal((2, V)).astype(np.float32)
+    zt[0, [7, 260, 600, 995]] += np.float32(4.0)
+    zt[1, [12, 700]] += np.float32(5.0)
+    tree = helpers.star_tree(m, B)
+    qb = np.broadcast_to(zq[None], (B, 1, V))
+    tok, ex_r = orc.replay(qb, 1.0, tree, seed=41)
+    target = synth.path_keyed_rows(zt, tree["parent"], tree["depth"], tok, 0.5, seed=79)
+    out = orc.verify_rrs(target, qb, 1.0, tree, tok, seed=41, L=1)
+    first = out["tokens"][:, 0]
+    p_root = helpers.softmax64(synth.path_keyed_row(zt, [], 0.5, 79))
+    assert (out["len"] == 1).mean() > 0.2  # all children rejected reasonably often
+    assert helpers.chi2_pvalue(np.bincount(first, minlength=V), p_root) > P_MIN
+    two = out["len"] == 2
+    vals, cnt = np.unique(first[two], return_counts=True)
+    a = int(vals[np.argmax(cnt)])
+    sel = two & (first == a)
+    p_a = helpers.softmax64(synth.path_keyed_row(zt, [a], 0.5, 79))
+    assert helpers.chi2_pvalue(np.bincount(out["tokens"][sel, 1], minlength=V), p_a) > P_MIN
