@@ -202,10 +202,11 @@ int orc_row_stats(const orc_logits *rows, float temperature, int32_t K, double *
  *
  * Path score of a node at depth d reached through ranks (r_1..r_d):
  *     score = sum_j log q_j(y_j) = (sum_j x_{j, r_j}) - (sum_{j<=d} LSE_j)
- * held as the exact fp64 sum Sx of the x's plus the depth; key = Sx - CL[d] with
+ * held as the fp64 sum Sx of the x's (added in path order) and key = Sx - CL[d] with
  * CL[d] = LSE_1 + ... + LSE_d. Candidates pop in the order
- *     (key desc, depth asc, Sx desc, parent asc, rank asc),
- * a total order in which same-depth candidates compare through Sx exactly.               */
+ *     (key desc, depth asc, parent asc, rank asc).
+ * Same-depth candidates share CL[d], so equal Sx always means equal keys on every machine,
+ * and the tie goes to the earlier parent, then the lower rank.                           */
 typedef struct {
     double key, sx;
     int depth, parent, rank;
@@ -215,7 +216,6 @@ static int cand_before(const cand *a, const cand *b)
 {
     if (a->key != b->key) return a->key > b->key;
     if (a->depth != b->depth) return a->depth < b->depth;
-    if (a->sx != b->sx) return a->sx > b->sx;
     if (a->parent != b->parent) return a->parent < b->parent;
     return a->rank < b->rank;
 }
@@ -279,12 +279,15 @@ int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, i
             int best = 0;
             for (int f = 1; f < nf; ++f)
                 if (cand_before(&front[f], &front[best])) best = f;
-            /* Near-tie check: only keys of different depths depend on the log-normalisers;
-             * same-depth order is decided exactly through Sx. */
+            /* Near-tie check. Keys of different depths depend on the log-normalisers, which
+             * another implementation rounds differently; same-depth keys with different Sx can
+             * only tie through the rounding of Sx - CL[d]. Same-depth candidates with equal Sx
+             * tie exactly everywhere and are not near ties. */
             for (int f = 0; f < nf; ++f) {
-                if (f == best || front[f].depth == front[best].depth) continue;
+                if (f == best) continue;
+                if (front[f].depth == front[best].depth && front[f].sx == front[best].sx) continue;
                 double margin = front[best].key - front[f].key;
-                if (margin < mm) mm = margin;
+                if (front[f].depth != front[best].depth && margin < mm) mm = margin;
                 if (margin < key_eps * (1.0 + fabs(front[best].key))) ex = 1;
             }
             cand c = front[best];

@@ -43,53 +43,49 @@ struct BvArgs {
 };
 
 struct BlockRed {
-    double s[kWarps];
-    float m[kWarps];
+    MaxSum ms[kWarps];
+    FF ff[kWarps];
     unsigned long long k[kWarps];
-    double S;
-    float M;
+    MaxSum MS;
+    FF S;
     unsigned long long K;
 };
 
-// (max, sum exp) over the block; valid in every thread afterwards.
-__device__ void block_maxsum(BlockRed &sh, float m, double s, float &M, double &S) {
+// Softmax normaliser over the block (float-float); valid in every thread afterwards.
+__device__ MaxSum block_maxsum(BlockRed &sh, MaxSum v) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const float a = warp_max(m);
-    const double t = warp_sum_d(m == -INFINITY ? 0.0 : s * (double)expf(m - a));
-    if (lane == 0) {
-        sh.m[warp] = a;
-        sh.s[warp] = t;
-    }
+    v = warp_maxsum(v);
+    if (lane == 0) sh.ms[warp] = v;
     __syncthreads();
     if (warp == 0) {
-        const float bm = lane < kWarps ? sh.m[lane] : -INFINITY;
-        const double bs = lane < kWarps ? sh.s[lane] : 0.0;
-        const float aa = warp_max(bm);
-        const double tt = warp_sum_d(bm == -INFINITY ? 0.0 : bs * (double)expf(bm - aa));
-        if (lane == 0) {
-            sh.M = aa;
-            sh.S = tt;
-        }
+        const MaxSum w = warp_maxsum(lane < kWarps ? sh.ms[lane] : MaxSum{-INFINITY, FF{0.f, 0.f}});
+        if (lane == 0) sh.MS = w;
     }
     __syncthreads();
-    M = sh.M;
-    S = sh.S;
-    __syncthreads();
-}
-
-__device__ double block_sum(BlockRed &sh, double v) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const double t = warp_sum_d(v);
-    if (lane == 0) sh.s[warp] = t;
-    __syncthreads();
-    if (warp == 0) {
-        const double tt = warp_sum_d(lane < kWarps ? sh.s[lane] : 0.0);
-        if (lane == 0) sh.S = tt;
-    }
-    __syncthreads();
-    const double r = sh.S;
+    const MaxSum r = sh.MS;
     __syncthreads();
     return r;
+}
+
+__device__ FF block_sum(BlockRed &sh, FF v) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    v = warp_sum_ff(v);
+    if (lane == 0) sh.ff[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+        const FF w = warp_sum_ff(lane < kWarps ? sh.ff[lane] : FF{0.f, 0.f});
+        if (lane == 0) sh.S = w;
+    }
+    __syncthreads();
+    const FF r = sh.S;
+    __syncthreads();
+    return r;
+}
+
+__device__ __forceinline__ double lse_of(MaxSum v) {
+    if (!(v.s.hi > 0.f)) return -INFINITY;
+    const FF l = maxsum_lse(v);
+    return (double)l.hi + (double)l.lo;
 }
 
 __device__ unsigned long long block_argmax(BlockRed &sh, unsigned long long k) {
@@ -158,9 +154,7 @@ __global__ void __launch_bounds__(kThreads) k_bv_rows(BvArgs a) {
 #pragma unroll
             for (int k = 0; k < 8; ++k) s.add(expf(__fsub_rn(__fmul_rn(x[k], a.invT), m)));
         }
-    float M;
-    double S;
-    block_maxsum(sh, m, s.value(), M, S);
+    const MaxSum tot = block_maxsum(sh, MaxSum{m, s.ff()});
     double lse_q = 0.0;
     if (i < g) {
         const int r = qrow_index(a, b, i);
@@ -171,18 +165,16 @@ __global__ void __launch_bounds__(kThreads) k_bv_rows(BvArgs a) {
             for (int c = threadIdx.x; c < a.C; c += kThreads) mq = fmaxf(mq, st[c].x);
             const float mqw = mq;
             if (mqw != -INFINITY)
-                for (int c = threadIdx.x; c < a.C; c += kThreads) sq.add(st[c].y * expf(st[c].x - mqw));
+                for (int c = threadIdx.x; c < a.C; c += kThreads)
+                    sq.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, mqw))));
         } else if (threadIdx.x == 0) {
             raise_status(a.status, kDevBadIndex);
         }
-        float Mq;
-        double Sq;
-        block_maxsum(sh, mq, sq.value(), Mq, Sq);
-        lse_q = (double)Mq + log(Sq);
+        lse_q = lse_of(block_maxsum(sh, MaxSum{mq, sq.ff()}));
     }
     if (threadIdx.x == 0) {
         BvRow &o = a.rows[(int64_t)b * NN + i];
-        o.lse_t = (double)M + log(S);
+        o.lse_t = lse_of(tot);
         o.lse_q = lse_q;
     }
 }
@@ -251,7 +243,8 @@ __global__ void __launch_bounds__(kThreads) k_bv_resid(BvArgs a) {
             acc.add(fmaxf(__fsub_rn(__fmul_rn(w, p), q), 0.f));
         }
     }
-    const double S = block_sum(sh, acc.value());
+    const FF Sf = block_sum(sh, acc.ff());
+    const double S = (double)Sf.hi + (double)Sf.lo;
     if (threadIdx.x == 0) {
         BvRow &o = a.rows[(int64_t)b * NN + i];
         o.S = S;

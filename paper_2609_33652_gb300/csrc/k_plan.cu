@@ -7,11 +7,13 @@
 //   >= tau go through per-lane sorted lists, and a warp merge yields the top-K by
 //   (x desc, id asc). Results go to the workspace.
 // k_plan_heap, one CTA per tree: best-first expansion, popping N candidates. A candidate at
-//   depth d holds the exact fp64 sum Sx of its path's logits and the key Sx - CL[d],
+//   depth d holds the float-float sum Sx of its path's logits and the key Sx - CL[d],
 //   CL[d] = LSE_1 + ... + LSE_d (its draft path log-probability). Pop order: (key desc,
-//   depth asc, Sx desc, parent asc, rank asc). Popping (p, r) at depth d pushes the next
-//   sibling (p, r+1) and, below the depth cap, the first child (i, 0). Siblings are popped in
-//   rank order, so the children of u occupy child_ids[child_off[u] + rank] directly.
+//   depth asc, parent asc, rank asc), compared as integers (order-preserving image of the
+//   float-float key; no fp64 anywhere). Popping (p, r) at depth d
+//   pushes the next sibling (p, r+1) and, below the depth cap, the first child (i, 0).
+//   Siblings are popped in rank order, so the children of u occupy
+//   child_ids[child_off[u] + rank] directly.
 //
 // Both are latency-bound: the draft rows were streamed once by the statistics kernel and only
 // the few candidate chunks per row are read again.
@@ -30,7 +32,7 @@ struct TopkArgs {
     int B, R, V, C, L, K;
     const float2 *stats;
     float invT;
-    double *lse;       // [B*L]
+    float2 *lse;       // [B*L] row log-normalisers as float-float (hi, lo)
     float *topk_x;     // [B*L*K]
     int32_t *topk_id;  // [B*L*K]
 };
@@ -60,14 +62,17 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_row_topk(TopkArgs a) {
         }
     }
     __syncwarp();
-    // log-normaliser
+    // log-normaliser (float-float; the lane partials merge in a butterfly)
     float m = -INFINITY;
     for (int c = lane; c < C; c += 32) m = fmaxf(m, st[c].x);
-    m = warp_max(m);
     KahanF acc;
-    for (int c = lane; c < C; c += 32) acc.add(st[c].y * expf(st[c].x - m));
-    const double S = warp_sum_d(acc.value());
-    if (lane == 0) a.lse[row] = (double)m + log(S);
+    if (m != -INFINITY)
+        for (int c = lane; c < C; c += 32) acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
+    const MaxSum tot = warp_maxsum(MaxSum{m, acc.ff()});
+    if (lane == 0) {
+        const FF l = maxsum_lse(tot);
+        a.lse[row] = make_float2(l.hi, l.lo);
+    }
     // tau = K-th largest chunk maximum (-inf with fewer than K chunks)
     float tau = -INFINITY;
     if (C >= K) {
@@ -130,49 +135,88 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_row_topk(TopkArgs a) {
 
 struct HeapArgs {
     int L, N, K;
-    const double *lse;
+    const float2 *lse;
     const float *topk_x;
     const int32_t *topk_id;
     TreeDesc tree;
     uint32_t *status;
 };
 
-struct Cand {
-    double key, sx;
-    int meta;  // parent << 16 | depth << 8 | rank
+// A frontier candidate is a 96-bit integer key, larger = pops first:
+//   okey = order-preserving image of the float-float key (Sx - CL[depth]), high word from
+//          its head, low word from its tail;
+//   w3   = (255 - depth) << 24 | (65535 - parent) << 8 | (255 - rank)
+// so the order is (key desc, depth asc, parent asc, rank asc); an empty slot is (0, 0).
+// Path sums Sx are float-float sums of fp32 logits (TwoSum additions: exact while the
+// logits of a path span fewer than ~24 binades), so equal sums give equal keys bit for bit.
+__device__ __forceinline__ unsigned w3_of(int depth, int parent, int rank) {
+    return ((unsigned)(255 - depth) << 24) | ((unsigned)(65535 - parent) << 8) | (unsigned)(255 - rank);
+}
+__device__ __forceinline__ bool key_better(unsigned long long ka, unsigned wa, unsigned long long kb, unsigned wb) {
+    return ka > kb || (ka == kb && wa > wb);
+}
+__device__ __forceinline__ unsigned long long ord_ff(FF v) {
+    return ((unsigned long long)ord_f32(v.hi) << 32) | (unsigned long long)ord_f32(v.lo);
+}
+__device__ __forceinline__ FF ff_neg(FF v) { return FF{-v.hi, -v.lo}; }
+
+template <int S>
+struct Slots {
+    unsigned long long k[S];
+    unsigned w[S];
+    unsigned long long bk;  // the lane's best
+    unsigned bw;
+    int bs;
+    __device__ __forceinline__ void clear() {
+#pragma unroll
+        for (int s = 0; s < S; ++s) {
+            k[s] = 0ull;
+            w[s] = 0u;
+        }
+        bk = 0ull;
+        bw = 0u;
+        bs = 0;
+    }
+    __device__ __forceinline__ void put(int slot, unsigned long long kk, unsigned ww) {
+#pragma unroll
+        for (int s = 0; s < S; ++s)
+            if (s == slot) {
+                k[s] = kk;
+                w[s] = ww;
+            }
+    }
+    __device__ __forceinline__ void rescan() {
+        bk = 0ull;
+        bw = 0u;
+        bs = 0;
+#pragma unroll
+        for (int s = 0; s < S; ++s)
+            if (key_better(k[s], w[s], bk, bw)) {
+                bk = k[s];
+                bw = w[s];
+                bs = s;
+            }
+    }
 };
 
-__device__ __forceinline__ int meta_parent(int m) { return m >> 16; }
-__device__ __forceinline__ int meta_depth(int m) { return (m >> 8) & 0xff; }
-__device__ __forceinline__ int meta_rank(int m) { return m & 0xff; }
-
-// Does a pop before b?
-__device__ __forceinline__ bool cand_before(const Cand &a, const Cand &b) {
-    if (a.key != b.key) return a.key > b.key;
-    const int da = meta_depth(a.meta), db = meta_depth(b.meta);
-    if (da != db) return da < db;
-    if (a.sx != b.sx) return a.sx > b.sx;
-    const int pa = meta_parent(a.meta), pb = meta_parent(b.meta);
-    if (pa != pb) return pa < pb;
-    return meta_rank(a.meta) < meta_rank(b.meta);
-}
-
+// Best-first expansion for one tree with one warp. Each pop: a three-stage warp maximum of
+// the lanes' best keys (__reduce_max_sync on the high word, low word, tie word); the popped
+// candidate's slot takes its next sibling; its first child goes to the next round-robin
+// slot (children are numbered in creation order, lane = c % 32, slot = c / 32).
+template <int S>
 __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int L = a.L, N = a.N, K = a.K, NN = N + 1;
-    double *CL = reinterpret_cast<double *>(smem);   // [L+1]
-    double *f_key = CL + (L + 1);                    // [NN] frontier
-    double *f_sx = f_key + NN;                       // [NN]
-    double *n_sx = f_sx + NN;                        // [NN] node path sums
-    int32_t *f_meta = reinterpret_cast<int32_t *>(n_sx + NN);  // [NN]
-    int32_t *n_parent = f_meta + NN;                 // [NN]
+    FF *CL = reinterpret_cast<FF *>(smem);                         // [L+1]
+    FF *n_sx = CL + (L + 1);                                       // [NN] node path sums
+    int32_t *n_parent = reinterpret_cast<int32_t *>(n_sx + NN);    // [NN]
     int32_t *n_depth = n_parent + NN;
     int32_t *n_rank = n_depth + NN;
     int32_t *n_token = n_rank + NN;
-    int32_t *n_count = n_token + NN;                 // [NN]
-    float *n_score = reinterpret_cast<float *>(n_count + NN);  // [NN]
-    int32_t *tk_id = reinterpret_cast<int32_t *>(n_score + NN);  // [L*K]
-    float *tk_x = reinterpret_cast<float *>(tk_id + L * K);      // [L*K]
+    int32_t *n_count = n_token + NN;                               // [NN]
+    float *n_score = reinterpret_cast<float *>(n_count + NN);      // [NN]
+    int32_t *tk_id = reinterpret_cast<int32_t *>(n_score + NN);    // [L*K]
+    float *tk_x = reinterpret_cast<float *>(tk_id + L * K);        // [L*K]
 
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -187,10 +231,22 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
         n_rank[i] = 0;
         n_token[i] = -1;
         n_score[i] = 0.f;
+        n_sx[i] = FF{0.f, 0.f};
     }
-    if (threadIdx.x == 0) {
-        CL[0] = 0.0;
-        for (int d = 1; d <= L; ++d) CL[d] = CL[d - 1] + a.lse[(int64_t)b * L + d - 1];
+    if (warp == 0) {  // CL[d] = LSE_1 + ... + LSE_d (loads in parallel, sum in order)
+        if (lane < L) {
+            const float2 l = a.lse[(int64_t)b * L + lane];
+            CL[lane + 1] = FF{l.x, l.y};
+        }
+        if (lane + 32 < L) {
+            const float2 l = a.lse[(int64_t)b * L + lane + 32];
+            CL[lane + 33] = FF{l.x, l.y};
+        }
+        __syncwarp();
+        if (lane == 0) {
+            CL[0] = FF{0.f, 0.f};
+            for (int d = 1; d <= L; ++d) CL[d] = ff_add(CL[d - 1], CL[d]);
+        }
     }
     __syncthreads();
 
@@ -200,71 +256,69 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
             n_depth[0] = 0;
             n_rank[0] = -1;
             n_token[0] = -1;
-            n_score[0] = 0.f;
-            n_sx[0] = 0.0;
-            f_sx[0] = (double)tk_x[0];
-            f_key[0] = f_sx[0] - CL[1];
-            f_meta[0] = (0 << 16) | (1 << 8) | 0;
         }
-        int nf = 1;
+        Slots<S> fr;
+        fr.clear();
+        if (lane == 0) {  // the root's first child (depth 1, rank 0) is child number 0
+            const FF sx = ff_add(FF{0.f, 0.f}, FF{tk_x[0], 0.f});
+            fr.put(0, ord_ff(ff_add(sx, ff_neg(CL[1]))), w3_of(1, 0, 0));
+            fr.rescan();
+        }
+        int nchild = 1;
         __syncwarp();
         for (int i = 1; i <= N; ++i) {
-            Cand best{-INFINITY, 0.0, 0};
-            int bi = -1;
-            for (int f = lane; f < nf; f += 32) {
-                Cand c{f_key[f], f_sx[f], f_meta[f]};
-                if (bi < 0 || cand_before(c, best)) {
-                    best = c;
-                    bi = f;
-                }
-            }
-#pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-                Cand other;
-                other.key = __shfl_xor_sync(kFull, best.key, o);
-                other.sx = __shfl_xor_sync(kFull, best.sx, o);
-                other.meta = __shfl_xor_sync(kFull, best.meta, o);
-                const int oi = __shfl_xor_sync(kFull, bi, o);
-                if (oi >= 0 && (bi < 0 || cand_before(other, best))) {
-                    best = other;
-                    bi = oi;
-                }
-            }
-            if (bi < 0) {  // frontier exhausted: only with N above the tree's capacity
+            const unsigned hk = (unsigned)(fr.bk >> 32), lk = (unsigned)fr.bk;
+            const unsigned m1 = __reduce_max_sync(kFull, hk);
+            unsigned c = __ballot_sync(kFull, hk == m1);
+            const unsigned m2 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? lk : 0u);
+            c &= __ballot_sync(kFull, lk == m2);
+            const unsigned m3 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? fr.bw : 0u);
+            c &= __ballot_sync(kFull, fr.bw == m3);
+            if (m3 == 0u) {  // frontier exhausted: only with N above the tree's capacity
                 if (lane == 0) raise_status(a.status, kDevBadTree);
                 break;
             }
-            const int parent = meta_parent(best.meta), depth = meta_depth(best.meta), rank = meta_rank(best.meta);
+            const int winner = __ffs(c) - 1;
+            const int depth = 255 - (int)(m3 >> 24);
+            const int parent = 65535 - (int)((m3 >> 8) & 0xffffu);
+            const int rank = 255 - (int)(m3 & 0xffu);
+            FF sx = FF{0.f, 0.f};
+            if (lane == winner) {
+                // the popped path's sum, recomputed with the same additions as at creation
+                const FF sp = n_sx[parent];
+                sx = ff_add(sp, FF{tk_x[(depth - 1) * K + rank], 0.f});
+                n_sx[i] = sx;
+                if (rank + 1 < K) {  // the next sibling takes the freed slot
+                    const FF ss = ff_add(sp, FF{tk_x[(depth - 1) * K + rank + 1], 0.f});
+                    fr.put(fr.bs, ord_ff(ff_add(ss, ff_neg(CL[depth]))), w3_of(depth, parent, rank + 1));
+                } else {
+                    fr.put(fr.bs, 0ull, 0u);
+                }
+                fr.rescan();
+            }
             if (lane == 0) {
                 n_parent[i] = parent;
                 n_depth[i] = depth;
                 n_rank[i] = rank;
                 n_token[i] = tk_id[(depth - 1) * K + rank];
-                n_score[i] = (float)best.key;
-                n_sx[i] = best.sx;
-                // remove the popped entry, then push its next sibling and first child
-                const int last = nf - 1;
-                f_key[bi] = f_key[last];
-                f_sx[bi] = f_sx[last];
-                f_meta[bi] = f_meta[last];
-                int nn = last;
-                if (rank + 1 < K) {
-                    const double sx = n_sx[parent] + (double)tk_x[(depth - 1) * K + rank + 1];
-                    f_sx[nn] = sx;
-                    f_key[nn] = sx - CL[depth];
-                    f_meta[nn] = (parent << 16) | (depth << 8) | (rank + 1);
-                    ++nn;
-                }
-                if (depth < L) {
-                    const double sx = best.sx + (double)tk_x[depth * K + 0];
-                    f_sx[nn] = sx;
-                    f_key[nn] = sx - CL[depth + 1];
-                    f_meta[nn] = (i << 16) | ((depth + 1) << 8) | 0;
-                    ++nn;
-                }
-                nf = nn;
+                n_score[i] = f32_of_ord(m1);
             }
-            nf = __shfl_sync(kFull, nf, 0);
+            if (depth < L) {  // first child (i, 0), one level down
+                sx.hi = __shfl_sync(kFull, sx.hi, winner);
+                sx.lo = __shfl_sync(kFull, sx.lo, winner);
+                if (lane == (nchild & 31)) {
+                    const FF sc = ff_add(sx, FF{tk_x[depth * K + 0], 0.f});
+                    const unsigned long long ck = ord_ff(ff_add(sc, ff_neg(CL[depth + 1])));
+                    const unsigned cw = w3_of(depth + 1, i, 0);
+                    fr.put(nchild >> 5, ck, cw);
+                    if (key_better(ck, cw, fr.bk, fr.bw)) {
+                        fr.bk = ck;
+                        fr.bw = cw;
+                        fr.bs = nchild >> 5;
+                    }
+                }
+                ++nchild;
+            }
             __syncwarp();
         }
     }
@@ -311,7 +365,16 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
 
 size_t heap_smem_bytes(int L, int N, int K) {
     const size_t NN = (size_t)N + 1;
-    return (size_t)(L + 1) * 8 + 3 * NN * 8 + 7 * NN * 4 + 2 * (size_t)L * K * 4;
+    return (size_t)(L + 1) * sizeof(FF) + NN * sizeof(FF) + 6 * NN * 4 + 2 * (size_t)L * K * 4;
+}
+
+template <int S>
+cudaError_t launch_heap_t(const HeapArgs &h, int B, cudaStream_t s) {
+    const size_t smem = heap_smem_bytes(h.L, h.N, h.K);
+    cudaError_t e = cudaFuncSetAttribute(k_plan_heap<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    k_plan_heap<S><<<B, kHeapThreads, smem, s>>>(h);
+    return cudaGetLastError();
 }
 
 template <int KCAP, typename T>
@@ -329,9 +392,9 @@ cudaError_t launch_topk_t(const TopkArgs &a, cudaStream_t s) {
 PlanScratch plan_scratch(void *ws, int B, int N, int L, int K) {
     unsigned char *p = static_cast<unsigned char *>(ws) + kWsStatusBytes + (size_t)B * (N + 1) * kWsBvRowBytes;
     PlanScratch s;
-    s.lse = reinterpret_cast<double *>(p);
-    s.topk_x = reinterpret_cast<float *>(p + (size_t)B * L * sizeof(double));
-    s.topk_id = reinterpret_cast<int32_t *>(p + (size_t)B * L * sizeof(double) + (size_t)B * L * K * sizeof(float));
+    s.lse = reinterpret_cast<float2 *>(p);
+    s.topk_x = reinterpret_cast<float *>(p + (size_t)B * L * sizeof(float2));
+    s.topk_id = reinterpret_cast<int32_t *>(p + (size_t)B * L * sizeof(float2) + (size_t)B * L * K * sizeof(float));
     return s;
 }
 
@@ -368,11 +431,14 @@ cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N
     h.topk_id = sc.topk_id;
     h.tree = tree;
     h.status = static_cast<uint32_t *>(ws);
-    const size_t smem = heap_smem_bytes(L, N, K);
-    e = cudaFuncSetAttribute(k_plan_heap, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    k_plan_heap<<<draft.B, kHeapThreads, smem, s>>>(h);
-    return cudaGetLastError();
+    // frontier slots per lane: at most N + 1 first children are ever created
+    const int per_lane = (N + 1 + 31) / 32;
+    if (per_lane <= 1) return launch_heap_t<1>(h, draft.B, s);
+    if (per_lane <= 2) return launch_heap_t<2>(h, draft.B, s);
+    if (per_lane <= 4) return launch_heap_t<4>(h, draft.B, s);
+    if (per_lane <= 8) return launch_heap_t<8>(h, draft.B, s);
+    if (per_lane <= 16) return launch_heap_t<16>(h, draft.B, s);
+    return launch_heap_t<33>(h, draft.B, s);
 }
 
 }  // namespace tsb

@@ -4,8 +4,12 @@
 // the replay sampler (Sec. 3.2) all follow from these without touching the row again.
 //
 // HBM-bound: every logit is read once with 16-byte loads; 8 bytes are written per chunk.
-// One warp owns 4 consecutive chunks of a row (lane l holds logits 8l..8l+7 of each chunk),
-// issuing all of its loads before any arithmetic.
+// A warp owns groups of 8 consecutive chunks of a row (lane l holds logits 8l..8l+7 of each
+// chunk) and issues all 8 loads before any arithmetic; the grid is persistent (grid-stride
+// over groups) so there is no partial last wave. Per logit: one conversion, one max, one
+// fma, one ex2 and one add. Rounding to nearest is monotone, so the chunk maximum is taken on
+// the raw logits and scaled once: max_v fp32(z_v * invT) = fp32(max_v z_v * invT).
+// Non-finite logits are detected per chunk (an infinite maximum or a NaN sum).
 #include "tsb_device.cuh"
 #include "tsb_launch.h"
 
@@ -13,7 +17,56 @@ namespace tsb {
 namespace {
 
 constexpr int kWarps = 8;
-constexpr int kPerWarp = 4;  // chunks per warp
+constexpr int kPerWarp = 8;  // chunks per warp group
+
+template <typename T>
+struct Raw;  // 8 consecutive logits as raw 16-byte words
+template <>
+struct Raw<__nv_bfloat16> {
+    uint4 w;
+    __device__ __forceinline__ void load(const __nv_bfloat16 *row, int v0, int V) {
+        if (v0 + 8 <= V) {
+            w = __ldg(reinterpret_cast<const uint4 *>(row + v0));
+        } else {  // ragged tail: missing logits become -inf (0xff80)
+            const unsigned short *r = reinterpret_cast<const unsigned short *>(row);
+            unsigned short h[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) h[i] = (v0 + i < V) ? __ldg(r + v0 + i) : (unsigned short)0xff80u;
+            w.x = h[0] | ((uint32_t)h[1] << 16);
+            w.y = h[2] | ((uint32_t)h[3] << 16);
+            w.z = h[4] | ((uint32_t)h[5] << 16);
+            w.w = h[6] | ((uint32_t)h[7] << 16);
+        }
+    }
+    __device__ __forceinline__ void unpack(float z[8]) const {
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            z[2 * i] = __uint_as_float(u[i] << 16);
+            z[2 * i + 1] = __uint_as_float(u[i] & 0xffff0000u);
+        }
+    }
+};
+template <>
+struct Raw<float> {
+    float4 a, b;
+    __device__ __forceinline__ void load(const float *row, int v0, int V) {
+        if (v0 + 8 <= V) {
+            a = __ldg(reinterpret_cast<const float4 *>(row + v0));
+            b = __ldg(reinterpret_cast<const float4 *>(row + v0 + 4));
+        } else {
+            float z[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) z[i] = (v0 + i < V) ? __ldg(row + v0 + i) : -INFINITY;
+            a = make_float4(z[0], z[1], z[2], z[3]);
+            b = make_float4(z[4], z[5], z[6], z[7]);
+        }
+    }
+    __device__ __forceinline__ void unpack(float z[8]) const {
+        z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w;
+        z[4] = b.x; z[5] = b.y; z[6] = b.z; z[7] = b.w;
+    }
+};
 
 template <typename T>
 __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__ data, int R, int V,
@@ -21,64 +74,88 @@ __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__
                                                            int64_t groups_total, float invT,
                                                            float2 *__restrict__ stats, uint32_t *status) {
     const int lane = threadIdx.x & 31;
-    const int64_t gw = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5);
-    if (gw >= groups_total) return;
     const int groups = (C + kPerWarp - 1) / kPerWarp;
-    const int64_t row = gw / groups;
-    const int g = (int)(gw - row * groups);
-    const int b = (int)(row / R);
-    const int r = (int)(row - (int64_t)b * R);
-    const T *rp = data + (int64_t)b * bstride + (int64_t)r * rstride;
-    const int c0 = g * kPerWarp;
-    const int nc = min(kPerWarp, C - c0);
-
-    float x[kPerWarp][8];
-#pragma unroll
-    for (int k = 0; k < kPerWarp; ++k)
-        if (k < nc) Logit<T>::load8(rp, (c0 + k) * kChunk + lane * 8, V, x[k]);
-
+    const float c2 = __fmul_rn(invT, kLog2e);  // exp(x - m) = 2^(z invT log2e - m log2e)
     bool bad = false;
+    for (int64_t gw = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5); gw < groups_total;
+         gw += (int64_t)gridDim.x * kWarps) {
+        const int64_t row = gw / groups;
+        const int g = (int)(gw - row * groups);
+        const int b = (int)(row / R);
+        const int r = (int)(row - (int64_t)b * R);
+        const T *rp = data + (int64_t)b * bstride + (int64_t)r * rstride;
+        const int c0 = g * kPerWarp;
+        const int nc = min(kPerWarp, C - c0);
+        Raw<T> raw[kPerWarp];
 #pragma unroll
-    for (int k = 0; k < kPerWarp; ++k) {
-        if (k >= nc) break;  // warp-uniform
-        const int v0 = (c0 + k) * kChunk + lane * 8;
-        float m = -INFINITY;
+        for (int k = 0; k < kPerWarp; ++k)
+            if (k < nc) raw[k].load(rp, (c0 + k) * kChunk + lane * 8, V);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-            float xi = -INFINITY;
-            if (v0 + i < V) {
-                xi = __fmul_rn(x[k][i], invT);
-                bad |= !isfinite(xi);
+        for (int k = 0; k < kPerWarp; ++k) {
+            if (k >= nc) break;  // warp-uniform
+            float z[8];
+            raw[k].unpack(z);
+            float zm = z[0];
+#pragma unroll
+            for (int i = 1; i < 8; ++i) zm = fmaxf(zm, z[i]);
+            zm = warp_max(zm);
+            const float mc = __fmul_rn(zm, invT);
+            const float off = __fmul_rn(mc, kLog2e);
+            float s = 0.f;
+#pragma unroll
+            for (int i = 0; i < 8; ++i) s += fast_exp2(__fmaf_rn(z[i], c2, -off));
+            s = warp_sum(s);
+            if (lane == 0) {
+                stats[row * C + c0 + k] = make_float2(mc, s);
+                bad |= !(s == s) || isinf(mc);
             }
-            x[k][i] = xi;
-            m = fmaxf(m, xi);
         }
-        m = warp_max(m);
-        float s = 0.f;
-#pragma unroll
-        for (int i = 0; i < 8; ++i) s += fast_exp2(__fmul_rn(__fsub_rn(x[k][i], m), kLog2e));
-        s = warp_sum(s);
-        if (lane == 0) stats[row * C + c0 + k] = make_float2(m, s);
     }
-    if (__any_sync(kFull, bad) && lane == 0) raise_status(status, kDevNonFinite);
+    if (bad) raise_status(status, kDevNonFinite);
+}
+
+template <typename T>
+int blocks_per_sm() {
+    static int cached = 0;
+    if (cached == 0) {
+        int n = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, k_row_stats<T>, kWarps * 32, 0) != cudaSuccess || n < 1)
+            n = 1;
+        cached = n;
+    }
+    return cached;
+}
+
+int sm_count() {
+    static int cached = 0;
+    if (cached == 0) {
+        int dev = 0, n = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) !=
+                                                     cudaSuccess || n < 1)
+            n = 1;
+        cached = n;
+    }
+    return cached;
+}
+
+template <typename T>
+cudaError_t launch_t(const RowsDesc &rows, float invT, float2 *stats, uint32_t *status, cudaStream_t s) {
+    const int C = num_chunks(rows.V);
+    const int64_t groups_total = (int64_t)rows.B * rows.R * ((C + kPerWarp - 1) / kPerWarp);
+    const int64_t needed = (groups_total + kWarps - 1) / kWarps;
+    const int64_t resident = (int64_t)sm_count() * blocks_per_sm<T>();
+    const int64_t blocks = needed < resident ? needed : resident;
+    k_row_stats<T><<<(unsigned)blocks, kWarps * 32, 0, s>>>(static_cast<const T *>(rows.data), rows.R, rows.V,
+                                                             rows.batch_stride, rows.row_stride, C, groups_total,
+                                                             invT, stats, status);
+    return cudaGetLastError();
 }
 
 }  // namespace
 
 cudaError_t launch_row_stats(const RowsDesc &rows, float invT, float2 *stats, uint32_t *status, cudaStream_t s) {
-    const int C = num_chunks(rows.V);
-    const int64_t groups_total = (int64_t)rows.B * rows.R * ((C + kPerWarp - 1) / kPerWarp);
-    const int64_t blocks = (groups_total + kWarps - 1) / kWarps;
-    if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    if (rows.dtype == 1)
-        k_row_stats<__nv_bfloat16><<<(unsigned)blocks, kWarps * 32, 0, s>>>(
-            static_cast<const __nv_bfloat16 *>(rows.data), rows.R, rows.V, rows.batch_stride, rows.row_stride, C,
-            groups_total, invT, stats, status);
-    else
-        k_row_stats<float><<<(unsigned)blocks, kWarps * 32, 0, s>>>(static_cast<const float *>(rows.data), rows.R,
-                                                                     rows.V, rows.batch_stride, rows.row_stride, C,
-                                                                     groups_total, invT, stats, status);
-    return cudaGetLastError();
+    if (rows.dtype == 1) return launch_t<__nv_bfloat16>(rows, invT, stats, status, s);
+    return launch_t<float>(rows, invT, stats, status, s);
 }
 
 }  // namespace tsb

@@ -24,6 +24,8 @@
 // log(chunk mass) + G over chunks of 256 tokens, then the best token of the winning chunk.
 #include <cooperative_groups.h>
 
+#include <mutex>
+
 #include "tsb_device.cuh"
 #include "tsb_launch.h"
 
@@ -51,136 +53,155 @@ struct VerifyArgs {
     uint32_t *status;
 };
 
+// A partial of one cluster-wide reduction: two softmax normalisers (target row, q row), a
+// plain sum, and an argmax key carrying a token.
 struct alignas(16) Slot {
-    double s1, s2, z;
+    float m1, s1h, s1l, m2, s2h, s2l, zh, zl;
     unsigned long long key;
-    float m1, m2;
-    float hi1, lo1, hi2, lo2;  // log-normalisers as fp32 hi + lo (filled by the combine)
+    int tok, pad;
 };
 
-struct Scratch {
-    Slot slot[2];  // published partials, double-buffered across rounds
-    Slot res;      // combined result
-    double ws1[kWarps], ws2[kWarps], wz[kWarps];
-    unsigned long long wkey[kWarps];
-    float wm1[kWarps], wm2[kWarps];
-    float zs[kMaxK], ts[kMaxK];
-};
+enum : int { kRedLse = 1, kRedSum = 2, kRedArg = 4 };
 
-__device__ __forceinline__ float qratio(float q, float t) { return (q > 0.f && t > 0.f) ? __fdiv_rn(q, t) : 0.f; }
-
-// exp(x - LSE) with LSE = hi + lo; x = fp32(z) * invT
-__device__ __forceinline__ float prob_of(float x, float hi, float lo) { return expf(__fsub_rn(__fsub_rn(x, hi), lo)); }
-
-// p_i(y) from P0(y), Q(y): the same fp32 operations the element passes perform.
-__device__ __forceinline__ float point_residual(float p0, float q, const float *zs, const float *ts, int i) {
-    float p = p0;
-    for (int j = 0; j < i; ++j) {
-        const float r = fmaxf(__fsub_rn(p, qratio(q, ts[j])), 0.f);
-        p = __fdiv_rn(r, zs[j]);
-    }
-    return p;
+__device__ __forceinline__ Slot neutral_slot() {
+    Slot s;
+    s.m1 = s.m2 = -INFINITY;
+    s.s1h = s.s1l = s.s2h = s.s2l = s.zh = s.zl = 0.f;
+    s.key = 0ull;
+    s.tok = -1;
+    s.pad = 0;
+    return s;
 }
 
-// One cluster-wide reduction of (max, sum-exp) x2, a plain sum and an argmax key.
-__device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &cluster, float m1, double s1, float m2,
-                             double s2, double z, unsigned long long key) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    {
-        const float a1 = warp_max(m1), a2 = warp_max(m2);
-        const double t1 = warp_sum_d(m1 == -INFINITY ? 0.0 : s1 * (double)expf(m1 - a1));
-        const double t2 = warp_sum_d(m2 == -INFINITY ? 0.0 : s2 * (double)expf(m2 - a2));
-        const double tz = warp_sum_d(z);
-        const unsigned long long tk = warp_max_u64(key);
-        if (lane == 0) {
-            sh.wm1[warp] = a1;
-            sh.ws1[warp] = t1;
-            sh.wm2[warp] = a2;
-            sh.ws2[warp] = t2;
-            sh.wz[warp] = tz;
-            sh.wkey[warp] = tk;
+// Symmetric merge of the fields a reduction of this kind carries.
+template <int KIND>
+__device__ __forceinline__ Slot merge_slot(const Slot &a, const Slot &b) {
+    Slot r = a;
+    if (KIND & kRedLse) {
+        const MaxSum x = maxsum_merge(MaxSum{a.m1, FF{a.s1h, a.s1l}}, MaxSum{b.m1, FF{b.s1h, b.s1l}});
+        const MaxSum y = maxsum_merge(MaxSum{a.m2, FF{a.s2h, a.s2l}}, MaxSum{b.m2, FF{b.s2h, b.s2l}});
+        r.m1 = x.m;
+        r.s1h = x.s.hi;
+        r.s1l = x.s.lo;
+        r.m2 = y.m;
+        r.s2h = y.s.hi;
+        r.s2l = y.s.lo;
+    }
+    if (KIND & kRedSum) {
+        const FF z = ff_add(FF{a.zh, a.zl}, FF{b.zh, b.zl});
+        r.zh = z.hi;
+        r.zl = z.lo;
+    }
+    if (KIND & kRedArg) {
+        if (b.key > a.key) {
+            r.key = b.key;
+            r.tok = b.tok;
         }
     }
+    return r;
+}
+
+template <int KIND>
+__device__ __forceinline__ Slot warp_reduce_slot(Slot v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        Slot w = v;
+        if (KIND & kRedLse) {
+            w.m1 = __shfl_xor_sync(kFull, v.m1, o);
+            w.s1h = __shfl_xor_sync(kFull, v.s1h, o);
+            w.s1l = __shfl_xor_sync(kFull, v.s1l, o);
+            w.m2 = __shfl_xor_sync(kFull, v.m2, o);
+            w.s2h = __shfl_xor_sync(kFull, v.s2h, o);
+            w.s2l = __shfl_xor_sync(kFull, v.s2l, o);
+        }
+        if (KIND & kRedSum) {
+            w.zh = __shfl_xor_sync(kFull, v.zh, o);
+            w.zl = __shfl_xor_sync(kFull, v.zl, o);
+        }
+        if (KIND & kRedArg) {
+            w.key = __shfl_xor_sync(kFull, v.key, o);
+            w.tok = __shfl_xor_sync(kFull, v.tok, o);
+        }
+        v = merge_slot<KIND>(v, w);
+    }
+    return v;
+}
+
+struct Scratch {
+    Slot slot[2];        // published partials, double-buffered across rounds
+    Slot wpart[kWarps];  // per-warp partials of the current round
+    Slot res;            // combined result
+    FF L2t, L2q;         // log-normalisers of the target and q rows, times log2(e)
+    unsigned long long wbest[kWarps];
+    unsigned long long cbest;
+    float izs[kMaxK], its[kMaxK];  // 1/Z and 1/t of every rejection so far
+};
+
+// One cluster-wide reduction: warp butterflies, the CTA's warp partials in warp 0, the
+// cluster barrier, then warp 0 of every CTA reads the CS published partials (one per lane)
+// and combines them with the same butterfly, so every CTA obtains identical results.
+template <int KIND>
+__device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &cluster, Slot mine) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const Slot w = warp_reduce_slot<KIND>(mine);
+    if (lane == 0) sh.wpart[warp] = w;
     __syncthreads();
     if (warp == 0) {
-        const float b1 = lane < kWarps ? sh.wm1[lane] : -INFINITY;
-        const float b2 = lane < kWarps ? sh.wm2[lane] : -INFINITY;
-        const double c1 = lane < kWarps ? sh.ws1[lane] : 0.0;
-        const double c2 = lane < kWarps ? sh.ws2[lane] : 0.0;
-        const double cz = lane < kWarps ? sh.wz[lane] : 0.0;
-        const unsigned long long ck = lane < kWarps ? sh.wkey[lane] : 0ull;
-        const float a1 = warp_max(b1), a2 = warp_max(b2);
-        const double t1 = warp_sum_d(b1 == -INFINITY ? 0.0 : c1 * (double)expf(b1 - a1));
-        const double t2 = warp_sum_d(b2 == -INFINITY ? 0.0 : c2 * (double)expf(b2 - a2));
-        const double tz = warp_sum_d(cz);
-        const unsigned long long tk = warp_max_u64(ck);
-        if (lane == 0) {
-            Slot &s = sh.slot[par];
-            s.m1 = a1;
-            s.s1 = t1;
-            s.m2 = a2;
-            s.s2 = t2;
-            s.z = tz;
-            s.key = tk;
-        }
+        const Slot v = warp_reduce_slot<KIND>(lane < kWarps ? sh.wpart[lane] : neutral_slot());
+        if (lane == 0) sh.slot[par] = v;
     }
     cluster.sync();
-    if (threadIdx.x == 0) {
+    if (warp == 0) {
         const int CS = (int)cluster.num_blocks();
-        float M1 = -INFINITY, M2 = -INFINITY;
-        for (int r = 0; r < CS; ++r) {
-            const Slot *p = cluster.map_shared_rank(&sh.slot[par], r);
-            M1 = fmaxf(M1, p->m1);
-            M2 = fmaxf(M2, p->m2);
-        }
-        double S1 = 0.0, S2 = 0.0, Z = 0.0;
-        unsigned long long Kx = 0ull;
-        for (int r = 0; r < CS; ++r) {
-            const Slot *p = cluster.map_shared_rank(&sh.slot[par], r);
-            if (p->m1 != -INFINITY) S1 += p->s1 * (double)expf(p->m1 - M1);
-            if (p->m2 != -INFINITY) S2 += p->s2 * (double)expf(p->m2 - M2);
-            Z += p->z;
-            Kx = p->key > Kx ? p->key : Kx;
-        }
-        Slot &o = sh.res;
-        o.m1 = M1;
-        o.m2 = M2;
-        o.s1 = S1;
-        o.s2 = S2;
-        o.z = Z;
-        o.key = Kx;
-        o.hi1 = o.lo1 = o.hi2 = o.lo2 = 0.f;
-        if (S1 > 0.0) {
-            const double l1 = (double)M1 + log(S1);
-            o.hi1 = (float)l1;
-            o.lo1 = (float)(l1 - (double)o.hi1);
-        }
-        if (S2 > 0.0) {
-            const double l2 = (double)M2 + log(S2);
-            o.hi2 = (float)l2;
-            o.lo2 = (float)(l2 - (double)o.hi2);
+        const Slot v = warp_reduce_slot<KIND>(lane < CS ? *cluster.map_shared_rank(&sh.slot[par], lane)
+                                                        : neutral_slot());
+        if (lane == 0) {
+            sh.res = v;
+            if (KIND & kRedLse) {
+                const FF l1 = v.s1h > 0.f ? maxsum_lse(MaxSum{v.m1, FF{v.s1h, v.s1l}}) : FF{0.f, 0.f};
+                const FF l2 = v.s2h > 0.f ? maxsum_lse(MaxSum{v.m2, FF{v.s2h, v.s2l}}) : FF{0.f, 0.f};
+                sh.L2t = ff_times_log2e(l1);
+                sh.L2q = ff_times_log2e(l2);
+            }
         }
     }
     __syncthreads();
     par ^= 1;
 }
 
-// Per-thread online (max, sum of exp(x - max)) accumulation.
+// The residual after rejecting a slot: max(p - q/t, 0) with 1/t precomputed; one fma, so the
+// element passes and the point values produce the same bits.
+__device__ __forceinline__ float resid(float p, float q, float it) { return fmaxf(__fmaf_rn(-q, it, p), 0.f); }
+
+// p_i(y) from P0(y), Q(y): the same fp32 operations the element passes perform.
+__device__ __forceinline__ float point_residual(float p0, float q, const float *izs, const float *its, int i) {
+    float p = p0;
+    for (int j = 0; j < i; ++j) p = __fmul_rn(resid(p, q, its[j]), izs[j]);
+    return p;
+}
+
+// Per-thread online (max, sum of exp(x - max)) accumulation, eight logits at a time.
 struct OnlineLse {
     float m = -INFINITY;
     KahanF s;
-    __device__ __forceinline__ void add(float x) {
-        if (x > m) {
+    __device__ __forceinline__ MaxSum value() const { return MaxSum{m, s.ff()}; }
+    __device__ __forceinline__ void add8(const float x[8]) {
+        float gm = x[0];
+#pragma unroll
+        for (int k = 1; k < 8; ++k) gm = fmaxf(gm, x[k]);
+        if (gm == -INFINITY) return;
+        if (gm > m) {
             if (m != -INFINITY) {
-                const float scale = fast_exp2(__fmul_rn(__fsub_rn(m, x), kLog2e));
+                const float scale = fast_exp2(__fmul_rn(__fsub_rn(m, gm), kLog2e));
                 s.s = __fmul_rn(s.s, scale);
                 s.c = __fmul_rn(s.c, scale);
             }
-            m = x;
-            s.add(1.0f);
-        } else {
-            s.add(fast_exp2(__fmul_rn(__fsub_rn(x, m), kLog2e)));
+            m = gm;
         }
+        float t = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t += fast_exp2(__fmul_rn(__fsub_rn(x[k], m), kLog2e));
+        s.add(t);
     }
 };
 
@@ -202,103 +223,95 @@ struct Walk {
             float x[8];
             Logit<T>::load8(row, lo + 8 * g, a.V, x);
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                const bool in = lo + 8 * g + k < a.V;
-                const float xv = in ? __fmul_rn(x[k], a.invT) : -INFINITY;
-                P[8 * g + k] = xv;
-                if (lse && in) lse->add(xv);
-            }
+            for (int k = 0; k < 8; ++k) x[k] = (lo + 8 * g + k < a.V) ? __fmul_rn(x[k], a.invT) : -INFINITY;
+            reinterpret_cast<float4 *>(P)[2 * g] = make_float4(x[0], x[1], x[2], x[3]);
+            reinterpret_cast<float4 *>(P)[2 * g + 1] = make_float4(x[4], x[5], x[6], x[7]);
+            if (lse) lse->add8(x);
         }
     }
 
-    // argmax over the winning chunk of lw + G (warp 0 of the owner CTA computes it).
-    template <typename LW>
-    __device__ int element_argmax(int node, int c, LW lw) {
-        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-        unsigned long long best = 0ull;
-        const int i0c = c * kChunk - lo;  // chunk start in this CTA's slice
-        if (warp == 0 && i0c >= 0 && i0c < n) {
-            const int i0 = i0c + lane * 8, v0 = lo + i0;
-            const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
-            const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2) + 1u);
-#pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                if (i0 + k >= n) break;
-                const float l = lw(i0 + k, v0 + k);
-                if (l == -INFINITY) continue;
-                const float key = __fadd_rn(l, gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4]));
-                const unsigned long long pk = pack_key(key, (uint32_t)(v0 + k));
-                best = pk > best ? pk : best;
-            }
-        }
-        reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, best);
-        return sh.res.key == 0ull ? -1 : (int)key_id(sh.res.key);
-    }
-
-    // Two-level draw from log-weights lw(smem index, token) (-inf = no mass); chunk masses
-    // are log-sum-exp of the log-weights.
-    template <typename LW>
-    __device__ int draw_logits(int node, LW lw) {
+    // Two-level draw (chunk by Gumbel-max over chunk masses, then token by Gumbel-max inside
+    // the chunk) in one cluster round: every CTA picks its best chunk and that chunk's best
+    // token; the cluster keeps the pair with the largest chunk key. val(j, v) returns a
+    // log-weight (LOGITS) or a weight >= 0 for the element at smem index j, token v.
+    template <bool LOGITS, typename F>
+    __device__ int draw(int node, F val) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int nch = (n + kChunk - 1) / kChunk;
         unsigned long long best = 0ull;
         for (int cl = warp; cl < nch; cl += kWarps) {
             const int i0 = cl * kChunk + lane * 8;
             float v[8];
-            float mx = -INFINITY;
 #pragma unroll
-            for (int k = 0; k < 8; ++k) {
-                v[k] = (i0 + k < n) ? lw(i0 + k, lo + i0 + k) : -INFINITY;
-                mx = fmaxf(mx, v[k]);
-            }
-            mx = warp_max(mx);
-            float s = 0.f;
-            if (mx != -INFINITY) {
+            for (int k = 0; k < 8; ++k) v[k] = (i0 + k < n) ? val(i0 + k, lo + i0 + k) : (LOGITS ? -INFINITY : 0.f);
+            float A = -INFINITY;
+            if (LOGITS) {
+                float mx = -INFINITY;
 #pragma unroll
-                for (int k = 0; k < 8; ++k) s += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
+                for (int k = 0; k < 8; ++k) mx = fmaxf(mx, v[k]);
+                mx = warp_max(mx);
+                float sm = 0.f;
+                if (mx != -INFINITY) {
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) sm += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
+                }
+                sm = warp_sum(sm);
+                if (mx != -INFINITY) A = __fadd_rn(mx, logf(sm));
+            } else {
+                float sm = 0.f;
+#pragma unroll
+                for (int k = 0; k < 8; ++k) sm += v[k];
+                sm = warp_sum(sm);
+                if (sm > 0.f) A = logf(sm);
             }
-            s = warp_sum(s);
-            if (lane == 0 && mx != -INFINITY) {
+            if (lane == 0 && A != -INFINITY) {
                 const int c = (lo >> 8) + cl;
                 const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
-                const float key = __fadd_rn(__fadd_rn(mx, logf(s)), gumbel_of(w));
-                const unsigned long long pk = pack_key(key, (uint32_t)c);
+                const unsigned long long pk = pack_key(__fadd_rn(A, gumbel_of(w)), (uint32_t)c);
                 best = pk > best ? pk : best;
             }
         }
-        reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, best);
-        if (sh.res.key == 0ull) return -1;
-        return element_argmax(node, (int)key_id(sh.res.key), lw);
-    }
-
-    // Two-level draw from non-negative weights wf(smem index, token); chunk mass = sum w.
-    template <typename WF>
-    __device__ int draw_weights(int node, WF wf) {
-        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-        const int nch = (n + kChunk - 1) / kChunk;
-        unsigned long long best = 0ull;
-        for (int cl = warp; cl < nch; cl += kWarps) {
-            const int i0 = cl * kChunk + lane * 8;
-            float s = 0.f;
+        if (lane == 0) sh.wbest[warp] = best;
+        __syncthreads();
+        if (warp == 0) {
+            unsigned long long cb = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
+            // the best token inside this CTA's best chunk
+            unsigned long long tb = 0ull;
+            if (cb != 0ull) {
+                const int i0 = (int)key_id(cb) * kChunk - lo + lane * 8, v0 = lo + i0;
+                const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
+                const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2) + 1u);
 #pragma unroll
-            for (int k = 0; k < 8; ++k)
-                if (i0 + k < n) s += wf(i0 + k, lo + i0 + k);
-            s = warp_sum(s);
-            if (lane == 0 && s > 0.f) {
-                const int c = (lo >> 8) + cl;
-                const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
-                const float key = __fadd_rn(logf(s), gumbel_of(w));
-                const unsigned long long pk = pack_key(key, (uint32_t)c);
-                best = pk > best ? pk : best;
+                for (int k = 0; k < 8; ++k) {
+                    if (i0 + k >= n) break;
+                    const float x = val(i0 + k, v0 + k);
+                    float l;
+                    if (LOGITS) {
+                        if (x == -INFINITY) continue;
+                        l = x;
+                    } else {
+                        if (!(x > 0.f)) continue;
+                        l = logf(x);
+                    }
+                    const unsigned long long pk = pack_key(__fadd_rn(l, gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4])),
+                                                           (uint32_t)(v0 + k));
+                    tb = pk > tb ? pk : tb;
+                }
+                tb = warp_max_u64(tb);
+            }
+            if (lane == 0) {
+                sh.cbest = cb;
+                sh.wbest[0] = tb;
             }
         }
-        reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, 0.0, best);
-        if (sh.res.key == 0ull) return -1;
-        auto lw = [&](int i, int v) {
-            const float w = wf(i, v);
-            return w > 0.f ? logf(w) : -INFINITY;
-        };
-        return element_argmax(node, (int)key_id(sh.res.key), lw);
+        __syncthreads();
+        Slot mine = neutral_slot();
+        if (threadIdx.x == 0 && sh.cbest != 0ull) {
+            mine.key = sh.cbest;
+            mine.tok = (int)key_id(sh.wbest[0]);
+        }
+        reduce_round<kRedArg>(sh, par, cluster, mine);
+        return sh.res.key == 0ull ? -1 : sh.res.tok;
     }
 };
 
@@ -342,7 +355,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
         if (m == 0) {  // leaf: bonus token from the node's target row
             W.stage_target(trow, nullptr);
             __syncthreads();
-            final_tok = W.draw_logits(u, [&](int i, int) { return P[i]; });
+            final_tok = W.template draw<true>(u, [&](int i, int) { return P[i]; });
             break;
         }
         const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
@@ -361,11 +374,22 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
         KahanF s2;
         if (m2 != -INFINITY)
             for (int c = crank * kThreads + threadIdx.x; c < a.C; c += CS * kThreads)
-                s2.add(st[c].y * expf(st[c].x - m2));
-        reduce_round(sh, par, cluster, lt.m, lt.s.value(), m2, s2.value(), 0.0, 0ull);
-        const float lt_hi = sh.res.hi1, lt_lo = sh.res.lo1, lq_hi = sh.res.hi2, lq_lo = sh.res.lo2;
+                s2.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m2))));
+        {
+            Slot mine = neutral_slot();
+            const MaxSum t1 = lt.value();
+            mine.m1 = t1.m;
+            mine.s1h = t1.s.hi;
+            mine.s1l = t1.s.lo;
+            const FF q2 = s2.ff();
+            mine.m2 = m2;
+            mine.s2h = q2.hi;
+            mine.s2l = q2.lo;
+            reduce_round<kRedLse>(sh, par, cluster, mine);
+        }
+        const FF L2t = sh.L2t, L2q = sh.L2q;
 
-        double t = 1.0;
+        FF t = FF{1.f, 0.f};  // draft mass not yet drawn
         int accepted = -1;
         for (int i = 0; i < m; ++i) {
             const int c = kids[o + i];
@@ -374,75 +398,85 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
                 bad = true;
                 break;
             }
-            const float t_i = (float)t;
-            const float P0y = prob_of(__fmul_rn(Logit<T>::load1(trow, y), a.invT), lt_hi, lt_lo);
-            const float Qy = prob_of(__fmul_rn(Logit<T>::load1(qrow, y), a.invT), lq_hi, lq_lo);
-            const float pp = point_residual(P0y, Qy, sh.zs, sh.ts, i);
-            const float qp = qratio(Qy, t_i);
+            const float it = t.hi > 0.f ? __frcp_rn(t.hi) : 0.f;  // 1/t_i
+            const float P0y = exp_shifted(__fmul_rn(Logit<T>::load1(trow, y), a.invT), L2t);
+            const float Qy = exp_shifted(__fmul_rn(Logit<T>::load1(qrow, y), a.invT), L2q);
+            const float pp = point_residual(P0y, Qy, sh.izs, sh.its, i);
+            const float qp = __fmul_rn(Qy, it);
             const float U = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
             if (__fmul_rn(U, qp) < pp) {
                 accepted = c;
                 break;
             }
-            // p_i(v) of the element at smem index j
-            const float zprev = i > 0 ? sh.zs[i - 1] : 1.f;
-            auto p_of = [&](int j) { return i == 0 ? prob_of(P[j], lt_hi, lt_lo) : __fdiv_rn(P[j], zprev); };
+            // p_i(v) of the element at smem index j (P holds x before the first rejection,
+            // R_i afterwards)
+            const float izp = i > 0 ? sh.izs[i - 1] : 1.f;
+            auto p_of = [&](int j) { return i == 0 ? exp_shifted(P[j], L2t) : __fmul_rn(P[j], izp); };
             if (i == m - 1) {  // every slot rejected: final token from R_m = max(p_i - Q/t_i, 0)
                 if (i == 0) {  // the q slice was never staged: stage it (normalised) now
                     for (int g = threadIdx.x; g < groups; g += kThreads) {
                         float x[8];
                         Logit<T>::load8(qrow, lo + 8 * g, a.V, x);
 #pragma unroll
-                        for (int k = 0; k < 8; ++k) Qs[8 * g + k] = prob_of(__fmul_rn(x[k], a.invT), lq_hi, lq_lo);
+                        for (int k = 0; k < 8; ++k) Qs[8 * g + k] = exp_shifted(__fmul_rn(x[k], a.invT), L2q);
                     }
                     __syncthreads();
                 }
-                final_tok = W.draw_weights(u, [&](int j, int) {
-                    return fmaxf(__fsub_rn(p_of(j), qratio(Qs[j], t_i)), 0.f);
-                });
+                final_tok = W.template draw<false>(u, [&](int j, int) { return resid(p_of(j), Qs[j], it); });
                 if (final_tok < 0) {  // no residual mass (rounding only): the node's target row
                     __syncthreads();
                     W.stage_target(trow, nullptr);
                     __syncthreads();
-                    final_tok = W.draw_logits(u, [&](int j, int) { return P[j]; });
+                    final_tok = W.template draw<true>(u, [&](int j, int) { return P[j]; });
                 }
                 break;
             }
             // residual pass (the first one also stages the normalised q slice)
             KahanF zl;
             for (int g = threadIdx.x; g < groups; g += kThreads) {
-                float xq[8];
-                if (i == 0) Logit<T>::load8(qrow, lo + 8 * g, a.V, xq);
+                float q8[8], r8[8];
+                if (i == 0) {
+                    Logit<T>::load8(qrow, lo + 8 * g, a.V, q8);
+#pragma unroll
+                    for (int k = 0; k < 8; ++k) q8[k] = exp_shifted(__fmul_rn(q8[k], a.invT), L2q);
+                    reinterpret_cast<float4 *>(Qs)[2 * g] = make_float4(q8[0], q8[1], q8[2], q8[3]);
+                    reinterpret_cast<float4 *>(Qs)[2 * g + 1] = make_float4(q8[4], q8[5], q8[6], q8[7]);
+                } else {
+                    const float4 qa = reinterpret_cast<const float4 *>(Qs)[2 * g];
+                    const float4 qb = reinterpret_cast<const float4 *>(Qs)[2 * g + 1];
+                    q8[0] = qa.x; q8[1] = qa.y; q8[2] = qa.z; q8[3] = qa.w;
+                    q8[4] = qb.x; q8[5] = qb.y; q8[6] = qb.z; q8[7] = qb.w;
+                }
+                float sum8 = 0.f;
 #pragma unroll
                 for (int k = 0; k < 8; ++k) {
-                    const int j = 8 * g + k;
-                    if (lo + j >= a.V) break;
-                    float qv;
-                    if (i == 0) {
-                        qv = prob_of(__fmul_rn(xq[k], a.invT), lq_hi, lq_lo);
-                        Qs[j] = qv;
-                    } else {
-                        qv = Qs[j];
-                    }
-                    const float rr = fmaxf(__fsub_rn(p_of(j), qratio(qv, t_i)), 0.f);
-                    P[j] = rr;
-                    zl.add(rr);
+                    r8[k] = resid(p_of(8 * g + k), q8[k], it);  // padding: p = 0 (x = -inf), q = 0
+                    sum8 += r8[k];
                 }
+                reinterpret_cast<float4 *>(P)[2 * g] = make_float4(r8[0], r8[1], r8[2], r8[3]);
+                reinterpret_cast<float4 *>(P)[2 * g + 1] = make_float4(r8[4], r8[5], r8[6], r8[7]);
+                zl.add(sum8);
             }
-            reduce_round(sh, par, cluster, -INFINITY, 0.0, -INFINITY, 0.0, zl.value(), 0ull);
-            const double Z = sh.res.z;
-            if (!(Z > 0.0)) {  // no residual mass (rounding only): the node's target row
+            {
+                Slot mine = neutral_slot();
+                const FF z = zl.ff();
+                mine.zh = z.hi;
+                mine.zl = z.lo;
+                reduce_round<kRedSum>(sh, par, cluster, mine);
+            }
+            const float Z = sh.res.zh;
+            if (!(Z > 0.f)) {  // no residual mass (rounding only): the node's target row
                 W.stage_target(trow, nullptr);
                 __syncthreads();
-                final_tok = W.draw_logits(u, [&](int j, int) { return P[j]; });
+                final_tok = W.template draw<true>(u, [&](int j, int) { return P[j]; });
                 break;
             }
             if (threadIdx.x == 0) {
-                sh.zs[i] = (float)Z;
-                sh.ts[i] = t_i;
+                sh.izs[i] = __frcp_rn(Z);
+                sh.its[i] = it;
             }
             __syncthreads();
-            t -= (double)Qy;
+            t = ff_add(t, FF{-Qy, 0.f});
         }
         if (bad || accepted < 0) break;
         if (nacc >= a.L) {  // deeper than the depth cap: the tree arrays are inconsistent
@@ -468,29 +502,93 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
 
 constexpr size_t kSmemLimit = 210 * 1024;
 
-// Cluster size and chunk-aligned slice for a vocabulary: enough CTAs to spread a row, and
-// the two fp32 slices must fit in shared memory.
-int pick_cluster(int V, int *slice_out, size_t *smem_out) {
-    int cs = V >= 32768 ? 8 : V >= 8192 ? 4 : V >= 2048 ? 2 : 1;
-    for (;;) {
-        int slice = (V + cs - 1) / cs;
-        slice = (slice + kChunk - 1) / kChunk * kChunk;
-        const size_t smem = 2 * (size_t)slice * sizeof(float);
-        if (smem <= kSmemLimit) {
-            *slice_out = slice;
-            *smem_out = smem;
-            return cs;
-        }
-        if (cs == 16) return -1;
-        cs *= 2;
+// Chunk-aligned slice of each CTA and the dynamic shared memory it needs for cluster size cs.
+void slice_for(int V, int cs, int *slice_out, size_t *smem_out) {
+    int slice = (V + cs - 1) / cs;
+    slice = (slice + kChunk - 1) / kChunk * kChunk;
+    *slice_out = slice;
+    *smem_out = 2 * (size_t)slice * sizeof(float);
+}
+
+struct ClusterChoice {
+    int V, B, elem, cs;
+};
+
+// The cluster size for (V, B): the largest size up to 16 (above 8 the cluster is
+// non-portable) whose clusters can all be resident at once, so every tree walks in the same
+// wave; when no size fits the whole batch, the size with the most concurrently resident CTAs. Decisions are
+// cached per (V, B, element size); the cache is a pure function of the device.
+template <typename T>
+int choose_cluster(int V, int B, int *slice_out, size_t *smem_out) {
+    static ClusterChoice cache[16];
+    static int cache_n = 0;
+    static std::mutex mu;
+    {
+        std::lock_guard<std::mutex> g(mu);
+        for (int i = 0; i < cache_n; ++i)
+            if (cache[i].V == V && cache[i].B == B && cache[i].elem == (int)sizeof(T)) {
+                slice_for(V, cache[i].cs, slice_out, smem_out);
+                return cache[i].cs;
+            }
     }
+    const int lo_cs = V >= 32768 ? 4 : V >= 8192 ? 4 : V >= 2048 ? 2 : 1;
+    const int hi_cs = V >= 32768 ? 16 : lo_cs;
+    int chosen = -1, best_cs = -1;
+    long best_ctas = -1;
+    for (int cs = hi_cs; cs >= 1; --cs) {
+        int slice;
+        size_t smem;
+        slice_for(V, cs, &slice, &smem);
+        if (smem > kSmemLimit) break;  // smaller clusters only need more shared memory
+        if (cs < lo_cs && chosen < 0 && best_cs > 0) break;
+        if (cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
+            cudaSuccess)
+            continue;
+        if (cs > 8 && cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                          cudaSuccess)
+            continue;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3((unsigned)(B * cs), 1, 1);
+        cfg.blockDim = dim3(kThreads, 1, 1);
+        cfg.dynamicSmemBytes = smem;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = (unsigned)cs;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        int n = 0;
+        if (cudaOccupancyMaxActiveClusters(&n, k_verify_rrs<T>, &cfg) != cudaSuccess || n <= 0) continue;
+        if (n >= B) {
+            chosen = cs;
+            break;
+        }
+        if ((long)n * cs > best_ctas) {
+            best_ctas = (long)n * cs;
+            best_cs = cs;
+        }
+    }
+    if (chosen < 0) chosen = best_cs;
+    if (chosen < 0) {  // the slices do not fit below 16 CTAs: use 16 (non-portable)
+        int slice;
+        size_t smem;
+        slice_for(V, 16, &slice, &smem);
+        chosen = smem <= kSmemLimit ? 16 : -1;
+    }
+    if (chosen > 0) {
+        std::lock_guard<std::mutex> g(mu);
+        if (cache_n < 16) cache[cache_n++] = ClusterChoice{V, B, (int)sizeof(T), chosen};
+        slice_for(V, chosen, slice_out, smem_out);
+    }
+    return chosen;
 }
 
 template <typename T>
 cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     int slice = 0;
     size_t smem = 0;
-    const int cs = pick_cluster(a.V, &slice, &smem);
+    const int cs = choose_cluster<T>(a.V, B, &slice, &smem);
     if (cs < 0) return cudaErrorInvalidValue;
     a.slice = slice;
     cudaError_t e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -123,6 +123,120 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
     return v;
 }
 
+// ---------------------------------------------------------------------------------------
+// Float-float arithmetic (an unevaluated sum hi + lo of two fp32 values) for reductions that
+// need more than fp32 accuracy without touching the slow fp64 units.
+
+struct FF {
+    float hi, lo;
+};
+
+// Knuth's TwoSum: a + b = s + e exactly; symmetric in a and b bit for bit.
+__device__ __forceinline__ void two_sum(float a, float b, float &s, float &e) {
+    s = __fadd_rn(a, b);
+    const float bb = __fsub_rn(s, a);
+    e = __fadd_rn(__fsub_rn(a, __fsub_rn(s, bb)), __fsub_rn(b, bb));
+}
+
+__device__ __forceinline__ FF ff_add(FF a, FF b) {
+    float s, e;
+    two_sum(a.hi, b.hi, s, e);
+    e = __fadd_rn(e, __fadd_rn(a.lo, b.lo));
+    const float hi = __fadd_rn(s, e);
+    return FF{hi, __fsub_rn(e, __fsub_rn(hi, s))};
+}
+
+// a * f for f >= 0 (the product's rounding error is kept through an fma)
+__device__ __forceinline__ FF ff_scale(FF a, float f) {
+    const float p = __fmul_rn(a.hi, f);
+    const float err = __fmaf_rn(a.hi, f, -p);
+    const float lo = __fmaf_rn(a.lo, f, err);
+    const float hi = __fadd_rn(p, lo);
+    return FF{hi, __fsub_rn(lo, __fsub_rn(hi, p))};
+}
+
+__device__ __forceinline__ FF ff_shfl_xor(FF v, int o) {
+    return FF{__shfl_xor_sync(kFull, v.hi, o), __shfl_xor_sync(kFull, v.lo, o)};
+}
+
+__device__ __forceinline__ FF warp_sum_ff(FF v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = ff_add(v, ff_shfl_xor(v, o));
+    return v;
+}
+
+// A partial softmax normaliser: S = sum exp(x - m) over some set of logits.
+struct MaxSum {
+    float m;
+    FF s;
+};
+
+// Merge of two partial normalisers (symmetric bit for bit, so butterflies agree in all lanes).
+__device__ __forceinline__ MaxSum maxsum_merge(MaxSum a, MaxSum b) {
+    const float M = fmaxf(a.m, b.m);
+    if (M == -INFINITY) return MaxSum{M, FF{0.f, 0.f}};
+    const FF ta = a.m == -INFINITY ? FF{0.f, 0.f} : ff_scale(a.s, expf(__fsub_rn(a.m, M)));
+    const FF tb = b.m == -INFINITY ? FF{0.f, 0.f} : ff_scale(b.s, expf(__fsub_rn(b.m, M)));
+    return MaxSum{M, ff_add(ta, tb)};
+}
+
+__device__ __forceinline__ MaxSum warp_maxsum(MaxSum v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        MaxSum w{__shfl_xor_sync(kFull, v.m, o), ff_shfl_xor(v.s, o)};
+        v = maxsum_merge(v, w);
+    }
+    return v;
+}
+
+// log(S.hi + S.lo) for S > 0 as float-float, absolute error about 1e-7 at any magnitude:
+// S = f 2^k with f in [1, 2); log S = k ln2 + log f + S.lo/S.hi. ln 2 is split Cody-Waite
+// style into a head with 12 trailing zero bits (so k * head is exact) and a tail; logf is
+// only evaluated on [1, 2), where its result is below 0.7.
+__device__ __forceinline__ FF ff_log(FF S) {
+    constexpr float kLn2Head = 0.693145751953125f;        // 0x3F317200
+    constexpr float kLn2Tail = 1.4286068203094173e-06f;   // ln 2 - head
+    int e;
+    const float f = __fmul_rn(frexpf(S.hi, &e), 2.0f);
+    const float k = (float)(e - 1);
+    const float head = __fmul_rn(k, kLn2Head);
+    const float tail = __fadd_rn(__fmaf_rn(k, kLn2Tail, logf(f)), __fdiv_rn(S.lo, S.hi));
+    float s, err;
+    two_sum(head, tail, s, err);
+    return FF{s, err};
+}
+
+// log2(e) as a head (fp32 rounding) and a tail, so x * log2(e) is carried to ~2^-46.
+constexpr float kLog2eHi = 1.44269502162933349609375f;
+constexpr float kLog2eLo = 1.925963033500011e-08f;
+
+// (L.hi + L.lo) * log2(e) as float-float.
+__device__ __forceinline__ FF ff_times_log2e(FF L) {
+    const float hi = __fmul_rn(L.hi, kLog2eHi);
+    const float err = __fmaf_rn(L.hi, kLog2eHi, -hi);
+    const float lo = __fadd_rn(err, __fmaf_rn(L.hi, kLog2eLo, __fmul_rn(L.lo, kLog2eHi)));
+    const float h2 = __fadd_rn(hi, lo);
+    return FF{h2, __fsub_rn(lo, __fsub_rn(h2, hi))};
+}
+
+// e^(x - L) with L2 = L * log2(e) in float-float: the exponent x log2(e) - L2 is formed with
+// two fmas (exact products, one rounding each), then ex2. Relative error about
+// |x - L| 2^-24 + the ex2 approximation's few ulp; used identically wherever the same
+// probability must come out bit for bit (element passes and point values).
+__device__ __forceinline__ float exp_shifted(float x, FF L2) {
+    const float a = __fmaf_rn(x, kLog2eHi, -L2.hi);
+    const float b = __fmaf_rn(x, kLog2eLo, -L2.lo);
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(__fadd_rn(a, b)));
+    return y;
+}
+
+// m + log(S) of a normaliser as float-float (the row log-sum-exp).
+__device__ __forceinline__ FF maxsum_lse(MaxSum v) {
+    const FF l = ff_log(v.s);
+    return ff_add(FF{v.m, 0.f}, l);
+}
+
 // Compensated (Neumaier) accumulation in fp32.
 struct KahanF {
     float s = 0.f, c = 0.f;
@@ -135,7 +249,17 @@ struct KahanF {
         s = t;
     }
     __device__ __forceinline__ double value() const { return (double)s + (double)c; }
+    __device__ __forceinline__ FF ff() const {
+        const float hi = __fadd_rn(s, c);
+        return FF{hi, __fsub_rn(c, __fsub_rn(hi, s))};
+    }
 };
+
+// Order-preserving image of an fp64 value as u64 ("larger u64" = larger value; -0 == +0).
+__device__ __forceinline__ unsigned long long ord_f64(double d) {
+    const unsigned long long u = (unsigned long long)__double_as_longlong(d + 0.0);
+    return (u >> 63) ? ~u : (u | 0x8000000000000000ull);
+}
 
 // ---------------------------------------------------------------------------------------
 // Per-lane list of the CAP largest packed keys, kept sorted descending in registers.

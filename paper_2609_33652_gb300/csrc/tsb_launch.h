@@ -25,18 +25,18 @@ inline int num_chunks(int V) { return (V + 255) / 256; }
 // Workspace layout (caller-owned, 256-byte aligned):
 //   [0, 256)                       sticky status word
 //   B*(N+1) x 32 bytes             per-(tree, chain position) scalars of block verification
-//   B*L doubles, B*L*K floats,     per-draft-row log-normaliser and top-K (x, id) of the
-//   B*L*K int32                    first pass
+//   B*L float2, B*L*K floats,      per-draft-row log-normaliser (float-float) and top-K
+//   B*L*K int32                    (x, id) of the first pass
 constexpr size_t kWsStatusBytes = 256;
 constexpr size_t kWsBvRowBytes = 32;
 
 inline size_t workspace_bytes(int B, int N, int L, int K) {
-    return kWsStatusBytes + (size_t)B * ((size_t)N + 1) * kWsBvRowBytes + (size_t)B * L * sizeof(double) +
+    return kWsStatusBytes + (size_t)B * ((size_t)N + 1) * kWsBvRowBytes + (size_t)B * L * 2 * sizeof(float) +
            (size_t)B * L * K * (sizeof(float) + sizeof(int32_t));
 }
 
 struct PlanScratch {
-    double *lse;
+    float2 *lse;
     float *topk_x;
     int32_t *topk_id;
 };
