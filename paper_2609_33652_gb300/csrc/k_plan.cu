@@ -7,10 +7,9 @@
 //   >= tau go through per-lane sorted lists, and a warp merge yields the top-K by
 //   (x desc, id asc). Results go to the workspace.
 // k_plan_heap, one CTA per tree: best-first expansion, popping N candidates. A candidate at
-//   depth d holds the float-float sum Sx of its path's logits and the key Sx - CL[d],
-//   CL[d] = LSE_1 + ... + LSE_d (its draft path log-probability). Pop order: (key desc,
-//   depth asc, parent asc, rank asc), compared as integers (order-preserving image of the
-//   float-float key; no fp64 anywhere). Popping (p, r) at depth d
+//   depth d holds the sum Sx of its path's logits (exact, in 64-bit fixed point) and the key
+//   Sx - CL[d], CL[d] = LSE_1 + ... + LSE_d (its draft path log-probability). Pop order:
+//   (key desc, depth asc, parent asc, rank asc), compared as integers. Popping (p, r) at depth d
 //   pushes the next sibling (p, r+1) and, below the depth cap, the first child (i, 0).
 //   Siblings are popped in rank order, so the children of u occupy
 //   child_ids[child_off[u] + rank] directly.
@@ -80,11 +79,7 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_row_topk(TopkArgs a) {
         cl.clear();
         for (int c = lane; c < C; c += 32) cl.insert(pack_key(st[c].x, (uint32_t)c));
         uint64_t kth = 0;
-        for (int j = 0; j < K; ++j) {
-            const uint64_t best = warp_max_u64(cl.k[0]);
-            kth = best;
-            if (cl.k[0] == best) cl.pop_front();
-        }
+        for (int j = 0; j < K; ++j) kth = warp_pop_max(cl);
         tau = key_value(kth);
     }
     // top-K logits among the chunks whose maximum reaches tau, four chunks per batch
@@ -124,12 +119,11 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_row_topk(TopkArgs a) {
         }
     }
     for (int j = 0; j < K; ++j) {
-        const uint64_t best = warp_max_u64(el.k[0]);
+        const uint64_t best = warp_pop_max(el);
         if (lane == 0) {
             a.topk_id[(int64_t)row * K + j] = (int32_t)key_id(best);
             a.topk_x[(int64_t)row * K + j] = key_value(best);
         }
-        if (el.k[0] == best) el.pop_front();
     }
 }
 
@@ -142,23 +136,29 @@ struct HeapArgs {
     uint32_t *status;
 };
 
-// A frontier candidate is a 96-bit integer key, larger = pops first:
-//   okey = order-preserving image of the float-float key (Sx - CL[depth]), high word from
-//          its head, low word from its tail;
+// Path sums are kept in 64-bit fixed point with 2^-30 resolution: a logit x converts exactly
+// when |x| >= 2^-7 (its fp32 ulp is then a multiple of 2^-30), and sums stay exact up to
+// |Sx| < 2^33, so equal real path sums give equal integers and the expansion needs only
+// integer additions. The key of a candidate at depth d is Sx - CL[d], CL[d] rounded to the
+// same grid once per depth.
+// A frontier candidate is a 96-bit integer, larger = pops first:
+//   okey = key with its sign bit flipped (order-preserving as unsigned);
 //   w3   = (255 - depth) << 24 | (65535 - parent) << 8 | (255 - rank)
 // so the order is (key desc, depth asc, parent asc, rank asc); an empty slot is (0, 0).
-// Path sums Sx are float-float sums of fp32 logits (TwoSum additions: exact while the
-// logits of a path span fewer than ~24 binades), so equal sums give equal keys bit for bit.
+constexpr float kFixScale = 1073741824.0f;  // 2^30
+constexpr float kFixInv = 9.313225746154785e-10f;  // 2^-30
+
 __device__ __forceinline__ unsigned w3_of(int depth, int parent, int rank) {
     return ((unsigned)(255 - depth) << 24) | ((unsigned)(65535 - parent) << 8) | (unsigned)(255 - rank);
 }
 __device__ __forceinline__ bool key_better(unsigned long long ka, unsigned wa, unsigned long long kb, unsigned wb) {
     return ka > kb || (ka == kb && wa > wb);
 }
-__device__ __forceinline__ unsigned long long ord_ff(FF v) {
-    return ((unsigned long long)ord_f32(v.hi) << 32) | (unsigned long long)ord_f32(v.lo);
+__device__ __forceinline__ unsigned long long okey_of(long long key) {
+    return (unsigned long long)key ^ 0x8000000000000000ull;
 }
-__device__ __forceinline__ FF ff_neg(FF v) { return FF{-v.hi, -v.lo}; }
+__device__ __forceinline__ long long key_of_okey(unsigned long long o) { return (long long)(o ^ 0x8000000000000000ull); }
+__device__ __forceinline__ long long fix_of(float x) { return __float2ll_rn(__fmul_rn(x, kFixScale)); }
 
 template <int S>
 struct Slots {
@@ -207,22 +207,22 @@ template <int S>
 __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int L = a.L, N = a.N, K = a.K, NN = N + 1;
-    FF *CL = reinterpret_cast<FF *>(smem);                         // [L+1]
-    FF *n_sx = CL + (L + 1);                                       // [NN] node path sums
-    int32_t *n_parent = reinterpret_cast<int32_t *>(n_sx + NN);    // [NN]
+    long long *CL = reinterpret_cast<long long *>(smem);           // [L+1] fixed point
+    long long *n_sx = CL + (L + 1);                                // [NN] node path sums
+    long long *fx = n_sx + NN;                                     // [L*K] candidate logits
+    int32_t *n_parent = reinterpret_cast<int32_t *>(fx + L * K);   // [NN]
     int32_t *n_depth = n_parent + NN;
     int32_t *n_rank = n_depth + NN;
     int32_t *n_token = n_rank + NN;
     int32_t *n_count = n_token + NN;                               // [NN]
     float *n_score = reinterpret_cast<float *>(n_count + NN);      // [NN]
     int32_t *tk_id = reinterpret_cast<int32_t *>(n_score + NN);    // [L*K]
-    float *tk_x = reinterpret_cast<float *>(tk_id + L * K);        // [L*K]
 
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     for (int i = threadIdx.x; i < L * K; i += kHeapThreads) {
         tk_id[i] = a.topk_id[(int64_t)b * L * K + i];
-        tk_x[i] = a.topk_x[(int64_t)b * L * K + i];
+        fx[i] = fix_of(a.topk_x[(int64_t)b * L * K + i]);
     }
     for (int i = threadIdx.x; i < NN; i += kHeapThreads) {  // defined even if the expansion stops early
         n_count[i] = 0;
@@ -231,22 +231,26 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
         n_rank[i] = 0;
         n_token[i] = -1;
         n_score[i] = 0.f;
-        n_sx[i] = FF{0.f, 0.f};
+        n_sx[i] = 0;
     }
-    if (warp == 0) {  // CL[d] = LSE_1 + ... + LSE_d (loads in parallel, sum in order)
+    if (warp == 0) {  // CL[d] = LSE_1 + ... + LSE_d in float-float, then onto the fixed grid
+        FF l0 = FF{0.f, 0.f}, l1 = FF{0.f, 0.f};
         if (lane < L) {
-            const float2 l = a.lse[(int64_t)b * L + lane];
-            CL[lane + 1] = FF{l.x, l.y};
+            const float2 v = a.lse[(int64_t)b * L + lane];
+            l0 = FF{v.x, v.y};
         }
         if (lane + 32 < L) {
-            const float2 l = a.lse[(int64_t)b * L + lane + 32];
-            CL[lane + 33] = FF{l.x, l.y};
+            const float2 v = a.lse[(int64_t)b * L + lane + 32];
+            l1 = FF{v.x, v.y};
         }
-        __syncwarp();
-        if (lane == 0) {
-            CL[0] = FF{0.f, 0.f};
-            for (int d = 1; d <= L; ++d) CL[d] = ff_add(CL[d - 1], CL[d]);
+        FF acc = FF{0.f, 0.f};
+        for (int d = 0; d < L; ++d) {  // prefix sums in depth order (every lane, same values)
+            const FF l = d < 32 ? FF{__shfl_sync(kFull, l0.hi, d), __shfl_sync(kFull, l0.lo, d)}
+                                : FF{__shfl_sync(kFull, l1.hi, d - 32), __shfl_sync(kFull, l1.lo, d - 32)};
+            acc = ff_add(acc, l);
+            if (lane == 0) CL[d + 1] = fix_of(acc.hi) + fix_of(acc.lo);
         }
+        if (lane == 0) CL[0] = 0;
     }
     __syncthreads();
 
@@ -260,40 +264,46 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
         Slots<S> fr;
         fr.clear();
         if (lane == 0) {  // the root's first child (depth 1, rank 0) is child number 0
-            const FF sx = ff_add(FF{0.f, 0.f}, FF{tk_x[0], 0.f});
-            fr.put(0, ord_ff(ff_add(sx, ff_neg(CL[1]))), w3_of(1, 0, 0));
+            fr.put(0, okey_of(fx[0] - CL[1]), w3_of(1, 0, 0));
             fr.rescan();
         }
         int nchild = 1;
         __syncwarp();
         for (int i = 1; i <= N; ++i) {
-            const unsigned hk = (unsigned)(fr.bk >> 32), lk = (unsigned)fr.bk;
+            const unsigned hk = (unsigned)(fr.bk >> 32);
             const unsigned m1 = __reduce_max_sync(kFull, hk);
             unsigned c = __ballot_sync(kFull, hk == m1);
-            const unsigned m2 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? lk : 0u);
-            c &= __ballot_sync(kFull, lk == m2);
-            const unsigned m3 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? fr.bw : 0u);
-            c &= __ballot_sync(kFull, fr.bw == m3);
-            if (m3 == 0u) {  // frontier exhausted: only with N above the tree's capacity
+            if (__popc(c) > 1) {  // the high word ties: resolve with the low word, then w3
+                const unsigned lk = (unsigned)fr.bk;
+                const unsigned m2 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? lk : 0u);
+                c &= __ballot_sync(kFull, lk == m2);
+                if (__popc(c) > 1) {
+                    const unsigned m3 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? fr.bw : 0u);
+                    c &= __ballot_sync(kFull, fr.bw == m3);
+                }
+            }
+            const int winner = __ffs(c) - 1;
+            const unsigned long long wk = __shfl_sync(kFull, fr.bk, winner);
+            const unsigned ww = __shfl_sync(kFull, fr.bw, winner);
+            if (ww == 0u) {  // frontier exhausted: only with N above the tree's capacity
                 if (lane == 0) raise_status(a.status, kDevBadTree);
                 break;
             }
-            const int winner = __ffs(c) - 1;
-            const int depth = 255 - (int)(m3 >> 24);
-            const int parent = 65535 - (int)((m3 >> 8) & 0xffffu);
-            const int rank = 255 - (int)(m3 & 0xffu);
-            FF sx = FF{0.f, 0.f};
-            if (lane == winner) {
-                // the popped path's sum, recomputed with the same additions as at creation
-                const FF sp = n_sx[parent];
-                sx = ff_add(sp, FF{tk_x[(depth - 1) * K + rank], 0.f});
-                n_sx[i] = sx;
-                if (rank + 1 < K) {  // the next sibling takes the freed slot
-                    const FF ss = ff_add(sp, FF{tk_x[(depth - 1) * K + rank + 1], 0.f});
-                    fr.put(fr.bs, ord_ff(ff_add(ss, ff_neg(CL[depth]))), w3_of(depth, parent, rank + 1));
-                } else {
+            const int depth = 255 - (int)(ww >> 24);
+            const int parent = 65535 - (int)((ww >> 8) & 0xffffu);
+            const int rank = 255 - (int)(ww & 0xffu);
+            const bool sib = rank + 1 < K, kid = depth < L;
+            // every lane computes the popped path's sum and both new keys from broadcast loads;
+            // only the commits below differ per lane
+            const long long sp = n_sx[parent];
+            const long long sx = sp + fx[(depth - 1) * K + rank];
+            const long long ks = sp + (sib ? fx[(depth - 1) * K + rank + 1] : 0) - CL[depth];
+            const long long kc = sx + (kid ? fx[depth * K] : 0) - CL[kid ? depth + 1 : depth];
+            if (lane == winner) {  // the next sibling takes the freed slot
+                if (sib)
+                    fr.put(fr.bs, okey_of(ks), w3_of(depth, parent, rank + 1));
+                else
                     fr.put(fr.bs, 0ull, 0u);
-                }
                 fr.rescan();
             }
             if (lane == 0) {
@@ -301,14 +311,12 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
                 n_depth[i] = depth;
                 n_rank[i] = rank;
                 n_token[i] = tk_id[(depth - 1) * K + rank];
-                n_score[i] = f32_of_ord(m1);
+                n_score[i] = __fmul_rn(__ll2float_rn(key_of_okey(wk)), kFixInv);
+                n_sx[i] = sx;
             }
-            if (depth < L) {  // first child (i, 0), one level down
-                sx.hi = __shfl_sync(kFull, sx.hi, winner);
-                sx.lo = __shfl_sync(kFull, sx.lo, winner);
+            if (kid) {  // first child (i, 0), one level down, in the next round-robin slot
                 if (lane == (nchild & 31)) {
-                    const FF sc = ff_add(sx, FF{tk_x[depth * K + 0], 0.f});
-                    const unsigned long long ck = ord_ff(ff_add(sc, ff_neg(CL[depth + 1])));
+                    const unsigned long long ck = okey_of(kc);
                     const unsigned cw = w3_of(depth + 1, i, 0);
                     fr.put(nchild >> 5, ck, cw);
                     if (key_better(ck, cw, fr.bk, fr.bw)) {
@@ -365,7 +373,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
 
 size_t heap_smem_bytes(int L, int N, int K) {
     const size_t NN = (size_t)N + 1;
-    return (size_t)(L + 1) * sizeof(FF) + NN * sizeof(FF) + 6 * NN * 4 + 2 * (size_t)L * K * 4;
+    return (size_t)(L + 1) * 8 + NN * 8 + (size_t)L * K * 8 + 6 * NN * 4 + (size_t)L * K * 4;
 }
 
 template <int S>

@@ -51,9 +51,8 @@ template <int CAP>
 __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t *dst) {
     const int lane = threadIdx.x & 31;
     for (int j = 0; j < n; ++j) {
-        const uint64_t best = warp_max_u64(list.k[0]);
+        const uint64_t best = warp_pop_max(list);
         if (lane == 0) dst[j] = best;
-        if (best != 0ull && list.k[0] == best) list.pop_front();
     }
 }
 

@@ -20,55 +20,6 @@ constexpr int kWarps = 8;
 constexpr int kPerWarp = 8;  // chunks per warp group
 
 template <typename T>
-struct Raw;  // 8 consecutive logits as raw 16-byte words
-template <>
-struct Raw<__nv_bfloat16> {
-    uint4 w;
-    __device__ __forceinline__ void load(const __nv_bfloat16 *row, int v0, int V) {
-        if (v0 + 8 <= V) {
-            w = __ldg(reinterpret_cast<const uint4 *>(row + v0));
-        } else {  // ragged tail: missing logits become -inf (0xff80)
-            const unsigned short *r = reinterpret_cast<const unsigned short *>(row);
-            unsigned short h[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) h[i] = (v0 + i < V) ? __ldg(r + v0 + i) : (unsigned short)0xff80u;
-            w.x = h[0] | ((uint32_t)h[1] << 16);
-            w.y = h[2] | ((uint32_t)h[3] << 16);
-            w.z = h[4] | ((uint32_t)h[5] << 16);
-            w.w = h[6] | ((uint32_t)h[7] << 16);
-        }
-    }
-    __device__ __forceinline__ void unpack(float z[8]) const {
-        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            z[2 * i] = __uint_as_float(u[i] << 16);
-            z[2 * i + 1] = __uint_as_float(u[i] & 0xffff0000u);
-        }
-    }
-};
-template <>
-struct Raw<float> {
-    float4 a, b;
-    __device__ __forceinline__ void load(const float *row, int v0, int V) {
-        if (v0 + 8 <= V) {
-            a = __ldg(reinterpret_cast<const float4 *>(row + v0));
-            b = __ldg(reinterpret_cast<const float4 *>(row + v0 + 4));
-        } else {
-            float z[8];
-#pragma unroll
-            for (int i = 0; i < 8; ++i) z[i] = (v0 + i < V) ? __ldg(row + v0 + i) : -INFINITY;
-            a = make_float4(z[0], z[1], z[2], z[3]);
-            b = make_float4(z[4], z[5], z[6], z[7]);
-        }
-    }
-    __device__ __forceinline__ void unpack(float z[8]) const {
-        z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w;
-        z[4] = b.x; z[5] = b.y; z[6] = b.z; z[7] = b.w;
-    }
-};
-
-template <typename T>
 __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__ data, int R, int V,
                                                            int64_t bstride, int64_t rstride, int C,
                                                            int64_t groups_total, float invT,
@@ -86,7 +37,7 @@ __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__
         const T *rp = data + (int64_t)b * bstride + (int64_t)r * rstride;
         const int c0 = g * kPerWarp;
         const int nc = min(kPerWarp, C - c0);
-        Raw<T> raw[kPerWarp];
+        RawGroup<T> raw[kPerWarp];
 #pragma unroll
         for (int k = 0; k < kPerWarp; ++k)
             if (k < nc) raw[k].load(rp, (c0 + k) * kChunk + lane * 8, V);

@@ -73,20 +73,10 @@ __device__ __forceinline__ Slot neutral_slot() {
     return s;
 }
 
-// Symmetric merge of the fields a reduction of this kind carries.
+// Symmetric merge of the plain-sum and argmax fields (normalisers are reduced separately).
 template <int KIND>
 __device__ __forceinline__ Slot merge_slot(const Slot &a, const Slot &b) {
     Slot r = a;
-    if (KIND & kRedLse) {
-        const MaxSum x = maxsum_merge(MaxSum{a.m1, FF{a.s1h, a.s1l}}, MaxSum{b.m1, FF{b.s1h, b.s1l}});
-        const MaxSum y = maxsum_merge(MaxSum{a.m2, FF{a.s2h, a.s2l}}, MaxSum{b.m2, FF{b.s2h, b.s2l}});
-        r.m1 = x.m;
-        r.s1h = x.s.hi;
-        r.s1l = x.s.lo;
-        r.m2 = y.m;
-        r.s2h = y.s.hi;
-        r.s2l = y.s.lo;
-    }
     if (KIND & kRedSum) {
         const FF z = ff_add(FF{a.zh, a.zl}, FF{b.zh, b.zl});
         r.zh = z.hi;
@@ -101,19 +91,27 @@ __device__ __forceinline__ Slot merge_slot(const Slot &a, const Slot &b) {
     return r;
 }
 
+// A normaliser rescaled to a larger reference maximum M (exp evaluated once).
+__device__ __forceinline__ FF rescale_to(float m, FF s, float M) {
+    return m == -INFINITY ? FF{0.f, 0.f} : (m == M ? s : ff_scale(s, expf(__fsub_rn(m, M))));
+}
+
 template <int KIND>
 __device__ __forceinline__ Slot warp_reduce_slot(Slot v) {
+    if (KIND & kRedLse) {  // maxima first, then every lane rescales once, then plain sums
+        const float M1 = warp_max(v.m1), M2 = warp_max(v.m2);
+        const FF a = warp_sum_ff(rescale_to(v.m1, FF{v.s1h, v.s1l}, M1));
+        const FF c = warp_sum_ff(rescale_to(v.m2, FF{v.s2h, v.s2l}, M2));
+        v.m1 = M1;
+        v.s1h = a.hi;
+        v.s1l = a.lo;
+        v.m2 = M2;
+        v.s2h = c.hi;
+        v.s2l = c.lo;
+    }
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         Slot w = v;
-        if (KIND & kRedLse) {
-            w.m1 = __shfl_xor_sync(kFull, v.m1, o);
-            w.s1h = __shfl_xor_sync(kFull, v.s1h, o);
-            w.s1l = __shfl_xor_sync(kFull, v.s1l, o);
-            w.m2 = __shfl_xor_sync(kFull, v.m2, o);
-            w.s2h = __shfl_xor_sync(kFull, v.s2h, o);
-            w.s2l = __shfl_xor_sync(kFull, v.s2l, o);
-        }
         if (KIND & kRedSum) {
             w.zh = __shfl_xor_sync(kFull, v.zh, o);
             w.zl = __shfl_xor_sync(kFull, v.zl, o);
@@ -218,16 +216,40 @@ struct Walk {
 
     // Stage x = fp32(z) * invT of this CTA's target slice into P; optionally accumulate the
     // target row's log-normaliser.
+    // Stage x = fp32(z) * invT of this CTA's target slice into P; optionally accumulate the
+    // target row's log-normaliser. Loads are issued in batches of kBatch groups per thread
+    // before any is used, so a slice costs one memory round trip per batch.
+    static constexpr int kBatch = sizeof(T) == 2 ? 6 : 3;
     __device__ void stage_target(const T *row, OnlineLse *lse) {
-        for (int g = threadIdx.x; g < groups(); g += kThreads) {
-            float x[8];
-            Logit<T>::load8(row, lo + 8 * g, a.V, x);
+        const int G = groups();
+        for (int g0 = threadIdx.x; g0 < G; g0 += kBatch * kThreads) {
+            RawGroup<T> raw[kBatch];
 #pragma unroll
-            for (int k = 0; k < 8; ++k) x[k] = (lo + 8 * g + k < a.V) ? __fmul_rn(x[k], a.invT) : -INFINITY;
-            reinterpret_cast<float4 *>(P)[2 * g] = make_float4(x[0], x[1], x[2], x[3]);
-            reinterpret_cast<float4 *>(P)[2 * g + 1] = make_float4(x[4], x[5], x[6], x[7]);
-            if (lse) lse->add8(x);
+            for (int e = 0; e < kBatch; ++e) {
+                const int g = g0 + e * kThreads;
+                if (g < G) raw[e].load(row, lo + 8 * g, a.V);
+            }
+#pragma unroll
+            for (int e = 0; e < kBatch; ++e) {
+                const int g = g0 + e * kThreads;
+                if (g >= G) break;
+                float x[8];
+                raw[e].unpack(x);
+#pragma unroll
+                for (int k = 0; k < 8; ++k) x[k] = __fmul_rn(x[k], a.invT);  // padding stays -inf
+                reinterpret_cast<float4 *>(P)[2 * g] = make_float4(x[0], x[1], x[2], x[3]);
+                reinterpret_cast<float4 *>(P)[2 * g + 1] = make_float4(x[4], x[5], x[6], x[7]);
+                if (lse) lse->add8(x);
+            }
         }
+    }
+
+    // Ask L2 for this CTA's slice of a row that is likely needed soon (one request per 128 B).
+    __device__ void prefetch_slice(const T *row) {
+        const char *base = reinterpret_cast<const char *>(row + lo);
+        const int bytes = n * (int)sizeof(T);
+        for (int off = threadIdx.x * 128; off < bytes; off += kThreads * 128)
+            asm volatile("prefetch.global.L2 [%0];" ::"l"(base + off));
     }
 
     // Two-level draw (chunk by Gumbel-max over chunk masses, then token by Gumbel-max inside
@@ -364,6 +386,13 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             break;
         }
         const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
+        {  // likely next reads: this node's q row (first rejection), the first child's target row
+            W.prefetch_slice(qrow);
+            const int c0 = kids[o];
+            if (c0 >= 1 && c0 <= a.N)
+                W.prefetch_slice(static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride +
+                                 (int64_t)c0 * a.t_rstride);
+        }
 
         // staging pass with the target log-normaliser; q row log-normaliser from its chunk stats
         OnlineLse lt;

@@ -288,15 +288,30 @@ struct TopList {
     }
 };
 
-// Merge the lanes' lists: out[j] (j < n) = j-th largest key over the warp (0 if fewer keys).
-// Every lane receives every key; n <= CAP. Keys must be distinct (they carry their id).
-template <int CAP>
-__device__ __forceinline__ void warp_merge_top(TopList<CAP> &list, int n, uint64_t *out) {
-    for (int j = 0; j < n; ++j) {
-        const uint64_t best = warp_max_u64(list.k[0]);
-        out[j] = best;
-        if (best != 0ull && list.k[0] == best) list.pop_front();
+// The largest of the lanes' 64-bit values (distinct unless zero): a hardware max over the
+// high words, then over the low words only among the lanes that tie. Returns the value to
+// every lane and the lane that holds it in *owner.
+__device__ __forceinline__ uint64_t warp_max_u64_owner(uint64_t v, int *owner) {
+    const int lane = threadIdx.x & 31;
+    const unsigned hi = (unsigned)(v >> 32);
+    const unsigned m1 = __reduce_max_sync(kFull, hi);
+    unsigned c = __ballot_sync(kFull, hi == m1);
+    if (__popc(c) > 1) {
+        const unsigned lo = (unsigned)v;
+        const unsigned m2 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? lo : 0u);
+        c &= __ballot_sync(kFull, lo == m2);
     }
+    *owner = __ffs(c) - 1;
+    return __shfl_sync(kFull, v, *owner);
+}
+
+// Take the warp's largest key out of the lanes' lists (0 when all lists are empty).
+template <int CAP>
+__device__ __forceinline__ uint64_t warp_pop_max(TopList<CAP> &list) {
+    int owner;
+    const uint64_t best = warp_max_u64_owner(list.k[0], &owner);
+    if ((threadIdx.x & 31) == owner && best != 0ull) list.pop_front();
+    return best;
 }
 
 // ---------------------------------------------------------------------------------------
@@ -342,6 +357,55 @@ struct Logit<__nv_bfloat16> {
     }
     __device__ __forceinline__ static float load1(const __nv_bfloat16 *row, int v) {
         return bf16_bits_to_f32(__ldg(reinterpret_cast<const unsigned short *>(row) + v));
+    }
+};
+
+template <typename T>
+struct RawGroup;  // 8 consecutive logits as raw 16-byte words (loaded now, unpacked later)
+template <>
+struct RawGroup<__nv_bfloat16> {
+    uint4 w;
+    __device__ __forceinline__ void load(const __nv_bfloat16 *row, int v0, int V) {
+        if (v0 + 8 <= V) {
+            w = __ldg(reinterpret_cast<const uint4 *>(row + v0));
+        } else {  // ragged tail: missing logits become -inf (0xff80)
+            const unsigned short *r = reinterpret_cast<const unsigned short *>(row);
+            unsigned short h[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) h[i] = (v0 + i < V) ? __ldg(r + v0 + i) : (unsigned short)0xff80u;
+            w.x = h[0] | ((uint32_t)h[1] << 16);
+            w.y = h[2] | ((uint32_t)h[3] << 16);
+            w.z = h[4] | ((uint32_t)h[5] << 16);
+            w.w = h[6] | ((uint32_t)h[7] << 16);
+        }
+    }
+    __device__ __forceinline__ void unpack(float z[8]) const {
+        const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            z[2 * i] = __uint_as_float(u[i] << 16);
+            z[2 * i + 1] = __uint_as_float(u[i] & 0xffff0000u);
+        }
+    }
+};
+template <>
+struct RawGroup<float> {
+    float4 a, b;
+    __device__ __forceinline__ void load(const float *row, int v0, int V) {
+        if (v0 + 8 <= V) {
+            a = __ldg(reinterpret_cast<const float4 *>(row + v0));
+            b = __ldg(reinterpret_cast<const float4 *>(row + v0 + 4));
+        } else {
+            float z[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) z[i] = (v0 + i < V) ? __ldg(row + v0 + i) : -INFINITY;
+            a = make_float4(z[0], z[1], z[2], z[3]);
+            b = make_float4(z[4], z[5], z[6], z[7]);
+        }
+    }
+    __device__ __forceinline__ void unpack(float z[8]) const {
+        z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w;
+        z[4] = b.x; z[5] = b.y; z[6] = b.z; z[7] = b.w;
     }
 };
 
