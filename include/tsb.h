@@ -22,7 +22,8 @@
  *     caller-supplied array) set bits in a sticky status word kept in the caller's workspace;
  *     tsb_device_status reads and clears it. Outputs of a call that set a bit are undefined.
  *   - Functions keep no global state and are safe to call from several host threads on
- *     different workspaces.
+ *     different workspaces. The one exception is tsb_plan_noalloc, whose scratch is a
+ *     static device array (see there).
  *   - Logits: element (b, r, v) is at data[b*batch_stride + r*row_stride + v], in elements.
  *     batch_stride may be 0 (every tree shares the same rows). Every row must start on a
  *     16-byte boundary (data, batch_stride*elem_size and row_stride*elem_size multiples of 16).
@@ -145,6 +146,37 @@ tsb_status tsb_row_stats(const tsb_logits *rows, float temperature, void *stats,
  * and temperature. Writes every array of *out. */
 tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats, size_t stats_bytes,
                     const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
+
+/* Size of the device scratch array behind tsb_plan_noalloc (1 MiB per device). */
+#define TSB_NOALLOC_SCRATCH_BYTES ((size_t)1 << 20)
+
+/* tsb_plan without a workspace and without any allocation. The paper has no counterpart:
+ * this is a calling convention, not a step of the method. It is for callers that cannot
+ * call cudaMalloc: a plug-in whose host program owns all device memory and hands it only
+ * its input and output tensors; a serving engine that reserves the device's memory up
+ * front for its own pool; a hot loop that cannot pay cudaMalloc's implicit device-wide
+ * synchronisation. It computes exactly what tsb_plan computes, with the same kernels,
+ * and writes the same *out.
+ *
+ * Scratch: a single static device array of TSB_NOALLOC_SCRATCH_BYTES that every device
+ * loading this library holds until the process exits. A configuration needs
+ * 256 + B*L*(8 + 8*K) bytes of it; larger ones return TSB_ERR_SHAPE before anything is
+ * launched (for example B <= 910 trees at L = 16, K = 8). All calls on a device share the
+ * array and it keeps the last call's contents, so calls whose kernels may overlap on the
+ * GPU (different streams, or different host threads, without ordering between them) race
+ * and give undefined outputs: order them on one stream or with events.
+ *
+ * Set-up: the first call on each device (with that device current) looks up the array's
+ * device address and caches it; make that first call before any stream capture on the
+ * device. The call allocates and frees nothing and calls no allocating library routine.
+ *
+ * dev_status: optional 4-byte aligned device word, owned by the caller, into which the
+ * device status bits (TSB_DEV_*) are OR-ed; the caller clears it (it may be the status
+ * word of a workspace set up by tsb_workspace_init, which tsb_device_status then reads).
+ * With NULL the bits go to a word inside the scratch that each call clears first and that
+ * nothing reads. Other arguments and errors as in tsb_plan. */
+tsb_status tsb_plan_noalloc(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats, size_t stats_bytes,
+                            const tsb_tree *out, uint32_t *dev_status, tsb_stream stream);
 
 /* Second pass (Sec. 3.2, Eq. replay-distribution; WoR as in App. A): for every parent u
  * with m_u children, draws m_u tokens without replacement from q_u = softmax(x of row

@@ -450,3 +450,50 @@ cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N
 }
 
 }  // namespace tsb
+
+namespace tsb {
+
+// The same two launches as launch_plan, with the per-draft-row scratch and the status word
+// given explicitly instead of being carved out of a caller workspace.
+cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
+                                const TreeDesc &tree, const PlanScratch &sc, uint32_t *status, cudaStream_t s) {
+    TopkArgs t;
+    t.draft = draft.data;
+    t.bstride = draft.batch_stride;
+    t.rstride = draft.row_stride;
+    t.B = draft.B;
+    t.R = draft.R;
+    t.V = draft.V;
+    t.C = num_chunks(draft.V);
+    t.L = L;
+    t.K = K;
+    t.stats = stats;
+    t.invT = invT;
+    t.lse = sc.lse;
+    t.topk_x = sc.topk_x;
+    t.topk_id = sc.topk_id;
+    cudaError_t e;
+    if (draft.dtype == 1)
+        e = K <= 8 ? launch_topk_t<8, __nv_bfloat16>(t, s) : launch_topk_t<32, __nv_bfloat16>(t, s);
+    else
+        e = K <= 8 ? launch_topk_t<8, float>(t, s) : launch_topk_t<32, float>(t, s);
+    if (e != cudaSuccess) return e;
+    HeapArgs h;
+    h.L = L;
+    h.N = N;
+    h.K = K;
+    h.lse = sc.lse;
+    h.topk_x = sc.topk_x;
+    h.topk_id = sc.topk_id;
+    h.tree = tree;
+    h.status = status;
+    const int per_lane = (N + 1 + 31) / 32;
+    if (per_lane <= 1) return launch_heap_t<1>(h, draft.B, s);
+    if (per_lane <= 2) return launch_heap_t<2>(h, draft.B, s);
+    if (per_lane <= 4) return launch_heap_t<4>(h, draft.B, s);
+    if (per_lane <= 8) return launch_heap_t<8>(h, draft.B, s);
+    if (per_lane <= 16) return launch_heap_t<16>(h, draft.B, s);
+    return launch_heap_t<33>(h, draft.B, s);
+}
+
+}  // namespace tsb

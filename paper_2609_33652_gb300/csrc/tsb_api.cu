@@ -3,6 +3,8 @@
 #include <math.h>
 #include <stdint.h>
 
+#include <mutex>
+
 #include "../../include/tsb.h"
 #include "tsb_launch.h"
 
@@ -215,3 +217,81 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------
+// tsb_plan_noalloc: the first pass for callers that may not allocate device memory.
+//
+// Its scratch (the first pass's per-draft-row log-normaliser and top-K list, plus a status
+// word used when the caller gives none) lives in one file-scope device array of
+// TSB_NOALLOC_SCRATCH_BYTES. Every device that loads this library holds the array until the
+// process exits, and every call on that device shares it.
+namespace {
+
+constexpr size_t kNoallocBytes = TSB_NOALLOC_SCRATCH_BYTES;
+static_assert(kNoallocBytes % 256 == 0 && kNoallocBytes > kStatusBytes, "scratch size");
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocBytes];
+
+// In host code g_noalloc_scratch names a host-side shadow, not device memory: the device
+// address is looked up once per device and cached here.
+constexpr int kNoallocMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[kNoallocMaxDevices];  // guarded by g_noalloc_mu
+
+// Device address of the scratch array on the current device (set-up on the first call there).
+tsb_status noalloc_scratch(unsigned char **out) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoallocMaxDevices) return TSB_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!g_noalloc_ptr[dev]) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return TSB_ERR_CUDA;
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = static_cast<unsigned char *>(g_noalloc_ptr[dev]);
+    return TSB_OK;
+}
+
+// Bytes of the scratch one configuration uses: status word, then per draft row a float2
+// log-normaliser, K floats and K int32 (the same per-row record as the workspace's).
+size_t noalloc_need(const tsb_cfg *c) {
+    const size_t rows = (size_t)c->B * (size_t)c->L;
+    return kStatusBytes + rows * sizeof(float2) + rows * (size_t)c->K * (sizeof(float) + sizeof(int32_t));
+}
+
+}  // namespace
+
+extern "C" tsb_status tsb_plan_noalloc(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats,
+                                       size_t stats_bytes, const tsb_tree *out, uint32_t *dev_status,
+                                       tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_logits(draft, cfg->B, cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(draft_stats, stats_bytes, cfg->B, draft->R, cfg->V);
+    if (st != TSB_OK) return st;
+    if (!out || !out->parent || !out->depth || !out->rank || !out->plan_token || !out->score || !out->child_off ||
+        !out->child_ids)
+        return TSB_ERR_ARG;
+    if (dev_status && !aligned(dev_status, sizeof(uint32_t))) return TSB_ERR_ARG;
+    if (noalloc_need(cfg) > kNoallocBytes) return TSB_ERR_SHAPE;
+    unsigned char *base = nullptr;
+    st = noalloc_scratch(&base);
+    if (st != TSB_OK) return st;
+    uint32_t *status = dev_status;
+    if (!status) {
+        // bits nobody reads, but the word is OR-ed into: start it at zero on every call
+        status = reinterpret_cast<uint32_t *>(base);
+        if (cudaMemsetAsync(status, 0, sizeof(uint32_t), (cudaStream_t)stream) != cudaSuccess) return TSB_ERR_CUDA;
+    }
+    // The top-K launch writes every (lse, x, id) entry the frontier launch reads, so the
+    // rest of the scratch needs no clearing.
+    const size_t rows = (size_t)cfg->B * (size_t)cfg->L;
+    tsb::PlanScratch sc;
+    sc.lse = reinterpret_cast<float2 *>(base + kStatusBytes);
+    sc.topk_x = reinterpret_cast<float *>(base + kStatusBytes + rows * sizeof(float2));
+    sc.topk_id = reinterpret_cast<int32_t *>(base + kStatusBytes + rows * sizeof(float2) +
+                                             rows * (size_t)cfg->K * sizeof(float));
+    return cuda_status(tsb::launch_plan_scratch(rows_of(draft), static_cast<const float2 *>(draft_stats), cfg->L,
+                                                cfg->N, cfg->K, inv_temperature(cfg->temperature), tree_of(out), sc,
+                                                status, (cudaStream_t)stream));
+}

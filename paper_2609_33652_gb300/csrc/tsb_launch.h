@@ -46,6 +46,8 @@ cudaError_t launch_row_stats(const RowsDesc &rows, float invT, float2 *stats, ui
 
 cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
                         const TreeDesc &tree, void *ws, cudaStream_t s);
+cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
+                                const TreeDesc &tree, const PlanScratch &sc, uint32_t *status, cudaStream_t s);
 
 cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
                           int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token, uint32_t *status,

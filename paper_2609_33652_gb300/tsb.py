@@ -26,7 +26,8 @@ TSB_DEV_NONFINITE, TSB_DEV_BAD_INDEX, TSB_DEV_BAD_TREE = 0x1, 0x2, 0x4
 TSB_CHUNK = 256
 
 EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_bytes", "tsb_workspace_init",
-           "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify")
+           "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify", "tsb_plan_noalloc")
+TSB_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
 class TsbError(RuntimeError):
@@ -78,6 +79,7 @@ def load():
         "tsb_device_status": (_I32, [_P, _P, _P]),
         "tsb_row_stats": (_I32, [_P, ctypes.c_float, _P, _SZ, _P, _SZ, _P]),
         "tsb_plan": (_I32, [_P, _P, _P, _SZ, _P, _P, _SZ, _P]),
+        "tsb_plan_noalloc": (_I32, [_P, _P, _P, _SZ, _P, _P, _P]),
         "tsb_replay": (_I32, [_P, _P, _P, _SZ, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
         "tsb_verify": (_I32, [_P, _I32, _P, _P, _P, _SZ, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
     }
@@ -171,6 +173,17 @@ def tsb_plan(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, ws:
     t = tree_struct(tree)
     _check(load().tsb_plan(ctypes.byref(cfg), ctypes.byref(d), _ptr(stats), stats.numel() * stats.element_size(),
                            ctypes.byref(t), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)), "tsb_plan")
+
+
+def tsb_plan_noalloc(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, dev_status=None, stream=None):
+    """tsb_plan with the library's static device scratch instead of a workspace; the C call
+    allocates nothing. ``dev_status``: optional int32 CUDA tensor whose first word receives
+    the device status bits."""
+    d = logits_desc(draft)
+    t = tree_struct(tree)
+    _check(load().tsb_plan_noalloc(ctypes.byref(cfg), ctypes.byref(d), _ptr(stats),
+                                   stats.numel() * stats.element_size(), ctypes.byref(t), _ptr(dev_status),
+                                   _stream(stream)), "tsb_plan_noalloc")
 
 
 def tsb_replay(cfg: Cfg, qrows: torch.Tensor, qstats: torch.Tensor, qrow_of_node, tree: dict, seed: int,
