@@ -4,10 +4,11 @@
 // One thread-block cluster per tree. CTA r of the cluster owns the chunk-aligned vocabulary
 // slice [r*slice, (r+1)*slice) and keeps that slice of the current node in shared memory as
 // fp32: P holds the target logits, later the current residual; Q holds the normalised draft
-// law once it is needed. Scalars (log-normalisers, residual masses, argmax keys) are combined
-// across the cluster through distributed shared memory: each CTA publishes its partial, the
-// cluster barrier orders the writes, and every CTA combines all partials in rank order, so
-// all CTAs hold bitwise identical values and take identical decisions.
+// law once a rejection needs it. Scalars (the target log-normaliser, residual masses, argmax
+// keys) are combined across the cluster through distributed shared memory: each CTA
+// publishes its partial, the cluster barrier orders the writes, and every CTA combines all
+// partials in rank order, so all CTAs hold bitwise identical values and take identical
+// decisions.
 //
 // Walk at node u with children y_1..y_m (slot order), P0 = softmax(target row u),
 // Q = softmax(q row of u), t_0 = 1:
@@ -17,11 +18,17 @@
 //   A rejected token has p_{i+1} = 0 from then on, which is exactly the exclusion of drawn
 //   tokens from the renormalised draft law. Each pass is O(1) per element: P keeps R_i and
 //   p_i(v) = P[v] / Z_i; the point value p_i(y) repeats the same fp32 operations from P0(y).
-// Per node: one staging pass (the target log-normaliser is accumulated while staging); the
-// q row is staged by the first rejection pass only, so a node whose first child is accepted
-// reads one row. Final tokens (all children rejected: from R_m; leaf: bonus from the target
-// row) are drawn with the two-level Gumbel-max of the contract: chunk keys
-// log(chunk mass) + G over chunks of 256 tokens, then the best token of the winning chunk.
+// Final tokens (all children rejected: from R_m; leaf: bonus from the target row) are drawn
+// with the two-level Gumbel-max of the randomness contract: chunk keys log(chunk mass) + G
+// over chunks of 256 tokens, then the best token of the winning chunk.
+//
+// Scheduling. The tree's topology is copied to shared memory once. At every node, while
+// warps 0..13 stage the target slice (one batch of loads per warp, then the online
+// log-normaliser), warp 14 computes the q row's log-normaliser from its chunk statistics
+// (every CTA computes the same value, so it needs no cluster round) and warp 15 fetches the
+// children's tokens, their target and q logits and their acceptance uniforms. Element
+// passes give lane l the elements 4l..4l+3 and 128+4l..128+4l+3 of each 256-token chunk, so
+// every shared-memory access is a conflict-free 16-byte vector.
 #include <cooperative_groups.h>
 
 #include <mutex>
@@ -36,6 +43,9 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
+constexpr int kStageWarps = 14;       // warps that stage the target slice
+constexpr int kQWarp = 14;            // q-row log-normaliser
+constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
 
 struct VerifyArgs {
     const void *target;
@@ -53,42 +63,23 @@ struct VerifyArgs {
     uint32_t *status;
 };
 
-// A partial of one cluster-wide reduction: two softmax normalisers (target row, q row), a
-// plain sum, and an argmax key carrying a token.
+// A partial of one cluster-wide reduction: a softmax normaliser (max, float-float sum), a
+// plain float-float sum, and an argmax key carrying a token.
 struct alignas(16) Slot {
-    float m1, s1h, s1l, m2, s2h, s2l, zh, zl;
+    float m, sh, sl, zh, zl;
+    int tok;
     unsigned long long key;
-    int tok, pad;
 };
 
 enum : int { kRedLse = 1, kRedSum = 2, kRedArg = 4 };
 
 __device__ __forceinline__ Slot neutral_slot() {
     Slot s;
-    s.m1 = s.m2 = -INFINITY;
-    s.s1h = s.s1l = s.s2h = s.s2l = s.zh = s.zl = 0.f;
-    s.key = 0ull;
+    s.m = -INFINITY;
+    s.sh = s.sl = s.zh = s.zl = 0.f;
     s.tok = -1;
-    s.pad = 0;
+    s.key = 0ull;
     return s;
-}
-
-// Symmetric merge of the plain-sum and argmax fields (normalisers are reduced separately).
-template <int KIND>
-__device__ __forceinline__ Slot merge_slot(const Slot &a, const Slot &b) {
-    Slot r = a;
-    if (KIND & kRedSum) {
-        const FF z = ff_add(FF{a.zh, a.zl}, FF{b.zh, b.zl});
-        r.zh = z.hi;
-        r.zl = z.lo;
-    }
-    if (KIND & kRedArg) {
-        if (b.key > a.key) {
-            r.key = b.key;
-            r.tok = b.tok;
-        }
-    }
-    return r;
 }
 
 // A normaliser rescaled to a larger reference maximum M (exp evaluated once).
@@ -98,29 +89,22 @@ __device__ __forceinline__ FF rescale_to(float m, FF s, float M) {
 
 template <int KIND>
 __device__ __forceinline__ Slot warp_reduce_slot(Slot v) {
-    if (KIND & kRedLse) {  // maxima first, then every lane rescales once, then plain sums
-        const float M1 = warp_max(v.m1), M2 = warp_max(v.m2);
-        const FF a = warp_sum_ff(rescale_to(v.m1, FF{v.s1h, v.s1l}, M1));
-        const FF c = warp_sum_ff(rescale_to(v.m2, FF{v.s2h, v.s2l}, M2));
-        v.m1 = M1;
-        v.s1h = a.hi;
-        v.s1l = a.lo;
-        v.m2 = M2;
-        v.s2h = c.hi;
-        v.s2l = c.lo;
+    if (KIND & kRedLse) {  // maximum first, then every lane rescales once, then a plain sum
+        const float M = warp_max(v.m);
+        const FF a = warp_sum_ff(rescale_to(v.m, FF{v.sh, v.sl}, M));
+        v.m = M;
+        v.sh = a.hi;
+        v.sl = a.lo;
     }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        Slot w = v;
-        if (KIND & kRedSum) {
-            w.zh = __shfl_xor_sync(kFull, v.zh, o);
-            w.zl = __shfl_xor_sync(kFull, v.zl, o);
-        }
-        if (KIND & kRedArg) {
-            w.key = __shfl_xor_sync(kFull, v.key, o);
-            w.tok = __shfl_xor_sync(kFull, v.tok, o);
-        }
-        v = merge_slot<KIND>(v, w);
+    if (KIND & kRedSum) {
+        const FF z = warp_sum_ff(FF{v.zh, v.zl});
+        v.zh = z.hi;
+        v.zl = z.lo;
+    }
+    if (KIND & kRedArg) {
+        int owner;
+        v.key = warp_max_u64_owner(v.key, &owner);
+        v.tok = __shfl_sync(kFull, v.tok, owner);
     }
     return v;
 }
@@ -131,13 +115,17 @@ struct Scratch {
     Slot res;            // combined result
     FF L2t, L2q;         // log-normalisers of the target and q rows, times log2(e)
     unsigned long long wbest[kWarps];
-    unsigned long long cbest;
-    float izs[kMaxK], its[kMaxK];  // 1/Z and 1/t of every rejection so far
+    unsigned long long cbest, tbest;
+    float izs[kMaxK], its[kMaxK];             // 1/Z and 1/t of every rejection so far
+    float cxt[kMaxK], cxq[kMaxK], cu[kMaxK];  // children: target x, q x, acceptance uniform
+    int cnode[kMaxK];
+    int cbad;
+    float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
 };
 
-// One cluster-wide reduction: warp butterflies, the CTA's warp partials in warp 0, the
+// One cluster-wide reduction: warp reductions, the CTA's warp partials in warp 0, the
 // cluster barrier, then warp 0 of every CTA reads the CS published partials (one per lane)
-// and combines them with the same butterfly, so every CTA obtains identical results.
+// and combines them the same way, so every CTA obtains identical results.
 template <int KIND>
 __device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &cluster, Slot mine) {
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -156,10 +144,8 @@ __device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &clu
         if (lane == 0) {
             sh.res = v;
             if (KIND & kRedLse) {
-                const FF l1 = v.s1h > 0.f ? maxsum_lse(MaxSum{v.m1, FF{v.s1h, v.s1l}}) : FF{0.f, 0.f};
-                const FF l2 = v.s2h > 0.f ? maxsum_lse(MaxSum{v.m2, FF{v.s2h, v.s2l}}) : FF{0.f, 0.f};
-                sh.L2t = ff_times_log2e(l1);
-                sh.L2q = ff_times_log2e(l2);
+                const FF l = v.sh > 0.f ? maxsum_lse(MaxSum{v.m, FF{v.sh, v.sl}}) : FF{0.f, 0.f};
+                sh.L2t = ff_times_log2e(l);
             }
         }
     }
@@ -178,15 +164,13 @@ __device__ __forceinline__ float point_residual(float p0, float q, const float *
     return p;
 }
 
-// Per-thread online (max, sum of exp(x - max)) accumulation, eight logits at a time.
+// Per-thread online (max, sum of exp(x - max)) accumulation, four logits at a time.
 struct OnlineLse {
     float m = -INFINITY;
     KahanF s;
     __device__ __forceinline__ MaxSum value() const { return MaxSum{m, s.ff()}; }
-    __device__ __forceinline__ void add8(const float x[8]) {
-        float gm = x[0];
-#pragma unroll
-        for (int k = 1; k < 8; ++k) gm = fmaxf(gm, x[k]);
+    __device__ __forceinline__ void add4(const float x[4]) {
+        const float gm = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
         if (gm == -INFINITY) return;
         if (gm > m) {
             if (m != -INFINITY) {
@@ -198,48 +182,66 @@ struct OnlineLse {
         }
         float t = 0.f;
 #pragma unroll
-        for (int k = 0; k < 8; ++k) t += fast_exp2(__fmul_rn(__fsub_rn(x[k], m), kLog2e));
+        for (int k = 0; k < 4; ++k) t += fast_exp2(__fmul_rn(__fsub_rn(x[k], m), kLog2e));
         s.add(t);
     }
 };
+
+__device__ __forceinline__ float4 ld4(const float *p, int j) { return *reinterpret_cast<const float4 *>(p + j); }
+__device__ __forceinline__ void st4(float *p, int j, float a, float b, float c, float d) {
+    *reinterpret_cast<float4 *>(p + j) = make_float4(a, b, c, d);
+}
 
 template <typename T>
 struct Walk {
     const VerifyArgs &a;
     Scratch &sh;
     const cg::cluster_group &cluster;
-    float *P, *Qs;
+    float *P, *Q;
     int &par;
-    int b, lo, n, crank;
+    int b, lo, n, nch;
 
-    __device__ int groups() const { return (n + 7) >> 3; }
+    // Shared-memory index of lane `lane`'s quad h (0 or 1) in local chunk cl.
+    static __device__ __forceinline__ int quad_at(int cl, int h, int lane) { return cl * kChunk + h * 128 + 4 * lane; }
 
-    // Stage x = fp32(z) * invT of this CTA's target slice into P; optionally accumulate the
-    // target row's log-normaliser.
-    // Stage x = fp32(z) * invT of this CTA's target slice into P; optionally accumulate the
-    // target row's log-normaliser. Loads are issued in batches of kBatch groups per thread
-    // before any is used, so a slice costs one memory round trip per batch.
-    static constexpr int kBatch = sizeof(T) == 2 ? 6 : 3;
-    __device__ void stage_target(const T *row, OnlineLse *lse) {
-        const int G = groups();
-        for (int g0 = threadIdx.x; g0 < G; g0 += kBatch * kThreads) {
-            RawGroup<T> raw[kBatch];
+    // Stage x = fp32(z) * invT of this CTA's slice of `row` into dst (warps 0..nw-1; logits
+    // past the vocabulary become -inf), optionally with the online log-normaliser, or store
+    // exp(x - L) instead of x (the normalised law). Loads are issued in batches of kB chunks
+    // per warp before any is used, so a slice costs one memory round trip per batch.
+    template <bool NORMALISE>
+    __device__ void stage(const T *row, float *dst, int nw, OnlineLse *lse, FF L2) {
+        constexpr int kB = sizeof(T) == 2 ? 8 : 4;
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        if (warp >= nw) return;
+        const int end = lo + n;
+        for (int c0 = warp; c0 < nch; c0 += nw * kB) {
+            RawQuad<T> raw[kB][2];
 #pragma unroll
-            for (int e = 0; e < kBatch; ++e) {
-                const int g = g0 + e * kThreads;
-                if (g < G) raw[e].load(row, lo + 8 * g, a.V);
+            for (int e = 0; e < kB; ++e) {
+                const int cl = c0 + e * nw;
+                if (cl < nch) {
+                    raw[e][0].load(row, lo + quad_at(cl, 0, lane), end);
+                    raw[e][1].load(row, lo + quad_at(cl, 1, lane), end);
+                }
             }
 #pragma unroll
-            for (int e = 0; e < kBatch; ++e) {
-                const int g = g0 + e * kThreads;
-                if (g >= G) break;
-                float x[8];
-                raw[e].unpack(x);
+            for (int e = 0; e < kB; ++e) {
+                const int cl = c0 + e * nw;
+                if (cl >= nch) break;
 #pragma unroll
-                for (int k = 0; k < 8; ++k) x[k] = __fmul_rn(x[k], a.invT);  // padding stays -inf
-                reinterpret_cast<float4 *>(P)[2 * g] = make_float4(x[0], x[1], x[2], x[3]);
-                reinterpret_cast<float4 *>(P)[2 * g + 1] = make_float4(x[4], x[5], x[6], x[7]);
-                if (lse) lse->add8(x);
+                for (int h = 0; h < 2; ++h) {
+                    float x[4];
+                    raw[e][h].unpack(x);
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) x[k] = __fmul_rn(x[k], a.invT);  // padding stays -inf
+                    if (NORMALISE) {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) x[k] = exp_shifted(x[k], L2);
+                    } else if (lse) {
+                        lse->add4(x);
+                    }
+                    st4(dst, quad_at(cl, h, lane), x[0], x[1], x[2], x[3]);
+                }
             }
         }
     }
@@ -254,23 +256,21 @@ struct Walk {
 
     // Two-level draw (chunk by Gumbel-max over chunk masses, then token by Gumbel-max inside
     // the chunk) in one cluster round: every CTA picks its best chunk and that chunk's best
-    // token; the cluster keeps the pair with the largest chunk key. val(j, v) returns a
-    // log-weight (LOGITS) or a weight >= 0 for the element at smem index j, token v.
+    // token; the cluster keeps the pair with the largest chunk key. wt(j, w) fills w[0..3]
+    // with the quad at shared-memory index j: log-weights (LOGITS) or weights >= 0.
     template <bool LOGITS, typename F>
-    __device__ int draw(int node, F val) {
+    __device__ int draw(int node, F wt) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-        const int nch = (n + kChunk - 1) / kChunk;
-        unsigned long long best = 0ull;
+        // 1. chunk log-masses, one warp per chunk
         for (int cl = warp; cl < nch; cl += kWarps) {
-            const int i0 = cl * kChunk + lane * 8;
             float v[8];
-#pragma unroll
-            for (int k = 0; k < 8; ++k) v[k] = (i0 + k < n) ? val(i0 + k, lo + i0 + k) : (LOGITS ? -INFINITY : 0.f);
+            wt(quad_at(cl, 0, lane), v);
+            wt(quad_at(cl, 1, lane), v + 4);
             float A = -INFINITY;
             if (LOGITS) {
-                float mx = -INFINITY;
+                float mx = v[0];
 #pragma unroll
-                for (int k = 0; k < 8; ++k) mx = fmaxf(mx, v[k]);
+                for (int k = 1; k < 8; ++k) mx = fmaxf(mx, v[k]);
                 mx = warp_max(mx);
                 float sm = 0.f;
                 if (mx != -INFINITY) {
@@ -286,62 +286,119 @@ struct Walk {
                 sm = warp_sum(sm);
                 if (sm > 0.f) A = logf(sm);
             }
-            if (lane == 0 && A != -INFINITY) {
+            if (lane == 0) sh.clog[cl] = A;
+        }
+        __syncthreads();
+        // 2. chunk keys, one thread per chunk, and the CTA's best chunk
+        unsigned long long best = 0ull;
+        for (int cl = threadIdx.x; cl < nch; cl += kThreads) {
+            const float A = sh.clog[cl];
+            if (A != -INFINITY) {
                 const int c = (lo >> 8) + cl;
                 const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
                 const unsigned long long pk = pack_key(__fadd_rn(A, gumbel_of(w)), (uint32_t)c);
                 best = pk > best ? pk : best;
             }
         }
+        best = warp_max_u64(best);
         if (lane == 0) sh.wbest[warp] = best;
         __syncthreads();
+        // 3. warp 0: the best token inside this CTA's best chunk
         if (warp == 0) {
-            unsigned long long cb = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
-            // the best token inside this CTA's best chunk
+            const unsigned long long cb = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
             unsigned long long tb = 0ull;
             if (cb != 0ull) {
-                const int i0 = (int)key_id(cb) * kChunk - lo + lane * 8, v0 = lo + i0;
-                const Words4 w0 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
-                const Words4 w1 = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2) + 1u);
+                const int cl = (int)key_id(cb) - (lo >> 8);
 #pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    if (i0 + k >= n) break;
-                    const float x = val(i0 + k, v0 + k);
-                    float l;
-                    if (LOGITS) {
-                        if (x == -INFINITY) continue;
-                        l = x;
-                    } else {
-                        if (!(x > 0.f)) continue;
-                        l = logf(x);
+                for (int h = 0; h < 2; ++h) {
+                    const int j = quad_at(cl, h, lane), v0 = lo + j;
+                    float v[4];
+                    wt(j, v);
+                    const Words4 w = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        float l;
+                        if (LOGITS) {
+                            if (v[k] == -INFINITY) continue;
+                            l = v[k];
+                        } else {
+                            if (!(v[k] > 0.f)) continue;
+                            l = logf(v[k]);
+                        }
+                        const unsigned long long pk = pack_key(__fadd_rn(l, gumbel_of(w.w[k])), (uint32_t)(v0 + k));
+                        tb = pk > tb ? pk : tb;
                     }
-                    const unsigned long long pk = pack_key(__fadd_rn(l, gumbel_of(k < 4 ? w0.w[k] : w1.w[k - 4])),
-                                                           (uint32_t)(v0 + k));
-                    tb = pk > tb ? pk : tb;
                 }
                 tb = warp_max_u64(tb);
             }
             if (lane == 0) {
                 sh.cbest = cb;
-                sh.wbest[0] = tb;
+                sh.tbest = tb;
             }
         }
         __syncthreads();
         Slot mine = neutral_slot();
         if (threadIdx.x == 0 && sh.cbest != 0ull) {
             mine.key = sh.cbest;
-            mine.tok = (int)key_id(sh.wbest[0]);
+            mine.tok = (int)key_id(sh.tbest);
         }
         reduce_round<kRedArg>(sh, par, cluster, mine);
         return sh.res.key == 0ull ? -1 : sh.res.tok;
     }
+
+    // Bonus draw from the logits of `row` (a leaf, or a residual without mass).
+    __device__ int draw_from_row(const T *row, int node) {
+        __syncthreads();
+        stage<false>(row, P, kWarps, nullptr, FF{0.f, 0.f});
+        __syncthreads();
+        return draw<true>(node, [&](int j, float *v) {
+            const float4 x = ld4(P, j);
+            v[0] = x.x;
+            v[1] = x.y;
+            v[2] = x.z;
+            v[3] = x.w;
+        });
+    }
 };
+
+// Log-normaliser of a q row from its chunk statistics (m_c, s_c), by one warp, times
+// log2(e): the maximum of the m_c, then sum s_c exp(m_c - M) (loads issued eight at a time;
+// the same code on the same data in every CTA gives the same bits).
+__device__ FF q_log_normaliser(const float2 *st, int C) {
+    constexpr int kB = 8;
+    const int lane = threadIdx.x & 31;
+    float m = -INFINITY;
+    for (int c0 = lane; c0 < C; c0 += 32 * kB) {
+        float v[kB];
+#pragma unroll
+        for (int e = 0; e < kB; ++e) v[e] = c0 + 32 * e < C ? __ldg(&st[c0 + 32 * e]).x : -INFINITY;
+#pragma unroll
+        for (int e = 0; e < kB; ++e) m = fmaxf(m, v[e]);
+    }
+    m = warp_max(m);
+    KahanF s;
+    if (m != -INFINITY)
+        for (int c0 = lane; c0 < C; c0 += 32 * kB) {
+            float2 v[kB];
+#pragma unroll
+            for (int e = 0; e < kB; ++e)
+                v[e] = c0 + 32 * e < C ? __ldg(&st[c0 + 32 * e]) : make_float2(-INFINITY, 0.f);
+#pragma unroll
+            for (int e = 0; e < kB; ++e)
+                if (v[e].x != -INFINITY) s.add(__fmul_rn(v[e].y, expf(__fsub_rn(v[e].x, m))));
+        }
+    const FF S = warp_sum_ff(s.ff());
+    return S.hi > 0.f ? ff_times_log2e(maxsum_lse(MaxSum{m, S})) : FF{0.f, 0.f};
+}
+
+// Shared-memory bytes of the tree's topology copy.
+inline size_t topo_bytes(int N) { return (size_t)(4 * N + 5) * sizeof(int32_t); }
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     extern __shared__ __align__(16) float dyn[];
     float *P = dyn;
-    float *Qs = dyn + a.slice;
+    float *Q = dyn + a.slice;
     __shared__ Scratch sh;
 
     cg::cluster_group cluster = cg::this_cluster();
@@ -351,36 +408,47 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     const int NN = a.N + 1;
     const int lo = crank * a.slice;
     const int n = max(0, min(a.V - lo, a.slice));
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const bool writer = crank == 0 && threadIdx.x == 0;
     int par = 0;
-    Walk<T> W{a, sh, cluster, P, Qs, par, b, lo, n, crank};
-    const int groups = W.groups();
+    Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
 
-    const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
-    const int32_t *kids = a.child_ids + (int64_t)b * a.N;
-    const int32_t *tok = a.token + (int64_t)b * NN;
+    // the tree's topology: child_off [N+2], child_ids [N], token [N+1], q row of node [N+1]
+    int32_t *s_off = reinterpret_cast<int32_t *>(dyn + 2 * a.slice);
+    int32_t *s_kid = s_off + (NN + 1);
+    int32_t *s_tok = s_kid + a.N;
+    int32_t *s_row = s_tok + NN;
+    {
+        const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+        const int32_t *kids = a.child_ids + (int64_t)b * a.N;
+        const int32_t *tok = a.token + (int64_t)b * NN;
+        const int32_t *row = a.qrow_of_node ? a.qrow_of_node + (int64_t)b * NN : a.depth + (int64_t)b * NN;
+        for (int i = threadIdx.x; i <= NN; i += kThreads) s_off[i] = __ldg(off + i);
+        for (int i = threadIdx.x; i < a.N; i += kThreads) s_kid[i] = __ldg(kids + i);
+        for (int i = threadIdx.x; i < NN; i += kThreads) {
+            s_tok[i] = __ldg(tok + i);
+            s_row[i] = __ldg(row + i);
+        }
+    }
     int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
     int32_t *onode = a.out_nodes + (int64_t)b * a.L;
 
-    cluster.sync();  // every CTA of the cluster runs before any distributed access
+    cluster.sync();  // topology visible; every CTA of the cluster runs before any distributed access
 
     int u = 0, nacc = 0, final_tok = -1;
     bool bad = false;
     for (int step = 0; step <= a.L; ++step) {
-        const int o = off[u], m = off[u + 1] - o;
+        const int o = s_off[u], m = s_off[u + 1] - o;
         if (m < 0 || m > kMaxK || o < 0 || o + m > a.N) {
             bad = true;
             break;
         }
         const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
-        __syncthreads();
         if (m == 0) {  // leaf: bonus token from the node's target row
-            W.stage_target(trow, nullptr);
-            __syncthreads();
-            final_tok = W.template draw<true>(u, [&](int i, int) { return P[i]; });
+            final_tok = W.draw_from_row(trow, u);
             break;
         }
-        const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
+        const int r = s_row[u];
         if (r < 0 || r >= a.q_R) {
             bad = true;
             break;
@@ -388,103 +456,113 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
         const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
         {  // likely next reads: this node's q row (first rejection), the first child's target row
             W.prefetch_slice(qrow);
-            const int c0 = kids[o];
+            const int c0 = s_kid[o];
             if (c0 >= 1 && c0 <= a.N)
                 W.prefetch_slice(static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride +
                                  (int64_t)c0 * a.t_rstride);
         }
+        __syncthreads();  // the previous node's readers of P, Q and the child data are done
 
-        // staging pass with the target log-normaliser; q row log-normaliser from its chunk stats
+        // staging (warps 0..13) with the target log-normaliser; q normaliser (warp 14);
+        // child data (warp 15)
         OnlineLse lt;
-        W.stage_target(trow, &lt);
-        const float2 *st = a.qstats + ((int64_t)b * a.q_R + r) * a.C;
-        float m2 = -INFINITY;
-        for (int c = crank * kThreads + threadIdx.x; c < a.C; c += CS * kThreads) m2 = fmaxf(m2, st[c].x);
-        KahanF s2;
-        if (m2 != -INFINITY)
-            for (int c = crank * kThreads + threadIdx.x; c < a.C; c += CS * kThreads)
-                s2.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m2))));
+        if (warp < kStageWarps) {
+            W.template stage<false>(trow, P, kStageWarps, &lt, FF{0.f, 0.f});
+        } else if (warp == kQWarp) {
+            const FF L2q = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
+            if (lane == 0) sh.L2q = L2q;
+        } else {
+            bool cb = false;
+            if (lane < m) {
+                const int c = s_kid[o + lane];
+                const int y = (c >= 1 && c <= a.N) ? s_tok[c] : -1;
+                if (y < 0 || y >= a.V) {
+                    cb = true;
+                } else {
+                    sh.cxt[lane] = __fmul_rn(Logit<T>::load1(trow, y), a.invT);
+                    sh.cxq[lane] = __fmul_rn(Logit<T>::load1(qrow, y), a.invT);
+                    sh.cu[lane] = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
+                    sh.cnode[lane] = c;
+                }
+            }
+            cb = __any_sync(kFull, cb);
+            if (lane == 0) sh.cbad = cb ? 1 : 0;
+        }
         {
             Slot mine = neutral_slot();
             const MaxSum t1 = lt.value();
-            mine.m1 = t1.m;
-            mine.s1h = t1.s.hi;
-            mine.s1l = t1.s.lo;
-            const FF q2 = s2.ff();
-            mine.m2 = m2;
-            mine.s2h = q2.hi;
-            mine.s2l = q2.lo;
+            mine.m = t1.m;
+            mine.sh = t1.s.hi;
+            mine.sl = t1.s.lo;
             reduce_round<kRedLse>(sh, par, cluster, mine);
         }
+        if (sh.cbad) {
+            bad = true;
+            break;
+        }
         const FF L2t = sh.L2t, L2q = sh.L2q;
-
         FF t = FF{1.f, 0.f};  // draft mass not yet drawn
         int accepted = -1;
+        bool q_staged = false;
         for (int i = 0; i < m; ++i) {
-            const int c = kids[o + i];
-            const int y = (c >= 1 && c <= a.N) ? tok[c] : -1;
-            if (y < 0 || y >= a.V) {
-                bad = true;
-                break;
-            }
             const float it = t.hi > 0.f ? __frcp_rn(t.hi) : 0.f;  // 1/t_i
-            const float P0y = exp_shifted(__fmul_rn(Logit<T>::load1(trow, y), a.invT), L2t);
-            const float Qy = exp_shifted(__fmul_rn(Logit<T>::load1(qrow, y), a.invT), L2q);
+            const float P0y = exp_shifted(sh.cxt[i], L2t);
+            const float Qy = exp_shifted(sh.cxq[i], L2q);
             const float pp = point_residual(P0y, Qy, sh.izs, sh.its, i);
             const float qp = __fmul_rn(Qy, it);
-            const float U = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
-            if (__fmul_rn(U, qp) < pp) {
-                accepted = c;
+            if (__fmul_rn(sh.cu[i], qp) < pp) {
+                accepted = sh.cnode[i];
                 break;
             }
-            // p_i(v) of the element at smem index j (P holds x before the first rejection,
-            // R_i afterwards)
+            if (!q_staged) {  // the normalised q slice, once per node
+                W.template stage<true>(qrow, Q, kWarps, nullptr, L2q);
+                __syncthreads();
+                q_staged = true;
+            }
+            // p_i(v) of the quad at smem index j (P holds x before the first rejection, R_i
+            // afterwards)
             const float izp = i > 0 ? sh.izs[i - 1] : 1.f;
-            auto p_of = [&](int j) { return i == 0 ? exp_shifted(P[j], L2t) : __fmul_rn(P[j], izp); };
+            auto p_quad = [&](int j, float *p) {
+                const float4 x = ld4(P, j);
+                if (i == 0) {
+                    p[0] = exp_shifted(x.x, L2t);
+                    p[1] = exp_shifted(x.y, L2t);
+                    p[2] = exp_shifted(x.z, L2t);
+                    p[3] = exp_shifted(x.w, L2t);
+                } else {
+                    p[0] = __fmul_rn(x.x, izp);
+                    p[1] = __fmul_rn(x.y, izp);
+                    p[2] = __fmul_rn(x.z, izp);
+                    p[3] = __fmul_rn(x.w, izp);
+                }
+            };
             if (i == m - 1) {  // every slot rejected: final token from R_m = max(p_i - Q/t_i, 0)
-                if (i == 0) {  // the q slice was never staged: stage it (normalised) now
-                    for (int g = threadIdx.x; g < groups; g += kThreads) {
-                        float x[8];
-                        Logit<T>::load8(qrow, lo + 8 * g, a.V, x);
-#pragma unroll
-                        for (int k = 0; k < 8; ++k) Qs[8 * g + k] = exp_shifted(__fmul_rn(x[k], a.invT), L2q);
-                    }
-                    __syncthreads();
-                }
-                final_tok = W.template draw<false>(u, [&](int j, int) { return resid(p_of(j), Qs[j], it); });
-                if (final_tok < 0) {  // no residual mass (rounding only): the node's target row
-                    __syncthreads();
-                    W.stage_target(trow, nullptr);
-                    __syncthreads();
-                    final_tok = W.template draw<true>(u, [&](int j, int) { return P[j]; });
-                }
+                final_tok = W.template draw<false>(u, [&](int j, float *v) {
+                    float p[4];
+                    p_quad(j, p);
+                    const float4 q = ld4(Q, j);
+                    v[0] = resid(p[0], q.x, it);
+                    v[1] = resid(p[1], q.y, it);
+                    v[2] = resid(p[2], q.z, it);
+                    v[3] = resid(p[3], q.w, it);
+                });
+                if (final_tok < 0) final_tok = W.draw_from_row(trow, u);  // no residual mass (rounding)
                 break;
             }
-            // residual pass (the first one also stages the normalised q slice)
+            // residual pass: R_{i+1} into P and its mass
             KahanF zl;
-            for (int g = threadIdx.x; g < groups; g += kThreads) {
-                float q8[8], r8[8];
-                if (i == 0) {
-                    Logit<T>::load8(qrow, lo + 8 * g, a.V, q8);
+            for (int cl = warp; cl < W.nch; cl += kWarps) {
 #pragma unroll
-                    for (int k = 0; k < 8; ++k) q8[k] = exp_shifted(__fmul_rn(q8[k], a.invT), L2q);
-                    reinterpret_cast<float4 *>(Qs)[2 * g] = make_float4(q8[0], q8[1], q8[2], q8[3]);
-                    reinterpret_cast<float4 *>(Qs)[2 * g + 1] = make_float4(q8[4], q8[5], q8[6], q8[7]);
-                } else {
-                    const float4 qa = reinterpret_cast<const float4 *>(Qs)[2 * g];
-                    const float4 qb = reinterpret_cast<const float4 *>(Qs)[2 * g + 1];
-                    q8[0] = qa.x; q8[1] = qa.y; q8[2] = qa.z; q8[3] = qa.w;
-                    q8[4] = qb.x; q8[5] = qb.y; q8[6] = qb.z; q8[7] = qb.w;
+                for (int h = 0; h < 2; ++h) {
+                    const int j = Walk<T>::quad_at(cl, h, lane);
+                    float p[4];
+                    p_quad(j, p);
+                    const float4 q = ld4(Q, j);  // padding: p = 0 (x = -inf), q = 0
+                    const float r0 = resid(p[0], q.x, it), r1 = resid(p[1], q.y, it);
+                    const float r2 = resid(p[2], q.z, it), r3 = resid(p[3], q.w, it);
+                    st4(P, j, r0, r1, r2, r3);
+                    zl.add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
                 }
-                float sum8 = 0.f;
-#pragma unroll
-                for (int k = 0; k < 8; ++k) {
-                    r8[k] = resid(p_of(8 * g + k), q8[k], it);  // padding: p = 0 (x = -inf), q = 0
-                    sum8 += r8[k];
-                }
-                reinterpret_cast<float4 *>(P)[2 * g] = make_float4(r8[0], r8[1], r8[2], r8[3]);
-                reinterpret_cast<float4 *>(P)[2 * g + 1] = make_float4(r8[4], r8[5], r8[6], r8[7]);
-                zl.add(sum8);
             }
             {
                 Slot mine = neutral_slot();
@@ -495,9 +573,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             }
             const float Z = sh.res.zh;
             if (!(Z > 0.f)) {  // no residual mass (rounding only): the node's target row
-                W.stage_target(trow, nullptr);
-                __syncthreads();
-                final_tok = W.template draw<true>(u, [&](int j, int) { return P[j]; });
+                final_tok = W.draw_from_row(trow, u);
                 break;
             }
             if (threadIdx.x == 0) {
@@ -513,7 +589,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             break;
         }
         if (writer) {
-            otok[nacc] = tok[accepted];
+            otok[nacc] = s_tok[accepted];
             onode[nacc] = accepted;
         }
         ++nacc;
@@ -531,32 +607,34 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
 
 constexpr size_t kSmemLimit = 210 * 1024;
 
-// Chunk-aligned slice of each CTA and the dynamic shared memory it needs for cluster size cs.
-void slice_for(int V, int cs, int *slice_out, size_t *smem_out) {
+// Chunk-aligned slice of each CTA and the dynamic shared memory it needs for cluster size cs
+// (SIZE_MAX when the slice exceeds the per-CTA chunk table).
+void slice_for(int V, int N, int cs, int *slice_out, size_t *smem_out) {
     int slice = (V + cs - 1) / cs;
     slice = (slice + kChunk - 1) / kChunk * kChunk;
     *slice_out = slice;
-    *smem_out = 2 * (size_t)slice * sizeof(float);
+    *smem_out = slice > kMaxSliceChunks * kChunk ? (size_t)-1 : 2 * (size_t)slice * sizeof(float) + topo_bytes(N);
 }
 
 struct ClusterChoice {
-    int V, B, elem, cs;
+    int V, N, B, elem, cs;
 };
 
-// The cluster size for (V, B): the largest size up to 16 (above 8 the cluster is
+// The cluster size for (V, N, B): the largest size up to 16 (above 8 the cluster is
 // non-portable) whose clusters can all be resident at once, so every tree walks in the same
-// wave; when no size fits the whole batch, the size with the most concurrently resident CTAs. Decisions are
-// cached per (V, B, element size); the cache is a pure function of the device.
+// wave; when no size fits the whole batch, the size with the most concurrently resident
+// CTAs. Decisions are cached per (V, N, B, element size); the cache is a pure function of
+// the device.
 template <typename T>
-int choose_cluster(int V, int B, int *slice_out, size_t *smem_out) {
+int choose_cluster(int V, int N, int B, int *slice_out, size_t *smem_out) {
     static ClusterChoice cache[16];
     static int cache_n = 0;
     static std::mutex mu;
     {
         std::lock_guard<std::mutex> g(mu);
         for (int i = 0; i < cache_n; ++i)
-            if (cache[i].V == V && cache[i].B == B && cache[i].elem == (int)sizeof(T)) {
-                slice_for(V, cache[i].cs, slice_out, smem_out);
+            if (cache[i].V == V && cache[i].N == N && cache[i].B == B && cache[i].elem == (int)sizeof(T)) {
+                slice_for(V, N, cache[i].cs, slice_out, smem_out);
                 return cache[i].cs;
             }
     }
@@ -567,7 +645,7 @@ int choose_cluster(int V, int B, int *slice_out, size_t *smem_out) {
     for (int cs = hi_cs; cs >= 1; --cs) {
         int slice;
         size_t smem;
-        slice_for(V, cs, &slice, &smem);
+        slice_for(V, N, cs, &slice, &smem);
         if (smem > kSmemLimit) break;  // smaller clusters only need more shared memory
         if (cs < lo_cs && chosen < 0 && best_cs > 0) break;
         if (cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) !=
@@ -602,13 +680,13 @@ int choose_cluster(int V, int B, int *slice_out, size_t *smem_out) {
     if (chosen < 0) {  // the slices do not fit below 16 CTAs: use 16 (non-portable)
         int slice;
         size_t smem;
-        slice_for(V, 16, &slice, &smem);
+        slice_for(V, N, 16, &slice, &smem);
         chosen = smem <= kSmemLimit ? 16 : -1;
     }
     if (chosen > 0) {
         std::lock_guard<std::mutex> g(mu);
-        if (cache_n < 16) cache[cache_n++] = ClusterChoice{V, B, (int)sizeof(T), chosen};
-        slice_for(V, chosen, slice_out, smem_out);
+        if (cache_n < 16) cache[cache_n++] = ClusterChoice{V, N, B, (int)sizeof(T), chosen};
+        slice_for(V, N, chosen, slice_out, smem_out);
     }
     return chosen;
 }
@@ -617,7 +695,7 @@ template <typename T>
 cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     int slice = 0;
     size_t smem = 0;
-    const int cs = choose_cluster<T>(a.V, B, &slice, &smem);
+    const int cs = choose_cluster<T>(a.V, a.N, B, &slice, &smem);
     if (cs < 0) return cudaErrorInvalidValue;
     a.slice = slice;
     cudaError_t e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);

@@ -409,6 +409,52 @@ struct RawGroup<float> {
     }
 };
 
+template <typename T>
+struct RawQuad;  // 4 consecutive logits as raw words (8 bytes of bf16 or 16 of fp32)
+template <>
+struct RawQuad<__nv_bfloat16> {
+    uint2 w;
+    // logits v0..v0+3 (v0 a multiple of 4); those at or beyond `end` become -inf (0xff80)
+    __device__ __forceinline__ void load(const __nv_bfloat16 *row, int v0, int end) {
+        if (v0 + 4 <= end) {
+            w = __ldg(reinterpret_cast<const uint2 *>(row + v0));
+        } else {
+            const unsigned short *r = reinterpret_cast<const unsigned short *>(row);
+            unsigned short h[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) h[i] = (v0 + i < end) ? __ldg(r + v0 + i) : (unsigned short)0xff80u;
+            w.x = h[0] | ((uint32_t)h[1] << 16);
+            w.y = h[2] | ((uint32_t)h[3] << 16);
+        }
+    }
+    __device__ __forceinline__ void unpack(float z[4]) const {
+        z[0] = __uint_as_float(w.x << 16);
+        z[1] = __uint_as_float(w.x & 0xffff0000u);
+        z[2] = __uint_as_float(w.y << 16);
+        z[3] = __uint_as_float(w.y & 0xffff0000u);
+    }
+};
+template <>
+struct RawQuad<float> {
+    float4 w;
+    __device__ __forceinline__ void load(const float *row, int v0, int end) {
+        if (v0 + 4 <= end) {
+            w = __ldg(reinterpret_cast<const float4 *>(row + v0));
+        } else {
+            float z[4];
+#pragma unroll
+            for (int i = 0; i < 4; ++i) z[i] = (v0 + i < end) ? __ldg(row + v0 + i) : -INFINITY;
+            w = make_float4(z[0], z[1], z[2], z[3]);
+        }
+    }
+    __device__ __forceinline__ void unpack(float z[4]) const {
+        z[0] = w.x;
+        z[1] = w.y;
+        z[2] = w.z;
+        z[3] = w.w;
+    }
+};
+
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
