@@ -3,7 +3,8 @@
 
 Workload (batched serving): B=16 trees, V=151,936, draft block L=16, N=64 planned nodes,
 top-k 8, T=1, bf16 logits; target rows [16, 65, V] = the node's depth row + N(0, 0.7^2).
-A step = tsb_row_stats + tsb_plan + tsb_replay + tsb_verify on one batch (4 kernel launches).
+A step = tsb_row_stats + tsb_plan + tsb_replay + tsb_verify on one batch (5 kernel launches:
+the planner launches its per-row top-K kernel and its frontier kernel).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tsb|reference]
 
@@ -39,6 +40,7 @@ FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
 L2_BYTES = 129 * 1024 * 1024
 KERNELS = ("tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify")
+LAUNCHES_PER_STEP = {"tsb_row_stats": 1, "tsb_plan": 2, "tsb_replay": 1, "tsb_verify": 1}
 KERNEL_SOURCES = {"tsb_row_stats": "k_row_stats.cu", "tsb_plan": "k_plan.cu", "tsb_replay": "k_replay.cu",
                   "tsb_verify": "k_verify.cu"}
 
@@ -320,7 +322,7 @@ def run_tsb(args):
         "per_kernel_us": {n: round(v, 3) for n, v in kern_us.items()},
         "per_kernel_gbs": per_kernel_gbs,
         "roofline": roofline,
-        "gpu_launches": 4 * K,
+        "gpu_launches": sum(LAUNCHES_PER_STEP.values()) * K,
         "clocks": clocks.summary(),
         "e2e": e2e,
         "cpu_baseline": cpu,

@@ -4,12 +4,14 @@
 // the replay sampler (Sec. 3.2) all follow from these without touching the row again.
 //
 // HBM-bound: every logit is read once with 16-byte loads; 8 bytes are written per chunk.
-// A warp owns groups of 8 consecutive chunks of a row (lane l holds logits 8l..8l+7 of each
-// chunk) and issues all 8 loads before any arithmetic; the grid is persistent (grid-stride
-// over groups) so there is no partial last wave. Per logit: one conversion, one max, one
-// fma, one ex2 and one add. Rounding to nearest is monotone, so the chunk maximum is taken on
-// the raw logits and scaled once: max_v fp32(z_v * invT) = fp32(max_v z_v * invT).
-// Non-finite logits are detected per chunk (an infinite maximum or a NaN sum).
+// Eight lanes own one chunk (lane g of the group reads logits 8g..8g+7 of each 64-logit
+// quarter, so a group's load instruction covers 128 contiguous bytes), a warp owns four
+// chunks at a time and issues two such units' loads before any arithmetic. The grid is
+// persistent (grid-stride over units), so there is no partial last wave. Per logit: one
+// conversion, one max, one fma, one ex2 and one add; per chunk only three shuffle levels.
+// Rounding to nearest is monotone, so the chunk maximum is taken on the raw logits and
+// scaled once: max_v fp32(z_v * invT) = fp32(max_v z_v * invT). Non-finite logits are
+// detected per chunk (an infinite maximum or a NaN sum).
 #include "tsb_device.cuh"
 #include "tsb_launch.h"
 
@@ -17,47 +19,74 @@ namespace tsb {
 namespace {
 
 constexpr int kWarps = 8;
-constexpr int kPerWarp = 8;  // chunks per warp group
+constexpr int kUnitChunks = 4;  // chunks per warp unit (8 lanes each)
+constexpr int kUnits = 2;       // units per warp iteration (loads in flight together)
 
 template <typename T>
 __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__ data, int R, int V,
                                                            int64_t bstride, int64_t rstride, int C,
-                                                           int64_t groups_total, float invT,
+                                                           int64_t units_total, float invT,
                                                            float2 *__restrict__ stats, uint32_t *status) {
-    const int lane = threadIdx.x & 31;
-    const int groups = (C + kPerWarp - 1) / kPerWarp;
-    const float c2 = __fmul_rn(invT, kLog2e);  // exp(x - m) = 2^(z invT log2e - m log2e)
+    const int lane = threadIdx.x & 31, g = lane & 7, q = lane >> 3;
+    const int upr = (C + kUnitChunks - 1) / kUnitChunks;  // units per row
+    const float c2 = __fmul_rn(invT, kLog2e);             // exp(x - m) = 2^(z invT log2e - m log2e)
     bool bad = false;
-    for (int64_t gw = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5); gw < groups_total;
-         gw += (int64_t)gridDim.x * kWarps) {
-        const int64_t row = gw / groups;
-        const int g = (int)(gw - row * groups);
-        const int b = (int)(row / R);
-        const int r = (int)(row - (int64_t)b * R);
-        const T *rp = data + (int64_t)b * bstride + (int64_t)r * rstride;
-        const int c0 = g * kPerWarp;
-        const int nc = min(kPerWarp, C - c0);
-        RawGroup<T> raw[kPerWarp];
+    const int64_t stride = (int64_t)gridDim.x * kWarps;
+    for (int64_t u0 = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5); u0 < units_total; u0 += stride * kUnits) {
+        RawGroup<T> raw[kUnits][4];
+        int64_t row_of[kUnits];
+        int c_of[kUnits];
 #pragma unroll
-        for (int k = 0; k < kPerWarp; ++k)
-            if (k < nc) raw[k].load(rp, (c0 + k) * kChunk + lane * 8, V);
+        for (int e = 0; e < kUnits; ++e) {
+            const int64_t un = u0 + e * stride;
+            c_of[e] = -1;
+            row_of[e] = 0;
+            if (un >= units_total) continue;
+            const int64_t row = un / upr;
+            const int c = (int)(un - row * upr) * kUnitChunks + q;
+            row_of[e] = row;
+            if (c >= C) continue;
+            c_of[e] = c;
+            const int b = (int)(row / R);
+            const int r = (int)(row - (int64_t)b * R);
+            const T *rp = data + (int64_t)b * bstride + (int64_t)r * rstride;
 #pragma unroll
-        for (int k = 0; k < kPerWarp; ++k) {
-            if (k >= nc) break;  // warp-uniform
-            float z[8];
-            raw[k].unpack(z);
-            float zm = z[0];
+            for (int k = 0; k < 4; ++k) raw[e][k].load(rp, c * kChunk + k * 64 + g * 8, V);
+        }
 #pragma unroll
-            for (int i = 1; i < 8; ++i) zm = fmaxf(zm, z[i]);
-            zm = warp_max(zm);
+        for (int e = 0; e < kUnits; ++e) {
+            const int c = c_of[e];
+            float zm = -INFINITY;
+            if (c >= 0) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    float z[8];
+                    raw[e][k].unpack(z);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
+                }
+            }
+            // the group's maximum (xor 4, 2, 1 stay inside the 8-lane group)
+            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
+            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
+            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
             const float mc = __fmul_rn(zm, invT);
             const float off = __fmul_rn(mc, kLog2e);
             float s = 0.f;
+            if (c >= 0) {
 #pragma unroll
-            for (int i = 0; i < 8; ++i) s += fast_exp2(__fmaf_rn(z[i], c2, -off));
-            s = warp_sum(s);
-            if (lane == 0) {
-                stats[row * C + c0 + k] = make_float2(mc, s);
+                for (int k = 0; k < 4; ++k) {
+                    float z[8];
+                    raw[e][k].unpack(z);  // unpacked again rather than kept: fewer registers
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) s += fast_exp2(__fmaf_rn(z[i], c2, -off));
+                }
+            }
+            s += __shfl_xor_sync(kFull, s, 4);
+            s += __shfl_xor_sync(kFull, s, 2);
+            s += __shfl_xor_sync(kFull, s, 1);
+            if (c >= 0 && g == 0) {
+                stats[row_of[e] * C + c] = make_float2(mc, s);
                 bad |= !(s == s) || isinf(mc);
             }
         }
@@ -92,12 +121,12 @@ int sm_count() {
 template <typename T>
 cudaError_t launch_t(const RowsDesc &rows, float invT, float2 *stats, uint32_t *status, cudaStream_t s) {
     const int C = num_chunks(rows.V);
-    const int64_t groups_total = (int64_t)rows.B * rows.R * ((C + kPerWarp - 1) / kPerWarp);
-    const int64_t needed = (groups_total + kWarps - 1) / kWarps;
+    const int64_t units_total = (int64_t)rows.B * rows.R * ((C + kUnitChunks - 1) / kUnitChunks);
+    const int64_t needed = (units_total + kWarps - 1) / kWarps;
     const int64_t resident = (int64_t)sm_count() * blocks_per_sm<T>();
     const int64_t blocks = needed < resident ? needed : resident;
     k_row_stats<T><<<(unsigned)blocks, kWarps * 32, 0, s>>>(static_cast<const T *>(rows.data), rows.R, rows.V,
-                                                             rows.batch_stride, rows.row_stride, C, groups_total,
+                                                             rows.batch_stride, rows.row_stride, C, units_total,
                                                              invT, stats, status);
     return cudaGetLastError();
 }
