@@ -22,13 +22,18 @@
 // with the two-level Gumbel-max of the randomness contract: chunk keys log(chunk mass) + G
 // over chunks of 256 tokens, then the best token of the winning chunk.
 //
-// Scheduling. The tree's topology is copied to shared memory once. At every node, while
-// warps 0..13 stage the target slice (one batch of loads per warp, then the online
-// log-normaliser), warp 14 computes the q row's log-normaliser from its chunk statistics
-// (every CTA computes the same value, so it needs no cluster round) and warp 15 fetches the
-// children's tokens, their target and q logits and their acceptance uniforms. Element
-// passes give lane l the elements 4l..4l+3 and 128+4l..128+4l+3 of each 256-token chunk, so
-// every shared-memory access is a conflict-free 16-byte vector.
+// Scheduling. A pre-pass kernel (all SMs, bandwidth-bound) computes the target
+// log-normaliser of the M highest-scoring nodes (ids below M, pop order) and, for per-depth
+// q rows, every q row's log-normaliser. The walk kernel copies the tree's topology, the
+// children's target and q logits and their acceptance uniforms to shared memory once. At a
+// node below M it needs no staging and no cluster round: every CTA takes the same decisions
+// from the same inputs, and the slice is staged only if a rejection needs the residual. At
+// any other node warps 0..13 (0..14 for per-depth q rows) stage the target slice (one batch
+// of loads per warp, then the online log-normaliser) while warp 14 computes a per-node q
+// row's log-normaliser from its chunk statistics. Element passes give lane l the elements
+// 4l..4l+3 and 128+4l..128+4l+3 of each 256-token chunk, so every shared-memory access is a
+// conflict-free 16-byte vector. Which path computes a node's normaliser depends only on its
+// id, so results do not depend on timing.
 #include <cooperative_groups.h>
 
 #include <mutex>
@@ -46,6 +51,22 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kStageWarps = 14;       // warps that stage the target slice
 constexpr int kQWarp = 14;            // q-row log-normaliser
 constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
+constexpr int kPreTop = 8;            // highest-scoring node ids the pre-pass covers
+constexpr int kMaxDepthRows = 64;     // per-depth q rows (depth cap L <= 64)
+constexpr int kPreThreads = 1024;
+
+// Pre-pass results, one 32-byte workspace slot per (tree, node) (the slots block
+// verification uses for its own per-position scalars): l2t = target log-normaliser of node u
+// (u in the pre-computed set), l2q = log-normaliser of per-depth q row u; both float-float,
+// times log2(e). Pre-computed set of a tree: its internal nodes with ids below kPreTop (the
+// highest-scoring nodes in pop order; the root is visited by every walk). Measured on the
+// batched workload, covering the first-child chain as well cost more bandwidth than it saved.
+struct alignas(16) PreRow {
+    float2 l2t, l2q;
+    float pad[4];
+};
+static_assert(sizeof(PreRow) == kWsBvRowBytes, "pre-pass slot size");
+
 
 struct VerifyArgs {
     const void *target;
@@ -61,6 +82,10 @@ struct VerifyArgs {
     uint64_t seed;
     int32_t *out_tokens, *out_nodes, *out_len;
     uint32_t *status;
+    PreRow *pre;  // [B, N+1]
+    int M;        // node ids below M with children are pre-computed
+    int Lq;       // per-depth q rows whose normaliser the pre-pass computes (0 for per-node rows)
+    int B;
 };
 
 // A partial of one cluster-wide reduction: a softmax normaliser (max, float-float sum), a
@@ -116,11 +141,11 @@ struct Scratch {
     FF L2t, L2q;         // log-normalisers of the target and q rows, times log2(e)
     unsigned long long wbest[kWarps];
     unsigned long long cbest, tbest;
-    float izs[kMaxK], its[kMaxK];             // 1/Z and 1/t of every rejection so far
-    float cxt[kMaxK], cxq[kMaxK], cu[kMaxK];  // children: target x, q x, acceptance uniform
-    int cnode[kMaxK];
+    float izs[kMaxK], its[kMaxK];  // 1/Z and 1/t of every rejection so far
     int cbad;
+    int path[kMaxDepthRows];      // accepted node ids (written out after the walk)
     float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
+    FF l2q[kMaxDepthRows];        // per-depth q log-normalisers (times log2 e)
 };
 
 // One cluster-wide reduction: warp reductions, the CTA's warp partials in warp 0, the
@@ -303,37 +328,32 @@ struct Walk {
         best = warp_max_u64(best);
         if (lane == 0) sh.wbest[warp] = best;
         __syncthreads();
-        // 3. warp 0: the best token inside this CTA's best chunk
-        if (warp == 0) {
-            const unsigned long long cb = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
-            unsigned long long tb = 0ull;
-            if (cb != 0ull) {
-                const int cl = (int)key_id(cb) - (lo >> 8);
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const int j = quad_at(cl, h, lane), v0 = lo + j;
-                    float v[4];
-                    wt(j, v);
-                    const Words4 w = draw_block(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)(v0 >> 2));
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        float l;
-                        if (LOGITS) {
-                            if (v[k] == -INFINITY) continue;
-                            l = v[k];
-                        } else {
-                            if (!(v[k] > 0.f)) continue;
-                            l = logf(v[k]);
-                        }
-                        const unsigned long long pk = pack_key(__fadd_rn(l, gumbel_of(w.w[k])), (uint32_t)(v0 + k));
-                        tb = pk > tb ? pk : tb;
-                    }
-                }
-                tb = warp_max_u64(tb);
+        // 3. the best token inside this CTA's best chunk: one element per thread (threads
+        //    0..255), then the CTA's maximum
+        const unsigned long long cb = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
+        unsigned long long tb = 0ull;
+        if (cb != 0ull && threadIdx.x < kChunk) {
+            const int cl = (int)key_id(cb) - (lo >> 8);
+            const int e = threadIdx.x, j = cl * kChunk + (e & ~3), v = lo + cl * kChunk + e;
+            float q4[4];
+            wt(j, q4);
+            const float x = q4[e & 3];
+            const bool live = LOGITS ? x != -INFINITY : x > 0.f;
+            if (live) {
+                const float l = LOGITS ? x : logf(x);
+                const uint32_t w = draw_word(a.seed, kFinal, (uint32_t)b, (uint32_t)node, (uint32_t)v);
+                tb = pack_key(__fadd_rn(l, gumbel_of(w)), (uint32_t)v);
             }
+        }
+        tb = warp_max_u64(tb);
+        __syncthreads();  // every warp has read sh.wbest
+        if (lane == 0) sh.wbest[warp] = tb;
+        __syncthreads();
+        if (warp == 0) {
+            const unsigned long long t = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
             if (lane == 0) {
                 sh.cbest = cb;
-                sh.tbest = tb;
+                sh.tbest = t;
             }
         }
         __syncthreads();
@@ -391,8 +411,116 @@ __device__ FF q_log_normaliser(const float2 *st, int C) {
     return S.hi > 0.f ? ff_times_log2e(maxsum_lse(MaxSum{m, S})) : FF{0.f, 0.f};
 }
 
-// Shared-memory bytes of the tree's topology copy.
-inline size_t topo_bytes(int N) { return (size_t)(4 * N + 5) * sizeof(int32_t); }
+// Shared-memory bytes of the tree's copy: per node its pre-computed target log-normaliser
+// (float-float) and whether it has one; topology (child_off [N+2], child_ids [N], token [N+1],
+// q row of node [N+1]); per child slot its parent, target logit, q logit and uniform.
+inline size_t topo_bytes(int N) {
+    return (size_t)(N + 1) * sizeof(float2) + (size_t)(6 * N + 6) * sizeof(int32_t) + (size_t)3 * N * sizeof(float);
+}
+
+// Pre-pass. CTAs [0, B*M): CTA (b, j) streams target row j of tree b for its log-normaliser
+// (if node j has children).
+// Eight lanes own one 256-logit chunk (lane g reads logits 8g..8g+7 of each 64-logit
+// quarter); a warp takes four consecutive chunks per unit and two units (bf16; one for fp32)
+// per iteration, and every lane of a warp runs the same iterations and every shuffle (chunks
+// past the row contribute nothing). Each group folds its chunks' (max, sum) into a float-float
+// accumulator; groups, then warps, merge in a fixed order. CTAs from B*M on: one warp per
+// per-depth q row (tree b, depth d < Lq), from its chunk statistics.
+template <typename T>
+__global__ void __launch_bounds__(kPreThreads) k_verify_pre(VerifyArgs a) {
+    __shared__ Slot part[kPreThreads / 32];
+    constexpr int nwarps = kPreThreads / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int NN = a.N + 1;
+    const int ntarget = a.B * a.M;
+    if ((int)blockIdx.x >= ntarget) {  // q-row log-normalisers, one warp each
+        const int task = ((int)blockIdx.x - ntarget) * nwarps + warp;
+        if (task >= a.B * a.Lq) return;  // warp-uniform; no barrier in this branch
+        const int b = task / a.Lq, d = task - (task / a.Lq) * a.Lq;
+        const FF L2q = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + d) * a.C, a.C);
+        if (lane == 0) a.pre[(int64_t)b * NN + d].l2q = make_float2(L2q.hi, L2q.lo);
+        return;
+    }
+    const int b = (int)blockIdx.x / a.M, j = (int)blockIdx.x - ((int)blockIdx.x / a.M) * a.M;
+    {  // leaves need no normaliser
+        const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+        if (__ldg(off + j + 1) - __ldg(off + j) <= 0) return;  // uniform over the CTA
+    }
+    const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)j * a.t_rstride;
+    const int g = lane & 7, q = lane >> 3;
+    const float c2 = __fmul_rn(a.invT, kLog2e);
+    constexpr int kSweep = nwarps * 4;          // chunks covered by one unit of every warp
+    constexpr int kU = sizeof(T) == 2 ? 2 : 1;  // units in flight per warp (register budget)
+    float macc = -INFINITY;
+    FF sacc = FF{0.f, 0.f};
+    for (int c0 = warp * 4; c0 < a.C; c0 += kU * kSweep) {  // uniform over the warp
+        RawGroup<T> raw[kU][4];
+#pragma unroll
+        for (int e = 0; e < kU; ++e) {
+            const int c = c0 + e * kSweep + q;
+            if (c < a.C)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) raw[e][k].load(row, c * kChunk + k * 64 + g * 8, a.V);
+        }
+#pragma unroll
+        for (int e = 0; e < kU; ++e) {
+            const int c = c0 + e * kSweep + q;
+            const bool live = c < a.C;
+            float zm = -INFINITY;
+            if (live) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    float z[8];
+                    raw[e][k].unpack(z);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
+                }
+            }
+            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
+            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
+            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
+            const float mc = __fmul_rn(zm, a.invT);
+            const float off = __fmul_rn(mc, kLog2e);
+            float sc = 0.f;
+            if (live && mc != -INFINITY) {
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                    float z[8];
+                    raw[e][k].unpack(z);
+#pragma unroll
+                    for (int i = 0; i < 8; ++i) sc += fast_exp2(__fmaf_rn(z[i], c2, -off));
+                }
+            }
+            sc += __shfl_xor_sync(kFull, sc, 4);
+            sc += __shfl_xor_sync(kFull, sc, 2);
+            sc += __shfl_xor_sync(kFull, sc, 1);
+            if (live && mc != -INFINITY) {
+                if (mc > macc) {
+                    sacc = rescale_to(macc, sacc, mc);
+                    macc = mc;
+                }
+                sacc = ff_add(sacc, FF{mc == macc ? sc : __fmul_rn(sc, expf(__fsub_rn(mc, macc))), 0.f});
+            }
+        }
+    }
+    Slot mine = neutral_slot();
+    if (g == 0) {  // one contribution per group (its eight lanes hold the same values)
+        mine.m = macc;
+        mine.sh = sacc.hi;
+        mine.sl = sacc.lo;
+    }
+    const Slot w = warp_reduce_slot<kRedLse>(mine);
+    if (lane == 0) part[warp] = w;
+    __syncthreads();
+    if (warp == 0) {
+        const Slot v = warp_reduce_slot<kRedLse>(lane < nwarps ? part[lane] : neutral_slot());
+        if (lane == 0) {
+            const FF l = v.sh > 0.f ? maxsum_lse(MaxSum{v.m, FF{v.sh, v.sl}}) : FF{0.f, 0.f};
+            const FF L2 = ff_times_log2e(l);
+            a.pre[(int64_t)b * NN + j].l2t = make_float2(L2.hi, L2.lo);
+        }
+    }
+}
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
@@ -410,114 +538,160 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     const int n = max(0, min(a.V - lo, a.slice));
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const bool writer = crank == 0 && threadIdx.x == 0;
+    const bool per_depth = a.qrow_of_node == nullptr;
     int par = 0;
     Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
 
-    // the tree's topology: child_off [N+2], child_ids [N], token [N+1], q row of node [N+1]
-    int32_t *s_off = reinterpret_cast<int32_t *>(dyn + 2 * a.slice);
+    // the tree's copy in shared memory
+    FF *s_l2t = reinterpret_cast<FF *>(dyn + 2 * a.slice);  // [N+1] pre-computed normalisers
+    int32_t *s_pre = reinterpret_cast<int32_t *>(s_l2t + NN);  // [N+1] 1 if pre-computed
+    int32_t *s_off = s_pre + NN;
     int32_t *s_kid = s_off + (NN + 1);
     int32_t *s_tok = s_kid + a.N;
     int32_t *s_row = s_tok + NN;
+    int32_t *s_ps = s_row + NN;                             // [N] parent of each child slot
+    float *s_cxt = reinterpret_cast<float *>(s_ps + a.N);  // [N] per child slot
+    float *s_cxq = s_cxt + a.N;
+    float *s_cu = s_cxq + a.N;
     {
         const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
         const int32_t *kids = a.child_ids + (int64_t)b * a.N;
         const int32_t *tok = a.token + (int64_t)b * NN;
-        const int32_t *row = a.qrow_of_node ? a.qrow_of_node + (int64_t)b * NN : a.depth + (int64_t)b * NN;
+        const int32_t *row = per_depth ? a.depth + (int64_t)b * NN : a.qrow_of_node + (int64_t)b * NN;
         for (int i = threadIdx.x; i <= NN; i += kThreads) s_off[i] = __ldg(off + i);
-        for (int i = threadIdx.x; i < a.N; i += kThreads) s_kid[i] = __ldg(kids + i);
+        for (int i = threadIdx.x; i < a.N; i += kThreads) {
+            s_kid[i] = __ldg(kids + i);
+            s_ps[i] = -1;
+        }
         for (int i = threadIdx.x; i < NN; i += kThreads) {
             s_tok[i] = __ldg(tok + i);
             s_row[i] = __ldg(row + i);
         }
+        for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
+            const float2 v = a.pre[(int64_t)b * NN + i].l2q;
+            sh.l2q[i] = FF{v.x, v.y};
+        }
+        if (threadIdx.x == 0) sh.cbad = 0;
+    }
+    __syncthreads();
+    {  // every valid internal node claims its child slots
+        bool bad_here = false;
+        for (int u = threadIdx.x; u < NN; u += kThreads) {
+            const int o = s_off[u], m = s_off[u + 1] - o;
+            if (m == 0) continue;
+            const int r = s_row[u];
+            if (m < 0 || m > kMaxK || o < 0 || o + m > a.N || r < 0 || r >= a.q_R || (per_depth && r >= a.Lq)) {
+                bad_here = true;
+                continue;
+            }
+            for (int i = 0; i < m; ++i) s_ps[o + i] = u;
+        }
+        if (bad_here) sh.cbad = 1;
+    }
+    __syncthreads();
+    for (int u = threadIdx.x; u < NN; u += kThreads) {  // the pre-computed set, as the pre-pass saw it
+        const bool p = u < a.M && s_off[u + 1] - s_off[u] > 0;
+        s_pre[u] = p ? 1 : 0;
+        if (p) {
+            const float2 v = a.pre[(int64_t)b * NN + u].l2t;
+            s_l2t[u] = FF{v.x, v.y};
+        }
+    }
+    {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
+        bool bad_here = false;
+        for (int j = threadIdx.x; j < a.N; j += kThreads) {
+            const int u = s_ps[j];
+            if (u < 0) continue;  // not a child slot of a valid node (never read by the walk)
+            const int c = s_kid[j];
+            const int y = (c >= 1 && c <= a.N) ? s_tok[c] : -1;
+            if (y < 0 || y >= a.V) {
+                bad_here = true;
+                continue;
+            }
+            const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
+            const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)s_row[u] * a.q_rstride;
+            s_cxt[j] = __fmul_rn(Logit<T>::load1(trow, y), a.invT);
+            s_cxq[j] = __fmul_rn(Logit<T>::load1(qrow, y), a.invT);
+            s_cu[j] = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
+        }
+        if (bad_here) sh.cbad = 1;
     }
     int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
     int32_t *onode = a.out_nodes + (int64_t)b * a.L;
 
-    cluster.sync();  // topology visible; every CTA of the cluster runs before any distributed access
+    cluster.sync();  // the copy is complete; every CTA of the cluster runs before any distributed access
 
     int u = 0, nacc = 0, final_tok = -1;
-    bool bad = false;
-    for (int step = 0; step <= a.L; ++step) {
+    bool bad = sh.cbad != 0;  // every CTA checked the same arrays
+    for (int step = 0; step <= a.L && !bad; ++step) {
         const int o = s_off[u], m = s_off[u + 1] - o;
-        if (m < 0 || m > kMaxK || o < 0 || o + m > a.N) {
-            bad = true;
-            break;
-        }
         const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
         if (m == 0) {  // leaf: bonus token from the node's target row
             final_tok = W.draw_from_row(trow, u);
             break;
         }
         const int r = s_row[u];
-        if (r < 0 || r >= a.q_R) {
-            bad = true;
-            break;
-        }
         const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
-        {  // likely next reads: this node's q row (first rejection), the first child's target row
-            W.prefetch_slice(qrow);
-            const int c0 = s_kid[o];
-            if (c0 >= 1 && c0 <= a.N)
-                W.prefetch_slice(static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride +
-                                 (int64_t)c0 * a.t_rstride);
-        }
-        __syncthreads();  // the previous node's readers of P, Q and the child data are done
-
-        // staging (warps 0..13) with the target log-normaliser; q normaliser (warp 14);
-        // child data (warp 15)
-        OnlineLse lt;
-        if (warp < kStageWarps) {
-            W.template stage<false>(trow, P, kStageWarps, &lt, FF{0.f, 0.f});
-        } else if (warp == kQWarp) {
-            const FF L2q = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
-            if (lane == 0) sh.L2q = L2q;
-        } else {
-            bool cb = false;
-            if (lane < m) {
-                const int c = s_kid[o + lane];
-                const int y = (c >= 1 && c <= a.N) ? s_tok[c] : -1;
-                if (y < 0 || y >= a.V) {
-                    cb = true;
-                } else {
-                    sh.cxt[lane] = __fmul_rn(Logit<T>::load1(trow, y), a.invT);
-                    sh.cxq[lane] = __fmul_rn(Logit<T>::load1(qrow, y), a.invT);
-                    sh.cu[lane] = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
-                    sh.cnode[lane] = c;
+        const bool pre = s_pre[u] != 0;
+        bool staged = !pre;  // P holds this node's x
+        FF L2t, L2q;
+        if (pre) {
+            L2t = s_l2t[u];
+            if (per_depth) {
+                L2q = sh.l2q[r];
+            } else {
+                __syncthreads();
+                if (warp == kQWarp) {
+                    const FF v = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
+                    if (lane == 0) sh.L2q = v;
                 }
+                __syncthreads();
+                L2q = sh.L2q;
             }
-            cb = __any_sync(kFull, cb);
-            if (lane == 0) sh.cbad = cb ? 1 : 0;
-        }
-        {
+        } else {
+            {  // likely next reads: this node's q row (first rejection), the first child's target row
+                W.prefetch_slice(qrow);
+                W.prefetch_slice(static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride +
+                                 (int64_t)s_kid[o] * a.t_rstride);
+            }
+            __syncthreads();  // earlier readers of P and Q are done
+            // staging with the target log-normaliser; a per-node q row's normaliser on warp 14
+            const int nstage = per_depth ? kStageWarps + 1 : kStageWarps;
+            OnlineLse lt;
+            if (warp < nstage) {
+                W.template stage<false>(trow, P, nstage, &lt, FF{0.f, 0.f});
+            } else if (warp == kQWarp) {
+                const FF v = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
+                if (lane == 0) sh.L2q = v;
+            }
             Slot mine = neutral_slot();
             const MaxSum t1 = lt.value();
             mine.m = t1.m;
             mine.sh = t1.s.hi;
             mine.sl = t1.s.lo;
             reduce_round<kRedLse>(sh, par, cluster, mine);
+            L2t = sh.L2t;
+            L2q = per_depth ? sh.l2q[r] : sh.L2q;
         }
-        if (sh.cbad) {
-            bad = true;
-            break;
-        }
-        const FF L2t = sh.L2t, L2q = sh.L2q;
         FF t = FF{1.f, 0.f};  // draft mass not yet drawn
         int accepted = -1;
         bool q_staged = false;
         for (int i = 0; i < m; ++i) {
             const float it = t.hi > 0.f ? __frcp_rn(t.hi) : 0.f;  // 1/t_i
-            const float P0y = exp_shifted(sh.cxt[i], L2t);
-            const float Qy = exp_shifted(sh.cxq[i], L2q);
+            const float P0y = exp_shifted(s_cxt[o + i], L2t);
+            const float Qy = exp_shifted(s_cxq[o + i], L2q);
             const float pp = point_residual(P0y, Qy, sh.izs, sh.its, i);
             const float qp = __fmul_rn(Qy, it);
-            if (__fmul_rn(sh.cu[i], qp) < pp) {
-                accepted = sh.cnode[i];
+            if (__fmul_rn(s_cu[o + i], qp) < pp) {
+                accepted = s_kid[o + i];
                 break;
             }
-            if (!q_staged) {  // the normalised q slice, once per node
+            if (!staged || !q_staged) {  // the slices a rejection needs, once per node
+                __syncthreads();         // earlier readers of P and Q are done
+                if (!staged) W.template stage<false>(trow, P, kWarps, nullptr, FF{0.f, 0.f});
                 W.template stage<true>(qrow, Q, kWarps, nullptr, L2q);
                 __syncthreads();
-                q_staged = true;
+                staged = q_staged = true;
             }
             // p_i(v) of the quad at smem index j (P holds x before the first rejection, R_i
             // afterwards)
@@ -583,20 +757,21 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             __syncthreads();
             t = ff_add(t, FF{-Qy, 0.f});
         }
-        if (bad || accepted < 0) break;
+        if (accepted < 0) break;
         if (nacc >= a.L) {  // deeper than the depth cap: the tree arrays are inconsistent
             bad = true;
             break;
         }
-        if (writer) {
-            otok[nacc] = s_tok[accepted];
-            onode[nacc] = accepted;
-        }
+        if (writer) sh.path[nacc] = accepted;  // no global store while cluster barriers follow
         ++nacc;
         u = accepted;
     }
     if (writer) {
         if (bad) raise_status(a.status, kDevBadTree);
+        for (int k = 0; k < nacc; ++k) {
+            otok[k] = s_tok[sh.path[k]];
+            onode[k] = sh.path[k];
+        }
         otok[nacc] = final_tok;
         for (int k = nacc + 1; k <= a.L; ++k) otok[k] = -1;
         for (int k = nacc; k < a.L; ++k) onode[k] = -1;
@@ -704,6 +879,13 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
         e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
     }
+    const int64_t pre_blocks = (int64_t)B * a.M + ((int64_t)B * a.Lq + kPreThreads / 32 - 1) / (kPreThreads / 32);
+    if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    if (pre_blocks > 0) {
+        k_verify_pre<T><<<(unsigned)pre_blocks, kPreThreads, 0, s>>>(a);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)(B * cs), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
@@ -752,6 +934,11 @@ cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const f
     a.out_nodes = out_nodes;
     a.out_len = out_len;
     a.status = status;
+    // the pre-pass results use the workspace's per-(tree, node) slots (status word is ws[0])
+    a.pre = reinterpret_cast<PreRow *>(reinterpret_cast<char *>(status) + kWsStatusBytes);
+    a.M = N + 1 < kPreTop ? N + 1 : kPreTop;
+    a.Lq = qrow_of_node ? 0 : (L < N + 1 ? L : N + 1);
+    a.B = B;
     if (target.dtype == 1) return launch_rrs_t<__nv_bfloat16>(a, B, s);
     return launch_rrs_t<float>(a, B, s);
 }

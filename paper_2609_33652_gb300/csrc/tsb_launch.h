@@ -24,7 +24,8 @@ inline int num_chunks(int V) { return (V + 255) / 256; }
 
 // Workspace layout (caller-owned, 256-byte aligned):
 //   [0, 256)                       sticky status word
-//   B*(N+1) x 32 bytes             per-(tree, chain position) scalars of block verification
+//   B*(N+1) x 32 bytes             per-(tree, node) scalars: block verification's per-position
+//                                  values, or the verifier pre-pass's log-normalisers
 //   B*L float2, B*L*K floats,      per-draft-row log-normaliser (float-float) and top-K
 //   B*L*K int32                    (x, id) of the first pass
 constexpr size_t kWsStatusBytes = 256;
