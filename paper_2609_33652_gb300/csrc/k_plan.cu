@@ -1,11 +1,12 @@
 // First pass (Sec. 3.1; max-heap expansion as in DDTree, Sec. 2.2 / App. B.3), two kernels.
 //
-// k_row_topk, one warp per draft row (every row of the batch in parallel): the row's chunk
-//   statistics are staged in shared memory, merged into the log-normaliser LSE_d, and give
-//   tau = the K-th largest chunk maximum, a lower bound on the K-th largest logit (K distinct
-//   chunk maxima reach it). Only chunks whose maximum reaches tau are re-read; their logits
-//   >= tau go through per-lane sorted lists, and a warp merge yields the top-K by
-//   (x desc, id asc). Results go to the workspace.
+// k_row_topk, one 4-warp CTA per draft row (every row of the batch in parallel): the row's
+//   chunk statistics are staged in shared memory (one round of loads), merged into the
+//   log-normaliser LSE_d, and give tau = the K-th largest chunk maximum, a lower bound on the
+//   K-th largest logit (K distinct chunk maxima reach it). Only chunks whose maximum reaches
+//   tau are re-read, spread over the warps; their logits >= tau go through per-lane sorted
+//   lists, and warp then CTA merges yield the top-K by (x desc, id asc). Results go to the
+//   workspace.
 // k_plan_heap, one CTA per tree: best-first expansion, popping N candidates. A candidate at
 //   depth d holds the sum Sx of its path's logits (exact, in 64-bit fixed point) and the key
 //   Sx - CL[d], CL[d] = LSE_1 + ... + LSE_d (its draft path log-probability). Pop order:
@@ -22,7 +23,8 @@
 namespace tsb {
 namespace {
 
-constexpr int kTopkWarps = 4;
+constexpr int kTopkThreads = 128;
+constexpr int kTopkWarps = kTopkThreads / 32;
 constexpr int kHeapThreads = 128;
 
 struct TopkArgs {
@@ -36,57 +38,86 @@ struct TopkArgs {
     int32_t *topk_id;  // [B*L*K]
 };
 
+// Top n keys of a warp's lanes' lists into dst[0..n) (lane 0 writes).
+template <int CAP>
+__device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t *dst) {
+    for (int j = 0; j < n; ++j) {
+        const uint64_t best = warp_pop_max(list);
+        if ((threadIdx.x & 31) == 0) dst[j] = best;
+    }
+}
+
 template <int KCAP, typename T>
-__global__ void __launch_bounds__(kTopkWarps * 32) k_row_topk(TopkArgs a) {
-    extern __shared__ __align__(16) float2 st_all[];
+__global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
+    extern __shared__ __align__(16) float2 st[];  // [C] the row's chunk statistics
+    __shared__ uint64_t wl[kTopkWarps][KCAP];
+    __shared__ float wm[kTopkWarps], wsh[kTopkWarps], wsl[kTopkWarps];
+    __shared__ float s_tau;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int row = blockIdx.x * kTopkWarps + warp;
-    if (row >= a.B * a.L) return;  // warp-uniform; no block-wide barrier below
+    const int row = blockIdx.x;
     const int b = row / a.L, d = row - (row / a.L) * a.L;
     const int C = a.C, K = a.K;
-    float2 *st = st_all + (size_t)warp * C;
     const float2 *gst = a.stats + ((int64_t)b * a.R + d) * C;
-    // stage the row's chunk statistics (eight independent loads in flight per lane)
-    for (int c0 = lane; c0 < C; c0 += 32 * 8) {
+    // 1. stage the statistics (eight loads in flight per thread); per-thread maximum and list
+    //    of chunk maxima
+    TopList<KCAP> cl;
+    cl.clear();
+    float m = -INFINITY;
+    for (int c0 = threadIdx.x; c0 < C; c0 += kTopkThreads * 8) {
         float2 v[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int c = c0 + 32 * k;
-            v[k] = c < C ? gst[c] : make_float2(-INFINITY, 0.f);
+        for (int e = 0; e < 8; ++e) {
+            const int c = c0 + kTopkThreads * e;
+            v[e] = c < C ? __ldg(&gst[c]) : make_float2(-INFINITY, 0.f);
         }
 #pragma unroll
-        for (int k = 0; k < 8; ++k) {
-            const int c = c0 + 32 * k;
-            if (c < C) st[c] = v[k];
+        for (int e = 0; e < 8; ++e) {
+            const int c = c0 + kTopkThreads * e;
+            if (c < C) {
+                st[c] = v[e];
+                m = fmaxf(m, v[e].x);
+                cl.insert(pack_key(v[e].x, (uint32_t)c));
+            }
         }
     }
-    __syncwarp();
-    // log-normaliser (float-float; the lane partials merge in a butterfly)
-    float m = -INFINITY;
-    for (int c = lane; c < C; c += 32) m = fmaxf(m, st[c].x);
+    // 2. log-normaliser partials (float-float) over the thread's own chunks, then per warp
     KahanF acc;
     if (m != -INFINITY)
-        for (int c = lane; c < C; c += 32) acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
-    const MaxSum tot = warp_maxsum(MaxSum{m, acc.ff()});
+        for (int c = threadIdx.x; c < C; c += kTopkThreads)
+            acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
+    const MaxSum ms = warp_maxsum(MaxSum{m, acc.ff()});
     if (lane == 0) {
-        const FF l = maxsum_lse(tot);
-        a.lse[row] = make_float2(l.hi, l.lo);
+        wm[warp] = ms.m;
+        wsh[warp] = ms.s.hi;
+        wsl[warp] = ms.s.lo;
     }
-    // tau = K-th largest chunk maximum (-inf with fewer than K chunks)
-    float tau = -INFINITY;
-    if (C >= K) {
-        TopList<KCAP> cl;
-        cl.clear();
-        for (int c = lane; c < C; c += 32) cl.insert(pack_key(st[c].x, (uint32_t)c));
+    // 3. each warp's K largest chunk maxima
+    warp_top_to(cl, K, wl[warp]);
+    __syncthreads();
+    if (warp == 0) {
+        MaxSum v = lane < kTopkWarps ? MaxSum{wm[lane], FF{wsh[lane], wsl[lane]}} : MaxSum{-INFINITY, FF{0.f, 0.f}};
+        v = warp_maxsum(v);
+        if (lane == 0) {
+            const FF l = maxsum_lse(v);
+            a.lse[row] = make_float2(l.hi, l.lo);
+        }
+        // tau = K-th largest chunk maximum (-inf with fewer than K chunks): a lower bound on
+        // the K-th largest logit, since K distinct chunk maxima reach it
+        TopList<KCAP> t;
+        t.clear();
+        for (int e = lane; e < kTopkWarps * K; e += 32) t.insert(wl[e / K][e % K]);
         uint64_t kth = 0;
-        for (int j = 0; j < K; ++j) kth = warp_pop_max(cl);
-        tau = key_value(kth);
+        for (int j = 0; j < K; ++j) kth = warp_pop_max(t);
+        if (lane == 0) s_tau = C >= K ? key_value(kth) : -INFINITY;
     }
-    // top-K logits among the chunks whose maximum reaches tau, four chunks per batch
+    __syncthreads();
+    const float tau = s_tau;
+    // 4. the logits >= tau of the chunks whose maximum reaches tau; a chunk goes to the warp
+    //    that scans it, four chunks' loads per batch
     const T *rowp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
     TopList<KCAP> el;
     el.clear();
-    for (int cb = 0; cb < C; cb += 32) {
+    for (int cb = warp * 32; cb < C; cb += kTopkThreads) {
         const int c = cb + lane;
         unsigned mask = __ballot_sync(kFull, c < C && st[c].x >= tau);
         while (mask) {
@@ -118,11 +149,19 @@ __global__ void __launch_bounds__(kTopkWarps * 32) k_row_topk(TopkArgs a) {
             }
         }
     }
-    for (int j = 0; j < K; ++j) {
-        const uint64_t best = warp_pop_max(el);
-        if (lane == 0) {
-            a.topk_id[(int64_t)row * K + j] = (int32_t)key_id(best);
-            a.topk_x[(int64_t)row * K + j] = key_value(best);
+    // 5. per warp top-K, then the CTA's
+    warp_top_to(el, K, wl[warp]);  // warp 0 finished reading wl before the barrier above
+    __syncthreads();
+    if (warp == 0) {
+        TopList<KCAP> t;
+        t.clear();
+        for (int e = lane; e < kTopkWarps * K; e += 32) t.insert(wl[e / K][e % K]);
+        for (int j = 0; j < K; ++j) {
+            const uint64_t best = warp_pop_max(t);
+            if (lane == 0) {
+                a.topk_id[(int64_t)row * K + j] = (int32_t)key_id(best);
+                a.topk_x[(int64_t)row * K + j] = key_value(best);
+            }
         }
     }
 }
@@ -160,47 +199,66 @@ __device__ __forceinline__ unsigned long long okey_of(long long key) {
 __device__ __forceinline__ long long key_of_okey(unsigned long long o) { return (long long)(o ^ 0x8000000000000000ull); }
 __device__ __forceinline__ long long fix_of(float x) { return __float2ll_rn(__fmul_rn(x, kFixScale)); }
 
+// A 32-bit image of an okey, monotone non-decreasing: keys in [-2^41, 2^41) (|log-probability|
+// below 2048) at 2^-20 resolution, clamped outside; an empty slot (0) maps to 0. Equal images
+// are resolved on the full key.
+__device__ __forceinline__ unsigned coarse_of(unsigned long long okey) {
+    constexpr unsigned long long kBase = 0x8000000000000000ull - (1ull << 41);
+    if (okey < kBase) return 0u;
+    const unsigned long long c = (okey - kBase) >> 10;
+    return c > 0xffffffffull ? 0xffffffffu : (unsigned)c;
+}
+
 template <int S>
 struct Slots {
-    unsigned long long k[S];
-    unsigned w[S];
-    unsigned long long bk;  // the lane's best
+    unsigned long long k[S];  // okey
+    unsigned w[S];            // tie word
+    long long x[S];           // the candidate's path sum Sx (fixed point)
+    unsigned long long bk;    // the lane's best
     unsigned bw;
+    long long bx;
     int bs;
     __device__ __forceinline__ void clear() {
 #pragma unroll
         for (int s = 0; s < S; ++s) {
             k[s] = 0ull;
             w[s] = 0u;
+            x[s] = 0;
         }
         bk = 0ull;
         bw = 0u;
+        bx = 0;
         bs = 0;
     }
-    __device__ __forceinline__ void put(int slot, unsigned long long kk, unsigned ww) {
+    // Predicated writes of slot `slot` (every lane runs the same instructions).
+    __device__ __forceinline__ void put_if(bool p, int slot, unsigned long long kk, unsigned ww, long long xx) {
 #pragma unroll
-        for (int s = 0; s < S; ++s)
-            if (s == slot) {
-                k[s] = kk;
-                w[s] = ww;
-            }
+        for (int s = 0; s < S; ++s) {
+            const bool hit = p && s == slot;
+            k[s] = hit ? kk : k[s];
+            w[s] = hit ? ww : w[s];
+            x[s] = hit ? xx : x[s];
+        }
     }
     __device__ __forceinline__ void rescan() {
         bk = 0ull;
         bw = 0u;
+        bx = 0;
         bs = 0;
 #pragma unroll
-        for (int s = 0; s < S; ++s)
-            if (key_better(k[s], w[s], bk, bw)) {
-                bk = k[s];
-                bw = w[s];
-                bs = s;
-            }
+        for (int s = 0; s < S; ++s) {
+            const bool better = key_better(k[s], w[s], bk, bw);
+            bk = better ? k[s] : bk;
+            bw = better ? w[s] : bw;
+            bx = better ? x[s] : bx;
+            bs = better ? s : bs;
+        }
     }
 };
 
-// Best-first expansion for one tree with one warp. Each pop: a three-stage warp maximum of
-// the lanes' best keys (__reduce_max_sync on the high word, low word, tie word); the popped
+// Best-first expansion for one tree with one warp. Each pop: a warp maximum of the lanes'
+// best keys, one __reduce_max_sync on a 32-bit monotone image of the key, refined on the
+// full key (high word, low word, tie word) only among lanes whose images tie; the popped
 // candidate's slot takes its next sibling; its first child goes to the next round-robin
 // slot (children are numbered in creation order, lane = c % 32, slot = c / 32).
 template <int S>
@@ -208,7 +266,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     extern __shared__ __align__(16) unsigned char smem[];
     const int L = a.L, N = a.N, K = a.K, NN = N + 1;
     long long *CL = reinterpret_cast<long long *>(smem);           // [L+1] fixed point
-    long long *n_sx = CL + (L + 1);                                // [NN] node path sums
+    long long *n_sx = CL + (L + 1);                                // [NN] raw pop keys
     long long *fx = n_sx + NN;                                     // [L*K] candidate logits
     int32_t *n_parent = reinterpret_cast<int32_t *>(fx + L * K);   // [NN]
     int32_t *n_depth = n_parent + NN;
@@ -254,26 +312,28 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     }
     __syncthreads();
 
+    // The expansion (warp 0). Per pop the critical path is the warp maximum, three shuffles,
+    // the decode, independent shared loads of the candidate logits and depth normalisers, and
+    // predicated slot updates: no dependent load of the parent's path sum (each slot carries
+    // its own) and no divergent branch. Each pop's tie word and key are stored raw and
+    // decoded after the loop by all threads.
+    unsigned *rec_w = reinterpret_cast<unsigned *>(n_rank);  // [NN], 0 = not popped
+    long long *rec_k = n_sx;                                  // [NN]
     if (warp == 0) {
-        if (lane == 0) {
-            n_parent[0] = -1;
-            n_depth[0] = 0;
-            n_rank[0] = -1;
-            n_token[0] = -1;
-        }
         Slots<S> fr;
         fr.clear();
-        if (lane == 0) {  // the root's first child (depth 1, rank 0) is child number 0
-            fr.put(0, okey_of(fx[0] - CL[1]), w3_of(1, 0, 0));
-            fr.rescan();
-        }
+        // the root's first child (depth 1, rank 0) is child number 0: lane 0, slot 0
+        fr.put_if(lane == 0, 0, okey_of(fx[0] - CL[1]), w3_of(1, 0, 0), fx[0]);
+        fr.rescan();
         int nchild = 1;
-        __syncwarp();
         for (int i = 1; i <= N; ++i) {
-            const unsigned hk = (unsigned)(fr.bk >> 32);
-            const unsigned m1 = __reduce_max_sync(kFull, hk);
-            unsigned c = __ballot_sync(kFull, hk == m1);
-            if (__popc(c) > 1) {  // the high word ties: resolve with the low word, then w3
+            const unsigned ck = coarse_of(fr.bk);
+            const unsigned m0 = __reduce_max_sync(kFull, ck);
+            unsigned c = __ballot_sync(kFull, ck == m0);
+            if (__popc(c) > 1) {  // coarse keys tie: the full key (high word, low word), then w3
+                const unsigned hk = (unsigned)(fr.bk >> 32);
+                const unsigned m1 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? hk : 0u);
+                c &= __ballot_sync(kFull, hk == m1);
                 const unsigned lk = (unsigned)fr.bk;
                 const unsigned m2 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? lk : 0u);
                 c &= __ballot_sync(kFull, lk == m2);
@@ -285,6 +345,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
             const int winner = __ffs(c) - 1;
             const unsigned long long wk = __shfl_sync(kFull, fr.bk, winner);
             const unsigned ww = __shfl_sync(kFull, fr.bw, winner);
+            const long long wx = __shfl_sync(kFull, fr.bx, winner);
             if (ww == 0u) {  // frontier exhausted: only with N above the tree's capacity
                 if (lane == 0) raise_status(a.status, kDevBadTree);
                 break;
@@ -293,42 +354,42 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
             const int parent = 65535 - (int)((ww >> 8) & 0xffffu);
             const int rank = 255 - (int)(ww & 0xffu);
             const bool sib = rank + 1 < K, kid = depth < L;
-            // every lane computes the popped path's sum and both new keys from broadcast loads;
-            // only the commits below differ per lane
-            const long long sp = n_sx[parent];
-            const long long sx = sp + fx[(depth - 1) * K + rank];
-            const long long ks = sp + (sib ? fx[(depth - 1) * K + rank + 1] : 0) - CL[depth];
-            const long long kc = sx + (kid ? fx[depth * K] : 0) - CL[kid ? depth + 1 : depth];
-            if (lane == winner) {  // the next sibling takes the freed slot
-                if (sib)
-                    fr.put(fr.bs, okey_of(ks), w3_of(depth, parent, rank + 1));
-                else
-                    fr.put(fr.bs, 0ull, 0u);
-                fr.rescan();
-            }
+            const long long fr0 = fx[(depth - 1) * K + rank];
+            const long long fn = sib ? fx[(depth - 1) * K + rank + 1] : 0;
+            const long long f0 = kid ? fx[depth * K] : 0;
+            const long long cd = CL[depth], cd1 = kid ? CL[depth + 1] : 0;
+            const long long xs = wx - fr0 + fn, xc = wx + f0;  // sibling's and first child's Sx
+            // the next sibling takes the popped slot; the first child the next round-robin slot
+            fr.put_if(lane == winner, fr.bs, sib ? okey_of(xs - cd) : 0ull, sib ? w3_of(depth, parent, rank + 1) : 0u,
+                      xs);
+            fr.put_if(kid && lane == (nchild & 31), nchild >> 5, okey_of(xc - cd1), w3_of(depth + 1, i, 0), xc);
+            fr.rescan();
             if (lane == 0) {
-                n_parent[i] = parent;
-                n_depth[i] = depth;
-                n_rank[i] = rank;
-                n_token[i] = tk_id[(depth - 1) * K + rank];
-                n_score[i] = __fmul_rn(__ll2float_rn(key_of_okey(wk)), kFixInv);
-                n_sx[i] = sx;
+                rec_w[i] = ww;
+                rec_k[i] = (long long)wk;
             }
-            if (kid) {  // first child (i, 0), one level down, in the next round-robin slot
-                if (lane == (nchild & 31)) {
-                    const unsigned long long ck = okey_of(kc);
-                    const unsigned cw = w3_of(depth + 1, i, 0);
-                    fr.put(nchild >> 5, ck, cw);
-                    if (key_better(ck, cw, fr.bk, fr.bw)) {
-                        fr.bk = ck;
-                        fr.bw = cw;
-                        fr.bs = nchild >> 5;
-                    }
-                }
-                ++nchild;
-            }
-            __syncwarp();
+            nchild += kid ? 1 : 0;
         }
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < NN; i += kHeapThreads) {  // decode the records
+        if (i == 0) {
+            n_parent[0] = -1;
+            n_depth[0] = 0;
+            n_rank[0] = -1;
+            n_token[0] = -1;
+            n_score[0] = 0.f;
+            continue;
+        }
+        const unsigned ww = rec_w[i];
+        if (ww == 0u) continue;  // not popped (the expansion stopped early)
+        const int depth = 255 - (int)(ww >> 24);
+        const int rank = 255 - (int)(ww & 0xffu);
+        n_parent[i] = 65535 - (int)((ww >> 8) & 0xffffu);
+        n_depth[i] = depth;
+        n_rank[i] = rank;
+        n_token[i] = tk_id[(depth - 1) * K + rank];
+        n_score[i] = __fmul_rn(__ll2float_rn(key_of_okey((unsigned long long)rec_k[i])), kFixInv);
     }
     __syncthreads();
 
@@ -387,11 +448,10 @@ cudaError_t launch_heap_t(const HeapArgs &h, int B, cudaStream_t s) {
 
 template <int KCAP, typename T>
 cudaError_t launch_topk_t(const TopkArgs &a, cudaStream_t s) {
-    const size_t smem = (size_t)kTopkWarps * a.C * sizeof(float2);
+    const size_t smem = (size_t)a.C * sizeof(float2);
     cudaError_t e = cudaFuncSetAttribute(k_row_topk<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    const int rows = a.B * a.L;
-    k_row_topk<KCAP, T><<<(rows + kTopkWarps - 1) / kTopkWarps, kTopkWarps * 32, smem, s>>>(a);
+    k_row_topk<KCAP, T><<<(unsigned)(a.B * a.L), kTopkThreads, smem, s>>>(a);
     return cudaGetLastError();
 }
 
@@ -443,6 +503,7 @@ cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N
     const int per_lane = (N + 1 + 31) / 32;
     if (per_lane <= 1) return launch_heap_t<1>(h, draft.B, s);
     if (per_lane <= 2) return launch_heap_t<2>(h, draft.B, s);
+    if (per_lane <= 3) return launch_heap_t<3>(h, draft.B, s);
     if (per_lane <= 4) return launch_heap_t<4>(h, draft.B, s);
     if (per_lane <= 8) return launch_heap_t<8>(h, draft.B, s);
     if (per_lane <= 16) return launch_heap_t<16>(h, draft.B, s);
@@ -490,6 +551,7 @@ cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int 
     const int per_lane = (N + 1 + 31) / 32;
     if (per_lane <= 1) return launch_heap_t<1>(h, draft.B, s);
     if (per_lane <= 2) return launch_heap_t<2>(h, draft.B, s);
+    if (per_lane <= 3) return launch_heap_t<3>(h, draft.B, s);
     if (per_lane <= 4) return launch_heap_t<4>(h, draft.B, s);
     if (per_lane <= 8) return launch_heap_t<8>(h, draft.B, s);
     if (per_lane <= 16) return launch_heap_t<16>(h, draft.B, s);

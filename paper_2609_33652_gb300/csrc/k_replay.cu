@@ -14,7 +14,7 @@
 // be among the top m_u: the joint law is exactly that of flat Gumbel-top-k over V tokens,
 // at ceil(V/256) + m_u*256 draws per parent instead of V.
 //
-// One CTA of 8 warps per (tree, node); nodes without children return at once. Chunk keys are
+// One CTA of 4 warps per (tree, node); nodes without children return at once. Chunk keys are
 // spread over the CTA (four chunks per thread share one Philox block), each warp then takes
 // one kept chunk, and per-warp candidate lists are merged in shared memory.
 #include "tsb_device.cuh"
@@ -23,8 +23,11 @@
 namespace tsb {
 namespace {
 
-constexpr int kWarps = 8;
+constexpr int kWarps = 4;
 constexpr int kThreads = kWarps * 32;
+// 4 warps and at most 64 registers: eight CTAs per SM, so a batch's B*(N+1) CTAs (1,040 at
+// B=16, N=64) are resident in one wave (leaf nodes' CTAs exit at once).
+constexpr int kMinBlocks = 8;
 
 struct ReplayArgs {
     const void *q;
@@ -67,7 +70,7 @@ __device__ __forceinline__ void merge_warps(const uint64_t (*cand)[CAP], int n, 
 }
 
 template <int KCAP, typename T>
-__global__ void __launch_bounds__(kThreads) k_replay(ReplayArgs a) {
+__global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay(ReplayArgs a) {
     __shared__ uint64_t cand[kWarps][KCAP];
     __shared__ uint64_t sel[KCAP];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
