@@ -38,13 +38,18 @@ struct TopkArgs {
     int32_t *topk_id;  // [B*L*K]
 };
 
-// Top n keys of a warp's lanes' lists into dst[0..n) (lane 0 writes).
+// Top n keys of a warp's lanes' lists into dst[0..n) (lane 0 writes; zeros once the lists
+// are empty, without further pops).
 template <int CAP>
 __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t *dst) {
-    for (int j = 0; j < n; ++j) {
+    int j = 0;
+    for (; j < n; ++j) {
         const uint64_t best = warp_pop_max(list);
         if ((threadIdx.x & 31) == 0) dst[j] = best;
+        if (best == 0ull) break;  // uniform over the warp
     }
+    if ((threadIdx.x & 31) == 0)
+        for (++j; j < n; ++j) dst[j] = 0ull;
 }
 
 template <int KCAP, typename T>

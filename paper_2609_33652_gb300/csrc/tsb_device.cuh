@@ -286,6 +286,12 @@ struct TopList {
         for (int i = 0; i < CAP - 1; ++i) k[i] = k[i + 1];
         k[CAP - 1] = 0ull;
     }
+    // pop_front where p holds, as selects (no branch: every lane runs the same instructions)
+    __device__ __forceinline__ void pop_front_if(bool p) {
+#pragma unroll
+        for (int i = 0; i < CAP - 1; ++i) k[i] = p ? k[i + 1] : k[i];
+        k[CAP - 1] = p ? 0ull : k[CAP - 1];
+    }
 };
 
 // The largest of the lanes' 64-bit values (distinct unless zero): a hardware max over the
@@ -310,7 +316,7 @@ template <int CAP>
 __device__ __forceinline__ uint64_t warp_pop_max(TopList<CAP> &list) {
     int owner;
     const uint64_t best = warp_max_u64_owner(list.k[0], &owner);
-    if ((threadIdx.x & 31) == owner && best != 0ull) list.pop_front();
+    list.pop_front_if((threadIdx.x & 31) == owner && best != 0ull);
     return best;
 }
 
