@@ -127,6 +127,7 @@ __device__ __forceinline__ const T *qrow_ptr(const BvArgs &a, int b, int r) {
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) k_bv_rows(BvArgs a) {
+    pdl_begin();
     __shared__ BlockRed sh;
     const int g = a.N, NN = a.N + 1;
     const int b = blockIdx.x / NN, i = blockIdx.x - b * NN;
@@ -203,6 +204,7 @@ __device__ float chain_weights(const BvArgs &a, int b, int upto, float *w_all) {
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) k_bv_resid(BvArgs a) {
+    pdl_begin();
     __shared__ BlockRed sh;
     __shared__ float w_sh;
     __shared__ int ok_sh;
@@ -254,6 +256,7 @@ __global__ void __launch_bounds__(kThreads) k_bv_resid(BvArgs a) {
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads) k_bv_final(BvArgs a) {
+    pdl_begin();
     __shared__ BlockRed sh;
     __shared__ int tau_sh, ok_sh;
     __shared__ float wtau_sh;
@@ -392,14 +395,11 @@ __global__ void __launch_bounds__(kThreads) k_bv_final(BvArgs a) {
 template <typename T>
 cudaError_t launch_bv_t(const BvArgs &a, int B, cudaStream_t s) {
     const int NN = a.N + 1;
-    k_bv_rows<T><<<(unsigned)(B * NN), kThreads, 0, s>>>(a);
-    cudaError_t e = cudaGetLastError();
+    cudaError_t e = launch_pdl(k_bv_rows<T>, dim3((unsigned)(B * NN)), dim3(kThreads), 0, s, 0, a);
     if (e != cudaSuccess) return e;
-    k_bv_resid<T><<<(unsigned)(B * a.N), kThreads, 0, s>>>(a);
-    e = cudaGetLastError();
+    e = launch_pdl(k_bv_resid<T>, dim3((unsigned)(B * a.N)), dim3(kThreads), 0, s, 0, a);
     if (e != cudaSuccess) return e;
-    k_bv_final<T><<<(unsigned)B, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(k_bv_final<T>, dim3((unsigned)B), dim3(kThreads), 0, s, 0, a);
 }
 
 }  // namespace

@@ -54,6 +54,7 @@ __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t 
 
 template <int KCAP, typename T>
 __global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
+    pdl_begin();
     extern __shared__ __align__(16) float2 st[];  // [C] the row's chunk statistics
     __shared__ uint64_t wl[kTopkWarps][KCAP];
     __shared__ float wm[kTopkWarps], wsh[kTopkWarps], wsl[kTopkWarps];
@@ -268,6 +269,7 @@ struct Slots {
 // slot (children are numbered in creation order, lane = c % 32, slot = c / 32).
 template <int S>
 __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
+    pdl_begin();
     extern __shared__ __align__(16) unsigned char smem[];
     const int L = a.L, N = a.N, K = a.K, NN = N + 1;
     long long *CL = reinterpret_cast<long long *>(smem);           // [L+1] fixed point
@@ -447,8 +449,7 @@ cudaError_t launch_heap_t(const HeapArgs &h, int B, cudaStream_t s) {
     const size_t smem = heap_smem_bytes(h.L, h.N, h.K);
     cudaError_t e = cudaFuncSetAttribute(k_plan_heap<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_plan_heap<S><<<B, kHeapThreads, smem, s>>>(h);
-    return cudaGetLastError();
+    return launch_pdl(k_plan_heap<S>, dim3((unsigned)B), dim3(kHeapThreads), smem, s, 0, h);
 }
 
 template <int KCAP, typename T>
@@ -456,8 +457,7 @@ cudaError_t launch_topk_t(const TopkArgs &a, cudaStream_t s) {
     const size_t smem = (size_t)a.C * sizeof(float2);
     cudaError_t e = cudaFuncSetAttribute(k_row_topk<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    k_row_topk<KCAP, T><<<(unsigned)(a.B * a.L), kTopkThreads, smem, s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(k_row_topk<KCAP, T>, dim3((unsigned)(a.B * a.L)), dim3(kTopkThreads), smem, s, 0, a);
 }
 
 }  // namespace

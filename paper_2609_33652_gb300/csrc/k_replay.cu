@@ -71,6 +71,7 @@ __device__ __forceinline__ void merge_warps(const uint64_t (*cand)[CAP], int n, 
 
 template <int KCAP, typename T>
 __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay(ReplayArgs a) {
+    pdl_begin();
     __shared__ uint64_t cand[kWarps][KCAP];
     __shared__ uint64_t sel[KCAP];
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -176,8 +177,7 @@ template <int KCAP, typename T>
 cudaError_t launch_replay_t(const ReplayArgs &a, cudaStream_t s) {
     const int64_t blocks = (int64_t)a.B * (a.N + 1);
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    k_replay<KCAP, T><<<(unsigned)blocks, kThreads, 0, s>>>(a);
-    return cudaGetLastError();
+    return launch_pdl(k_replay<KCAP, T>, dim3((unsigned)blocks), dim3(kThreads), 0, s, 0, a);
 }
 
 }  // namespace

@@ -27,6 +27,7 @@ __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__
                                                            int64_t bstride, int64_t rstride, int C,
                                                            int64_t units_total, float invT,
                                                            float2 *__restrict__ stats, uint32_t *status) {
+    pdl_begin();
     const int lane = threadIdx.x & 31, g = lane & 7, q = lane >> 3;
     const int upr = (C + kUnitChunks - 1) / kUnitChunks;  // units per row
     const float c2 = __fmul_rn(invT, kLog2e);             // exp(x - m) = 2^(z invT log2e - m log2e)
@@ -125,10 +126,9 @@ cudaError_t launch_t(const RowsDesc &rows, float invT, float2 *stats, uint32_t *
     const int64_t needed = (units_total + kWarps - 1) / kWarps;
     const int64_t resident = (int64_t)sm_count() * blocks_per_sm<T>();
     const int64_t blocks = needed < resident ? needed : resident;
-    k_row_stats<T><<<(unsigned)blocks, kWarps * 32, 0, s>>>(static_cast<const T *>(rows.data), rows.R, rows.V,
-                                                             rows.batch_stride, rows.row_stride, C, units_total,
-                                                             invT, stats, status);
-    return cudaGetLastError();
+    return launch_pdl(k_row_stats<T>, dim3((unsigned)blocks), dim3(kWarps * 32), 0, s, 0,
+                      static_cast<const T *>(rows.data), rows.R, rows.V, rows.batch_stride, rows.row_stride, C,
+                      units_total, invT, stats, status);
 }
 
 }  // namespace

@@ -428,6 +428,7 @@ inline size_t topo_bytes(int N) {
 // per-depth q row (tree b, depth d < Lq), from its chunk statistics.
 template <typename T>
 __global__ void __launch_bounds__(kPreThreads) k_verify_pre(VerifyArgs a) {
+    pdl_begin();
     __shared__ Slot part[kPreThreads / 32];
     constexpr int nwarps = kPreThreads / 32;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -524,6 +525,7 @@ __global__ void __launch_bounds__(kPreThreads) k_verify_pre(VerifyArgs a) {
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
+    pdl_begin();
     extern __shared__ __align__(16) float dyn[];
     float *P = dyn;
     float *Q = dyn + a.slice;
@@ -882,25 +884,10 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     const int64_t pre_blocks = (int64_t)B * a.M + ((int64_t)B * a.Lq + kPreThreads / 32 - 1) / (kPreThreads / 32);
     if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     if (pre_blocks > 0) {
-        k_verify_pre<T><<<(unsigned)pre_blocks, kPreThreads, 0, s>>>(a);
-        e = cudaGetLastError();
+        e = launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), 0, s, 0, a);
         if (e != cudaSuccess) return e;
     }
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3((unsigned)(B * cs), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = (unsigned)cs;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, k_verify_rrs<T>, a);
-    if (e != cudaSuccess) return e;
-    return cudaGetLastError();
+    return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
 
 }  // namespace

@@ -461,6 +461,17 @@ struct RawQuad<float> {
     }
 };
 
+// Programmatic dependent launch. Every kernel of the library starts with pdl_begin(): it
+// waits until the kernel launched before it on the stream has completed and its memory is
+// visible (griddepcontrol.wait; immediate when there is no programmatic dependency), then
+// lets the next kernel on the stream be launched (griddepcontrol.launch_dependents). No
+// global memory is touched before the wait, so launches with the programmatic-serialisation
+// attribute only overlap a kernel's launch and CTA scheduling with its predecessor's tail.
+__device__ __forceinline__ void pdl_begin() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ float fast_exp2(float x) {
     float y;
     asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
