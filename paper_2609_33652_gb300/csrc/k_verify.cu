@@ -189,26 +189,21 @@ __device__ __forceinline__ float point_residual(float p0, float q, const float *
     return p;
 }
 
-// Per-thread online (max, sum of exp(x - max)) accumulation, four logits at a time.
+// Per-thread (max, sum of exp(x - max)) accumulation: batches are added as a maximum first
+// (rebase) and then a plain sum of exponentials relative to the running maximum.
 struct OnlineLse {
     float m = -INFINITY;
     KahanF s;
     __device__ __forceinline__ MaxSum value() const { return MaxSum{m, s.ff()}; }
-    __device__ __forceinline__ void add4(const float x[4]) {
-        const float gm = fmaxf(fmaxf(x[0], x[1]), fmaxf(x[2], x[3]));
-        if (gm == -INFINITY) return;
-        if (gm > m) {
+    __device__ __forceinline__ void rebase(float bm) {
+        if (bm > m) {
             if (m != -INFINITY) {
-                const float scale = fast_exp2(__fmul_rn(__fsub_rn(m, gm), kLog2e));
+                const float scale = fast_exp2(__fmul_rn(__fsub_rn(m, bm), kLog2e));
                 s.s = __fmul_rn(s.s, scale);
                 s.c = __fmul_rn(s.c, scale);
             }
-            m = gm;
+            m = bm;
         }
-        float t = 0.f;
-#pragma unroll
-        for (int k = 0; k < 4; ++k) t += fast_exp2(__fmul_rn(__fsub_rn(x[k], m), kLog2e));
-        s.add(t);
     }
 };
 
@@ -249,6 +244,22 @@ struct Walk {
                     raw[e][1].load(row, lo + quad_at(cl, 1, lane), end);
                 }
             }
+            if (!NORMALISE && lse) {  // the batch's maximum first (rounding is monotone: max z, then * invT)
+                float zm = -INFINITY;
+#pragma unroll
+                for (int e = 0; e < kB; ++e) {
+                    if (c0 + e * nw >= nch) break;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h) {
+                        float z[4];
+                        raw[e][h].unpack(z);
+                        zm = fmaxf(zm, fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
+                    }
+                }
+                lse->rebase(__fmul_rn(zm, a.invT));
+            }
+            const float mref = (!NORMALISE && lse) ? lse->m : 0.f;
+            float t0 = 0.f, t1 = 0.f;
 #pragma unroll
             for (int e = 0; e < kB; ++e) {
                 const int cl = c0 + e * nw;
@@ -262,12 +273,18 @@ struct Walk {
                     if (NORMALISE) {
 #pragma unroll
                         for (int k = 0; k < 4; ++k) x[k] = exp_shifted(x[k], L2);
-                    } else if (lse) {
-                        lse->add4(x);
+                    } else if (lse && lse->m != -INFINITY) {
+                        // exp(x - m) = 2^((x - m) log2 e): the difference first, so the exponent
+                        // carries no rounding of m itself
+                        t0 += fast_exp2(__fmul_rn(__fsub_rn(x[0], mref), kLog2e)) +
+                              fast_exp2(__fmul_rn(__fsub_rn(x[1], mref), kLog2e));
+                        t1 += fast_exp2(__fmul_rn(__fsub_rn(x[2], mref), kLog2e)) +
+                              fast_exp2(__fmul_rn(__fsub_rn(x[3], mref), kLog2e));
                     }
                     st4(dst, quad_at(cl, h, lane), x[0], x[1], x[2], x[3]);
                 }
             }
+            if (!NORMALISE && lse && lse->m != -INFINITY) lse->s.add(__fadd_rn(t0, t1));
         }
     }
 

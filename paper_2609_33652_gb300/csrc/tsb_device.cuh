@@ -99,10 +99,12 @@ __device__ __forceinline__ float key_value(uint64_t k) { return f32_of_ord((uint
 
 // ---------------------------------------------------------------------------------------
 // Warp reductions (butterfly: every lane ends with the result).
+// Warp maximum of a float in one instruction (redux.sync.max.f32, sm_100a family); like
+// fmaxf, NaN inputs are ignored unless every input is NaN.
 __device__ __forceinline__ float warp_max(float v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(kFull, v, o));
-    return v;
+    float r;
+    asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
+    return r;
 }
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
