@@ -3,8 +3,9 @@
 
 Workload (batched serving): B=16 trees, V=151,936, draft block L=16, N=64 planned nodes,
 top-k 8, T=1, bf16 logits; target rows [16, 65, V] = the node's depth row + N(0, 0.7^2).
-A step = tsb_row_stats + tsb_plan + tsb_replay + tsb_verify on one batch (5 kernel launches:
-the planner launches its per-row top-K kernel and its frontier kernel).
+A step = tsb_plan_rows + tsb_replay + tsb_verify on one batch (5 kernel launches: the planner
+streams each draft row once for its chunk statistics and top-K, then runs the frontier
+kernel; the verifier runs its pre-pass and its walk).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tsb|reference]
 
@@ -42,10 +43,9 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
 L2_BYTES = 129 * 1024 * 1024
-KERNELS = ("tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify")
-LAUNCHES_PER_STEP = {"tsb_row_stats": 1, "tsb_plan": 2, "tsb_replay": 1, "tsb_verify": 1}
-KERNEL_SOURCES = {"tsb_row_stats": "k_row_stats.cu", "tsb_plan": "k_plan.cu", "tsb_replay": "k_replay.cu",
-                  "tsb_verify": "k_verify.cu"}
+KERNELS = ("tsb_plan_rows", "tsb_replay", "tsb_verify")
+LAUNCHES_PER_STEP = {"tsb_plan_rows": 2, "tsb_replay": 1, "tsb_verify": 2}
+KERNEL_SOURCES = {"tsb_plan_rows": "k_plan.cu", "tsb_replay": "k_replay.cu", "tsb_verify": "k_verify.cu"}
 
 
 def parse():
@@ -267,7 +267,7 @@ def run_tsb(args):
     # Per-call durations: a second pass over the same prepared steps with an event before the
     # first call and after each call (on the launching stream).
     KA = min(K, 300)
-    events = [[torch.cuda.Event(enable_timing=True) for _ in range(5)] for _ in range(KA)]
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(len(KERNELS) + 1)] for _ in range(KA)]
     for k in range(KA):
         steps[k].run(events[k])
     torch.cuda.synchronize()
@@ -297,9 +297,8 @@ def run_tsb(args):
     C = (w["V"] + 255) // 256
     es = 2 if w["dtype"] == "bf16" else 4
     kernel_bytes = {
-        "tsb_row_stats": B * L * w["V"] * es + B * L * C * 8,
+        "tsb_plan_rows": B * L * w["V"] * es + B * L * C * 8,
         "tsb_verify": float(target_bytes.mean()),
-        "tsb_plan": B * L * C * 8,
         "tsb_replay": B * w["N"] * (C * 8),
     }
     achieved = kernel_bytes[dom] / (kern_us[dom] * 1e-6) / 1e9

@@ -7,6 +7,7 @@
  *
  *   tsb_row_stats   draft rows            -> chunk statistics (max, sum of exp)
  *   tsb_plan        draft rows + stats    -> frozen topology T (first pass, Sec. 3.1)
+ *   tsb_plan_rows   draft rows            -> their statistics + T, in one pass over the rows
  *   tsb_replay      q rows + stats + T    -> one fresh token per node (second pass, Sec. 3.2)
  *   tsb_verify      target rows + q rows + T + tokens -> accepted path and final token
  *                   (recursive rejection sampling, Sec. 2.3 and App. A; or block verification
@@ -146,6 +147,16 @@ tsb_status tsb_row_stats(const tsb_logits *rows, float temperature, void *stats,
  * and temperature. Writes every array of *out. */
 tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats, size_t stats_bytes,
                     const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
+
+/* tsb_row_stats of draft rows 0..L-1 and tsb_plan in one pass over those rows: each draft
+ * row is streamed once by one CTA, which writes the row's chunk statistics to draft_stats
+ * (layout and bits exactly as tsb_row_stats writes them; rows L..R-1 are not written) and then
+ * runs the first pass's top-K on them while the candidate chunks are still in L2; then the
+ * best-first expansion as in tsb_plan (Sec. 3.1, App. B.3). draft_stats: float2-aligned
+ * device buffer of tsb_stats_bytes(B, R, V), an output here. Other arguments and errors as in
+ * tsb_plan; non-finite logits set TSB_DEV_NONFINITE. */
+tsb_status tsb_plan_rows(const tsb_cfg *cfg, const tsb_logits *draft, void *draft_stats, size_t stats_bytes,
+                         const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
 
 /* Size of the device scratch array behind tsb_plan_noalloc (1 MiB per device). */
 #define TSB_NOALLOC_SCRATCH_BYTES ((size_t)1 << 20)

@@ -24,7 +24,7 @@ namespace tsb {
 namespace {
 
 constexpr int kTopkThreads = 128;
-constexpr int kTopkWarps = kTopkThreads / 32;
+constexpr int kRowPlanThreads = 512;
 constexpr int kHeapThreads = 128;
 
 struct TopkArgs {
@@ -32,6 +32,8 @@ struct TopkArgs {
     int64_t bstride, rstride;
     int B, R, V, C, L, K;
     const float2 *stats;
+    float2 *stats_out;  // k_row_stats_topk: the statistics it writes ([B][R][C])
+    uint32_t *status;
     float invT;
     float2 *lse;       // [B*L] row log-normalisers as float-float (hi, lo)
     float *topk_x;     // [B*L*K]
@@ -52,78 +54,69 @@ __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t 
         for (++j; j < n; ++j) dst[j] = 0ull;
 }
 
-template <int KCAP, typename T>
-__global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
-    pdl_begin();
-    extern __shared__ __align__(16) float2 st[];  // [C] the row's chunk statistics
-    __shared__ uint64_t wl[kTopkWarps][KCAP];
-    __shared__ float wm[kTopkWarps], wsh[kTopkWarps], wsl[kTopkWarps];
+// The top-K pass of one draft row from its chunk statistics st[0..C) in shared memory (all NT
+// threads of the CTA call it, after a barrier that follows the last write of st): the
+// float-float log-normaliser, tau = the K-th largest chunk maximum (a lower bound on the K-th
+// largest logit, since K distinct chunk maxima reach it), the logits >= tau of the chunks whose
+// maximum reaches tau (a chunk goes to the warp that scans it, four chunks' loads per batch),
+// then per-warp and CTA merges. Writes lse[row], topk_x / topk_id [row][K].
+template <int KCAP, int NT, typename T>
+__device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st) {
+    constexpr int NW = NT / 32;
+    static_assert(NW >= 2, "warps 0 and 1 merge in parallel");
+    __shared__ uint64_t wl[NW][KCAP];
+    __shared__ float wm[4], wsh[4], wsl[4];
     __shared__ float s_tau;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    const int row = blockIdx.x;
     const int b = row / a.L, d = row - (row / a.L) * a.L;
     const int C = a.C, K = a.K;
-    const float2 *gst = a.stats + ((int64_t)b * a.R + d) * C;
-    // 1. stage the statistics (eight loads in flight per thread); per-thread maximum and list
-    //    of chunk maxima
+    // 1. per-thread list of chunk maxima; log-normaliser partials over a fixed partition of
+    //    kLseThreads threads (whatever NT is, so every caller sums in the same order)
     TopList<KCAP> cl;
     cl.clear();
-    float m = -INFINITY;
-    for (int c0 = threadIdx.x; c0 < C; c0 += kTopkThreads * 8) {
-        float2 v[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const int c = c0 + kTopkThreads * e;
-            v[e] = c < C ? __ldg(&gst[c]) : make_float2(-INFINITY, 0.f);
-        }
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-            const int c = c0 + kTopkThreads * e;
-            if (c < C) {
-                st[c] = v[e];
-                m = fmaxf(m, v[e].x);
-                cl.insert(pack_key(v[e].x, (uint32_t)c));
-            }
+    for (int c = threadIdx.x; c < C; c += NT) cl.insert(pack_key(st[c].x, (uint32_t)c));
+    constexpr int kLseThreads = 128, kLseWarps = kLseThreads / 32;
+    static_assert(NT >= kLseThreads, "the partition needs kLseThreads threads");
+    if (threadIdx.x < kLseThreads) {
+        float m = -INFINITY;
+        for (int c = threadIdx.x; c < C; c += kLseThreads) m = fmaxf(m, st[c].x);
+        KahanF acc;
+        if (m != -INFINITY)
+            for (int c = threadIdx.x; c < C; c += kLseThreads)
+                acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
+        const MaxSum ms = warp_maxsum(MaxSum{m, acc.ff()});
+        if (lane == 0) {
+            wm[warp] = ms.m;
+            wsh[warp] = ms.s.hi;
+            wsl[warp] = ms.s.lo;
         }
     }
-    // 2. log-normaliser partials (float-float) over the thread's own chunks, then per warp
-    KahanF acc;
-    if (m != -INFINITY)
-        for (int c = threadIdx.x; c < C; c += kTopkThreads)
-            acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
-    const MaxSum ms = warp_maxsum(MaxSum{m, acc.ff()});
-    if (lane == 0) {
-        wm[warp] = ms.m;
-        wsh[warp] = ms.s.hi;
-        wsl[warp] = ms.s.lo;
-    }
-    // 3. each warp's K largest chunk maxima
+    // 2. each warp's K largest chunk maxima
     warp_top_to(cl, K, wl[warp]);
     __syncthreads();
     if (warp == 0) {
-        MaxSum v = lane < kTopkWarps ? MaxSum{wm[lane], FF{wsh[lane], wsl[lane]}} : MaxSum{-INFINITY, FF{0.f, 0.f}};
+        MaxSum v = lane < kLseWarps ? MaxSum{wm[lane], FF{wsh[lane], wsl[lane]}} : MaxSum{-INFINITY, FF{0.f, 0.f}};
         v = warp_maxsum(v);
         if (lane == 0) {
             const FF l = maxsum_lse(v);
             a.lse[row] = make_float2(l.hi, l.lo);
         }
-        // tau = K-th largest chunk maximum (-inf with fewer than K chunks): a lower bound on
-        // the K-th largest logit, since K distinct chunk maxima reach it
+    } else if (warp == 1) {  // in parallel with warp 0
+        // tau = K-th largest chunk maximum (-inf with fewer than K chunks)
         TopList<KCAP> t;
         t.clear();
-        for (int e = lane; e < kTopkWarps * K; e += 32) t.insert(wl[e / K][e % K]);
+        for (int e = lane; e < NW * K; e += 32) t.insert(wl[e / K][e % K]);
         uint64_t kth = 0;
         for (int j = 0; j < K; ++j) kth = warp_pop_max(t);
         if (lane == 0) s_tau = C >= K ? key_value(kth) : -INFINITY;
     }
     __syncthreads();
     const float tau = s_tau;
-    // 4. the logits >= tau of the chunks whose maximum reaches tau; a chunk goes to the warp
-    //    that scans it, four chunks' loads per batch
+    // 3. the logits >= tau of the chunks whose maximum reaches tau
     const T *rowp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
     TopList<KCAP> el;
     el.clear();
-    for (int cb = warp * 32; cb < C; cb += kTopkThreads) {
+    for (int cb = warp * 32; cb < C; cb += NT) {
         const int c = cb + lane;
         unsigned mask = __ballot_sync(kFull, c < C && st[c].x >= tau);
         while (mask) {
@@ -155,13 +148,13 @@ __global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
             }
         }
     }
-    // 5. per warp top-K, then the CTA's
-    warp_top_to(el, K, wl[warp]);  // warp 0 finished reading wl before the barrier above
+    // 4. per warp top-K, then the CTA's
+    warp_top_to(el, K, wl[warp]);  // wl was last read before the barrier above
     __syncthreads();
     if (warp == 0) {
         TopList<KCAP> t;
         t.clear();
-        for (int e = lane; e < kTopkWarps * K; e += 32) t.insert(wl[e / K][e % K]);
+        for (int e = lane; e < NW * K; e += 32) t.insert(wl[e / K][e % K]);
         for (int j = 0; j < K; ++j) {
             const uint64_t best = warp_pop_max(t);
             if (lane == 0) {
@@ -170,6 +163,80 @@ __global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
             }
         }
     }
+}
+
+// One 4-warp CTA per draft row: stage the row's chunk statistics (one round of loads), then
+// the top-K pass.
+template <int KCAP, typename T>
+__global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
+    pdl_begin();
+    extern __shared__ __align__(16) float2 st[];  // [C] the row's chunk statistics
+    const int row = blockIdx.x;
+    const int b = row / a.L, d = row - (row / a.L) * a.L;
+    const int C = a.C;
+    const float2 *gst = a.stats + ((int64_t)b * a.R + d) * C;
+    for (int c0 = threadIdx.x; c0 < C; c0 += kTopkThreads * 8) {  // eight loads in flight per thread
+        float2 v[8];
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int c = c0 + kTopkThreads * e;
+            v[e] = c < C ? __ldg(&gst[c]) : make_float2(-INFINITY, 0.f);
+        }
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const int c = c0 + kTopkThreads * e;
+            if (c < C) st[c] = v[e];
+        }
+    }
+    __syncthreads();
+    topk_from_stats<KCAP, kTopkThreads, T>(a, row, st);
+}
+
+// One 16-warp CTA per draft row, streaming the row once: the chunk statistics exactly as
+// k_row_stats computes them (same per-chunk code, so the same bits), written to the caller's
+// statistics buffer and kept in shared memory, then the top-K pass, whose candidate chunks
+// are then still in L2. Two CTAs per SM (K <= 8), so up to 2 rows per SM run in one wave.
+template <int KCAP, typename T>
+__global__ void __launch_bounds__(kRowPlanThreads, KCAP <= 8 ? 2 : 1) k_row_stats_topk(TopkArgs a) {
+    pdl_begin();
+    extern __shared__ __align__(16) float2 st[];  // [C]
+    constexpr int NW = kRowPlanThreads / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, g = lane & 7, q = lane >> 3;
+    const int row = blockIdx.x;
+    const int b = row / a.L, d = row - (row / a.L) * a.L;
+    const int C = a.C;
+    const T *rp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
+    float2 *gst = a.stats_out + ((int64_t)b * a.R + d) * C;
+    const float c2 = __fmul_rn(a.invT, kLog2e);
+    const int units = (C + 3) / 4;  // four chunks (eight lanes each) per warp unit
+    constexpr int kU = sizeof(T) == 2 ? 2 : 1;  // units in flight per warp (register budget)
+    bool bad = false;
+    for (int u0 = warp; u0 < units; u0 += kU * NW) {  // uniform over the warp
+        RawGroup<T> raw[kU][4];
+#pragma unroll
+        for (int e = 0; e < kU; ++e) {
+            const int c = (u0 + e * NW) * 4 + q;
+            if (u0 + e * NW < units && c < C)
+#pragma unroll
+                for (int k = 0; k < 4; ++k) raw[e][k].load(rp, c * kChunk + k * 64 + g * 8, a.V);
+        }
+#pragma unroll
+        for (int e = 0; e < kU; ++e) {
+            const int c = (u0 + e * NW) * 4 + q;
+            const bool live = u0 + e * NW < units && c < C;
+            float mc, sc;
+            chunk_stats8<T>(raw[e], live, a.invT, c2, &mc, &sc);
+            if (live && g == 0) {
+                const float2 v = make_float2(mc, sc);
+                gst[c] = v;
+                st[c] = v;
+                bad |= !(sc == sc) || isinf(mc);
+            }
+        }
+    }
+    if (bad) raise_status(a.status, kDevNonFinite);
+    __syncthreads();
+    topk_from_stats<KCAP, kRowPlanThreads, T>(a, row, st);
 }
 
 struct HeapArgs {
@@ -460,6 +527,61 @@ cudaError_t launch_topk_t(const TopkArgs &a, cudaStream_t s) {
     return launch_pdl(k_row_topk<KCAP, T>, dim3((unsigned)(a.B * a.L)), dim3(kTopkThreads), smem, s, 0, a);
 }
 
+template <int KCAP, typename T>
+cudaError_t launch_stats_topk_t(const TopkArgs &a, cudaStream_t s) {
+    const size_t smem = (size_t)a.C * sizeof(float2);
+    cudaError_t e =
+        cudaFuncSetAttribute(k_row_stats_topk<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_row_stats_topk<KCAP, T>, dim3((unsigned)(a.B * a.L)), dim3(kRowPlanThreads), smem, s, 0, a);
+}
+
+// The frontier kernel with as many slots per lane as N + 1 first children need.
+cudaError_t launch_heap(const HeapArgs &h, int B, cudaStream_t s) {
+    const int per_lane = (h.N + 1 + 31) / 32;
+    if (per_lane <= 1) return launch_heap_t<1>(h, B, s);
+    if (per_lane <= 2) return launch_heap_t<2>(h, B, s);
+    if (per_lane <= 3) return launch_heap_t<3>(h, B, s);
+    if (per_lane <= 4) return launch_heap_t<4>(h, B, s);
+    if (per_lane <= 8) return launch_heap_t<8>(h, B, s);
+    if (per_lane <= 16) return launch_heap_t<16>(h, B, s);
+    return launch_heap_t<33>(h, B, s);
+}
+
+TopkArgs topk_args(const RowsDesc &draft, const float2 *stats, int L, int K, float invT, const PlanScratch &sc) {
+    TopkArgs t;
+    t.draft = draft.data;
+    t.bstride = draft.batch_stride;
+    t.rstride = draft.row_stride;
+    t.B = draft.B;
+    t.R = draft.R;
+    t.V = draft.V;
+    t.C = num_chunks(draft.V);
+    t.L = L;
+    t.K = K;
+    t.stats = stats;
+    t.stats_out = nullptr;
+    t.status = nullptr;
+    t.invT = invT;
+    t.lse = sc.lse;
+    t.topk_x = sc.topk_x;
+    t.topk_id = sc.topk_id;
+    return t;
+}
+
+HeapArgs heap_args(int L, int N, int K, const PlanScratch &sc, const TreeDesc &tree, uint32_t *status) {
+    HeapArgs h;
+    h.L = L;
+    h.N = N;
+    h.K = K;
+    h.lse = sc.lse;
+    h.topk_x = sc.topk_x;
+    h.topk_id = sc.topk_id;
+    h.tree = tree;
+    h.status = status;
+    return h;
+}
+
 }  // namespace
 
 PlanScratch plan_scratch(void *ws, int B, int N, int L, int K) {
@@ -474,45 +596,29 @@ PlanScratch plan_scratch(void *ws, int B, int N, int L, int K) {
 cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
                         const TreeDesc &tree, void *ws, cudaStream_t s) {
     const PlanScratch sc = plan_scratch(ws, draft.B, N, L, K);
-    TopkArgs t;
-    t.draft = draft.data;
-    t.bstride = draft.batch_stride;
-    t.rstride = draft.row_stride;
-    t.B = draft.B;
-    t.R = draft.R;
-    t.V = draft.V;
-    t.C = num_chunks(draft.V);
-    t.L = L;
-    t.K = K;
-    t.stats = stats;
-    t.invT = invT;
-    t.lse = sc.lse;
-    t.topk_x = sc.topk_x;
-    t.topk_id = sc.topk_id;
+    const TopkArgs t = topk_args(draft, stats, L, K, invT, sc);
     cudaError_t e;
     if (draft.dtype == 1)
         e = K <= 8 ? launch_topk_t<8, __nv_bfloat16>(t, s) : launch_topk_t<32, __nv_bfloat16>(t, s);
     else
         e = K <= 8 ? launch_topk_t<8, float>(t, s) : launch_topk_t<32, float>(t, s);
     if (e != cudaSuccess) return e;
-    HeapArgs h;
-    h.L = L;
-    h.N = N;
-    h.K = K;
-    h.lse = sc.lse;
-    h.topk_x = sc.topk_x;
-    h.topk_id = sc.topk_id;
-    h.tree = tree;
-    h.status = static_cast<uint32_t *>(ws);
-    // frontier slots per lane: at most N + 1 first children are ever created
-    const int per_lane = (N + 1 + 31) / 32;
-    if (per_lane <= 1) return launch_heap_t<1>(h, draft.B, s);
-    if (per_lane <= 2) return launch_heap_t<2>(h, draft.B, s);
-    if (per_lane <= 3) return launch_heap_t<3>(h, draft.B, s);
-    if (per_lane <= 4) return launch_heap_t<4>(h, draft.B, s);
-    if (per_lane <= 8) return launch_heap_t<8>(h, draft.B, s);
-    if (per_lane <= 16) return launch_heap_t<16>(h, draft.B, s);
-    return launch_heap_t<33>(h, draft.B, s);
+    return launch_heap(heap_args(L, N, K, sc, tree, static_cast<uint32_t *>(ws)), draft.B, s);
+}
+
+cudaError_t launch_plan_rows(const RowsDesc &draft, float2 *stats_out, int L, int N, int K, float invT,
+                             const TreeDesc &tree, void *ws, cudaStream_t s) {
+    const PlanScratch sc = plan_scratch(ws, draft.B, N, L, K);
+    TopkArgs t = topk_args(draft, nullptr, L, K, invT, sc);
+    t.stats_out = stats_out;
+    t.status = static_cast<uint32_t *>(ws);
+    cudaError_t e;
+    if (draft.dtype == 1)
+        e = K <= 8 ? launch_stats_topk_t<8, __nv_bfloat16>(t, s) : launch_stats_topk_t<32, __nv_bfloat16>(t, s);
+    else
+        e = K <= 8 ? launch_stats_topk_t<8, float>(t, s) : launch_stats_topk_t<32, float>(t, s);
+    if (e != cudaSuccess) return e;
+    return launch_heap(heap_args(L, N, K, sc, tree, static_cast<uint32_t *>(ws)), draft.B, s);
 }
 
 }  // namespace tsb
@@ -523,44 +629,14 @@ namespace tsb {
 // given explicitly instead of being carved out of a caller workspace.
 cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
                                 const TreeDesc &tree, const PlanScratch &sc, uint32_t *status, cudaStream_t s) {
-    TopkArgs t;
-    t.draft = draft.data;
-    t.bstride = draft.batch_stride;
-    t.rstride = draft.row_stride;
-    t.B = draft.B;
-    t.R = draft.R;
-    t.V = draft.V;
-    t.C = num_chunks(draft.V);
-    t.L = L;
-    t.K = K;
-    t.stats = stats;
-    t.invT = invT;
-    t.lse = sc.lse;
-    t.topk_x = sc.topk_x;
-    t.topk_id = sc.topk_id;
+    const TopkArgs t = topk_args(draft, stats, L, K, invT, sc);
     cudaError_t e;
     if (draft.dtype == 1)
         e = K <= 8 ? launch_topk_t<8, __nv_bfloat16>(t, s) : launch_topk_t<32, __nv_bfloat16>(t, s);
     else
         e = K <= 8 ? launch_topk_t<8, float>(t, s) : launch_topk_t<32, float>(t, s);
     if (e != cudaSuccess) return e;
-    HeapArgs h;
-    h.L = L;
-    h.N = N;
-    h.K = K;
-    h.lse = sc.lse;
-    h.topk_x = sc.topk_x;
-    h.topk_id = sc.topk_id;
-    h.tree = tree;
-    h.status = status;
-    const int per_lane = (N + 1 + 31) / 32;
-    if (per_lane <= 1) return launch_heap_t<1>(h, draft.B, s);
-    if (per_lane <= 2) return launch_heap_t<2>(h, draft.B, s);
-    if (per_lane <= 3) return launch_heap_t<3>(h, draft.B, s);
-    if (per_lane <= 4) return launch_heap_t<4>(h, draft.B, s);
-    if (per_lane <= 8) return launch_heap_t<8>(h, draft.B, s);
-    if (per_lane <= 16) return launch_heap_t<16>(h, draft.B, s);
-    return launch_heap_t<33>(h, draft.B, s);
+    return launch_heap(heap_args(L, N, K, sc, tree, status), draft.B, s);
 }
 
 }  // namespace tsb

@@ -57,35 +57,8 @@ __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__
 #pragma unroll
         for (int e = 0; e < kUnits; ++e) {
             const int c = c_of[e];
-            float zm = -INFINITY;
-            if (c >= 0) {
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    float z[8];
-                    raw[e][k].unpack(z);
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
-                }
-            }
-            // the group's maximum (xor 4, 2, 1 stay inside the 8-lane group)
-            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
-            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
-            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
-            const float mc = __fmul_rn(zm, invT);
-            const float off = __fmul_rn(mc, kLog2e);
-            float s = 0.f;
-            if (c >= 0) {
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    float z[8];
-                    raw[e][k].unpack(z);  // unpacked again rather than kept: fewer registers
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) s += fast_exp2(__fmaf_rn(z[i], c2, -off));
-                }
-            }
-            s += __shfl_xor_sync(kFull, s, 4);
-            s += __shfl_xor_sync(kFull, s, 2);
-            s += __shfl_xor_sync(kFull, s, 1);
+            float mc, s;
+            chunk_stats8<T>(raw[e], c >= 0, invT, c2, &mc, &s);
             if (c >= 0 && g == 0) {
                 stats[row_of[e] * C + c] = make_float2(mc, s);
                 bad |= !(s == s) || isinf(mc);

@@ -168,6 +168,22 @@ tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *dra
                                         (cudaStream_t)stream));
 }
 
+tsb_status tsb_plan_rows(const tsb_cfg *cfg, const tsb_logits *draft, void *draft_stats, size_t stats_bytes,
+                         const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_logits(draft, cfg->B, cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(draft_stats, stats_bytes, cfg->B, draft->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!out || !out->parent || !out->depth || !out->rank || !out->plan_token || !out->score || !out->child_off ||
+        !out->child_ids)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_plan_rows(rows_of(draft), static_cast<float2 *>(draft_stats), cfg->L, cfg->N,
+                                             cfg->K, inv_temperature(cfg->temperature), tree_of(out), ws,
+                                             (cudaStream_t)stream));
+}
+
 tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,
                       const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
                       size_t ws_bytes, tsb_stream stream) {

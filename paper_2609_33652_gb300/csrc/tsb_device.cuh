@@ -482,4 +482,45 @@ __device__ __forceinline__ float fast_exp2(float x) {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Statistics of one 256-logit chunk held by an 8-lane group (lane g holds logits 8g..8g+7 of
+// each 64-logit quarter, raw[k] = quarter k): the maximum m_c = fp32(max z * invT) and
+// s_c = sum 2^(z c2 - m_c log2 e) with c2 = invT log2 e, in a fixed order, then xor 4, 2, 1
+// inside the group. Every lane of the warp must call it (the shuffles are warp-wide); a group
+// with live == false contributes -inf / 0. Shared by the statistics kernels so that they
+// produce the same bits.
+template <typename T>
+__device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool live, float invT, float c2,
+                                             float *mc_out, float *s_out) {
+    float zm = -INFINITY;
+    if (live) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float z[8];
+            raw[k].unpack(z);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
+        }
+    }
+    zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
+    zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
+    zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
+    const float mc = __fmul_rn(zm, invT);
+    const float off = __fmul_rn(mc, kLog2e);
+    float s = 0.f;
+    if (live) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+            float z[8];
+            raw[k].unpack(z);  // unpacked again rather than kept: fewer registers
+#pragma unroll
+            for (int i = 0; i < 8; ++i) s += fast_exp2(__fmaf_rn(z[i], c2, -off));
+        }
+    }
+    s += __shfl_xor_sync(kFull, s, 4);
+    s += __shfl_xor_sync(kFull, s, 2);
+    s += __shfl_xor_sync(kFull, s, 1);
+    *mc_out = mc;
+    *s_out = s;
+}
+
 }  // namespace tsb

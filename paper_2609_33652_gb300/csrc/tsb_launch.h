@@ -75,6 +75,8 @@ cudaError_t launch_row_stats(const RowsDesc &rows, float invT, float2 *stats, ui
 
 cudaError_t launch_plan(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
                         const TreeDesc &tree, void *ws, cudaStream_t s);
+cudaError_t launch_plan_rows(const RowsDesc &draft, float2 *stats_out, int L, int N, int K, float invT,
+                             const TreeDesc &tree, void *ws, cudaStream_t s);
 cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
                                 const TreeDesc &tree, const PlanScratch &sc, uint32_t *status, cudaStream_t s);
 

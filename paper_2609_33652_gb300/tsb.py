@@ -26,7 +26,8 @@ TSB_DEV_NONFINITE, TSB_DEV_BAD_INDEX, TSB_DEV_BAD_TREE = 0x1, 0x2, 0x4
 TSB_CHUNK = 256
 
 EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_bytes", "tsb_workspace_init",
-           "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify", "tsb_plan_noalloc")
+           "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify", "tsb_plan_noalloc",
+           "tsb_plan_rows")
 TSB_NOALLOC_SCRATCH_BYTES = 1 << 20
 
 
@@ -80,6 +81,7 @@ def load():
         "tsb_row_stats": (_I32, [_P, ctypes.c_float, _P, _SZ, _P, _SZ, _P]),
         "tsb_plan": (_I32, [_P, _P, _P, _SZ, _P, _P, _SZ, _P]),
         "tsb_plan_noalloc": (_I32, [_P, _P, _P, _SZ, _P, _P, _P]),
+        "tsb_plan_rows": (_I32, [_P, _P, _P, _SZ, _P, _P, _SZ, _P]),
         "tsb_replay": (_I32, [_P, _P, _P, _SZ, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
         "tsb_verify": (_I32, [_P, _I32, _P, _P, _P, _SZ, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
     }
@@ -175,6 +177,15 @@ def tsb_plan(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, ws:
                            ctypes.byref(t), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)), "tsb_plan")
 
 
+def tsb_plan_rows(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, ws: torch.Tensor, stream=None):
+    """tsb_row_stats of draft rows 0..L-1 (written into ``stats``) and tsb_plan in one pass."""
+    d = logits_desc(draft)
+    t = tree_struct(tree)
+    _check(load().tsb_plan_rows(ctypes.byref(cfg), ctypes.byref(d), _ptr(stats), stats.numel() * stats.element_size(),
+                                ctypes.byref(t), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)),
+           "tsb_plan_rows")
+
+
 def tsb_plan_noalloc(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, dev_status=None, stream=None):
     """tsb_plan with the library's static device scratch instead of a workspace; the C call
     allocates nothing. ``dev_status``: optional int32 CUDA tensor whose first word receives
@@ -241,11 +252,12 @@ class TsbBuffers:
 
 class PreparedStep:
     """One plan -> replay -> verify step with every ctypes argument built in advance, so a
-    timing loop pays only the C calls. ``calls`` holds (name, function, args) for
-    tsb_row_stats, tsb_plan, tsb_replay and tsb_verify in launch order."""
+    timing loop pays only the C calls. ``calls`` holds (name, function, args) in launch order:
+    tsb_plan_rows, tsb_replay, tsb_verify (``fused``, the default), or tsb_row_stats,
+    tsb_plan, tsb_replay, tsb_verify."""
 
     def __init__(self, buf: TsbBuffers, draft: torch.Tensor, target: torch.Tensor, seed: int, mode=TSB_VERIFY_RRS,
-                 out_tokens=None, out_nodes=None, out_len=None, stream=None):
+                 out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True):
         lib = load()
         self._keep = []
         s = _stream(stream)
@@ -261,11 +273,15 @@ class PreparedStep:
         ol = buf.out_len if out_len is None else out_len
         self._keep += [ot, on, ol]
         seed = int(seed) & (2**64 - 1)
-        self.calls = [
-            ("tsb_row_stats", lib.tsb_row_stats,
-             (ctypes.byref(dd), ctypes.c_float(cfg.temperature), _ptr(buf.stats), sb, _ptr(buf.ws), wb, s)),
-            ("tsb_plan", lib.tsb_plan, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb, ctypes.byref(tr),
-                                        _ptr(buf.ws), wb, s)),
+        if fused:
+            plan = [("tsb_plan_rows", lib.tsb_plan_rows, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb,
+                                                          ctypes.byref(tr), _ptr(buf.ws), wb, s))]
+        else:
+            plan = [("tsb_row_stats", lib.tsb_row_stats,
+                     (ctypes.byref(dd), ctypes.c_float(cfg.temperature), _ptr(buf.stats), sb, _ptr(buf.ws), wb, s)),
+                    ("tsb_plan", lib.tsb_plan, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb,
+                                                ctypes.byref(tr), _ptr(buf.ws), wb, s))]
+        self.calls = plan + [
             ("tsb_replay", lib.tsb_replay, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb, None,
                                             ctypes.byref(tr), seed, _ptr(buf.token), _ptr(buf.ws), wb, s)),
             ("tsb_verify", lib.tsb_verify, (ctypes.byref(cfg), int(mode), ctypes.byref(dt), ctypes.byref(dd),
@@ -274,8 +290,8 @@ class PreparedStep:
         ]
 
     def run(self, events=None):
-        """Launch the four calls; with ``events`` (five torch.cuda.Event), record one before
-        the first call and one after each."""
+        """Launch the calls; with ``events`` (len(calls) + 1 torch.cuda.Event), record one
+        before the first call and one after each."""
         if events is not None:
             events[0].record()
         for i, (name, fn, args) in enumerate(self.calls):

@@ -96,6 +96,27 @@ def test_plan_validation(lib):
     assert lib.tsb_workspace_bytes(ctypes.byref(cfg1)) == 256 + 4 * 7 * 32 + 4 * 2 * (8 + 8 * 2)
 
 
+def test_plan_rows_validation(lib):
+    good = tsb.make_cfg(4, 16, 64, 8, 1024, 1.0)
+    d = _logits(4, 16, 1024)
+
+    def call(cfg=good, draft=d, stats=FAKE, stats_bytes=1 << 30, ws=FAKE, ws_bytes=1 << 30, tree=None):
+        t = tree if tree is not None else _tree()
+        return lib.tsb_plan_rows(ctypes.byref(cfg) if cfg is not None else None, ctypes.byref(draft), stats,
+                                 stats_bytes, ctypes.byref(t), ws, ws_bytes, None)
+
+    assert call(cfg=None) == ARG
+    assert call(stats=None) == ARG
+    assert call(stats=FAKE + 4) == WS
+    assert call(stats_bytes=4 * 16 * 4 * 8 - 8) == WS
+    assert call(draft=_logits(4, 15, 1024)) == SHAPE
+    assert call(draft=_logits(4, 16, 1024, dtype=2)) == DTYPE
+    assert call(ws_bytes=255) == WS
+    t = _tree()
+    t.score = None
+    assert call(tree=t) == ARG
+
+
 def test_replay_verify_validation(lib):
     cfg = tsb.make_cfg(2, 4, 8, 4, 64, 1.0)
     q = _logits(2, 4, 64)

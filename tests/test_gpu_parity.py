@@ -156,6 +156,40 @@ def test_edges_broadcast_rows():
     assert len({tuple(t) for t in tok}) > 1
 
 
+@pytest.mark.parametrize("B,R,L,N,K,V,kind,dtype", [
+    (16, 16, 16, 64, 8, 151936, "planted", "bf16"),  # the batched workload
+    (3, 6, 4, 40, 12, 5003, "normal3", "f32"),       # ragged V, K > 8, rows beyond L
+    (64, 4, 4, 8, 4, 32, "normal2", "f32"),          # tiny rows, one chunk
+])
+def test_plan_rows_matches_separate_calls(B, R, L, N, K, V, kind, dtype):
+    """tsb_plan_rows = tsb_row_stats (rows < L, same bits) + tsb_plan (same tree)."""
+    draft = _draft(B, R, V, kind, dtype, 71)
+    ref = tsb.TsbBuffers.allocate(B, L, N, K, V, 1.0, draft_rows=R, device=DEV)
+    tsb.tsb_row_stats(draft, 1.0, ref.stats, ref.ws)
+    tsb.tsb_plan(ref.cfg, draft, ref.stats, ref.tree, ref.ws)
+    got = tsb.TsbBuffers.allocate(B, L, N, K, V, 1.0, draft_rows=R, device=DEV)
+    got.stats.fill_(-7.0)
+    tsb.tsb_plan_rows(got.cfg, draft, got.stats, got.tree, got.ws)
+    torch.cuda.synchronize()
+    check_status(ref)
+    check_status(got)
+    C = (V + 255) // 256
+    rs = ref.stats.view(B, R, C, 2)
+    gs = got.stats.view(B, R, C, 2)
+    assert torch.equal(gs[:, :L], rs[:, :L])
+    assert bool((gs[:, L:] == -7.0).all())  # rows the plan does not read are not written
+    for k in ("parent", "depth", "rank", "plan_token", "score", "child_off", "child_ids"):
+        assert torch.equal(got.tree[k], ref.tree[k]), k
+
+
+def test_plan_rows_flags_nonfinite():
+    draft = _draft(2, 3, 512, "normal3", "f32", 15).clone()
+    draft[1, 2, 100] = float("inf")
+    buf = tsb.TsbBuffers.allocate(2, 3, 10, 3, 512, 1.0, device=DEV)
+    tsb.tsb_plan_rows(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+    assert tsb.tsb_device_status(buf.ws) & tsb.TSB_DEV_NONFINITE
+
+
 def test_determinism_and_launch_independence():
     w = synth.WORKLOADS["tiny"]
     draft = _draft(32, w["L"], 2000, "normal3", "bf16", 14)
