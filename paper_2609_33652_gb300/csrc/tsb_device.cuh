@@ -488,19 +488,38 @@ constexpr float kLog2e = 1.4426950408889634f;
 // inside the group. Every lane of the warp must call it (the shuffles are warp-wide); a group
 // with live == false contributes -inf / 0. Shared by the statistics kernels so that they
 // produce the same bits.
+// Maximum of a lane's 32 raw logits (exact: the maximum of bf16 values is a bf16 value).
+__device__ __forceinline__ float group_max32(const RawGroup<float> (&raw)[4]) {
+    float zm = -INFINITY;
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        float z[8];
+        raw[k].unpack(z);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
+    }
+    return zm;
+}
+__device__ __forceinline__ float group_max32(const RawGroup<__nv_bfloat16> (&raw)[4]) {
+    // packed bf16x2 maxima: 16 instructions for 32 logits
+    __nv_bfloat162 h[4];
+#pragma unroll
+    for (int k = 0; k < 4; ++k) {
+        const uint4 w = raw[k].w;
+        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&w.x);
+        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&w.y);
+        const __nv_bfloat162 c = *reinterpret_cast<const __nv_bfloat162 *>(&w.z);
+        const __nv_bfloat162 d = *reinterpret_cast<const __nv_bfloat162 *>(&w.w);
+        h[k] = __hmax2(__hmax2(a, b), __hmax2(c, d));
+    }
+    const __nv_bfloat162 m2 = __hmax2(__hmax2(h[0], h[1]), __hmax2(h[2], h[3]));
+    return fmaxf(__low2float(m2), __high2float(m2));
+}
+
 template <typename T>
 __device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool live, float invT, float c2,
                                              float *mc_out, float *s_out) {
-    float zm = -INFINITY;
-    if (live) {
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-            float z[8];
-            raw[k].unpack(z);
-#pragma unroll
-            for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
-        }
-    }
+    float zm = live ? group_max32(raw) : -INFINITY;
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
