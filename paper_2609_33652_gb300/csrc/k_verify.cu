@@ -53,7 +53,7 @@ constexpr int kQWarp = 14;            // q-row log-normaliser
 constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
 constexpr int kPreTop = 8;            // highest-scoring node ids the pre-pass covers
 constexpr int kMaxDepthRows = 64;     // per-depth q rows (depth cap L <= 64)
-constexpr int kPreThreads = 1024;
+constexpr int kPreThreads = 512;
 
 // Pre-pass results, one 32-byte workspace slot per (tree, node) (the slots block
 // verification uses for its own per-position scalars): l2t = target log-normaliser of node u
@@ -435,22 +435,22 @@ inline size_t topo_bytes(int N) {
     return (size_t)(N + 1) * sizeof(float2) + (size_t)(6 * N + 6) * sizeof(int32_t) + (size_t)3 * N * sizeof(float);
 }
 
-// Pre-pass. CTAs [0, B*M): CTA (b, j) streams target row j of tree b for its log-normaliser
-// (if node j has children).
-// Eight lanes own one 256-logit chunk (lane g reads logits 8g..8g+7 of each 64-logit
-// quarter); a warp takes four consecutive chunks per unit and two units (bf16; one for fp32)
-// per iteration, and every lane of a warp runs the same iterations and every shuffle (chunks
-// past the row contribute nothing). Each group folds its chunks' (max, sum) into a float-float
-// accumulator; groups, then warps, merge in a fixed order. CTAs from B*M on: one warp per
-// per-depth q row (tree b, depth d < Lq), from its chunk statistics.
+// Pre-pass, in clusters of two CTAs. Clusters [0, B*M): cluster (b, j) streams target row j of
+// tree b (if node j has children), each CTA half of its four-chunk units: the chunk statistics
+// of every 256-logit chunk (eight lanes per chunk, two units in flight per warp, the same
+// per-chunk code as the row statistics kernel) into shared memory; rank 0 gathers rank 1's
+// half through distributed shared memory and computes the row's log-normaliser over a fixed
+// 128-thread partition of all chunks, merged in a fixed order. Later CTAs: one warp per
+// per-depth q row (tree b, depth d < Lq), from its chunk statistics (no cluster barrier).
 template <typename T>
-__global__ void __launch_bounds__(kPreThreads) k_verify_pre(VerifyArgs a) {
+__global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     pdl_begin();
-    __shared__ Slot part[kPreThreads / 32];
+    extern __shared__ __align__(16) float2 pst[];  // [C] the row's chunk statistics
+    __shared__ Slot part[4];
     constexpr int nwarps = kPreThreads / 32;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int NN = a.N + 1;
-    const int ntarget = a.B * a.M;
+    const int ntarget = 2 * a.B * a.M;  // even: a cluster is all target or all q-row CTAs
     if ((int)blockIdx.x >= ntarget) {  // q-row log-normalisers, one warp each
         const int task = ((int)blockIdx.x - ntarget) * nwarps + warp;
         if (task >= a.B * a.Lq) return;  // warp-uniform; no barrier in this branch
@@ -459,79 +459,65 @@ __global__ void __launch_bounds__(kPreThreads) k_verify_pre(VerifyArgs a) {
         if (lane == 0) a.pre[(int64_t)b * NN + d].l2q = make_float2(L2q.hi, L2q.lo);
         return;
     }
-    const int b = (int)blockIdx.x / a.M, j = (int)blockIdx.x - ((int)blockIdx.x / a.M) * a.M;
-    {  // leaves need no normaliser
+    cg::cluster_group cluster = cg::this_cluster();
+    const int half = (int)cluster.block_rank();
+    const int pair = (int)blockIdx.x >> 1;
+    const int b = pair / a.M, j = pair - (pair / a.M) * a.M;
+    {  // leaves need no normaliser (both CTAs of the cluster return)
         const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
-        if (__ldg(off + j + 1) - __ldg(off + j) <= 0) return;  // uniform over the CTA
+        if (__ldg(off + j + 1) - __ldg(off + j) <= 0) return;
     }
     const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)j * a.t_rstride;
     const int g = lane & 7, q = lane >> 3;
     const float c2 = __fmul_rn(a.invT, kLog2e);
-    constexpr int kSweep = nwarps * 4;          // chunks covered by one unit of every warp
+    const int C = a.C, units = (C + 3) / 4;
+    const int ulo = half == 0 ? 0 : (units + 1) / 2, uhi = half == 0 ? (units + 1) / 2 : units;
     constexpr int kU = sizeof(T) == 2 ? 2 : 1;  // units in flight per warp (register budget)
-    float macc = -INFINITY;
-    FF sacc = FF{0.f, 0.f};
-    for (int c0 = warp * 4; c0 < a.C; c0 += kU * kSweep) {  // uniform over the warp
+    for (int u0 = ulo + warp; u0 < uhi; u0 += kU * nwarps) {  // uniform over the warp
         RawGroup<T> raw[kU][4];
 #pragma unroll
         for (int e = 0; e < kU; ++e) {
-            const int c = c0 + e * kSweep + q;
-            if (c < a.C)
+            const int c = (u0 + e * nwarps) * 4 + q;
+            if (u0 + e * nwarps < uhi && c < C)
 #pragma unroll
                 for (int k = 0; k < 4; ++k) raw[e][k].load(row, c * kChunk + k * 64 + g * 8, a.V);
         }
 #pragma unroll
         for (int e = 0; e < kU; ++e) {
-            const int c = c0 + e * kSweep + q;
-            const bool live = c < a.C;
-            float zm = -INFINITY;
-            if (live) {
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    float z[8];
-                    raw[e][k].unpack(z);
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) zm = fmaxf(zm, z[i]);
-                }
-            }
-            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
-            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
-            zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
-            const float mc = __fmul_rn(zm, a.invT);
-            const float off = __fmul_rn(mc, kLog2e);
-            float sc = 0.f;
-            if (live && mc != -INFINITY) {
-#pragma unroll
-                for (int k = 0; k < 4; ++k) {
-                    float z[8];
-                    raw[e][k].unpack(z);
-#pragma unroll
-                    for (int i = 0; i < 8; ++i) sc += fast_exp2(__fmaf_rn(z[i], c2, -off));
-                }
-            }
-            sc += __shfl_xor_sync(kFull, sc, 4);
-            sc += __shfl_xor_sync(kFull, sc, 2);
-            sc += __shfl_xor_sync(kFull, sc, 1);
-            if (live && mc != -INFINITY) {
-                if (mc > macc) {
-                    sacc = rescale_to(macc, sacc, mc);
-                    macc = mc;
-                }
-                sacc = ff_add(sacc, FF{mc == macc ? sc : __fmul_rn(sc, expf(__fsub_rn(mc, macc))), 0.f});
-            }
+            const int c = (u0 + e * nwarps) * 4 + q;
+            const bool live = u0 + e * nwarps < uhi && c < C;
+            float mc, sc;
+            chunk_stats8<T>(raw[e], live, a.invT, c2, &mc, &sc);
+            if (live && g == 0) pst[c] = make_float2(mc, sc);
         }
     }
-    Slot mine = neutral_slot();
-    if (g == 0) {  // one contribution per group (its eight lanes hold the same values)
-        mine.m = macc;
-        mine.sh = sacc.hi;
-        mine.sl = sacc.lo;
+    cluster.sync();  // both halves written
+    if (half == 1) {
+        cluster.sync();  // rank 0 has copied this half
+        return;
     }
-    const Slot w = warp_reduce_slot<kRedLse>(mine);
-    if (lane == 0) part[warp] = w;
+    {
+        const float2 *other = cluster.map_shared_rank(pst, 1);
+        for (int c = (units + 1) / 2 * 4 + threadIdx.x; c < C; c += kPreThreads) pst[c] = other[c];
+    }
+    cluster.sync();  // rank 1 may leave; rank 0's copy is complete (the barrier also orders the CTA)
+    if (warp < 4) {  // the log-normaliser over threads 0..127, then warps 0..3 in order
+        float m = -INFINITY;
+        for (int c = threadIdx.x; c < C; c += 128) m = fmaxf(m, pst[c].x);
+        KahanF acc;
+        if (m != -INFINITY)
+            for (int c = threadIdx.x; c < C; c += 128) acc.add(__fmul_rn(pst[c].y, expf(__fsub_rn(pst[c].x, m))));
+        Slot mine = neutral_slot();
+        const FF sv = acc.ff();
+        mine.m = m;
+        mine.sh = sv.hi;
+        mine.sl = sv.lo;
+        const Slot w = warp_reduce_slot<kRedLse>(mine);
+        if (lane == 0) part[warp] = w;
+    }
     __syncthreads();
     if (warp == 0) {
-        const Slot v = warp_reduce_slot<kRedLse>(lane < nwarps ? part[lane] : neutral_slot());
+        const Slot v = warp_reduce_slot<kRedLse>(lane < 4 ? part[lane] : neutral_slot());
         if (lane == 0) {
             const FF l = v.sh > 0.f ? maxsum_lse(MaxSum{v.m, FF{v.sh, v.sl}}) : FF{0.f, 0.f};
             const FF L2 = ff_times_log2e(l);
@@ -898,10 +884,14 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
         e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
     }
-    const int64_t pre_blocks = (int64_t)B * a.M + ((int64_t)B * a.Lq + kPreThreads / 32 - 1) / (kPreThreads / 32);
+    int64_t pre_blocks = 2 * (int64_t)B * a.M + ((int64_t)B * a.Lq + kPreThreads / 32 - 1) / (kPreThreads / 32);
+    pre_blocks += pre_blocks & 1;  // whole clusters of two (a spare q-row CTA finds no task)
     if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     if (pre_blocks > 0) {
-        e = launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), 0, s, 0, a);
+        const size_t psmem = (size_t)a.C * sizeof(float2);
+        e = cudaFuncSetAttribute(k_verify_pre<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+        if (e != cudaSuccess) return e;
+        e = launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), psmem, s, 2, a);
         if (e != cudaSuccess) return e;
     }
     return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
