@@ -206,6 +206,16 @@ def algorithmic_bytes(w, sets, out_len, out_nodes):
     return draft_bytes, visited * row, staged_q * row, visited
 
 
+def max_over_ranks(value: float, dist, device) -> float:
+    """The largest of the ranks' values (every rank gets it): a job's time is its slowest
+    replica's. ``device`` is where the process group's backend reduces (cuda for nccl)."""
+    import torch
+
+    t = torch.tensor([float(value)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def run_tsb(args):
     import torch
 
@@ -272,9 +282,7 @@ def run_tsb(args):
         steps[k].run(events[k])
     torch.cuda.synchronize()
     if dist is not None:
-        t = torch.tensor([total_ms], device=device, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        total_ms = float(t.item())
+        total_ms = max_over_ranks(total_ms, dist, device)
     for st in sets:
         if tsb.tsb_device_status(st["buf"].ws) != 0:
             raise RuntimeError("device status bits set during the timed region")
