@@ -417,12 +417,15 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
                 }
             }
             const int winner = __ffs(c) - 1;
-            const unsigned long long wk = __shfl_sync(kFull, fr.bk, winner);
             const unsigned ww = __shfl_sync(kFull, fr.bw, winner);
             const long long wx = __shfl_sync(kFull, fr.bx, winner);
             if (ww == 0u) {  // frontier exhausted: only with N above the tree's capacity
                 if (lane == 0) raise_status(a.status, kDevBadTree);
                 break;
+            }
+            if (lane == winner) {  // the pop's record, before its slot is overwritten
+                rec_w[i] = ww;
+                rec_k[i] = (long long)fr.bk;
             }
             const int depth = 255 - (int)(ww >> 24);
             const int parent = 65535 - (int)((ww >> 8) & 0xffffu);
@@ -438,10 +441,6 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
                       xs);
             fr.put_if(kid && lane == (nchild & 31), nchild >> 5, okey_of(xc - cd1), w3_of(depth + 1, i, 0), xc);
             fr.rescan();
-            if (lane == 0) {
-                rec_w[i] = ww;
-                rec_k[i] = (long long)wk;
-            }
             nchild += kid ? 1 : 0;
         }
     }
@@ -536,16 +535,19 @@ cudaError_t launch_stats_topk_t(const TopkArgs &a, cudaStream_t s) {
     return launch_pdl(k_row_stats_topk<KCAP, T>, dim3((unsigned)(a.B * a.L)), dim3(kRowPlanThreads), smem, s, 0, a);
 }
 
-// The frontier kernel with as many slots per lane as N + 1 first children need.
+// The frontier kernel with as many slots per lane as N first children need.
 cudaError_t launch_heap(const HeapArgs &h, int B, cudaStream_t s) {
-    const int per_lane = (h.N + 1 + 31) / 32;
+    // Child numbers 0..N-1 need slots: child number c is created by pop c at the earliest, so
+    // number N can only come from the last pop and is never popped (its slot index N / 32 may
+    // lie past the last slot, where the predicated write matches no slot).
+    const int per_lane = (h.N + 31) / 32;
     if (per_lane <= 1) return launch_heap_t<1>(h, B, s);
     if (per_lane <= 2) return launch_heap_t<2>(h, B, s);
     if (per_lane <= 3) return launch_heap_t<3>(h, B, s);
     if (per_lane <= 4) return launch_heap_t<4>(h, B, s);
     if (per_lane <= 8) return launch_heap_t<8>(h, B, s);
     if (per_lane <= 16) return launch_heap_t<16>(h, B, s);
-    return launch_heap_t<33>(h, B, s);
+    return launch_heap_t<32>(h, B, s);  // N <= 1024
 }
 
 TopkArgs topk_args(const RowsDesc &draft, const float2 *stats, int L, int K, float invT, const PlanScratch &sc) {

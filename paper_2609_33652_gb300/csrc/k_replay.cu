@@ -95,11 +95,17 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
     const T *row = static_cast<const T *>(a.q) + (int64_t)b * a.bstride + (int64_t)r * a.rstride;
     const uint32_t ub = (uint32_t)b, un = (uint32_t)u;
     const int msel = min(m, a.C);
+    // One child: the draw is the Gumbel-max token, i.e. the top chunk by K_c and inside it the
+    // token with the largest raw key g_v (its shifted key is K_c itself and every other key of
+    // the chunk lies below K_c), so running maxima replace the lists and no key is shifted.
+    // The same loops serve both cases (one copy of the key arithmetic).
+    const bool single = m == 1;  // uniform over the CTA
 
     // 1. chunk keys: thread t takes chunks 4t..4t+3 (+1024k), one Philox block each
     {
         TopList<KCAP> cl;
         cl.clear();
+        uint64_t best = 0ull;
         for (int c4 = threadIdx.x * 4; c4 < a.C; c4 += 4 * kThreads) {
             const Words4 w = draw_block(a.seed, kReplayChunk, ub, un, (uint32_t)(c4 >> 2));
 #pragma unroll
@@ -108,18 +114,37 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
                 if (c < a.C) {
                     const float2 s = st[c];
                     const float Kc = (s.x + logf(s.y)) + gumbel_of(w.w[i]);
-                    cl.insert(pack_key(Kc, (uint32_t)c));
+                    const uint64_t k = pack_key(Kc, (uint32_t)c);
+                    if (single)
+                        best = k > best ? k : best;
+                    else
+                        cl.insert(k);
                 }
             }
         }
-        warp_top_to(cl, msel, cand[warp]);
+        if (single) {
+            best = warp_max_u64(best);
+            if (lane == 0) cand[warp][0] = best;
+        } else {
+            warp_top_to(cl, msel, cand[warp]);
+        }
     }
     __syncthreads();
-    if (warp == 0) merge_warps<KCAP>(cand, msel, sel);
+    if (warp == 0) {
+        if (single) {
+            const uint64_t v = warp_max_u64(lane < kWarps ? cand[lane][0] : 0ull);
+            if (lane == 0) sel[0] = v;
+        } else {
+            merge_warps<KCAP>(cand, msel, sel);
+        }
+    }
     __syncthreads();
 
     // 2. element keys of each kept chunk (one warp per chunk), shifted to the chunk key
     {
+        // K*, the smallest kept chunk key, bounds the drawn keys from below when m chunks are
+        // kept (m <= C)
+        const float kstar = msel == m ? key_value(sel[msel - 1]) : -INFINITY;
         TopList<KCAP> el;
         el.clear();
         for (int s = warp; s < msel; s += kWarps) {
@@ -144,16 +169,38 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
                 }
             }
             zk = warp_max_u64(zk);
+            if (single) {  // warp 0 only (msel = 1)
+                const int child = kids[0];
+                if (lane == 0) {
+                    if (child > 0 && child < NN)
+                        a.token[(int64_t)b * NN + child] = (int32_t)key_id(zk);
+                    else
+                        raise_status(a.status, kDevBadTree);
+                }
+                continue;
+            }
             const float Z = key_value(zk);
             const uint32_t jmax = key_id(zk);
+            // The m kept chunks' maxima hold keys K_c >= K* (the m-th chunk key), so a key below
+            // K* is never drawn. The shifted key grows with g, and k_v >= K* exactly when
+            //   g_v >= g* = Z - softplus((Z - K*) + log(-expm1(K* - T_c))),
+            // so only elements with g_v >= g* - margin (rounding of g* and of the keys) get a
+            // shifted key and a list entry.
+            float gmin = -INFINITY;
+            if (kstar != -INFINITY) {
+                const float w = __fadd_rn(__fsub_rn(Z, kstar), logf(-expm1f(__fsub_rn(kstar, Tc))));
+                const float sp = w == -INFINITY ? 0.f : fmaxf(w, 0.f) + log1pf(expf(-fabsf(w)));
+                gmin = __fsub_rn(__fsub_rn(Z, sp), 1e-3f * (1.f + fabsf(Z)));
+            }
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
-                if (v0 + i >= a.V) continue;
+                if (v0 + i >= a.V || !(g[i] >= gmin)) continue;
                 const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_key(Tc, Z, g[i]);
                 el.insert(pack_key(k, (uint32_t)(v0 + i)));
             }
         }
-        __syncthreads();  // the chunk lists in cand[] are no longer needed
+        if (single) return;  // uniform over the CTA
+        __syncthreads();     // the chunk lists in cand[] are no longer needed
         warp_top_to(el, m, cand[warp]);
     }
     __syncthreads();

@@ -6,7 +6,7 @@ import torch
 
 import helpers
 import oracle
-from gpu_harness import check_status, gpu_plan, run_step
+from gpu_harness import Report, check_status, compare_plan, gpu_plan, run_step
 from paper_2609_33652_gb300 import synth, tsb
 
 pytestmark = pytest.mark.gpu
@@ -180,6 +180,35 @@ def test_plan_rows_matches_separate_calls(B, R, L, N, K, V, kind, dtype):
     assert bool((gs[:, L:] == -7.0).all())  # rows the plan does not read are not written
     for k in ("parent", "depth", "rank", "plan_token", "score", "child_off", "child_ids"):
         assert torch.equal(got.tree[k], ref.tree[k]), k
+
+
+@pytest.mark.parametrize("B,L,N,K,V,kind,dtype", [
+    (2, 4, 1024, 32, 5003, "normal3", "f32"),   # the largest budget, 33 frontier slots per lane
+    (2, 64, 1024, 2, 1000, "planted", "bf16"),  # the deepest tree (64 levels)
+    (3, 16, 500, 8, 5003, "planted", "bf16"),   # 16 slots per lane
+    (3, 16, 200, 4, 2048, "normal2", "f32"),    # 8 slots per lane
+])
+def test_plan_large_budgets(B, L, N, K, V, kind, dtype):
+    """Topology of large and deep budgets against the oracle's best-first expansion."""
+    draft = _draft(B, L, V, kind, dtype, 1010 + N)
+    buf = gpu_plan(draft, L, N, K, 1.0)
+    check_status(buf)
+    ref = oracle.plan(synth.to_host(draft), 1.0, N, K, L)
+    rep = Report()
+    same = compare_plan(buf, ref, rep, list(range(B)))
+    g = {k: v.cpu().numpy() for k, v in buf.tree.items()}
+    for b in range(B):
+        if same[b]:
+            continue
+        # a tree with flagged near ties that differs: still a best-first expansion, i.e. a
+        # valid tree whose path scores are the oracle's top-N scores up to the near ties
+        par, dep, rk = g["parent"][b], g["depth"][b], g["rank"][b]
+        assert (par[1:] < np.arange(1, N + 1)).all() and (dep[1:] == dep[par[1:]] + 1).all()
+        for u in range(N + 1):
+            kids = g["child_ids"][b][g["child_off"][b][u]:g["child_off"][b][u + 1]]
+            assert (par[kids] == u).all() and (rk[kids] == np.arange(len(kids))).all()
+        np.testing.assert_allclose(np.sort(g["score"][b]), np.sort(ref["score"][b]), rtol=1e-5, atol=1e-5)
+    assert sum(same.values()) >= 1 or all(ref["exempt"]), rep
 
 
 def test_plan_rows_flags_nonfinite():
