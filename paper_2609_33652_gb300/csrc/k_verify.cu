@@ -48,7 +48,6 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
-constexpr int kStageWarps = 14;       // warps that stage the target slice
 constexpr int kQWarp = 14;            // q-row log-normaliser
 constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
 constexpr int kPreTop = 8;            // highest-scoring node ids the pre-pass covers
@@ -146,6 +145,7 @@ struct Scratch {
     int path[kMaxDepthRows];      // accepted node ids (written out after the walk)
     float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
     FF l2q[kMaxDepthRows];        // per-depth q log-normalisers (times log2 e)
+    float2 cst[2][kMaxSliceChunks];  // chunk statistics of the slice, alternating per staged node
 };
 
 // One cluster-wide reduction: warp reductions, the CTA's warp partials in warp 0, the
@@ -189,27 +189,36 @@ __device__ __forceinline__ float point_residual(float p0, float q, const float *
     return p;
 }
 
-// Per-thread (max, sum of exp(x - max)) accumulation: batches are added as a maximum first
-// (rebase) and then a plain sum of exponentials relative to the running maximum.
-struct OnlineLse {
-    float m = -INFINITY;
-    KahanF s;
-    __device__ __forceinline__ MaxSum value() const { return MaxSum{m, s.ff()}; }
-    __device__ __forceinline__ void rebase(float bm) {
-        if (bm > m) {
-            if (m != -INFINITY) {
-                const float scale = fast_exp2(__fmul_rn(__fsub_rn(m, bm), kLog2e));
-                s.s = __fmul_rn(s.s, scale);
-                s.c = __fmul_rn(s.c, scale);
-            }
-            m = bm;
-        }
-    }
-};
-
 __device__ __forceinline__ float4 ld4(const float *p, int j) { return *reinterpret_cast<const float4 *>(p + j); }
 __device__ __forceinline__ void st4(float *p, int j, float a, float b, float c, float d) {
     *reinterpret_cast<float4 *>(p + j) = make_float4(a, b, c, d);
+}
+
+// A row's log-normaliser from its chunk statistics (m_c, s_c) in shared memory, over a fixed
+// partition: thread t < 128 takes chunks t, t + 128, ... (their maximum, then a Kahan sum of
+// s_c e^(m_c - m)), each of warps 0..3 merges its lanes (lse_part), and warp 0 merges the
+// four warps in order (lse_final, result times log2 e). Every kernel that needs a target
+// row's normaliser calls these two functions, kept out of line, so the value does not depend
+// on which kernel or CTA computed it.
+__device__ __noinline__ Slot lse_part(const float2 *pst, int C) {
+    float m = -INFINITY;
+    for (int c = threadIdx.x; c < C; c += 128) m = fmaxf(m, pst[c].x);
+    KahanF acc;
+    if (m != -INFINITY)
+        for (int c = threadIdx.x; c < C; c += 128) acc.add(__fmul_rn(pst[c].y, expf(__fsub_rn(pst[c].x, m))));
+    Slot mine = neutral_slot();
+    const FF sv = acc.ff();
+    mine.m = m;
+    mine.sh = sv.hi;
+    mine.sl = sv.lo;
+    return warp_reduce_slot<kRedLse>(mine);
+}
+
+__device__ __noinline__ FF lse_final(const Slot *part) {
+    const int lane = threadIdx.x & 31;
+    const Slot v = warp_reduce_slot<kRedLse>(lane < 4 ? part[lane] : neutral_slot());
+    const FF l = v.sh > 0.f ? maxsum_lse(MaxSum{v.m, FF{v.sh, v.sl}}) : FF{0.f, 0.f};
+    return ff_times_log2e(l);
 }
 
 template <typename T>
@@ -225,11 +234,11 @@ struct Walk {
     static __device__ __forceinline__ int quad_at(int cl, int h, int lane) { return cl * kChunk + h * 128 + 4 * lane; }
 
     // Stage x = fp32(z) * invT of this CTA's slice of `row` into dst (warps 0..nw-1; logits
-    // past the vocabulary become -inf), optionally with the online log-normaliser, or store
-    // exp(x - L) instead of x (the normalised law). Loads are issued in batches of kB chunks
-    // per warp before any is used, so a slice costs one memory round trip per batch.
+    // past the vocabulary become -inf), or store exp(x - L) instead of x (the normalised
+    // law). Loads are issued in batches of kB chunks per warp before any is used, so a slice
+    // costs one memory round trip per batch.
     template <bool NORMALISE>
-    __device__ void stage(const T *row, float *dst, int nw, OnlineLse *lse, FF L2) {
+    __device__ void stage(const T *row, float *dst, int nw, FF L2) {
         constexpr int kB = sizeof(T) == 2 ? 8 : 4;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         if (warp >= nw) return;
@@ -244,22 +253,6 @@ struct Walk {
                     raw[e][1].load(row, lo + quad_at(cl, 1, lane), end);
                 }
             }
-            if (!NORMALISE && lse) {  // the batch's maximum first (rounding is monotone: max z, then * invT)
-                float zm = -INFINITY;
-#pragma unroll
-                for (int e = 0; e < kB; ++e) {
-                    if (c0 + e * nw >= nch) break;
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        float z[4];
-                        raw[e][h].unpack(z);
-                        zm = fmaxf(zm, fmaxf(fmaxf(z[0], z[1]), fmaxf(z[2], z[3])));
-                    }
-                }
-                lse->rebase(__fmul_rn(zm, a.invT));
-            }
-            const float mref = (!NORMALISE && lse) ? lse->m : 0.f;
-            float t0 = 0.f, t1 = 0.f;
 #pragma unroll
             for (int e = 0; e < kB; ++e) {
                 const int cl = c0 + e * nw;
@@ -273,19 +266,82 @@ struct Walk {
                     if (NORMALISE) {
 #pragma unroll
                         for (int k = 0; k < 4; ++k) x[k] = exp_shifted(x[k], L2);
-                    } else if (lse && lse->m != -INFINITY) {
-                        // exp(x - m) = 2^((x - m) log2 e): the difference first, so the exponent
-                        // carries no rounding of m itself
-                        t0 += fast_exp2(__fmul_rn(__fsub_rn(x[0], mref), kLog2e)) +
-                              fast_exp2(__fmul_rn(__fsub_rn(x[1], mref), kLog2e));
-                        t1 += fast_exp2(__fmul_rn(__fsub_rn(x[2], mref), kLog2e)) +
-                              fast_exp2(__fmul_rn(__fsub_rn(x[3], mref), kLog2e));
                     }
                     st4(dst, quad_at(cl, h, lane), x[0], x[1], x[2], x[3]);
                 }
             }
-            if (!NORMALISE && lse && lse->m != -INFINITY) lse->s.add(__fadd_rn(t0, t1));
         }
+    }
+
+    // Stage this CTA's slice of `row` in the chunk-statistics layout (eight lanes per 256-logit
+    // chunk, lane g holding logits 8g..8g+7 of each 64-logit quarter; four chunks per warp and
+    // unit, two units in flight for bf16): the statistics of every chunk of the slice into
+    // cst[] (the per-chunk code of the statistics kernels) and, with dst, x = fp32(z) * invT
+    // into dst (logits past the vocabulary become -inf). Every warp takes part.
+    __device__ void stage_chunks(const T *row, float *dst, float2 *cst) {
+        constexpr int kU = sizeof(T) == 2 ? 2 : 1;
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        const int g = lane & 7, q = lane >> 3;
+        const float c2 = __fmul_rn(a.invT, kLog2e);
+        const int units = (nch + 3) / 4;
+        for (int u0 = warp; u0 < units; u0 += kU * kWarps) {  // uniform over the warp
+            RawGroup<T> raw[kU][4];
+#pragma unroll
+            for (int e = 0; e < kU; ++e) {
+                const int cl = (u0 + e * kWarps) * 4 + q;
+                if (u0 + e * kWarps < units && cl < nch)
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) raw[e][k].load(row, lo + cl * kChunk + k * 64 + g * 8, a.V);
+            }
+#pragma unroll
+            for (int e = 0; e < kU; ++e) {
+                const int cl = (u0 + e * kWarps) * 4 + q;
+                const bool live = u0 + e * kWarps < units && cl < nch;
+                float mc, sc;
+                chunk_stats8<T>(raw[e], live, a.invT, c2, &mc, &sc);
+                if (live && g == 0) cst[cl] = make_float2(mc, sc);
+                if (dst && live) {
+#pragma unroll
+                    for (int k = 0; k < 4; ++k) {
+                        float z[8];
+                        raw[e][k].unpack(z);
+                        const int j = cl * kChunk + k * 64 + g * 8;
+                        st4(dst, j, __fmul_rn(z[0], a.invT), __fmul_rn(z[1], a.invT), __fmul_rn(z[2], a.invT),
+                            __fmul_rn(z[3], a.invT));
+                        st4(dst, j + 4, __fmul_rn(z[4], a.invT), __fmul_rn(z[5], a.invT), __fmul_rn(z[6], a.invT),
+                            __fmul_rn(z[7], a.invT));
+                    }
+                }
+            }
+        }
+    }
+
+    // The log-normaliser of a row whose chunk statistics every CTA of the cluster has staged
+    // into its cst[] (slice / 256 chunks per CTA): each CTA gathers all of them into `tmp`
+    // through distributed shared memory and computes the value itself (identical in every
+    // CTA); warp kQWarp meanwhile runs `side`. Ends with the value in sh.L2t.
+    template <typename F>
+    __device__ void gather_lse(const float2 *cst, float2 *tmp, F side) {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        cluster.sync();  // every CTA's chunk statistics are written
+        const int per = a.slice / kChunk;
+        for (int c = threadIdx.x; c < a.C; c += kThreads) {
+            const int r = c / per;
+            tmp[c] = *cluster.map_shared_rank(&cst[c - r * per], r);
+        }
+        __syncthreads();
+        if (warp < 4) {
+            const Slot w = lse_part(tmp, a.C);
+            if (lane == 0) sh.wpart[warp] = w;
+        } else if (warp == kQWarp) {
+            side();
+        }
+        __syncthreads();
+        if (warp == 0) {
+            const FF L2 = lse_final(sh.wpart);
+            if (lane == 0) sh.L2t = L2;
+        }
+        __syncthreads();
     }
 
     // Ask L2 for this CTA's slice of a row that is likely needed soon (one request per 128 B).
@@ -386,7 +442,7 @@ struct Walk {
     // Bonus draw from the logits of `row` (a leaf, or a residual without mass).
     __device__ int draw_from_row(const T *row, int node) {
         __syncthreads();
-        stage<false>(row, P, kWarps, nullptr, FF{0.f, 0.f});
+        stage<false>(row, P, kWarps, FF{0.f, 0.f});
         __syncthreads();
         return draw<true>(node, [&](int j, float *v) {
             const float4 x = ld4(P, j);
@@ -502,27 +558,13 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     }
     cluster.sync();  // rank 1 may leave; rank 0's copy is complete (the barrier also orders the CTA)
     if (warp < 4) {  // the log-normaliser over threads 0..127, then warps 0..3 in order
-        float m = -INFINITY;
-        for (int c = threadIdx.x; c < C; c += 128) m = fmaxf(m, pst[c].x);
-        KahanF acc;
-        if (m != -INFINITY)
-            for (int c = threadIdx.x; c < C; c += 128) acc.add(__fmul_rn(pst[c].y, expf(__fsub_rn(pst[c].x, m))));
-        Slot mine = neutral_slot();
-        const FF sv = acc.ff();
-        mine.m = m;
-        mine.sh = sv.hi;
-        mine.sl = sv.lo;
-        const Slot w = warp_reduce_slot<kRedLse>(mine);
+        const Slot w = lse_part(pst, C);
         if (lane == 0) part[warp] = w;
     }
     __syncthreads();
     if (warp == 0) {
-        const Slot v = warp_reduce_slot<kRedLse>(lane < 4 ? part[lane] : neutral_slot());
-        if (lane == 0) {
-            const FF l = v.sh > 0.f ? maxsum_lse(MaxSum{v.m, FF{v.sh, v.sl}}) : FF{0.f, 0.f};
-            const FF L2 = ff_times_log2e(l);
-            a.pre[(int64_t)b * NN + j].l2t = make_float2(L2.hi, L2.lo);
-        }
+        const FF L2 = lse_final(part);
+        if (lane == 0) a.pre[(int64_t)b * NN + j].l2t = make_float2(L2.hi, L2.lo);
     }
 }
 
@@ -626,7 +668,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
 
     cluster.sync();  // the copy is complete; every CTA of the cluster runs before any distributed access
 
-    int u = 0, nacc = 0, final_tok = -1;
+    int u = 0, nacc = 0, final_tok = -1, ncst = 0;
     bool bad = sh.cbad != 0;  // every CTA checked the same arrays
     for (int step = 0; step <= a.L && !bad; ++step) {
         const int o = s_off[u], m = s_off[u + 1] - o;
@@ -660,21 +702,18 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
                                  (int64_t)s_kid[o] * a.t_rstride);
             }
             __syncthreads();  // earlier readers of P and Q are done
-            // staging with the target log-normaliser; a per-node q row's normaliser on warp 14
-            const int nstage = per_depth ? kStageWarps + 1 : kStageWarps;
-            OnlineLse lt;
-            if (warp < nstage) {
-                W.template stage<false>(trow, P, nstage, &lt, FF{0.f, 0.f});
-            } else if (warp == kQWarp) {
-                const FF v = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
-                if (lane == 0) sh.L2q = v;
-            }
-            Slot mine = neutral_slot();
-            const MaxSum t1 = lt.value();
-            mine.m = t1.m;
-            mine.sh = t1.s.hi;
-            mine.sl = t1.s.lo;
-            reduce_round<kRedLse>(sh, par, cluster, mine);
+            // x into P with the slice's chunk statistics, then the row's log-normaliser from all
+            // chunks of the cluster (gathered into Q, free until the node's first rejection);
+            // a per-node q row's normaliser on warp 14 meanwhile
+            float2 *cst = sh.cst[ncst];
+            ncst ^= 1;  // a CTA may stage its next node while another still reads this one
+            W.stage_chunks(trow, P, cst);
+            W.gather_lse(cst, reinterpret_cast<float2 *>(Q), [&] {
+                if (!per_depth) {
+                    const FF v = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
+                    if (lane == 0) sh.L2q = v;
+                }
+            });
             L2t = sh.L2t;
             L2q = per_depth ? sh.l2q[r] : sh.L2q;
         }
@@ -693,8 +732,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             }
             if (!staged || !q_staged) {  // the slices a rejection needs, once per node
                 __syncthreads();         // earlier readers of P and Q are done
-                if (!staged) W.template stage<false>(trow, P, kWarps, nullptr, FF{0.f, 0.f});
-                W.template stage<true>(qrow, Q, kWarps, nullptr, L2q);
+                if (!staged) W.template stage<false>(trow, P, kWarps, FF{0.f, 0.f});
+                W.template stage<true>(qrow, Q, kWarps, L2q);
                 __syncthreads();
                 staged = q_staged = true;
             }
