@@ -54,65 +54,109 @@ __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t 
         for (++j; j < n; ++j) dst[j] = 0ull;
 }
 
+// Number of keys in keys[0..n) larger than v (the keys are distinct).
+__device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t v) {
+    int r = 0;
+    for (int j = 0; j < n; ++j) r += keys[j] > v ? 1 : 0;
+    return r;
+}
+
 // The top-K pass of one draft row from its chunk statistics st[0..C) in shared memory (all NT
-// threads of the CTA call it, after a barrier that follows the last write of st): the
-// float-float log-normaliser, tau = the K-th largest chunk maximum (a lower bound on the K-th
-// largest logit, since K distinct chunk maxima reach it), the logits >= tau of the chunks whose
-// maximum reaches tau (a chunk goes to the warp that scans it, four chunks' loads per batch),
-// then per-warp and CTA merges. Writes lse[row], topk_x / topk_id [row][K].
+// threads of the CTA call it, after a barrier that follows the last write of st; cand has room
+// for C keys): the float-float log-normaliser; tau = the K-th largest chunk maximum (a lower
+// bound on the K-th largest logit, since K distinct chunk maxima reach it), found by rank
+// among the chunk keys that reach a cheap lower bound (the K-th largest of the warps' top
+// keys); the logits >= tau of the chunks whose maximum reaches tau (a chunk goes to the warp
+// that scans it, four chunks' loads per batch), ranked in shared memory (per-warp lists and
+// merges when more than C logits reach tau). Writes lse[row], topk_x / topk_id [row][K].
 template <int KCAP, int NT, typename T>
-__device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st) {
+__device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st, uint64_t *cand) {
     constexpr int NW = NT / 32;
-    static_assert(NW >= 2, "warps 0 and 1 merge in parallel");
+    static_assert(NW >= 2, "warps 0 and 1 work in parallel");
+    constexpr int kLseThreads = 128, kLseWarps = kLseThreads / 32;
+    static_assert(NT >= kLseThreads, "the partition needs kLseThreads threads");
+    constexpr int kLseWarp0 = NW - kLseWarps;  // the log-normaliser runs on the last four warps
     __shared__ uint64_t wl[NW][KCAP];
     __shared__ float wm[4], wsh[4], wsl[4];
     __shared__ float s_tau;
+    __shared__ uint64_t s_lb;
+    __shared__ int s_n, s_n2;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int b = row / a.L, d = row - (row / a.L) * a.L;
     const int C = a.C, K = a.K;
-    // 1. per-thread list of chunk maxima; log-normaliser partials over a fixed partition of
-    //    kLseThreads threads (whatever NT is, so every caller sums in the same order)
+    const int r = (K + NW - 1) / NW;  // each warp's share of the lower bound (NW * r <= 32)
+    // 1. per-thread list of chunk keys; log-normaliser partials over a fixed partition of
+    //    kLseThreads threads (the same for every caller, so every caller sums in one order)
     TopList<KCAP> cl;
     cl.clear();
     for (int c = threadIdx.x; c < C; c += NT) cl.insert(pack_key(st[c].x, (uint32_t)c));
-    constexpr int kLseThreads = 128, kLseWarps = kLseThreads / 32;
-    static_assert(NT >= kLseThreads, "the partition needs kLseThreads threads");
-    if (threadIdx.x < kLseThreads) {
+    if (warp >= kLseWarp0) {
+        const int t = threadIdx.x - kLseWarp0 * 32;
         float m = -INFINITY;
-        for (int c = threadIdx.x; c < C; c += kLseThreads) m = fmaxf(m, st[c].x);
+        for (int c = t; c < C; c += kLseThreads) m = fmaxf(m, st[c].x);
         KahanF acc;
         if (m != -INFINITY)
-            for (int c = threadIdx.x; c < C; c += kLseThreads)
-                acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
+            for (int c = t; c < C; c += kLseThreads) acc.add(__fmul_rn(st[c].y, expf(__fsub_rn(st[c].x, m))));
         const MaxSum ms = warp_maxsum(MaxSum{m, acc.ff()});
         if (lane == 0) {
-            wm[warp] = ms.m;
-            wsh[warp] = ms.s.hi;
-            wsl[warp] = ms.s.lo;
+            wm[warp - kLseWarp0] = ms.m;
+            wsh[warp - kLseWarp0] = ms.s.hi;
+            wsl[warp - kLseWarp0] = ms.s.lo;
         }
     }
-    // 2. each warp's K largest chunk maxima
-    warp_top_to(cl, K, wl[warp]);
+    // 2. each warp's r largest chunk keys
+    for (int j = 0; j < r; ++j) {
+        const uint64_t best = warp_pop_max(cl);
+        if (lane == 0) wl[warp][j] = best;
+    }
     __syncthreads();
     if (warp == 0) {
+        // 3. lower bound of tau (= the K-th largest chunk key): the K-th largest of the warps'
+        //    keys (K distinct chunk keys reach it), or 0 when they hold fewer than K keys
+        const uint64_t v = lane < NW * r ? wl[lane / r][lane - (lane / r) * r] : 0ull;
+        int rk = 0, nz = 0;
+        for (int j = 0; j < 32; ++j) {
+            const uint64_t w = __shfl_sync(kFull, v, j);
+            rk += w > v ? 1 : 0;
+            nz += w != 0ull ? 1 : 0;
+        }
+        if (nz < K) {
+            if (lane == 0) s_lb = 0ull;
+        } else if (v != 0ull && rk == K - 1) {
+            s_lb = v;
+        }
+        if (lane == 0) {
+            s_tau = -INFINITY;  // fewer than K chunks
+            s_n = 0;
+            s_n2 = 0;
+        }
+    } else if (warp == 1) {  // in parallel with warp 0
         MaxSum v = lane < kLseWarps ? MaxSum{wm[lane], FF{wsh[lane], wsl[lane]}} : MaxSum{-INFINITY, FF{0.f, 0.f}};
         v = warp_maxsum(v);
         if (lane == 0) {
             const FF l = maxsum_lse(v);
             a.lse[row] = make_float2(l.hi, l.lo);
         }
-    } else if (warp == 1) {  // in parallel with warp 0
-        // tau = K-th largest chunk maximum (-inf with fewer than K chunks)
-        TopList<KCAP> t;
-        t.clear();
-        for (int e = lane; e < NW * K; e += 32) t.insert(wl[e / K][e % K]);
-        uint64_t kth = 0;
-        for (int j = 0; j < K; ++j) kth = warp_pop_max(t);
-        if (lane == 0) s_tau = C >= K ? key_value(kth) : -INFINITY;
+    }
+    __syncthreads();
+    // 4. the chunk keys at or above the bound, then tau by rank among them
+    const uint64_t lb = s_lb;
+    for (int c = threadIdx.x; c < C; c += NT) {
+        const uint64_t k = pack_key(st[c].x, (uint32_t)c);
+        if (k >= lb) cand[atomicAdd(&s_n, 1)] = k;
+    }
+    __syncthreads();
+    if (C >= K) {
+        const int n = s_n;
+        for (int i = threadIdx.x; i < n; i += NT) {
+            const uint64_t v = cand[i];
+            if (rank_among(cand, n, v) == K - 1) s_tau = key_value(v);
+        }
     }
     __syncthreads();
     const float tau = s_tau;
-    // 3. the logits >= tau of the chunks whose maximum reaches tau
+    // 5. the logits >= tau of the chunks whose maximum reaches tau: into cand (up to C of them)
+    //    and into per-lane lists for the case of more
     const T *rowp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
     TopList<KCAP> el;
     el.clear();
@@ -143,13 +187,31 @@ __device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st) {
                 for (int i = 0; i < 8; ++i) {
                     if (v0 + i >= a.V) continue;
                     const float xi = __fmul_rn(x[k][i], a.invT);
-                    if (xi >= tau) el.insert(pack_key(xi, (uint32_t)(v0 + i)));
+                    if (xi >= tau) {
+                        const uint64_t key = pack_key(xi, (uint32_t)(v0 + i));
+                        el.insert(key);
+                        const int idx = atomicAdd(&s_n2, 1);
+                        if (idx < C) cand[idx] = key;
+                    }
                 }
             }
         }
     }
-    // 4. per warp top-K, then the CTA's
-    warp_top_to(el, K, wl[warp]);  // wl was last read before the barrier above
+    __syncthreads();
+    const int n2 = s_n2;
+    if (n2 <= C) {  // 6. the top K by rank (at least K logits reach tau)
+        for (int i = threadIdx.x; i < n2; i += NT) {
+            const uint64_t v = cand[i];
+            const int rk = rank_among(cand, n2, v);
+            if (rk < K) {
+                a.topk_id[(int64_t)row * K + rk] = (int32_t)key_id(v);
+                a.topk_x[(int64_t)row * K + rk] = key_value(v);
+            }
+        }
+        return;
+    }
+    // 6'. more than C logits reach tau (ties, flat rows): per warp top-K, then the CTA's
+    warp_top_to(el, K, wl[warp]);  // wl was last read before the barriers above
     __syncthreads();
     if (warp == 0) {
         TopList<KCAP> t;
@@ -189,7 +251,7 @@ __global__ void __launch_bounds__(kTopkThreads) k_row_topk(TopkArgs a) {
         }
     }
     __syncthreads();
-    topk_from_stats<KCAP, kTopkThreads, T>(a, row, st);
+    topk_from_stats<KCAP, kTopkThreads, T>(a, row, st, reinterpret_cast<uint64_t *>(st + C));
 }
 
 // One 16-warp CTA per draft row, streaming the row once: the chunk statistics exactly as
@@ -236,7 +298,7 @@ __global__ void __launch_bounds__(kRowPlanThreads, KCAP <= 8 ? 2 : 1) k_row_stat
     }
     if (bad) raise_status(a.status, kDevNonFinite);
     __syncthreads();
-    topk_from_stats<KCAP, kRowPlanThreads, T>(a, row, st);
+    topk_from_stats<KCAP, kRowPlanThreads, T>(a, row, st, reinterpret_cast<uint64_t *>(st + C));
 }
 
 struct HeapArgs {
@@ -520,7 +582,7 @@ cudaError_t launch_heap_t(const HeapArgs &h, int B, cudaStream_t s) {
 
 template <int KCAP, typename T>
 cudaError_t launch_topk_t(const TopkArgs &a, cudaStream_t s) {
-    const size_t smem = (size_t)a.C * sizeof(float2);
+    const size_t smem = (size_t)a.C * (sizeof(float2) + sizeof(uint64_t));  // statistics, candidates
     cudaError_t e = cudaFuncSetAttribute(k_row_topk<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(k_row_topk<KCAP, T>, dim3((unsigned)(a.B * a.L)), dim3(kTopkThreads), smem, s, 0, a);
@@ -528,7 +590,7 @@ cudaError_t launch_topk_t(const TopkArgs &a, cudaStream_t s) {
 
 template <int KCAP, typename T>
 cudaError_t launch_stats_topk_t(const TopkArgs &a, cudaStream_t s) {
-    const size_t smem = (size_t)a.C * sizeof(float2);
+    const size_t smem = (size_t)a.C * (sizeof(float2) + sizeof(uint64_t));  // statistics, candidates
     cudaError_t e =
         cudaFuncSetAttribute(k_row_stats_topk<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;

@@ -211,6 +211,48 @@ def test_plan_large_budgets(B, L, N, K, V, kind, dtype):
     assert sum(same.values()) >= 1 or all(ref["exempt"]), rep
 
 
+def _topk_scratch(buf, B, L, N, K):
+    """The first pass's per-row top-K (x, id) from the workspace: after the 256-byte header and
+    B*(N+1) 32-byte slots come B*L float2 log-normalisers, B*L*K x, B*L*K ids."""
+    off = 256 + B * (N + 1) * 32 + B * L * 8
+    x = buf.ws[off:off + B * L * K * 4].view(torch.float32).view(B * L, K).cpu().numpy()
+    ids = buf.ws[off + B * L * K * 4:off + B * L * K * 8].view(torch.int32).view(B * L, K).cpu().numpy()
+    return x, ids
+
+
+@pytest.mark.parametrize("dtype,K", [("f32", 8), ("bf16", 12), ("f32", 32)])
+@pytest.mark.parametrize("fused", [False, True])
+def test_topk_rows_exact(dtype, K, fused):
+    """Per-row top-K by (x desc, id asc) against a host sort, on rows with heavy ties: a flat
+    row (every logit reaches tau), a row whose maximum repeats 100 times, a planted row, and
+    random rows (ragged V)."""
+    B, L, N, V = 2, 4, 16, 5003
+    g = torch.Generator().manual_seed(77)
+    z = torch.randn(B, L, V, generator=g) * 3
+    z[0, 1] = 0.5
+    pos = torch.randperm(V, generator=g)[:100]
+    z[0, 2, pos] = z[0, 2].max() + 1.0
+    z[0, 3, 1234] = 12.0
+    rows = z.to(torch.bfloat16 if dtype == "bf16" else torch.float32)
+    stride = (V + 7) // 8 * 8
+    store = torch.zeros(B, L, stride, dtype=rows.dtype)
+    store[..., :V] = rows
+    draft = store.to(DEV)[..., :V]
+    buf = tsb.TsbBuffers.allocate(B, L, N, K, V, 1.0, device=DEV)
+    if fused:
+        tsb.tsb_plan_rows(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+    else:
+        tsb.tsb_row_stats(draft, 1.0, buf.stats, buf.ws)
+        tsb.tsb_plan(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+    check_status(buf)
+    gx, gid = _topk_scratch(buf, B, L, N, K)
+    x = rows.float().numpy().reshape(B * L, V)
+    for r in range(B * L):
+        order = np.lexsort((np.arange(V), -x[r]))[:K]
+        assert np.array_equal(gid[r], order), r
+        assert np.array_equal(gx[r], x[r][order]), r
+
+
 def test_plan_rows_flags_nonfinite():
     draft = _draft(2, 3, 512, "normal3", "f32", 15).clone()
     draft[1, 2, 100] = float("inf")
