@@ -54,13 +54,6 @@ __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t 
         for (++j; j < n; ++j) dst[j] = 0ull;
 }
 
-// Number of keys in keys[0..n) larger than v (the keys are distinct).
-__device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t v) {
-    int r = 0;
-    for (int j = 0; j < n; ++j) r += keys[j] > v ? 1 : 0;
-    return r;
-}
-
 // The top-K pass of one draft row from its chunk statistics st[0..C) in shared memory (all NT
 // threads of the CTA call it, after a barrier that follows the last write of st; cand has room
 // for C keys): the float-float log-normaliser; tau = the K-th largest chunk maximum (a lower

@@ -15,8 +15,12 @@
 // at ceil(V/256) + m_u*256 draws per parent instead of V.
 //
 // One CTA of 4 warps per (tree, node); nodes without children return at once. Chunk keys are
-// spread over the CTA (four chunks per thread share one Philox block), each warp then takes
-// one kept chunk, and per-warp candidate lists are merged in shared memory.
+// spread over the CTA (four chunks per thread share one Philox block) and kept in shared
+// memory; the top-m_u are ranked among those that reach a lower bound (the m_u-th largest of
+// the warps' few largest). Each warp then takes one kept chunk at a time; only elements whose
+// key can reach the m_u-th chunk key get a shifted key, and those are ranked in shared memory
+// (per-lane lists and merges when more of them than the buffer holds).
+// A parent with one child takes the Gumbel-max token directly (running maxima, no shift).
 #include "tsb_device.cuh"
 #include "tsb_launch.h"
 
@@ -69,11 +73,19 @@ __device__ __forceinline__ void merge_warps(const uint64_t (*cand)[CAP], int n, 
     warp_top_to(t, n, out);
 }
 
+// Shared-memory key buffer: every chunk key (C), then the chunk keys that reach the lower bound
+// (at most C) or up to max(C, kElemBuf) element keys.
+constexpr int kElemBuf = 512;
+__host__ __device__ inline int key_buf_len(int C) { return C + (C > kElemBuf ? C : kElemBuf); }
+
 template <int KCAP, typename T>
 __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay(ReplayArgs a) {
     pdl_begin();
     __shared__ uint64_t cand[kWarps][KCAP];
     __shared__ uint64_t sel[KCAP];
+    __shared__ uint64_t s_lb;
+    __shared__ int s_n, s_n2;
+    extern __shared__ uint64_t kbuf[];  // [key_buf_len(C)]
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int NN = a.N + 1;
     const int b = blockIdx.x / NN, u = blockIdx.x - (blockIdx.x / NN) * NN;
@@ -101,9 +113,13 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
     // The same loops serve both cases (one copy of the key arithmetic).
     const bool single = m == 1;  // uniform over the CTA
 
-    // 1. chunk keys: thread t takes chunks 4t..4t+3 (+1024k), one Philox block each
+    // 1. chunk keys: thread t takes chunks 4t..4t+3 (+1024k), one Philox block each; every key
+    //    goes to ckeys[c], each thread keeps its RR largest
+    constexpr int RR = KCAP / kWarps;  // >= rr = ceil(msel / kWarps): each warp's share below
+    uint64_t *ckeys = kbuf, *ebuf = kbuf + a.C;
+    const int ecap = key_buf_len(a.C) - a.C;
     {
-        TopList<KCAP> cl;
+        TopList<RR> cl;
         cl.clear();
         uint64_t best = 0ull;
         for (int c4 = threadIdx.x * 4; c4 < a.C; c4 += 4 * kThreads) {
@@ -115,27 +131,63 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
                     const float2 s = st[c];
                     const float Kc = (s.x + logf(s.y)) + gumbel_of(w.w[i]);
                     const uint64_t k = pack_key(Kc, (uint32_t)c);
-                    if (single)
+                    if (single) {
                         best = k > best ? k : best;
-                    else
+                    } else {
+                        ckeys[c] = k;
                         cl.insert(k);
+                    }
                 }
             }
         }
+        // the top msel chunk keys by rank among those that reach a lower bound: the msel-th
+        // largest of the warps' rr largest keys (every key when the warps hold fewer)
+        const int rr = (msel + kWarps - 1) / kWarps;  // kWarps * rr <= 32
         if (single) {
             best = warp_max_u64(best);
             if (lane == 0) cand[warp][0] = best;
         } else {
-            warp_top_to(cl, msel, cand[warp]);
+            for (int j = 0; j < rr; ++j) {
+                const uint64_t k = warp_pop_max(cl);
+                if (lane == 0) cand[warp][j] = k;
+            }
         }
-    }
-    __syncthreads();
-    if (warp == 0) {
-        if (single) {
-            const uint64_t v = warp_max_u64(lane < kWarps ? cand[lane][0] : 0ull);
-            if (lane == 0) sel[0] = v;
-        } else {
-            merge_warps<KCAP>(cand, msel, sel);
+        __syncthreads();
+        if (warp == 0) {
+            if (single) {
+                const uint64_t v = warp_max_u64(lane < kWarps ? cand[lane][0] : 0ull);
+                if (lane == 0) sel[0] = v;
+            } else {
+                const uint64_t v = lane < kWarps * rr ? cand[lane / rr][lane - (lane / rr) * rr] : 0ull;
+                int rk = 0, nz = 0;
+                for (int j = 0; j < kWarps * rr; ++j) {
+                    const uint64_t w = __shfl_sync(kFull, v, j);
+                    rk += w > v ? 1 : 0;
+                    nz += w != 0ull ? 1 : 0;
+                }
+                if (nz < msel) {
+                    if (lane == 0) s_lb = 0ull;  // every key
+                } else if (v != 0ull && rk == msel - 1) {
+                    s_lb = v;
+                }
+                if (lane == 0) {
+                    s_n = 0;
+                    s_n2 = 0;
+                }
+            }
+        }
+        __syncthreads();
+        if (!single) {  // the chunk keys that reach the bound, then the top msel by rank
+            const uint64_t lb = s_lb;
+            for (int c = threadIdx.x; c < a.C; c += kThreads)
+                if (ckeys[c] >= lb) ebuf[atomicAdd(&s_n, 1)] = ckeys[c];
+            __syncthreads();
+            const int n = s_n;
+            for (int i = threadIdx.x; i < n; i += kThreads) {
+                const uint64_t v = ebuf[i];
+                const int rk = rank_among(ebuf, n, v);
+                if (rk < msel) sel[rk] = v;
+            }
         }
     }
     __syncthreads();
@@ -196,12 +248,31 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
             for (int i = 0; i < 8; ++i) {
                 if (v0 + i >= a.V || !(g[i] >= gmin)) continue;
                 const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_key(Tc, Z, g[i]);
-                el.insert(pack_key(k, (uint32_t)(v0 + i)));
+                const uint64_t key = pack_key(k, (uint32_t)(v0 + i));
+                el.insert(key);
+                const int idx = atomicAdd(&s_n2, 1);
+                if (idx < ecap) ebuf[idx] = key;
             }
         }
         if (single) return;  // uniform over the CTA
         __syncthreads();     // the chunk lists in cand[] are no longer needed
-        warp_top_to(el, m, cand[warp]);
+        const int n2 = s_n2;
+        if (n2 <= ecap) {  // 3. the top-m keys by rank are the ordered draws
+            int32_t *tok = a.token + (int64_t)b * NN;
+            for (int i = threadIdx.x; i < n2; i += kThreads) {
+                const uint64_t v = ebuf[i];
+                const int rk = rank_among(ebuf, n2, v);
+                if (rk < m) {
+                    const int child = kids[rk];
+                    if (child > 0 && child < NN)
+                        tok[child] = (int32_t)key_id(v);
+                    else
+                        raise_status(a.status, kDevBadTree);
+                }
+            }
+            return;
+        }
+        warp_top_to(el, m, cand[warp]);  // more element keys than the buffer holds
     }
     __syncthreads();
 
@@ -224,7 +295,10 @@ template <int KCAP, typename T>
 cudaError_t launch_replay_t(const ReplayArgs &a, cudaStream_t s) {
     const int64_t blocks = (int64_t)a.B * (a.N + 1);
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    return launch_pdl(k_replay<KCAP, T>, dim3((unsigned)blocks), dim3(kThreads), 0, s, 0, a);
+    const size_t smem = (size_t)key_buf_len(a.C) * sizeof(uint64_t);
+    cudaError_t e = cudaFuncSetAttribute(k_replay<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_replay<KCAP, T>, dim3((unsigned)blocks), dim3(kThreads), smem, s, 0, a);
 }
 
 }  // namespace

@@ -296,6 +296,14 @@ struct TopList {
     }
 };
 
+// Number of keys in keys[0..n) larger than v (the keys are distinct); every thread of a warp
+// reading the same key is a shared-memory broadcast.
+__device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t v) {
+    int r = 0;
+    for (int j = 0; j < n; ++j) r += keys[j] > v ? 1 : 0;
+    return r;
+}
+
 // The largest of the lanes' 64-bit values (distinct unless zero): a hardware max over the
 // high words, then over the low words only among the lanes that tie. Returns the value to
 // every lane and the lane that holds it in *owner.

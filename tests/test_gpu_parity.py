@@ -105,6 +105,14 @@ def test_step_sweep_sampled(N, dtype):
     _assert_mostly_compared(rep, 0.9)
 
 
+def test_step_small_vocab_many_children():
+    """Parents with more children than vocabulary chunks (V=1000: 4 chunks, up to 8 children):
+    every element of the kept chunks is a replay candidate, more than the key buffer holds."""
+    draft = _draft(8, 4, 1000, "normal2", "f32", 31)
+    rep, _, _ = run_step(draft, 4, 40, 8, 1.0, seed=13, target_noise=0.7)
+    _assert_mostly_compared(rep, 0.9)
+
+
 def test_block_verification_chain():
     """Sampled chain (plan with K=1, replay = one draw per node) verified by block
     verification, on the batched workload's draft rows."""
