@@ -3,7 +3,7 @@
 //
 // One thread-block cluster per tree. CTA r of the cluster owns the chunk-aligned vocabulary
 // slice [r*slice, (r+1)*slice) and keeps that slice of the current node in shared memory as
-// fp32: P holds the target logits, later the current residual; Q holds the normalised draft
+// fp32: P holds the target logits, later their softmax P0; Q holds the normalised draft
 // law once a rejection needs it. Scalars (the target log-normaliser, residual masses, argmax
 // keys) are combined across the cluster through distributed shared memory: each CTA
 // publishes its partial, the cluster barrier orders the writes, and every CTA combines all
@@ -16,8 +16,12 @@
 //           on reject R_{i+1}(v) = max(p_i(v) - Q(v)/t_i, 0), Z_{i+1} = sum R_{i+1},
 //           p_{i+1} = R_{i+1}/Z_{i+1}, t_{i+1} = t_i - Q(y_i).
 //   A rejected token has p_{i+1} = 0 from then on, which is exactly the exclusion of drawn
-//   tokens from the renormalised draft law. Each pass is O(1) per element: P keeps R_i and
-//   p_i(v) = P[v] / Z_i; the point value p_i(y) repeats the same fp32 operations from P0(y).
+//   tokens from the renormalised draft law. The recursion has a closed form: subtracting
+//   non-negative multiples of Q and clamping at zero composes, so
+//   p_i(v) = max(P0(v) - A_i Q(v), 0) / D_i with A_{i+1} = A_i + D_i / t_i and D_{i+1} the
+//   mass of max(P0 - A_{i+1} Q, 0). P keeps P0 (a rejected token's entry set to zero), a pass
+//   per rejection reads P0 and Q and only sums, and the point value p_i(y) uses the same fp32
+//   operations as the element passes.
 // Final tokens (all children rejected: from R_m; leaf: bonus from the target row) are drawn
 // with the two-level Gumbel-max of the randomness contract: chunk keys log(chunk mass) + G
 // over chunks of 256 tokens, then the best token of the winning chunk.
@@ -140,7 +144,6 @@ struct Scratch {
     FF L2t, L2q;         // log-normalisers of the target and q rows, times log2(e)
     unsigned long long wbest[kWarps];
     unsigned long long cbest, tbest;
-    float izs[kMaxK], its[kMaxK];  // 1/Z and 1/t of every rejection so far
     int cbad;
     int path[kMaxDepthRows];      // accepted node ids (written out after the walk)
     float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
@@ -176,17 +179,6 @@ __device__ void reduce_round(Scratch &sh, int &par, const cg::cluster_group &clu
     }
     __syncthreads();
     par ^= 1;
-}
-
-// The residual after rejecting a slot: max(p - q/t, 0) with 1/t precomputed; one fma, so the
-// element passes and the point values produce the same bits.
-__device__ __forceinline__ float resid(float p, float q, float it) { return fmaxf(__fmaf_rn(-q, it, p), 0.f); }
-
-// p_i(y) from P0(y), Q(y): the same fp32 operations the element passes perform.
-__device__ __forceinline__ float point_residual(float p0, float q, const float *izs, const float *its, int i) {
-    float p = p0;
-    for (int j = 0; j < i; ++j) p = __fmul_rn(resid(p, q, its[j]), izs[j]);
-    return p;
 }
 
 __device__ __forceinline__ float4 ld4(const float *p, int j) { return *reinterpret_cast<const float4 *>(p + j); }
@@ -717,68 +709,75 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             L2t = sh.L2t;
             L2q = per_depth ? sh.l2q[r] : sh.L2q;
         }
+        // After i rejections p_i(v) = max(P0(v) - A_i Q(v), 0) / D_i with A_0 = 0, D_0 = 1,
+        // A_{i+1} = A_i + D_i / t_i and D_{i+1} = sum_v max(P0(v) - A_{i+1} Q(v), 0): the
+        // recursive residual max(p_i - Q/t_i, 0), renormalised, in closed form. A pass over the
+        // slice reads P0 and Q and writes nothing; a rejected token's P0 is set to zero.
         FF t = FF{1.f, 0.f};  // draft mass not yet drawn
         int accepted = -1;
         bool q_staged = false;
+        bool p_is_x = staged;  // P holds x (staged node) until its first pass stores P0
+        float A = 0.f, D = 1.f, iD = 1.f;
         for (int i = 0; i < m; ++i) {
             const float it = t.hi > 0.f ? __frcp_rn(t.hi) : 0.f;  // 1/t_i
             const float P0y = exp_shifted(s_cxt[o + i], L2t);
             const float Qy = exp_shifted(s_cxq[o + i], L2q);
-            const float pp = point_residual(P0y, Qy, sh.izs, sh.its, i);
+            const float pp = __fmul_rn(fmaxf(__fmaf_rn(-A, Qy, P0y), 0.f), iD);
             const float qp = __fmul_rn(Qy, it);
             if (__fmul_rn(s_cu[o + i], qp) < pp) {
                 accepted = s_kid[o + i];
                 break;
             }
+            __syncthreads();  // earlier readers of P and Q are done
             if (!staged || !q_staged) {  // the slices a rejection needs, once per node
-                __syncthreads();         // earlier readers of P and Q are done
-                if (!staged) W.template stage<false>(trow, P, kWarps, FF{0.f, 0.f});
+                if (!staged) W.template stage<true>(trow, P, kWarps, L2t);  // P0 directly
                 W.template stage<true>(qrow, Q, kWarps, L2q);
-                __syncthreads();
                 staged = q_staged = true;
+                __syncthreads();
             }
-            // p_i(v) of the quad at smem index j (P holds x before the first rejection, R_i
-            // afterwards)
-            const float izp = i > 0 ? sh.izs[i - 1] : 1.f;
-            auto p_quad = [&](int j, float *p) {
-                const float4 x = ld4(P, j);
-                if (i == 0) {
-                    p[0] = exp_shifted(x.x, L2t);
-                    p[1] = exp_shifted(x.y, L2t);
-                    p[2] = exp_shifted(x.z, L2t);
-                    p[3] = exp_shifted(x.w, L2t);
-                } else {
-                    p[0] = __fmul_rn(x.x, izp);
-                    p[1] = __fmul_rn(x.y, izp);
-                    p[2] = __fmul_rn(x.z, izp);
-                    p[3] = __fmul_rn(x.w, izp);
+            {  // the rejected token leaves the residual for good
+                const int y = s_tok[s_kid[o + i]];
+                if (threadIdx.x == 0 && y >= lo && y < lo + n) P[y - lo] = p_is_x ? -INFINITY : 0.f;
+            }
+            __syncthreads();
+            const float A1 = __fmaf_rn(D, it, A);
+            // max(P0 - A1 Q, 0) of the quad at shared-memory index j
+            auto w_quad = [&](int j, float *v) {
+                float4 x = ld4(P, j);
+                if (p_is_x) {
+                    x.x = exp_shifted(x.x, L2t);
+                    x.y = exp_shifted(x.y, L2t);
+                    x.z = exp_shifted(x.z, L2t);
+                    x.w = exp_shifted(x.w, L2t);
                 }
+                const float4 q = ld4(Q, j);
+                v[0] = fmaxf(__fmaf_rn(-A1, q.x, x.x), 0.f);
+                v[1] = fmaxf(__fmaf_rn(-A1, q.y, x.y), 0.f);
+                v[2] = fmaxf(__fmaf_rn(-A1, q.z, x.z), 0.f);
+                v[3] = fmaxf(__fmaf_rn(-A1, q.w, x.w), 0.f);
             };
-            if (i == m - 1) {  // every slot rejected: final token from R_m = max(p_i - Q/t_i, 0)
-                final_tok = W.template draw<false>(u, [&](int j, float *v) {
-                    float p[4];
-                    p_quad(j, p);
-                    const float4 q = ld4(Q, j);
-                    v[0] = resid(p[0], q.x, it);
-                    v[1] = resid(p[1], q.y, it);
-                    v[2] = resid(p[2], q.z, it);
-                    v[3] = resid(p[3], q.w, it);
-                });
+            if (i == m - 1) {  // every slot rejected: final token from R_m = max(P0 - A_m Q, 0)
+                final_tok = W.template draw<false>(u, w_quad);
                 if (final_tok < 0) final_tok = W.draw_from_row(trow, u);  // no residual mass (rounding)
                 break;
             }
-            // residual pass: R_{i+1} into P and its mass
+            // residual pass: the mass of R_{i+1} (storing P0 the first time P holds x)
             KahanF zl;
             for (int cl = warp; cl < W.nch; cl += kWarps) {
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
                     const int j = Walk<T>::quad_at(cl, h, lane);
-                    float p[4];
-                    p_quad(j, p);
-                    const float4 q = ld4(Q, j);  // padding: p = 0 (x = -inf), q = 0
-                    const float r0 = resid(p[0], q.x, it), r1 = resid(p[1], q.y, it);
-                    const float r2 = resid(p[2], q.z, it), r3 = resid(p[3], q.w, it);
-                    st4(P, j, r0, r1, r2, r3);
+                    float4 x = ld4(P, j);  // padding: P0 = 0 (x = -inf), Q = 0
+                    if (p_is_x) {
+                        x.x = exp_shifted(x.x, L2t);
+                        x.y = exp_shifted(x.y, L2t);
+                        x.z = exp_shifted(x.z, L2t);
+                        x.w = exp_shifted(x.w, L2t);
+                        st4(P, j, x.x, x.y, x.z, x.w);
+                    }
+                    const float4 q = ld4(Q, j);
+                    const float r0 = fmaxf(__fmaf_rn(-A1, q.x, x.x), 0.f), r1 = fmaxf(__fmaf_rn(-A1, q.y, x.y), 0.f);
+                    const float r2 = fmaxf(__fmaf_rn(-A1, q.z, x.z), 0.f), r3 = fmaxf(__fmaf_rn(-A1, q.w, x.w), 0.f);
                     zl.add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
                 }
             }
@@ -794,11 +793,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
                 final_tok = W.draw_from_row(trow, u);
                 break;
             }
-            if (threadIdx.x == 0) {
-                sh.izs[i] = __frcp_rn(Z);
-                sh.its[i] = it;
-            }
-            __syncthreads();
+            p_is_x = false;
+            A = A1;
+            D = Z;
+            iD = __frcp_rn(Z);
             t = ff_add(t, FF{-Qy, 0.f});
         }
         if (accepted < 0) break;
