@@ -32,9 +32,12 @@
 // children's target and q logits and their acceptance uniforms to shared memory once. At a
 // node below M it needs no staging and no cluster round: every CTA takes the same decisions
 // from the same inputs, and the slice is staged only if a rejection needs the residual. At
-// any other node warps 0..13 (0..14 for per-depth q rows) stage the target slice (one batch
-// of loads per warp, then the online log-normaliser) while warp 14 computes a per-node q
-// row's log-normaliser from its chunk statistics. Element passes give lane l the elements
+// any other node every warp stages the target slice in the chunk-statistics layout (x into
+// shared memory, each chunk's statistics beside it), every CTA gathers all chunk statistics
+// of the row through distributed shared memory and computes its log-normaliser, while warp
+// kQWarp computes a per-node q row's log-normaliser from its chunk statistics. 12 warps per
+// CTA: 160 registers a thread without spills (16 warps at 128 spilled in the walk's
+// hot paths and ran slower). Element passes give lane l the elements
 // 4l..4l+3 and 128+4l..128+4l+3 of each 256-token chunk, so every shared-memory access is a
 // conflict-free 16-byte vector. Which path computes a node's normaliser depends only on its
 // id, so results do not depend on timing.
@@ -50,9 +53,9 @@ namespace cg = cooperative_groups;
 namespace tsb {
 namespace {
 
-constexpr int kThreads = 512;
+constexpr int kThreads = 384;
 constexpr int kWarps = kThreads / 32;
-constexpr int kQWarp = 14;            // q-row log-normaliser
+constexpr int kQWarp = 10;            // q-row log-normaliser
 constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
 constexpr int kPreTop = 8;            // highest-scoring node ids the pre-pass covers
 constexpr int kMaxDepthRows = 64;     // per-depth q rows (depth cap L <= 64)
@@ -231,7 +234,7 @@ struct Walk {
     // costs one memory round trip per batch.
     template <bool NORMALISE>
     __device__ void stage(const T *row, float *dst, int nw, FF L2) {
-        constexpr int kB = sizeof(T) == 2 ? 8 : 4;
+        constexpr int kB = sizeof(T) == 2 ? 9 : 5;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         if (warp >= nw) return;
         const int end = lo + n;
@@ -696,7 +699,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             __syncthreads();  // earlier readers of P and Q are done
             // x into P with the slice's chunk statistics, then the row's log-normaliser from all
             // chunks of the cluster (gathered into Q, free until the node's first rejection);
-            // a per-node q row's normaliser on warp 14 meanwhile
+            // a per-node q row's normaliser on warp kQWarp meanwhile
             float2 *cst = sh.cst[ncst];
             ncst ^= 1;  // a CTA may stage its next node while another still reads this one
             W.stage_chunks(trow, P, cst);
