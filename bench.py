@@ -352,11 +352,37 @@ def run_tsb(args):
         dist.destroy_process_group()
 
 
+def bind_near_gpu(device):
+    """Run the host side on the CPUs local to the GPU (as the kernel reports them for its PCI
+    function), so that pinned buffers allocated afterwards sit in the near memory: a buffer
+    on the far socket slows every host-to-device copy. Returns the CPU list, or None where
+    the topology is not exposed (the affinity is then left alone)."""
+    import torch
+
+    try:
+        pr = torch.cuda.get_device_properties(device)
+        addr = f"{pr.pci_domain_id:04x}:{pr.pci_bus_id:02x}:{pr.pci_device_id:02x}.0"
+        with open(f"/sys/bus/pci/devices/{addr}/local_cpulist") as f:
+            spec = f.read().strip()
+        cpus = set()
+        for part in spec.split(","):
+            lo, _, hi = part.partition("-")
+            cpus.update(range(int(lo), int(hi or lo) + 1))
+        cpus &= os.sched_getaffinity(0)
+        if not cpus:
+            return None
+        os.sched_setaffinity(0, cpus)
+        return spec
+    except (AttributeError, OSError, ValueError):
+        return None
+
+
 def run_e2e(args, w, sets, device):
     import torch
 
     from paper_2609_33652_gb300 import tsb
 
+    near = bind_near_gpu(device)
     S = len(sets)
     E = args.e2e_steps
     h_draft = [st["draft"].cpu().pin_memory() for st in sets]
@@ -390,7 +416,7 @@ def run_e2e(args, w, sets, device):
     h2d = (sets[0]["draft"].numel() + sets[0]["target"].numel()) * es
     d2h = h_tok.numel() * 4 + h_len.numel() * 4
     return {"value": round(us, 3), "unit": "us/step", "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h),
-            "steps": E}
+            "steps": E, "host_cpus": near}
 
 
 # ---------------------------------------------------------------------------------------
