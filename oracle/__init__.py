@@ -22,6 +22,13 @@ Parity status of each function (what pins it, see tests/test_oracle_*.py):
                      (Eq. rs-overlap); chi-square of the sampled path against the target.
   verify_block     : exact enumeration of the extended output law (= target law);
                      gamma = 1 reduces to rejection sampling; E[tau] >= token-wise RS.
+  plan_expand      : equals the heap planner once the frontier holds N; brute-force
+                     path enumeration of the layer-wise frontiers; prefix closure; its
+                     i-th path probability never above the heap's.
+  replay_mixed     : deterministic slots vs a stable sort; chi-square of the sampled slot
+                     against q renormalised over the remaining tokens; m = 1 is the WoR draw.
+  verify_naive     : chi-square of the emitted tokens against the target law; acceptance
+                     frequency vs the closed form p(y) (Sec. 2.3); forced acceptances.
 """
 from __future__ import annotations
 
@@ -85,6 +92,10 @@ def _load():
         "orc_verify_rrs": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P,
                                 _P]),
         "orc_blockv_law": (_I, [_I, _I, _P, _P, _P, _P, _P, _P]),
+        "orc_plan_expand": (_I, [_P, ctypes.c_float, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, ctypes.c_double,
+                                 _P]),
+        "orc_replay_mixed": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, ctypes.c_uint64, _P, _P, _P]),
+        "orc_verify_naive": (_I, [_P, ctypes.c_float, _I, _I, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _P]),
         "orc_verify_block": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P,
                                   _P, _P, _P]),
     }
@@ -180,6 +191,28 @@ def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps:
     return tree
 
 
+def plan_expand(draft: np.ndarray, temperature: float, N: int, K: int, L: int, W: int, key_eps: float = 1e-6):
+    """Expand-then-prune first pass with frontier width W; same outputs as ``plan``."""
+    lib = _load()
+    B = draft.shape[0]
+    NN = N + 1
+    d, keep = _logits(draft)
+    out = {k: np.zeros(B * NN, dtype=np.int32) for k in ("parent", "depth", "rank", "plan_token")}
+    score = np.zeros(B * NN)
+    child_off = np.zeros(B * (NN + 1), dtype=np.int32)
+    child_ids = np.zeros(B * N, dtype=np.int32)
+    exempt = np.zeros(B, dtype=np.uint8)
+    _check(lib.orc_plan_expand(ctypes.byref(d), temperature, N, K, L, W, _ptr(out["parent"]), _ptr(out["depth"]),
+                               _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score), _ptr(child_off),
+                               _ptr(child_ids), key_eps, _ptr(exempt)), "plan_expand")
+    tree = {k: v.reshape(B, NN) for k, v in out.items()}
+    tree["score"] = score.reshape(B, NN)
+    tree["child_off"] = child_off.reshape(B, NN + 1)
+    tree["child_ids"] = child_ids.reshape(B, N)
+    tree["exempt"] = exempt.astype(bool)
+    return tree
+
+
 def _tree_ptrs(tree):
     return (_i32(tree["depth"]), _i32(tree["child_off"]), _i32(tree["child_ids"]))
 
@@ -204,6 +237,40 @@ def replay(q: np.ndarray, temperature: float, tree, seed: int, qrow_of_node=None
     _check(lib.orc_replay(ctypes.byref(d), temperature, _ptr(qr), NN - 1, _ptr(depth), _ptr(off), _ptr(ids),
                           int(seed), _ptr(bids), _ptr(token), _ptr(exempt)), "replay")
     return token.reshape(B, NN), exempt.reshape(B, NN).astype(bool)
+
+
+def replay_mixed(q: np.ndarray, temperature: float, tree, seed: int, qrow_of_node=None, batch_ids=None):
+    """Mixed sampling: tokens [B, N+1] (root -1) and a per-parent near-tie flag."""
+    lib = _load()
+    bids = _i32(batch_ids)
+    B = q.shape[0]
+    NN = tree["depth"].shape[1]
+    d, keep = _logits(q)
+    depth, off, ids = _tree_ptrs(tree)
+    qr = _i32(qrow_of_node)
+    token = np.zeros(B * NN, dtype=np.int32)
+    exempt = np.zeros(B * NN, dtype=np.uint8)
+    _check(lib.orc_replay_mixed(ctypes.byref(d), temperature, _ptr(qr), NN - 1, _ptr(depth), _ptr(off), _ptr(ids),
+                                int(seed), _ptr(bids), _ptr(token), _ptr(exempt)), "replay_mixed")
+    return token.reshape(B, NN), exempt.reshape(B, NN).astype(bool)
+
+
+def verify_naive(target: np.ndarray, temperature: float, tree, token, seed: int, L: int, batch_ids=None):
+    """Target-sample matching down the tree; outputs as ``verify_rrs``."""
+    lib = _load()
+    bids = _i32(batch_ids)
+    B = target.shape[0]
+    NN = tree["child_off"].shape[1] - 1
+    dt, keep_t = _logits(target)
+    off, ids = _i32(tree["child_off"]), _i32(tree["child_ids"])
+    tok = _i32(token)
+    otok = np.zeros(B * (L + 1), dtype=np.int32)
+    onode = np.zeros(B * L, dtype=np.int32)
+    olen = np.zeros(B, dtype=np.int32)
+    ex = np.zeros(B, dtype=np.uint8)
+    _check(lib.orc_verify_naive(ctypes.byref(dt), temperature, NN - 1, L, _ptr(off), _ptr(ids), _ptr(tok), int(seed),
+                                _ptr(bids), _ptr(otok), _ptr(onode), _ptr(olen), _ptr(ex)), "verify_naive")
+    return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool)}
 
 
 def verify_rrs(target: np.ndarray, q: np.ndarray, temperature: float, tree, token, seed: int, L: int,

@@ -812,3 +812,318 @@ int orc_verify_block(const orc_logits *target, const orc_logits *q, float temper
     free(x); free(Mb); free(Ms); free(resid); free(w); free(h); free(X);
     return 0;
 }
+
+/* ------------------------------------------------------------------------------------ */
+/* PLAN, expand-then-prune (the EAGLE-2-style first pass of Sec. 3.1 and App. B.3).
+ * Depth by depth, the W best candidates of the newest layer (its frontier) are expanded into
+ * their K children each (a node at the depth cap L gets none). Once every layer exists, the N
+ * best candidates of all layers are kept and numbered in the global order
+ *     (key desc, depth asc, parent's position in its layer asc, rank asc),
+ * with keys as in orc_plan (key = Sx - CL[d]). Inside a layer the order is the same one
+ * restricted to a depth, so a frontier is a prefix of its sorted layer and positions of
+ * same-depth parents order like their node numbers. A child's key never exceeds its parent's
+ * and its depth is larger, so the kept set is prefix-closed. With W >= N every node of the
+ * max-heap tree stays inside the frontiers (a node with n nodes before it in the global order
+ * has at most n before it in its layer) and both planners return the same tree; this is the
+ * sense in which App. B.3 says a wide enough frontier recovers the heap's solution.       */
+typedef struct {
+    double key, sx;
+    int depth, ppos, rank;
+    int num; /* node number once kept, 0 otherwise */
+} ept_cand;
+
+static int ept_before(const ept_cand *a, const ept_cand *b)
+{
+    if (a->key != b->key) return a->key > b->key;
+    if (a->depth != b->depth) return a->depth < b->depth;
+    if (a->ppos != b->ppos) return a->ppos < b->ppos;
+    return a->rank < b->rank;
+}
+
+static int ept_cmp(const void *pa, const void *pb)
+{
+    const ept_cand *a = (const ept_cand *)pa, *b = (const ept_cand *)pb;
+    return ept_before(a, b) ? -1 : (ept_before(b, a) ? 1 : 0);
+}
+
+/* adjacent entries in a sorted list whose order rounding could swap */
+static int ept_near(const ept_cand *a, const ept_cand *b, double key_eps)
+{
+    if (a->depth == b->depth && a->sx == b->sx) return 0; /* exact tie on every machine */
+    return a->key - b->key < key_eps * (1.0 + fabs(a->key));
+}
+
+int orc_plan_expand(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L, int32_t W,
+                    int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
+                    int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt)
+{
+    if (!draft || N < 1 || K < 1 || L < 1 || W < 1 || K > 64 || K > draft->V || draft->R < L) return -1;
+    if (!(temperature > 0.0f)) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = draft->V, NN = N + 1;
+    /* layer sizes: K at depth 1, min(W, previous) * K below */
+    int64_t total = 0, prev = 0;
+    int64_t *lstart = (int64_t *)malloc(sizeof(int64_t) * (L + 2));
+    if (!lstart) return -3;
+    for (int d = 1; d <= L; ++d) {
+        int64_t n = d == 1 ? K : (prev < W ? prev : W) * (int64_t)K;
+        lstart[d] = total;
+        total += n;
+        prev = n;
+    }
+    lstart[L + 1] = total;
+    if (total < N) { free(lstart); return -2; }
+    double *x = (double *)malloc(sizeof(double) * V);
+    double *CL = (double *)malloc(sizeof(double) * (L + 1));
+    int32_t *tid = (int32_t *)malloc(sizeof(int32_t) * L * K);
+    double *tx = (double *)malloc(sizeof(double) * L * K);
+    ept_cand *lay = (ept_cand *)malloc(sizeof(ept_cand) * (size_t)total);
+    ept_cand *all = (ept_cand *)malloc(sizeof(ept_cand) * (size_t)total);
+    int32_t *nchild = (int32_t *)malloc(sizeof(int32_t) * NN);
+    if (!x || !CL || !tid || !tx || !lay || !all || !nchild) return -3;
+    int rc = 0;
+    for (int b = 0; b < draft->B && rc == 0; ++b) {
+        CL[0] = 0.0;
+        for (int d = 0; d < L; ++d) {
+            read_row(draft, b, d, invT, x);
+            CL[d + 1] = CL[d] + logsumexp(x, V);
+            topk_row(x, V, K, tid + d * K, tx + d * K);
+        }
+        uint8_t ex = 0;
+        /* 1. layers, each sorted; the frontier of depth d is the first W of layer d */
+        for (int d = 1; d <= L; ++d) {
+            ept_cand *cur = lay + lstart[d];
+            int64_t n = 0;
+            if (d == 1) {
+                for (int r = 0; r < K; ++r, ++n) {
+                    cur[n].sx = tx[r];
+                    cur[n].ppos = 0;
+                    cur[n].rank = r;
+                }
+            } else {
+                const ept_cand *par = lay + lstart[d - 1];
+                const int64_t np = lstart[d] - lstart[d - 1], nf = np < W ? np : W;
+                for (int64_t f = 0; f < nf; ++f)
+                    for (int r = 0; r < K; ++r, ++n) {
+                        cur[n].sx = par[f].sx + tx[(d - 1) * K + r];
+                        cur[n].ppos = (int)f;
+                        cur[n].rank = r;
+                    }
+                if (np > W && ept_near(&par[W - 1], &par[W], key_eps)) ex = 1; /* frontier edge */
+            }
+            for (int64_t i = 0; i < n; ++i) {
+                cur[i].depth = d;
+                cur[i].key = cur[i].sx - CL[d];
+                cur[i].num = 0;
+            }
+            qsort(cur, (size_t)n, sizeof(ept_cand), ept_cmp);
+        }
+        /* 2. the N best of all layers, numbered in the global order. Each entry remembers its
+         *    layer position through (depth, index) so parents can be found after the sort. */
+        for (int64_t i = 0; i < total; ++i) {
+            all[i] = lay[i];
+            all[i].num = (int)i; /* temporarily: index into lay[] */
+        }
+        qsort(all, (size_t)total, sizeof(ept_cand), ept_cmp);
+        for (int64_t i = 0; i < N && i + 1 < total; ++i)
+            if (ept_near(&all[i], &all[i + 1], key_eps)) ex = 1; /* numbering and the budget edge */
+        int32_t *par = parent + (int64_t)b * NN, *dep = depth + (int64_t)b * NN;
+        int32_t *rk = rank + (int64_t)b * NN, *tok = plan_token + (int64_t)b * NN;
+        double *sc = score + (int64_t)b * NN;
+        par[0] = -1; dep[0] = 0; rk[0] = -1; tok[0] = -1; sc[0] = 0.0;
+        for (int i = 1; i <= N; ++i) lay[all[i - 1].num].num = i;
+        for (int i = 1; i <= N; ++i) {
+            const ept_cand *c = &all[i - 1];
+            int p = 0;
+            if (c->depth > 1) p = lay[lstart[c->depth - 1] + c->ppos].num;
+            if (c->depth > 1 && (p == 0 || p >= i)) { rc = -7; break; } /* not prefix-closed */
+            par[i] = p;
+            dep[i] = c->depth;
+            rk[i] = c->rank;
+            tok[i] = tid[(c->depth - 1) * K + c->rank];
+            sc[i] = c->key;
+        }
+        if (exempt) exempt[b] = ex;
+        /* child lists (CSR); siblings are kept in rank order, so slot = rank */
+        int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        for (int u = 0; u < NN; ++u) nchild[u] = 0;
+        for (int i = 1; i <= N && rc == 0; ++i) nchild[par[i]]++;
+        off[0] = 0;
+        for (int u = 0; u < NN; ++u) off[u + 1] = off[u] + nchild[u];
+        for (int i = 1; i <= N && rc == 0; ++i) {
+            if (rk[i] >= nchild[par[i]]) { rc = -7; break; } /* a sibling of lower rank is missing */
+            ids[off[par[i]] + rk[i]] = i;
+        }
+    }
+    free(lstart); free(x); free(CL); free(tid); free(tx); free(lay); free(all); free(nchild);
+    return rc;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* REPLAY with mixed sampling (Sec. 3.2 and App. A; the greedy draft sampling of Hu et al.
+ * 2025 that the paper pairs with its tree verifiers). For a parent u with m children, the
+ * first m-1 child slots take the m-1 most probable tokens of q_u, by (x desc, id asc), and the
+ * last slot takes one draw from q_u renormalised over the remaining tokens.
+ *
+ * The draw is the largest Gumbel key among the remaining tokens, with the keys of the
+ * hierarchical sampler of orc_replay (chunk keys K_c, element keys shifted to their chunk's
+ * maximum): the keys are jointly i.i.d. Gumbel(x_v), so the largest one over a fixed token set
+ * E' has law q restricted to E' and renormalised. A chunk without excluded tokens has its
+ * chunk key as its largest key, so only the chunks holding an excluded token and the best
+ * clean chunks need element keys (the second-best clean chunk only to flag near ties). With
+ * m = 1 nothing is excluded and the draw is orc_replay's single draw, token for token.     */
+int orc_replay_mixed(const orc_logits *q, float temperature, const int32_t *qrow_of_node, int32_t N,
+                     const int32_t *depth, const int32_t *child_off, const int32_t *child_ids, uint64_t seed,
+                     const int32_t *batch_ids, int32_t *token, uint8_t *exempt_node)
+{
+    if (!q || N < 0 || !(temperature > 0.0f)) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = q->V, C = (V + ORC_CHUNK - 1) / ORC_CHUNK, NN = N + 1;
+    double *x = (double *)malloc(sizeof(double) * V);
+    elem_key *ck = (elem_key *)malloc(sizeof(elem_key) * C);
+    uint8_t *excl = (uint8_t *)malloc(V), *dirty = (uint8_t *)malloc(C), *expand = (uint8_t *)malloc(C);
+    elem_key *ek = (elem_key *)malloc(sizeof(elem_key) * (size_t)V);
+    if (!x || !ck || !excl || !dirty || !expand || !ek) return -3;
+    for (int b = 0; b < q->B; ++b) {
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        const int bid = batch_of(batch_ids, b);
+        token[(int64_t)b * NN + 0] = -1;
+        for (int u = 0; u < NN; ++u) {
+            if (exempt_node) exempt_node[(int64_t)b * NN + u] = 0;
+            const int m = off[u + 1] - off[u];
+            if (m == 0) continue;
+            if (m > V) return -5;
+            const int r = replay_row_index(qrow_of_node, depth, (int64_t)b * NN + u);
+            if (r < 0 || r >= q->R) return -5;
+            read_row(q, b, r, invT, x);
+            /* 1. the m-1 deterministic slots: the most probable tokens in order */
+            int32_t top[64];
+            double topx[64];
+            if (m - 1 > 64) return -5;
+            if (m > 1) topk_row(x, V, m - 1, top, topx);
+            memset(excl, 0, V);
+            memset(dirty, 0, C);
+            for (int j = 0; j < m - 1; ++j) {
+                excl[top[j]] = 1;
+                dirty[top[j] / ORC_CHUNK] = 1;
+                token[(int64_t)b * NN + ids[off[u] + j]] = top[j];
+            }
+            /* 2. chunk keys; the two best clean chunks by (K desc, c asc) */
+            int best1 = -1, best2 = -1;
+            for (int c = 0; c < C; ++c) {
+                int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+                double uc = orc_uniform(seed, PURPOSE_REPLAY_CHUNK, bid, u, c);
+                ck[c].k = logsumexp(x + lo, hi - lo) + gumbel_of(uc);
+                ck[c].v = c;
+                ck[c].sens = gumbel_slope(uc);
+                if (dirty[c]) continue;
+                if (best1 < 0 || elem_before(&ck[c], &ck[best1])) {
+                    best2 = best1;
+                    best1 = c;
+                } else if (best2 < 0 || elem_before(&ck[c], &ck[best2])) {
+                    best2 = c;
+                }
+            }
+            for (int c = 0; c < C; ++c) expand[c] = dirty[c];
+            if (best1 >= 0) expand[best1] = 1;
+            if (best2 >= 0) expand[best2] = 1;
+            /* 3. shifted element keys of the expanded chunks; excluded tokens drop out */
+            int ne = 0;
+            for (int c = 0; c < C; ++c) {
+                if (!expand[c]) continue;
+                const double Tc = ck[c].k, uc_slope = ck[c].sens;
+                int lo = c * ORC_CHUNK, hi = lo + ORC_CHUNK < V ? lo + ORC_CHUNK : V;
+                double Z = -INFINITY, umax = 0.5;
+                int jmax = -1;
+                double *g = (double *)malloc(sizeof(double) * (hi - lo));
+                double *ug = (double *)malloc(sizeof(double) * (hi - lo));
+                if (!g || !ug) return -3;
+                for (int v = lo; v < hi; ++v) {
+                    ug[v - lo] = orc_uniform(seed, PURPOSE_REPLAY_ELEM, bid, u, v);
+                    g[v - lo] = x[v] + gumbel_of(ug[v - lo]);
+                    if (g[v - lo] > Z) { Z = g[v - lo]; jmax = v; umax = ug[v - lo]; }
+                }
+                for (int v = lo; v < hi; ++v) {
+                    if (excl[v]) continue;
+                    if (v == jmax) {
+                        ek[ne].k = Tc;
+                        ek[ne].sens = uc_slope;
+                    } else {
+                        double k = shift_key(Tc, Z, g[v - lo]);
+                        double s_own = gumbel_slope(ug[v - lo]) * exp(k - g[v - lo]);
+                        double s_T = uc_slope * exp(k - Tc);
+                        double s_Z = gumbel_slope(umax) * exp(k - Z);
+                        double s = s_own > s_T ? s_own : s_T;
+                        if (s_Z > s) s = s_Z;
+                        ek[ne].k = k;
+                        ek[ne].sens = s;
+                    }
+                    ek[ne].v = v;
+                    ++ne;
+                }
+                free(g);
+                free(ug);
+            }
+            if (ne == 0) return -5; /* cannot happen: V >= m leaves a token */
+            /* 4. the best remaining key is the sampled slot */
+            partial_sort(ek, ne, ne > 1 ? 2 : 1);
+            uint8_t ex = (ne > 1 && near_tie(&ek[0], &ek[1])) ? 1 : 0;
+            token[(int64_t)b * NN + ids[off[u] + m - 1]] = ek[0].v;
+            if (exempt_node) exempt_node[(int64_t)b * NN + u] = ex;
+        }
+    }
+    free(x); free(ck); free(excl); free(dirty); free(expand); free(ek);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* VERIFY by target-sample matching ("Naive" in Table 2, Sec. 2.3): at the current node u a
+ * token y is drawn from the target law p_u; if a child of u carries y (the first such slot),
+ * that child is accepted, y is emitted and the walk continues there; otherwise y itself is
+ * emitted as the final token and the walk stops. At a leaf the draw is the bonus token. Every
+ * emitted token is a draw from the target law at its prefix, whatever the candidates are, so
+ * the scheme is lossless for any tree and any way of filling it (deterministic first-pass
+ * tokens, WoR or mixed replay); a child with token v is accepted with probability p_u(v).
+ * The draw is the two-level Gumbel-max of sample_final on the target logits (purposes
+ * FINAL_CHUNK and FINAL, node u), the same draw as a bonus token.                        */
+int orc_verify_naive(const orc_logits *target, float temperature, int32_t N, int32_t L, const int32_t *child_off,
+                     const int32_t *child_ids, const int32_t *token, uint64_t seed, const int32_t *batch_ids,
+                     int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
+{
+    if (!target || N < 0 || L < 1 || !(temperature > 0.0f) || target->R < N + 1) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = target->V, NN = N + 1;
+    double *xt = (double *)malloc(sizeof(double) * V);
+    if (!xt) return -3;
+    for (int b = 0; b < target->B; ++b) {
+        const int64_t nb = (int64_t)b * NN;
+        const int bid = batch_of(batch_ids, b);
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        int32_t *otok = out_tokens + (int64_t)b * (L + 1), *onode = out_nodes + (int64_t)b * L;
+        for (int k = 0; k <= L; ++k) otok[k] = -1;
+        for (int k = 0; k < L; ++k) onode[k] = -1;
+        uint8_t ex = 0;
+        int u = 0, nacc = 0, y = -1;
+        for (;;) {
+            read_row(target, b, u, invT, xt);
+            y = sample_final(xt, 1, V, seed, bid, u, &ex);
+            int next = -1;
+            for (int i = off[u]; i < off[u + 1]; ++i) {
+                const int c = ids[i];
+                if (c < 1 || c > N) { free(xt); return -6; }
+                if (token[nb + c] == y) { next = c; break; }
+            }
+            if (next < 0 || nacc >= L) break;
+            otok[nacc] = y;
+            onode[nacc] = next;
+            ++nacc;
+            u = next;
+            y = -1;
+        }
+        otok[nacc] = y;
+        out_len[b] = nacc + 1;
+        if (exempt) exempt[b] = ex;
+    }
+    free(xt);
+    return 0;
+}
