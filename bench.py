@@ -57,6 +57,8 @@ def parse():
     ap.add_argument("--sets", type=int, default=8, help="independent input sets rotated across steps")
     ap.add_argument("--e2e-steps", type=int, default=40)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-variants", action="store_true", help="skip the other sampling / verification schemes")
+    ap.add_argument("--variant-steps", type=int, default=300)
     ap.add_argument("--workload", default="batched", choices=("batched", "batched128k"))
     args = ap.parse_args()
     if args.steps is None:
@@ -206,6 +208,67 @@ def algorithmic_bytes(w, sets, out_len, out_nodes):
     return draft_bytes, visited * row, staged_q * row, visited
 
 
+# Other sampling / verification schemes of the paper on the same workload (Table 2 and Sec.
+# 3.1): each runs eagerly like the headline step and is timed the same way (start and end
+# events only), followed by an event-separated pass for its per-call times.
+VARIANTS = (
+    ("mixed_replay_naive_verify", dict(replay="mixed", mode=2), False),
+    ("first_pass_tokens_naive_verify", dict(replay="plan", mode=2), False),
+    ("expand_prune_w10_wor_rrs", dict(width=10), False),
+    ("top1_chain_naive_verify", dict(replay="plan", mode=2), True),
+    ("sampled_chain_block_verify", dict(mode=1), True),
+)
+
+
+def run_variants(w, sets, device, steps=300, warmup=10):
+    import torch
+
+    from paper_2609_33652_gb300 import synth, tsb
+
+    B, L, S = w["B"], w["L"], len(sets)
+    chain_sets = []
+    for i, st in enumerate(sets):  # K = 1 chains of min(N, L) nodes on the same draft rows
+        buf = tsb.TsbBuffers.allocate(B, L, min(w["N"], L), 1, w["V"], w["T"], device=device)
+        tsb.tsb_row_stats(st["draft"], w["T"], buf.stats, buf.ws)
+        tsb.tsb_plan(buf.cfg, st["draft"], buf.stats, buf.tree, buf.ws)
+        target = synth.rows_from_depth(st["draft"], buf.tree["depth"], w["target_noise"], 5000 + i)
+        chain_sets.append(dict(draft=st["draft"], target=target, buf=buf))
+    torch.cuda.synchronize()
+    out = {}
+    for name, opts, chain in VARIANTS:
+        src = chain_sets if chain else sets
+        olen = torch.empty(steps, B, dtype=torch.int32, device=device)
+        otok = torch.empty(steps, B, L + 1, dtype=torch.int32, device=device)
+        onod = torch.empty(steps, B, L, dtype=torch.int32, device=device)
+        prep = [tsb.PreparedStep(src[k % S]["buf"], src[k % S]["draft"], src[k % S]["target"], 7_000_000 + k,
+                                 out_tokens=otok[k], out_nodes=onod[k], out_len=olen[k], **opts)
+                for k in range(steps)]
+        for k in range(min(warmup, steps)):
+            prep[k].run()
+        torch.cuda.synchronize()
+        t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        t0.record()
+        for p in prep:
+            p.run()
+        t1.record()
+        torch.cuda.synchronize()
+        us = t0.elapsed_time(t1) * 1e3 / steps
+        KA = min(steps, 100)
+        names = [c[0] for c in prep[0].calls]
+        ev = [[torch.cuda.Event(enable_timing=True) for _ in range(len(names) + 1)] for _ in range(KA)]
+        for k in range(KA):
+            prep[k].run(ev[k])
+        torch.cuda.synchronize()
+        for st in src:
+            if tsb.tsb_device_status(st["buf"].ws) != 0:
+                raise RuntimeError(f"device status bits set in variant {name}")
+        calls = {n: round(statistics.mean(ev[k][i].elapsed_time(ev[k][i + 1]) * 1e3 for k in range(KA)), 3)
+                 for i, n in enumerate(names)}
+        out[name] = {"us_per_step": round(us, 3), "per_call_us": calls,
+                     "mean_emitted_len": round(float(olen.float().mean().item()), 4), "steps": steps}
+    return out
+
+
 def max_over_ranks(value: float, dist, device) -> float:
     """The largest of the ranks' values (every rank gets it): a job's time is its slowest
     replica's. ``device`` is where the process group's backend reduces (cuda for nccl)."""
@@ -318,6 +381,7 @@ def run_tsb(args):
 
     # end to end through the C ABI with pinned host buffers
     e2e = run_e2e(args, w, sets, device) if args.e2e_steps > 0 else None
+    variants = run_variants(w, sets, device, steps=args.variant_steps) if not args.no_variants else None
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -343,6 +407,7 @@ def run_tsb(args):
         "gpu_launches": sum(LAUNCHES_PER_STEP.values()) * K,
         "clocks": clocks.summary(),
         "e2e": e2e,
+        "variants": variants,
         "cpu_baseline": cpu,
     }
     if rank == 0:

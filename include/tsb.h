@@ -64,11 +64,14 @@ typedef enum {
 typedef enum { TSB_F32 = 0, TSB_BF16 = 1 } tsb_dtype;
 
 typedef enum {
-    TSB_VERIFY_RRS = 0,  /* recursive rejection sampling, WoR candidates, any topology */
-    TSB_VERIFY_BLOCK = 1 /* block verification; the topology must be the chain 0->1->...->N */
+    TSB_VERIFY_RRS = 0,   /* recursive rejection sampling, WoR candidates, any topology */
+    TSB_VERIFY_BLOCK = 1, /* block verification; the topology must be the chain 0->1->...->N */
+    TSB_VERIFY_NAIVE = 2  /* target-sample matching: any topology, any way of filling it */
 } tsb_verify_mode;
 
 /* Limits (validated). */
+#define TSB_MAX_WIDTH 1024              /* frontier width of the expand-then-prune first pass */
+#define TSB_MAX_EXPAND_CANDIDATES 8192  /* candidates it may generate: K + (L-1) layers of <= W*K */
 #define TSB_CHUNK 256 /* fixed chunk of the chunk statistics and of the replay sampler */
 #define TSB_MAX_K 32
 #define TSB_MAX_L 64
@@ -158,6 +161,27 @@ tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *dra
 tsb_status tsb_plan_rows(const tsb_cfg *cfg, const tsb_logits *draft, void *draft_stats, size_t stats_bytes,
                          const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
 
+/* First pass by expand-then-prune (Sec. 3.1 and App. B.3: the EAGLE-2-style planner the paper
+ * uses for drafters that correct logits per prefix). Depth by depth, the `width` best
+ * candidates of the newest layer (its frontier) get their K children each (a node at depth L
+ * gets none); after the last depth the N best of all generated candidates are the nodes,
+ * numbered in the order (path log-probability desc, depth asc, parent's position in its layer
+ * asc, rank asc). Path scores, tokens and output layout are those of tsb_plan; with width >= N
+ * the tree is the max-heap tree of tsb_plan. Inside a layer the order is the same one, and a
+ * frontier is a prefix of its sorted layer.
+ * width: 1..TSB_MAX_WIDTH. The number of generated candidates, K + sum over depths 2..L of
+ * min(width, previous layer) * K, must be at least N and at most TSB_MAX_EXPAND_CANDIDATES,
+ * else TSB_ERR_SHAPE. A child whose rounded score came out above its parent's (a draft row
+ * with all its mass on one token) sets TSB_DEV_BAD_TREE.
+ * tsb_plan_expand takes the draft statistics as input like tsb_plan; tsb_plan_rows_expand
+ * computes and writes them in the same pass over the rows like tsb_plan_rows. Other arguments
+ * and errors as in tsb_plan / tsb_plan_rows. */
+tsb_status tsb_plan_expand(const tsb_cfg *cfg, int32_t width, const tsb_logits *draft, const void *draft_stats,
+                           size_t stats_bytes, const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
+tsb_status tsb_plan_rows_expand(const tsb_cfg *cfg, int32_t width, const tsb_logits *draft, void *draft_stats,
+                                size_t stats_bytes, const tsb_tree *out, void *ws, size_t ws_bytes,
+                                tsb_stream stream);
+
 /* Size of the device scratch array behind tsb_plan_noalloc (1 MiB per device). */
 #define TSB_NOALLOC_SCRATCH_BYTES ((size_t)1 << 20)
 
@@ -199,6 +223,17 @@ tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *q
                       const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
                       size_t ws_bytes, tsb_stream stream);
 
+/* Second pass with mixed sampling (Sec. 3.2 and App. A; the greedy draft sampling of Hu et
+ * al. 2025): for every parent u with m_u children, child slots 0..m_u-2 take the m_u-1 most
+ * probable tokens of q_u in order, by (x desc, id asc), and slot m_u-1 takes one draw from q_u
+ * renormalised over the other tokens: the largest Gumbel key among them, with the keys of
+ * tsb_replay's top-down construction (so with m_u = 1 the token is tsb_replay's). Arguments,
+ * layout and errors as in tsb_replay. Pair it with TSB_VERIFY_NAIVE: recursive rejection
+ * sampling assumes WoR candidates and is not lossless for these. */
+tsb_status tsb_replay_mixed(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,
+                            const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token,
+                            void *ws, size_t ws_bytes, tsb_stream stream);
+
 /* Verification on the frozen topology with the replayed tokens (Prop. 1).
  * TSB_VERIFY_RRS: from the root, test the children in slot order, accept child i iff
  *   U * q'(y_i) < p'(y_i) with q' the draft law renormalised over tokens not yet drawn and
@@ -207,6 +242,13 @@ tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *q
  *   children are rejected the final token is drawn from the last residual; at a leaf the
  *   bonus token is drawn from the node's target row.
  * TSB_VERIFY_BLOCK: block verification of the chain 0->1->...->N (requires N <= L).
+ * TSB_VERIFY_NAIVE: target-sample matching (Sec. 2.3, "Naive" in Table 2): from the root, draw
+ *   y from the node's target law (the two-level Gumbel-max of the bonus token); the first child
+ *   carrying y is accepted and the walk continues there, otherwise y is the final token. Each
+ *   emitted token is a draw from the target law, whatever the children hold, so it verifies the
+ *   first-pass tokens (plan_token) as well as WoR or mixed replays; a child with token v is
+ *   accepted with probability p(v). qrows, qstats and qrow_of_node are not used and may be
+ *   NULL. Every node's draw is computed in one parallel pass over all N+1 target rows.
  * target: [B, N+1, V], row u = target logits after the path to node u. qrows / qstats /
  * qrow_of_node as in tsb_replay. Outputs: out_tokens [B, L+1] (accepted tokens then the
  * final token, -1 after), out_nodes [B, L] (accepted node ids, -1 after), out_len [B]

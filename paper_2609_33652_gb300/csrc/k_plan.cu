@@ -327,6 +327,80 @@ __device__ __forceinline__ unsigned long long okey_of(long long key) {
 __device__ __forceinline__ long long key_of_okey(unsigned long long o) { return (long long)(o ^ 0x8000000000000000ull); }
 __device__ __forceinline__ long long fix_of(float x) { return __float2ll_rn(__fmul_rn(x, kFixScale)); }
 
+// CL[d] = LSE_1 + ... + LSE_d (d = 0..L) of one tree's draft rows, summed in float-float in
+// depth order and rounded onto the fixed grid once per depth. Called by one whole warp; lane 0
+// writes CL[0..L].
+__device__ __forceinline__ void depth_prefix_fixed(const float2 *lse, int L, long long *CL) {
+    const int lane = threadIdx.x & 31;
+    FF l0 = FF{0.f, 0.f}, l1 = FF{0.f, 0.f};
+    if (lane < L) {
+        const float2 v = lse[lane];
+        l0 = FF{v.x, v.y};
+    }
+    if (lane + 32 < L) {
+        const float2 v = lse[lane + 32];
+        l1 = FF{v.x, v.y};
+    }
+    FF acc = FF{0.f, 0.f};
+    for (int d = 0; d < L; ++d) {  // prefix sums in depth order (every lane, same values)
+        const FF l = d < 32 ? FF{__shfl_sync(kFull, l0.hi, d), __shfl_sync(kFull, l0.lo, d)}
+                            : FF{__shfl_sync(kFull, l1.hi, d - 32), __shfl_sync(kFull, l1.lo, d - 32)};
+        acc = ff_add(acc, l);
+        if (lane == 0) CL[d + 1] = fix_of(acc.hi) + fix_of(acc.lo);
+    }
+    if (lane == 0) CL[0] = 0;
+}
+
+// The tree's outputs from per-node arrays in shared memory (node 0 the root, nodes 1..N with
+// parent < node and siblings holding ranks 0..m-1): child lists by counting, an exclusive scan
+// (warp 0) and placement by rank, then the per-node arrays. n_count must hold zeros; it is
+// reused for the child-list starts. All NT threads of the CTA call it after a barrier.
+template <int NT>
+__device__ void emit_tree(int b, int N, const int32_t *n_parent, const int32_t *n_depth, const int32_t *n_rank,
+                          const int32_t *n_token, int32_t *n_count, const float *n_score, const TreeDesc &tree) {
+    const int NN = N + 1;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int i = 1 + threadIdx.x; i <= N; i += NT) atomicAdd(&n_count[n_parent[i]], 1);
+    __syncthreads();
+    int32_t *off = tree.child_off + (int64_t)b * (NN + 1);
+    if (warp == 0) {
+        const int per = (NN + 31) / 32;
+        const int lo = min(NN, lane * per), hi = min(NN, lo + per);
+        int s = 0;
+        for (int u = lo; u < hi; ++u) s += n_count[u];
+        int incl = s;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(kFull, incl, o);
+            if (lane >= o) incl += y;
+        }
+        int run = incl - s;
+        for (int u = lo; u < hi; ++u) {
+            const int c = n_count[u];
+            n_count[u] = run;  // now the start of u's children
+            off[u] = run;
+            run += c;
+        }
+        if (lane == 31) off[NN] = incl;
+    }
+    __syncthreads();
+    int32_t *ids = tree.child_ids + (int64_t)b * N;
+    for (int i = 1 + threadIdx.x; i <= N; i += NT) {
+        const int slot = n_count[n_parent[i]] + n_rank[i];
+        if (slot >= 0 && slot < N) ids[slot] = i;  // always, unless a tree check already failed
+    }
+    int32_t *par = tree.parent + (int64_t)b * NN, *dep = tree.depth + (int64_t)b * NN;
+    int32_t *rk = tree.rank + (int64_t)b * NN, *tok = tree.plan_token + (int64_t)b * NN;
+    float *sc = tree.score + (int64_t)b * NN;
+    for (int i = threadIdx.x; i < NN; i += NT) {
+        par[i] = n_parent[i];
+        dep[i] = n_depth[i];
+        rk[i] = n_rank[i];
+        tok[i] = n_token[i];
+        sc[i] = n_score[i];
+    }
+}
+
 // A 32-bit image of an okey, monotone non-decreasing: keys in [-2^41, 2^41) (|log-probability|
 // below 2048) at 2^-20 resolution, clamped outside; an empty slot (0) maps to 0. Equal images
 // are resolved on the full key.
@@ -420,25 +494,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
         n_score[i] = 0.f;
         n_sx[i] = 0;
     }
-    if (warp == 0) {  // CL[d] = LSE_1 + ... + LSE_d in float-float, then onto the fixed grid
-        FF l0 = FF{0.f, 0.f}, l1 = FF{0.f, 0.f};
-        if (lane < L) {
-            const float2 v = a.lse[(int64_t)b * L + lane];
-            l0 = FF{v.x, v.y};
-        }
-        if (lane + 32 < L) {
-            const float2 v = a.lse[(int64_t)b * L + lane + 32];
-            l1 = FF{v.x, v.y};
-        }
-        FF acc = FF{0.f, 0.f};
-        for (int d = 0; d < L; ++d) {  // prefix sums in depth order (every lane, same values)
-            const FF l = d < 32 ? FF{__shfl_sync(kFull, l0.hi, d), __shfl_sync(kFull, l0.lo, d)}
-                                : FF{__shfl_sync(kFull, l1.hi, d - 32), __shfl_sync(kFull, l1.lo, d - 32)};
-            acc = ff_add(acc, l);
-            if (lane == 0) CL[d + 1] = fix_of(acc.hi) + fix_of(acc.lo);
-        }
-        if (lane == 0) CL[0] = 0;
-    }
+    if (warp == 0) depth_prefix_fixed(a.lse + (int64_t)b * L, L, CL);
     __syncthreads();
 
     // The expansion (warp 0). Per pop the critical path is the warp maximum, three shuffles,
@@ -521,43 +577,196 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     }
     __syncthreads();
 
-    // child lists: count, exclusive scan (one warp), then place children by rank
-    for (int i = 1 + threadIdx.x; i <= N; i += kHeapThreads) atomicAdd(&n_count[n_parent[i]], 1);
+    emit_tree<kHeapThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
+}
+
+// ---------------------------------------------------------------------------------------
+// Expand-then-prune first pass (the EAGLE-2-style planner of Sec. 3.1 and App. B.3), one CTA
+// per tree. Layer 1 is the root's K children; layer d+1 holds the K children of each of the W
+// best candidates of layer d (its frontier), so layers stay at most W*K wide and L layers
+// deep. Every layer is kept sorted by (key desc, parent's position asc, rank asc): candidate
+// (f, r) of layer d+1 has sum Sx = Sx_f + x_{d,r}, and the candidates of frontier entry f' that
+// precede it are those whose logit exceeds Sx - Sx_f' (or reaches it when f' < f), a prefix of
+// the depth's sorted top-K logits found by binary search; its position is r plus those counts.
+// After the last layer, a candidate's place in the global order (key desc, depth asc, parent's
+// position asc, rank asc) is its layer position plus, for every other layer, the number of
+// entries above its key there (at or above it for shallower layers), again by binary search;
+// the N first are the nodes, numbered in that order. Keys are the 64-bit fixed-point path
+// sums of the max-heap planner, so same-depth comparisons are exact and a frontier holding N
+// candidates gives the heap's tree bit for bit.
+constexpr int kEptThreads = 512;
+constexpr int kEptGroup = 8;  // layers searched in lockstep per candidate
+
+struct EptArgs {
+    int L, N, K, W;
+    const float2 *lse;
+    const float *topk_x;
+    const int32_t *topk_id;
+    TreeDesc tree;
+    uint32_t *status;
+};
+
+size_t ept_smem_bytes(int L, int N, int K, int G) {
+    const size_t NN = (size_t)N + 1;
+    return (size_t)(L + 1) * 8 + (size_t)L * K * 8 + (size_t)G * 8 + (size_t)L * K * 4 + (size_t)G * 8 +
+           (size_t)(L + 2) * 4 + 6 * NN * 4;
+}
+
+__global__ void __launch_bounds__(kEptThreads) k_plan_ept(EptArgs a) {
+    pdl_begin();
+    extern __shared__ __align__(16) unsigned char smem[];
+    const int L = a.L, N = a.N, K = a.K, W = a.W, NN = N + 1;
+    const int G = (int)ept_layer_start(L + 1, K, W);
+    long long *CL = reinterpret_cast<long long *>(smem);          // [L+1]
+    long long *fx = CL + (L + 1);                                 // [L*K] candidate logits, fixed point
+    long long *skey = fx + L * K;                                 // [G] keys, each layer sorted
+    int32_t *tk_id = reinterpret_cast<int32_t *>(skey + G);       // [L*K]
+    int32_t *smeta = tk_id + L * K;                               // [G] (parent position << 8) | rank
+    int32_t *node_of = smeta + G;                                 // [G] node number, 0 if not kept
+    int32_t *lstart = node_of + G;                                // [L+2]
+    int32_t *n_parent = lstart + (L + 2);                         // [NN] each
+    int32_t *n_depth = n_parent + NN;
+    int32_t *n_rank = n_depth + NN;
+    int32_t *n_token = n_rank + NN;
+    int32_t *n_count = n_token + NN;
+    float *n_score = reinterpret_cast<float *>(n_count + NN);
+
+    const int b = blockIdx.x;
+    const int warp = threadIdx.x >> 5;
+    for (int i = threadIdx.x; i < L * K; i += kEptThreads) {
+        tk_id[i] = a.topk_id[(int64_t)b * L * K + i];
+        fx[i] = fix_of(a.topk_x[(int64_t)b * L * K + i]);
+    }
+    for (int i = threadIdx.x; i < NN; i += kEptThreads) {
+        n_count[i] = 0;
+        n_parent[i] = i == 0 ? -1 : 0;
+        n_depth[i] = 0;
+        n_rank[i] = i == 0 ? -1 : 0;
+        n_token[i] = -1;
+        n_score[i] = 0.f;
+    }
+    for (int d = 1 + threadIdx.x; d <= L + 1; d += kEptThreads) lstart[d] = (int)ept_layer_start(d, K, W);
+    if (warp == 0) depth_prefix_fixed(a.lse + (int64_t)b * L, L, CL);
     __syncthreads();
-    int32_t *off = a.tree.child_off + (int64_t)b * (NN + 1);
-    if (warp == 0) {
-        const int per = (NN + 31) / 32;
-        const int lo = min(NN, lane * per), hi = min(NN, lo + per);
-        int s = 0;
-        for (int u = lo; u < hi; ++u) s += n_count[u];
-        int incl = s;
+
+    // 1. layer 1 is sorted as built (the draft row's logits do not increase with rank)
+    for (int j = threadIdx.x; j < K; j += kEptThreads) {
+        skey[j] = fx[j] - CL[1];
+        smeta[j] = j;
+    }
+    __syncthreads();
+    // 2. layers 2..L, each placed at its sorted positions: a layer of at most one candidate per
+    //    thread by counting the candidates before each (index order j = f*K + r is the order of
+    //    equal keys), a wider one by binary searches over the depth's sorted logits
+    __shared__ long long tkey[kEptThreads];
+    int kbits = 0;  // steps of the binary search over a depth's K logits
+    while ((1 << kbits) <= K) ++kbits;
+    for (int d = 1; d < L; ++d) {
+        const int prev = lstart[d], nf = min(W, lstart[d + 1] - prev), base = lstart[d + 1];
+        const long long cd = CL[d], cd1 = CL[d + 1];
+        const long long *row = fx + d * K;  // logits of depth d+1, non-increasing in rank
+        if (nf * K <= kEptThreads) {  // uniform over the CTA
+            const int n = nf * K, j = threadIdx.x;
+            const int f = j / K, r = j - f * K;
+            long long key = 0;
+            if (j < n) {
+                key = skey[prev + f] + cd + row[r] - cd1;
+                tkey[j] = key;
+            }
+            __syncthreads();
+            if (j < n) {
+                int pos = 0;
+#pragma unroll 8
+                for (int i2 = 0; i2 < n; ++i2) {  // independent loads, eight in flight
+                    const long long k2 = tkey[i2];
+                    pos += (k2 > key || (k2 == key && i2 < j)) ? 1 : 0;
+                }
+                skey[base + pos] = key;
+                smeta[base + pos] = (f << 8) | r;
+            }
+            __syncthreads();  // before the next layer reads skey and rewrites tkey
+            continue;
+        }
+        for (int j = threadIdx.x; j < nf * K; j += kEptThreads) {
+            const int f = j / K, r = j - f * K;
+            const long long sx = skey[prev + f] + cd + row[r];
+            int pos = r;
+            for (int f2 = 0; f2 < nf; ++f2) {
+                if (f2 == f) continue;
+                const long long t = sx - (skey[prev + f2] + cd);
+                const bool incl = f2 < f;
+                int c = 0;  // logits of the depth above t (at or above t when incl)
+                for (int step = 1 << (kbits - 1); step > 0; step >>= 1)
+                    if (c + step <= K && (incl ? row[c + step - 1] >= t : row[c + step - 1] > t)) c += step;
+                pos += c;
+            }
+            skey[base + pos] = sx - cd1;
+            smeta[base + pos] = (f << 8) | r;
+        }
+        __syncthreads();
+    }
+    // 3. places in the global order; the first N are the nodes
+    int lbits = 0;  // steps of a binary search over a layer
+    while ((1 << lbits) <= W * K || (1 << lbits) <= K) ++lbits;
+    for (int idx = threadIdx.x; idx < G; idx += kEptThreads) {
+        int d = 1;
+        while (lstart[d + 1] <= idx) ++d;
+        int g = idx - lstart[d];
+        if (g >= N) {  // N candidates of its own layer come first
+            node_of[idx] = 0;
+            continue;
+        }
+        const long long k = skey[idx];
+        for (int d0 = 1; d0 <= L && g < N; d0 += kEptGroup) {
+            int c[kEptGroup], lo[kEptGroup], len[kEptGroup];
 #pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const int y = __shfl_up_sync(kFull, incl, o);
-            if (lane >= o) incl += y;
+            for (int q = 0; q < kEptGroup; ++q) {
+                const int d2 = d0 + q;
+                const bool live = d2 <= L && d2 != d;
+                c[q] = 0;
+                lo[q] = live ? lstart[d2] : 0;
+                len[q] = live ? lstart[d2 + 1] - lstart[d2] : 0;
+            }
+            for (int step = 1 << (lbits - 1); step > 0; step >>= 1) {
+                long long k2[kEptGroup];
+#pragma unroll
+                for (int q = 0; q < kEptGroup; ++q) {  // the group's loads issued together
+                    const bool in = c[q] + step <= len[q];
+                    k2[q] = skey[lo[q] + (in ? c[q] + step - 1 : 0)];
+                }
+#pragma unroll
+                for (int q = 0; q < kEptGroup; ++q) {
+                    const bool in = c[q] + step <= len[q];
+                    c[q] += (in && (d0 + q < d ? k2[q] >= k : k2[q] > k)) ? step : 0;
+                }
+            }
+#pragma unroll
+            for (int q = 0; q < kEptGroup; ++q) g += c[q];
         }
-        int run = incl - s;
-        for (int u = lo; u < hi; ++u) {
-            const int c = n_count[u];
-            n_count[u] = run;  // now the start of u's children
-            off[u] = run;
-            run += c;
-        }
-        if (lane == 31) off[NN] = incl;
+        node_of[idx] = g < N ? g + 1 : 0;
     }
     __syncthreads();
-    int32_t *ids = a.tree.child_ids + (int64_t)b * N;
-    for (int i = 1 + threadIdx.x; i <= N; i += kHeapThreads) ids[n_count[n_parent[i]] + n_rank[i]] = i;
-    int32_t *par = a.tree.parent + (int64_t)b * NN, *dep = a.tree.depth + (int64_t)b * NN;
-    int32_t *rk = a.tree.rank + (int64_t)b * NN, *tok = a.tree.plan_token + (int64_t)b * NN;
-    float *sc = a.tree.score + (int64_t)b * NN;
-    for (int i = threadIdx.x; i < NN; i += kHeapThreads) {
-        par[i] = n_parent[i];
-        dep[i] = n_depth[i];
-        rk[i] = n_rank[i];
-        tok[i] = n_token[i];
-        sc[i] = n_score[i];
+    bool bad = false;
+    for (int idx = threadIdx.x; idx < G; idx += kEptThreads) {
+        const int i = node_of[idx];
+        if (i == 0) continue;
+        int d = 1;
+        while (lstart[d + 1] <= idx) ++d;
+        const int meta = smeta[idx], f = meta >> 8, r = meta & 255;
+        int par = d == 1 ? 0 : node_of[lstart[d - 1] + f];
+        if (d > 1 && (par == 0 || par >= i)) {  // a child's key rounded above its parent's
+            bad = true;
+            par = 0;
+        }
+        n_parent[i] = par;
+        n_depth[i] = d;
+        n_rank[i] = r;
+        n_token[i] = tk_id[(d - 1) * K + r];
+        n_score[i] = __fmul_rn(__ll2float_rn(skey[idx]), kFixInv);
     }
+    if (bad) raise_status(a.status, kDevBadTree);
+    __syncthreads();
+    emit_tree<kEptThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
 }
 
 size_t heap_smem_bytes(int L, int N, int K) {
@@ -588,6 +797,14 @@ cudaError_t launch_stats_topk_t(const TopkArgs &a, cudaStream_t s) {
         cudaFuncSetAttribute(k_row_stats_topk<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     return launch_pdl(k_row_stats_topk<KCAP, T>, dim3((unsigned)(a.B * a.L)), dim3(kRowPlanThreads), smem, s, 0, a);
+}
+
+cudaError_t launch_ept(const EptArgs &e, int B, cudaStream_t s) {
+    const int G = (int)ept_layer_start(e.L + 1, e.K, e.W);
+    const size_t smem = ept_smem_bytes(e.L, e.N, e.K, G);
+    cudaError_t err = cudaFuncSetAttribute(k_plan_ept, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (err != cudaSuccess) return err;
+    return launch_pdl(k_plan_ept, dim3((unsigned)B), dim3(kEptThreads), smem, s, 0, e);
 }
 
 // The frontier kernel with as many slots per lane as N first children need.
@@ -676,6 +893,40 @@ cudaError_t launch_plan_rows(const RowsDesc &draft, float2 *stats_out, int L, in
         e = K <= 8 ? launch_stats_topk_t<8, float>(t, s) : launch_stats_topk_t<32, float>(t, s);
     if (e != cudaSuccess) return e;
     return launch_heap(heap_args(L, N, K, sc, tree, static_cast<uint32_t *>(ws)), draft.B, s);
+}
+
+// The per-row top-K pass (fused with the statistics when stats_out is given), then the
+// expand-then-prune planner with frontier width W.
+cudaError_t launch_plan_expand(const RowsDesc &draft, const float2 *stats, float2 *stats_out, int L, int N, int K,
+                               int W, float invT, const TreeDesc &tree, void *ws, cudaStream_t s) {
+    const PlanScratch sc = plan_scratch(ws, draft.B, N, L, K);
+    TopkArgs t = topk_args(draft, stats, L, K, invT, sc);
+    cudaError_t e;
+    if (stats_out) {
+        t.stats_out = stats_out;
+        t.status = static_cast<uint32_t *>(ws);
+        if (draft.dtype == 1)
+            e = K <= 8 ? launch_stats_topk_t<8, __nv_bfloat16>(t, s) : launch_stats_topk_t<32, __nv_bfloat16>(t, s);
+        else
+            e = K <= 8 ? launch_stats_topk_t<8, float>(t, s) : launch_stats_topk_t<32, float>(t, s);
+    } else {
+        if (draft.dtype == 1)
+            e = K <= 8 ? launch_topk_t<8, __nv_bfloat16>(t, s) : launch_topk_t<32, __nv_bfloat16>(t, s);
+        else
+            e = K <= 8 ? launch_topk_t<8, float>(t, s) : launch_topk_t<32, float>(t, s);
+    }
+    if (e != cudaSuccess) return e;
+    EptArgs ea;
+    ea.L = L;
+    ea.N = N;
+    ea.K = K;
+    ea.W = W;
+    ea.lse = sc.lse;
+    ea.topk_x = sc.topk_x;
+    ea.topk_id = sc.topk_id;
+    ea.tree = tree;
+    ea.status = static_cast<uint32_t *>(ws);
+    return launch_ept(ea, draft.B, s);
 }
 
 }  // namespace tsb

@@ -46,13 +46,6 @@ struct ReplayArgs {
     uint32_t *status;
 };
 
-// Gumbel key conditioned on the chunk maximum (stable form).
-__device__ __forceinline__ float shifted_key(float T, float Z, float g) {
-    const float u = T - g + log1pf(-expf(g - Z));
-    const float sp = fmaxf(u, 0.f) + log1pf(expf(-fabsf(u)));
-    return T - sp;
-}
-
 // Merge per-warp lists: each warp writes its top n keys to cand[warp][0..n).
 template <int CAP>
 __device__ __forceinline__ void warp_top_to(TopList<CAP> &list, int n, uint64_t *dst) {
@@ -247,7 +240,7 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
 #pragma unroll
             for (int i = 0; i < 8; ++i) {
                 if (v0 + i >= a.V || !(g[i] >= gmin)) continue;
-                const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_key(Tc, Z, g[i]);
+                const float k = ((uint32_t)(v0 + i) == jmax) ? Tc : shifted_gumbel_key(Tc, Z, g[i]);
                 const uint64_t key = pack_key(k, (uint32_t)(v0 + i));
                 el.insert(key);
                 const int idx = atomicAdd(&s_n2, 1);

@@ -88,11 +88,76 @@ tsb_status cuda_status(cudaError_t e) { return e == cudaSuccess ? TSB_OK : TSB_E
 
 float inv_temperature(float T) { return 1.0f / T; }
 
+// expand-then-prune: width in range, between N and kEptMaxCandidates candidates generated
+tsb_status check_width(const tsb_cfg *c, int32_t width) {
+    if (width < 1 || width > TSB_MAX_WIDTH) return TSB_ERR_SHAPE;
+    const int64_t G = tsb::ept_layer_start(c->L + 1, c->K, width);
+    if (G < c->N || G > tsb::kEptMaxCandidates) return TSB_ERR_SHAPE;
+    return TSB_OK;
+}
+
+tsb_status plan_expand_common(const tsb_cfg *cfg, int32_t width, const tsb_logits *draft, const void *stats_in,
+                              void *stats_out, size_t stats_bytes, const tsb_tree *out, void *ws, size_t ws_bytes,
+                              tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_width(cfg, width);
+    if (st != TSB_OK) return st;
+    st = check_logits(draft, cfg->B, cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(stats_in ? stats_in : stats_out, stats_bytes, cfg->B, draft->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!out || !out->parent || !out->depth || !out->rank || !out->plan_token || !out->score || !out->child_off ||
+        !out->child_ids)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_plan_expand(rows_of(draft), static_cast<const float2 *>(stats_in),
+                                               static_cast<float2 *>(stats_out), cfg->L, cfg->N, cfg->K, width,
+                                               inv_temperature(cfg->temperature), tree_of(out), ws,
+                                               (cudaStream_t)stream));
+}
+
+tsb_status replay_common(bool mixed, const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats,
+                         size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed,
+                         int32_t *token, void *ws, size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(qstats, stats_bytes, cfg->B, qrows->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!tree || !tree->child_off || !tree->child_ids || (!qrow_of_node && !tree->depth) || !token)
+        return TSB_ERR_ARG;
+    const auto launch = mixed ? tsb::launch_replay_mixed : tsb::launch_replay;
+    return cuda_status(launch(rows_of(qrows), static_cast<const float2 *>(qstats), qrow_of_node, cfg->B, cfg->N,
+                              cfg->K, tree_of(tree), inv_temperature(cfg->temperature), seed, token,
+                              static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+}
+
 }  // namespace
 
 extern "C" {
 
-int32_t tsb_version(void) { return 100; }
+tsb_status tsb_plan_expand(const tsb_cfg *cfg, int32_t width, const tsb_logits *draft, const void *draft_stats,
+                           size_t stats_bytes, const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream) {
+    if (!draft_stats) return TSB_ERR_ARG;
+    return plan_expand_common(cfg, width, draft, draft_stats, nullptr, stats_bytes, out, ws, ws_bytes, stream);
+}
+
+tsb_status tsb_plan_rows_expand(const tsb_cfg *cfg, int32_t width, const tsb_logits *draft, void *draft_stats,
+                                size_t stats_bytes, const tsb_tree *out, void *ws, size_t ws_bytes,
+                                tsb_stream stream) {
+    if (!draft_stats) return TSB_ERR_ARG;
+    return plan_expand_common(cfg, width, draft, nullptr, draft_stats, stats_bytes, out, ws, ws_bytes, stream);
+}
+
+tsb_status tsb_replay_mixed(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,
+                            const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token,
+                            void *ws, size_t ws_bytes, tsb_stream stream) {
+    return replay_common(true, cfg, qrows, qstats, stats_bytes, qrow_of_node, tree, seed, token, ws, ws_bytes,
+                         stream);
+}
+
+int32_t tsb_version(void) { return 200; }
 
 const char *tsb_status_str(tsb_status s) {
     switch (s) {
@@ -187,17 +252,8 @@ tsb_status tsb_plan_rows(const tsb_cfg *cfg, const tsb_logits *draft, void *draf
 tsb_status tsb_replay(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,
                       const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
                       size_t ws_bytes, tsb_stream stream) {
-    tsb_status st = check_cfg(cfg);
-    if (st != TSB_OK) return st;
-    st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
-    if (st == TSB_OK) st = check_stats(qstats, stats_bytes, cfg->B, qrows->R, cfg->V);
-    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
-    if (st != TSB_OK) return st;
-    if (!tree || !tree->child_off || !tree->child_ids || (!qrow_of_node && !tree->depth) || !token)
-        return TSB_ERR_ARG;
-    return cuda_status(tsb::launch_replay(rows_of(qrows), static_cast<const float2 *>(qstats), qrow_of_node, cfg->B,
-                                          cfg->N, cfg->K, tree_of(tree), inv_temperature(cfg->temperature), seed,
-                                          token, static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+    return replay_common(false, cfg, qrows, qstats, stats_bytes, qrow_of_node, tree, seed, token, ws, ws_bytes,
+                         stream);
 }
 
 tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target, const tsb_logits *qrows,
@@ -206,9 +262,18 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
                       int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream) {
     tsb_status st = check_cfg(cfg);
     if (st != TSB_OK) return st;
-    if (mode != TSB_VERIFY_RRS && mode != TSB_VERIFY_BLOCK) return TSB_ERR_ARG;
+    if (mode != TSB_VERIFY_RRS && mode != TSB_VERIFY_BLOCK && mode != TSB_VERIFY_NAIVE) return TSB_ERR_ARG;
     if (mode == TSB_VERIFY_BLOCK && cfg->N > cfg->L) return TSB_ERR_SHAPE;
     st = check_logits(target, cfg->B, cfg->N + 1, cfg->V);
+    if (mode == TSB_VERIFY_NAIVE) {  // no draft rows: only the target and the tree
+        if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+        if (st != TSB_OK) return st;
+        if (!tree || !tree->child_off || !tree->child_ids || !token || !out_tokens || !out_nodes || !out_len)
+            return TSB_ERR_ARG;
+        return cuda_status(tsb::launch_verify_naive(rows_of(target), cfg->B, cfg->N, cfg->L, tree_of(tree), token,
+                                                    inv_temperature(cfg->temperature), seed, out_tokens,
+                                                    out_nodes, out_len, ws, (cudaStream_t)stream));
+    }
     if (st == TSB_OK) st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
     if (st == TSB_OK && target->dtype != qrows->dtype) st = TSB_ERR_DTYPE;
     if (st == TSB_OK) st = check_stats(qstats, stats_bytes, cfg->B, qrows->R, cfg->V);

@@ -81,6 +81,15 @@ __device__ __forceinline__ float neg_log_uniform(uint32_t w) {
 // Standard Gumbel G = -log(-log U) of a draw word.
 __device__ __forceinline__ float gumbel_of(uint32_t w) { return -logf(neg_log_uniform(w)); }
 
+// Gumbel key g of the top-down construction shifted to the law conditional on its chunk's
+// maximum Z being T (Kool, van Hoof & Welling 2019, App. B; the stable softplus form):
+// T - softplus(T - g + log1p(-exp(g - Z))).
+__device__ __forceinline__ float shifted_gumbel_key(float T, float Z, float g) {
+    const float u = T - g + log1pf(-expf(g - Z));
+    const float sp = fmaxf(u, 0.f) + log1pf(expf(-fabsf(u)));
+    return T - sp;
+}
+
 // ---------------------------------------------------------------------------------------
 // Keys. A (value desc, id asc) order is packed into one u64 so that "larger u64 first" is
 // the order: high word = order-preserving image of the fp32 value, low word = ~id.
@@ -123,6 +132,52 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
         v = w > v ? w : v;
     }
     return v;
+}
+
+// Warp sums of U per-lane partials at once (U = 2, 4 or 8), for U chunks read side by side:
+// each halving step exchanges half of the remaining partials with the lane 16, 8, ... apart,
+// then the last partial is summed over the remaining lanes. On return every lane holds the
+// total of partial multi_sum_index<U>(lane); the lanes with lane % (32 / U) == 0 hold the U
+// totals once each. 2U - 1 + log2(32 / U) shuffles in place of 5U.
+template <int U>
+__device__ __forceinline__ int multi_sum_index(int lane) {
+    static_assert(U == 2 || U == 4 || U == 8, "U");
+    return U == 8 ? ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1)
+                  : (U == 4 ? ((lane >> 4) & 1) * 2 + ((lane >> 3) & 1) : (lane >> 4) & 1);
+}
+template <int U>
+__device__ __forceinline__ float warp_multi_sum(const float (&v)[U]) {
+    const int lane = threadIdx.x & 31;
+    float c8[8];
+#pragma unroll
+    for (int j = 0; j < U; ++j) c8[j] = v[j];
+    if (U == 8) {  // offset 16: keep four
+        const bool up = (lane & 16) != 0;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const float send = up ? c8[j] : c8[j + 4], keep = up ? c8[j + 4] : c8[j];
+            c8[j] = keep + __shfl_xor_sync(kFull, send, 16);
+        }
+    }
+    if (U >= 4) {  // keep two
+        const int off = U == 8 ? 8 : 16;
+        const bool up = (lane & off) != 0;
+#pragma unroll
+        for (int j = 0; j < 2; ++j) {
+            const float send = up ? c8[j] : c8[j + 2], keep = up ? c8[j + 2] : c8[j];
+            c8[j] = keep + __shfl_xor_sync(kFull, send, off);
+        }
+    }
+    const int off = U == 8 ? 4 : (U == 4 ? 8 : 16);  // keep one
+    {
+        const bool up = (lane & off) != 0;
+        const float send = up ? c8[0] : c8[1], keep = up ? c8[1] : c8[0];
+        c8[0] = keep + __shfl_xor_sync(kFull, send, off);
+    }
+    float y = c8[0];
+#pragma unroll
+    for (int o = off >> 1; o > 0; o >>= 1) y += __shfl_xor_sync(kFull, y, o);
+    return y;
 }
 
 // ---------------------------------------------------------------------------------------

@@ -64,6 +64,21 @@ inline size_t workspace_bytes(int B, int N, int L, int K) {
            (size_t)B * L * K * (sizeof(float) + sizeof(int32_t));
 }
 
+// Expand-then-prune first pass: layer d holds n_d candidates, n_1 = K and
+// n_{d+1} = min(W, n_d) * K; ept_layer_start(d) = n_1 + ... + n_{d-1}, so
+// ept_layer_start(L + 1) is the number of candidates generated. The planner keeps them all in
+// shared memory, at most kEptMaxCandidates.
+constexpr int kEptMaxCandidates = 8192;
+__host__ __device__ inline int64_t ept_layer_start(int d, int K, int W) {
+    int64_t start = 0, n = K;
+    for (int e = 1; e < d; ++e) {
+        start += n;
+        n = (n < W ? n : W) * (int64_t)K;
+        if (start > ((int64_t)1 << 40)) break;
+    }
+    return start;
+}
+
 struct PlanScratch {
     float2 *lse;
     float *topk_x;
@@ -80,9 +95,20 @@ cudaError_t launch_plan_rows(const RowsDesc &draft, float2 *stats_out, int L, in
 cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int L, int N, int K, float invT,
                                 const TreeDesc &tree, const PlanScratch &sc, uint32_t *status, cudaStream_t s);
 
+cudaError_t launch_plan_expand(const RowsDesc &draft, const float2 *stats, float2 *stats_out, int L, int N, int K,
+                               int W, float invT, const TreeDesc &tree, void *ws, cudaStream_t s);
+
 cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
                           int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token, uint32_t *status,
                           cudaStream_t s);
+
+cudaError_t launch_replay_mixed(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
+                                int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token,
+                                uint32_t *status, cudaStream_t s);
+
+cudaError_t launch_verify_naive(const RowsDesc &target, int B, int N, int L, const TreeDesc &tree,
+                                const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                                int32_t *out_nodes, int32_t *out_len, void *ws, cudaStream_t s);
 
 cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
                               const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,

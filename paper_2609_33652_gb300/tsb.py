@@ -21,14 +21,16 @@ TSB_OK = 0
 STATUS_NAMES = {0: "TSB_OK", 1: "TSB_ERR_ARG", 2: "TSB_ERR_SHAPE", 3: "TSB_ERR_DTYPE", 4: "TSB_ERR_ALIGN",
                 5: "TSB_ERR_WORKSPACE", 6: "TSB_ERR_CUDA", 7: "TSB_ERR_DEVICE"}
 TSB_F32, TSB_BF16 = 0, 1
-TSB_VERIFY_RRS, TSB_VERIFY_BLOCK = 0, 1
+TSB_VERIFY_RRS, TSB_VERIFY_BLOCK, TSB_VERIFY_NAIVE = 0, 1, 2
 TSB_DEV_NONFINITE, TSB_DEV_BAD_INDEX, TSB_DEV_BAD_TREE = 0x1, 0x2, 0x4
 TSB_CHUNK = 256
 
 EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_bytes", "tsb_workspace_init",
            "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify", "tsb_plan_noalloc",
-           "tsb_plan_rows")
+           "tsb_plan_rows", "tsb_plan_expand", "tsb_plan_rows_expand", "tsb_replay_mixed")
 TSB_NOALLOC_SCRATCH_BYTES = 1 << 20
+TSB_MAX_WIDTH = 1024
+TSB_MAX_EXPAND_CANDIDATES = 8192
 
 
 class TsbError(RuntimeError):
@@ -83,6 +85,9 @@ def load():
         "tsb_plan_noalloc": (_I32, [_P, _P, _P, _SZ, _P, _P, _P]),
         "tsb_plan_rows": (_I32, [_P, _P, _P, _SZ, _P, _P, _SZ, _P]),
         "tsb_replay": (_I32, [_P, _P, _P, _SZ, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
+        "tsb_replay_mixed": (_I32, [_P, _P, _P, _SZ, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
+        "tsb_plan_expand": (_I32, [_P, _I32, _P, _P, _SZ, _P, _P, _SZ, _P]),
+        "tsb_plan_rows_expand": (_I32, [_P, _I32, _P, _P, _SZ, _P, _P, _SZ, _P]),
         "tsb_verify": (_I32, [_P, _I32, _P, _P, _P, _SZ, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
     }
     for name, (res, args) in sig.items():
@@ -186,6 +191,26 @@ def tsb_plan_rows(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict
            "tsb_plan_rows")
 
 
+def tsb_plan_expand(cfg: Cfg, width: int, draft: torch.Tensor, stats: torch.Tensor, tree: dict, ws: torch.Tensor,
+                    stream=None):
+    """Expand-then-prune first pass with frontier width ``width`` (stats from tsb_row_stats)."""
+    d = logits_desc(draft)
+    t = tree_struct(tree)
+    _check(load().tsb_plan_expand(ctypes.byref(cfg), int(width), ctypes.byref(d), _ptr(stats),
+                                  stats.numel() * stats.element_size(), ctypes.byref(t), _ptr(ws),
+                                  ws.numel() * ws.element_size(), _stream(stream)), "tsb_plan_expand")
+
+
+def tsb_plan_rows_expand(cfg: Cfg, width: int, draft: torch.Tensor, stats: torch.Tensor, tree: dict,
+                         ws: torch.Tensor, stream=None):
+    """Statistics of draft rows 0..L-1 (written into ``stats``) and the expand-then-prune pass."""
+    d = logits_desc(draft)
+    t = tree_struct(tree)
+    _check(load().tsb_plan_rows_expand(ctypes.byref(cfg), int(width), ctypes.byref(d), _ptr(stats),
+                                       stats.numel() * stats.element_size(), ctypes.byref(t), _ptr(ws),
+                                       ws.numel() * ws.element_size(), _stream(stream)), "tsb_plan_rows_expand")
+
+
 def tsb_plan_noalloc(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, dev_status=None, stream=None):
     """tsb_plan with the library's static device scratch instead of a workspace; the C call
     allocates nothing. ``dev_status``: optional int32 CUDA tensor whose first word receives
@@ -206,14 +231,27 @@ def tsb_replay(cfg: Cfg, qrows: torch.Tensor, qstats: torch.Tensor, qrow_of_node
                              ws.numel() * ws.element_size(), _stream(stream)), "tsb_replay")
 
 
-def tsb_verify(cfg: Cfg, mode: int, target: torch.Tensor, qrows: torch.Tensor, qstats: torch.Tensor, qrow_of_node,
+def tsb_replay_mixed(cfg: Cfg, qrows: torch.Tensor, qstats: torch.Tensor, qrow_of_node, tree: dict, seed: int,
+                     token: torch.Tensor, ws: torch.Tensor, stream=None):
+    """Mixed sampling: the m-1 most probable tokens, then one draw from the rest."""
+    d = logits_desc(qrows)
+    t = tree_struct(tree)
+    _check(load().tsb_replay_mixed(ctypes.byref(cfg), ctypes.byref(d), _ptr(qstats),
+                                   qstats.numel() * qstats.element_size(), _ptr(qrow_of_node), ctypes.byref(t),
+                                   int(seed) & (2**64 - 1), _ptr(token), _ptr(ws), ws.numel() * ws.element_size(),
+                                   _stream(stream)), "tsb_replay_mixed")
+
+
+def tsb_verify(cfg: Cfg, mode: int, target: torch.Tensor, qrows, qstats, qrow_of_node,
                tree: dict, token: torch.Tensor, seed: int, out_tokens: torch.Tensor, out_nodes: torch.Tensor,
                out_len: torch.Tensor, ws: torch.Tensor, stream=None):
+    """``qrows`` / ``qstats`` may be None for TSB_VERIFY_NAIVE."""
     dt = logits_desc(target)
-    dq = logits_desc(qrows)
+    dq = logits_desc(qrows) if qrows is not None else None
     t = tree_struct(tree)
-    _check(load().tsb_verify(ctypes.byref(cfg), int(mode), ctypes.byref(dt), ctypes.byref(dq), _ptr(qstats),
-                             qstats.numel() * qstats.element_size(), _ptr(qrow_of_node), ctypes.byref(t), _ptr(token),
+    qsb = qstats.numel() * qstats.element_size() if qstats is not None else 0
+    _check(load().tsb_verify(ctypes.byref(cfg), int(mode), ctypes.byref(dt), ctypes.byref(dq) if dq is not None else None,
+                             _ptr(qstats), qsb, _ptr(qrow_of_node), ctypes.byref(t), _ptr(token),
                              int(seed) & (2**64 - 1), _ptr(out_tokens), _ptr(out_nodes), _ptr(out_len), _ptr(ws),
                              ws.numel() * ws.element_size(), _stream(stream)), "tsb_verify")
 
@@ -253,11 +291,13 @@ class TsbBuffers:
 class PreparedStep:
     """One plan -> replay -> verify step with every ctypes argument built in advance, so a
     timing loop pays only the C calls. ``calls`` holds (name, function, args) in launch order:
-    tsb_plan_rows, tsb_replay, tsb_verify (``fused``, the default), or tsb_row_stats,
-    tsb_plan, tsb_replay, tsb_verify."""
+    tsb_plan_rows (or, with ``width``, tsb_plan_rows_expand), tsb_replay (``replay="wor"``),
+    tsb_replay_mixed (``"mixed"``) or nothing (``"plan"``: the first pass's tokens are
+    verified), then tsb_verify in ``mode``. With ``fused=False`` the first pass is
+    tsb_row_stats + tsb_plan instead."""
 
     def __init__(self, buf: TsbBuffers, draft: torch.Tensor, target: torch.Tensor, seed: int, mode=TSB_VERIFY_RRS,
-                 out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True):
+                 out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True, width=None, replay="wor"):
         lib = load()
         self._keep = []
         s = _stream(stream)
@@ -273,7 +313,11 @@ class PreparedStep:
         ol = buf.out_len if out_len is None else out_len
         self._keep += [ot, on, ol]
         seed = int(seed) & (2**64 - 1)
-        if fused:
+        if width is not None:
+            plan = [("tsb_plan_rows_expand", lib.tsb_plan_rows_expand,
+                     (ctypes.byref(cfg), int(width), ctypes.byref(dd), _ptr(buf.stats), sb, ctypes.byref(tr),
+                      _ptr(buf.ws), wb, s))]
+        elif fused:
             plan = [("tsb_plan_rows", lib.tsb_plan_rows, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb,
                                                           ctypes.byref(tr), _ptr(buf.ws), wb, s))]
         else:
@@ -281,12 +325,22 @@ class PreparedStep:
                      (ctypes.byref(dd), ctypes.c_float(cfg.temperature), _ptr(buf.stats), sb, _ptr(buf.ws), wb, s)),
                     ("tsb_plan", lib.tsb_plan, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb,
                                                 ctypes.byref(tr), _ptr(buf.ws), wb, s))]
-        self.calls = plan + [
-            ("tsb_replay", lib.tsb_replay, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb, None,
-                                            ctypes.byref(tr), seed, _ptr(buf.token), _ptr(buf.ws), wb, s)),
-            ("tsb_verify", lib.tsb_verify, (ctypes.byref(cfg), int(mode), ctypes.byref(dt), ctypes.byref(dd),
-                                            _ptr(buf.stats), sb, None, ctypes.byref(tr), _ptr(buf.token), seed,
-                                            _ptr(ot), _ptr(on), _ptr(ol), _ptr(buf.ws), wb, s)),
+        tok = buf.tree["plan_token"] if replay == "plan" else buf.token
+        if replay == "plan":
+            rep = []
+        else:
+            fn, name = (lib.tsb_replay_mixed, "tsb_replay_mixed") if replay == "mixed" else (lib.tsb_replay,
+                                                                                              "tsb_replay")
+            rep = [(name, fn, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb, None, ctypes.byref(tr),
+                               seed, _ptr(tok), _ptr(buf.ws), wb, s))]
+        if mode == TSB_VERIFY_NAIVE:
+            qd, qs, qsb = None, None, 0
+        else:
+            qd, qs, qsb = ctypes.byref(dd), _ptr(buf.stats), sb
+        self.calls = plan + rep + [
+            ("tsb_verify", lib.tsb_verify, (ctypes.byref(cfg), int(mode), ctypes.byref(dt), qd, qs, qsb, None,
+                                            ctypes.byref(tr), _ptr(tok), seed, _ptr(ot), _ptr(on), _ptr(ol),
+                                            _ptr(buf.ws), wb, s)),
         ]
 
     def run(self, events=None):

@@ -24,11 +24,15 @@ import oracle
 from paper_2609_33652_gb300 import synth, tsb
 
 
-def gpu_plan(draft, L, N, K, T, stats_rows=None):
+def gpu_plan(draft, L, N, K, T, width=None):
+    """tsb_row_stats + tsb_plan (max-heap), or tsb_plan_expand with frontier ``width``."""
     B, R, V = draft.shape
     buf = tsb.TsbBuffers.allocate(B, L, N, K, V, T, draft_rows=R, device=draft.device)
     tsb.tsb_row_stats(draft, T, buf.stats, buf.ws)
-    tsb.tsb_plan(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+    if width is None:
+        tsb.tsb_plan(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+    else:
+        tsb.tsb_plan_expand(buf.cfg, width, draft, buf.stats, buf.tree, buf.ws)
     return buf
 
 
@@ -112,18 +116,20 @@ def compare_verify(gout, rout, same, rep: Report, trees):
 
 
 def run_step(draft, L, N, K, T, seed, target_noise=0.7, target_seed=2000, qrows=None, qrow_of_node=None,
-             trees=None, mode=tsb.TSB_VERIFY_RRS, target=None):
+             trees=None, mode=tsb.TSB_VERIFY_RRS, target=None, width=None, replay="wor"):
     """Full plan -> replay -> verify on both sides; returns the report, the GPU buffers and
     the GPU outputs. ``trees`` restricts the oracle to a sample of trees (large batches); the
-    oracle then draws with the sampled trees' own batch indices."""
+    oracle then draws with the sampled trees' own batch indices. ``width``: expand-then-prune
+    first pass with that frontier (default: max-heap). ``replay``: "wor" (tsb_replay), "mixed"
+    (tsb_replay_mixed) or "plan" (no replay: the first pass's tokens are verified)."""
     rep = Report()
-    buf = gpu_plan(draft, L, N, K, T)
+    buf = gpu_plan(draft, L, N, K, T, width)
     check_status(buf)
     B = draft.shape[0]
     sel = list(range(B)) if trees is None else list(trees)
     bids = np.array(sel, dtype=np.int32)
     h_draft = synth.to_host(draft[sel])
-    ref = oracle.plan(h_draft, T, N, K, L)
+    ref = oracle.plan(h_draft, T, N, K, L) if width is None else oracle.plan_expand(h_draft, T, N, K, L, width)
     same = compare_plan(buf, ref, rep, sel)
 
     if qrows is None:
@@ -137,9 +143,16 @@ def run_step(draft, L, N, K, T, seed, target_noise=0.7, target_seed=2000, qrows=
         qidx = qrow_of_node
         h_q = synth.to_host(qrows[sel])
         h_qidx = qrow_of_node[sel].cpu().numpy()
-    tsb.tsb_replay(buf.cfg, q, qstats, qidx, buf.tree, seed, buf.token, buf.ws)
+    if replay == "plan":
+        buf.token.copy_(buf.tree["plan_token"])
+        rtok, rex = ref["plan_token"], np.zeros(ref["plan_token"].shape, dtype=bool)
+    elif replay == "mixed":
+        tsb.tsb_replay_mixed(buf.cfg, q, qstats, qidx, buf.tree, seed, buf.token, buf.ws)
+        rtok, rex = oracle.replay_mixed(h_q, T, ref, seed, qrow_of_node=h_qidx, batch_ids=bids)
+    else:
+        tsb.tsb_replay(buf.cfg, q, qstats, qidx, buf.tree, seed, buf.token, buf.ws)
+        rtok, rex = oracle.replay(h_q, T, ref, seed, qrow_of_node=h_qidx, batch_ids=bids)
     check_status(buf)
-    rtok, rex = oracle.replay(h_q, T, ref, seed, qrow_of_node=h_qidx, batch_ids=bids)
     gtok = buf.token.cpu().numpy()
     same = compare_tokens(gtok, rtok, rex, host_tree(buf), same, rep, sel)
 
@@ -150,11 +163,17 @@ def run_step(draft, L, N, K, T, seed, target_noise=0.7, target_seed=2000, qrows=
                                                        target_noise, target_seed)[sel])
     else:
         h_target = synth.to_host(target[sel])
-    tsb.tsb_verify(buf.cfg, mode, target, q, qstats, qidx, buf.tree, buf.token, seed, buf.out_tokens,
-                   buf.out_nodes, buf.out_len, buf.ws)
+    if mode == tsb.TSB_VERIFY_NAIVE:  # no draft rows needed
+        tsb.tsb_verify(buf.cfg, mode, target, None, None, None, buf.tree, buf.token, seed, buf.out_tokens,
+                       buf.out_nodes, buf.out_len, buf.ws)
+    else:
+        tsb.tsb_verify(buf.cfg, mode, target, q, qstats, qidx, buf.tree, buf.token, seed, buf.out_tokens,
+                       buf.out_nodes, buf.out_len, buf.ws)
     check_status(buf)
     if mode == tsb.TSB_VERIFY_RRS:
         rout = oracle.verify_rrs(h_target, h_q, T, ref, rtok, seed, L, qrow_of_node=h_qidx, batch_ids=bids)
+    elif mode == tsb.TSB_VERIFY_NAIVE:
+        rout = oracle.verify_naive(h_target, T, ref, rtok, seed, L, batch_ids=bids)
     else:
         rout = oracle.verify_block(h_target, h_q, T, ref, rtok, seed, L, qrow_of_node=h_qidx, batch_ids=bids)
     gout = {"len": buf.out_len.cpu().numpy(), "tokens": buf.out_tokens.cpu().numpy(),

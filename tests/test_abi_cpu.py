@@ -135,11 +135,57 @@ def test_replay_verify_validation(lib):
         return lib.tsb_verify(ctypes.byref(cfg), mode, ctypes.byref(tg), ctypes.byref(q), FAKE, 1 << 30, None,
                               ctypes.byref(t), FAKE, 1, out, FAKE, FAKE, FAKE, 1 << 30, None)
 
-    assert verify(mode=2) == ARG
+    assert verify(mode=3) == ARG
     assert verify(target=_logits(2, 8, 64)) == SHAPE  # needs N+1 target rows
     assert verify(target=_logits(2, 9, 64, dtype=1)) == DTYPE  # target / q dtypes differ
     assert verify(out=None) == ARG
     assert verify(mode=1, cfg=tsb.make_cfg(2, 4, 5, 4, 64, 1.0)) == SHAPE  # block: chain longer than L
+
+
+def test_naive_and_mixed_validation(lib):
+    cfg = tsb.make_cfg(2, 4, 8, 4, 64, 1.0)
+    t = _tree()
+    tg = _logits(2, 9, 64)
+
+    def naive(target=tg, token=FAKE, out=FAKE, ws_bytes=1 << 30):
+        # target-sample matching takes no draft rows: qrows / qstats may be NULL
+        return lib.tsb_verify(ctypes.byref(cfg), tsb.TSB_VERIFY_NAIVE, ctypes.byref(target), None, None, 0, None,
+                              ctypes.byref(t), token, 1, out, FAKE, FAKE, FAKE, ws_bytes, None)
+
+    assert naive(target=_logits(2, 8, 64)) == SHAPE  # needs N+1 target rows
+    assert naive(target=_logits(2, 9, 64, dtype=2)) == DTYPE
+    assert naive(token=None) == ARG
+    assert naive(out=None) == ARG
+    assert naive(ws_bytes=255) == WS
+    q = _logits(2, 4, 64)
+
+    def mixed(q=q, token=FAKE, ws_bytes=1 << 30):
+        return lib.tsb_replay_mixed(ctypes.byref(cfg), ctypes.byref(q), FAKE, 1 << 30, None, ctypes.byref(t), 1,
+                                    token, FAKE, ws_bytes, None)
+
+    assert mixed(token=None) == ARG
+    assert mixed(q=_logits(2, 3, 64)) == SHAPE  # per-depth rows need L rows
+    assert mixed(ws_bytes=255) == WS
+
+
+def test_plan_expand_validation(lib):
+    good = tsb.make_cfg(4, 16, 64, 8, 1024, 1.0)
+    d = _logits(4, 16, 1024)
+
+    def call(width, cfg=good, draft=d, stats=FAKE, fused=False):
+        fn = lib.tsb_plan_rows_expand if fused else lib.tsb_plan_expand
+        return fn(ctypes.byref(cfg), width, ctypes.byref(draft), stats, 1 << 30, ctypes.byref(_tree()), FAKE,
+                  1 << 30, None)
+
+    for fused in (False, True):
+        assert call(0, fused=fused) == SHAPE
+        assert call(tsb.TSB_MAX_WIDTH + 1, fused=fused) == SHAPE
+        assert call(10, stats=None, fused=fused) == ARG
+        assert call(10, draft=_logits(4, 15, 1024), fused=fused) == SHAPE
+        # W = 1, K = 2, L = 3: 2 + 2 + 2 = 6 candidates cannot hold N = 7
+        assert call(1, cfg=tsb.make_cfg(4, 3, 7, 2, 1024, 1.0), draft=_logits(4, 3, 1024), fused=fused) == SHAPE
+        # K = 32, W = 64, L = 16: far more than TSB_MAX_EXPAND_CANDIDATES candidates
+        assert call(64, cfg=tsb.make_cfg(4, 16, 64, 32, 1024, 1.0), fused=fused) == SHAPE
 
 
 def test_workspace_and_status_validation(lib):
