@@ -584,18 +584,18 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
 // Expand-then-prune first pass (the EAGLE-2-style planner of Sec. 3.1 and App. B.3), one CTA
 // per tree. Layer 1 is the root's K children; layer d+1 holds the K children of each of the W
 // best candidates of layer d (its frontier), so layers stay at most W*K wide and L layers
-// deep. Every layer is kept sorted by (key desc, parent's position asc, rank asc): candidate
-// (f, r) of layer d+1 has sum Sx = Sx_f + x_{d,r}, and the candidates of frontier entry f' that
-// precede it are those whose logit exceeds Sx - Sx_f' (or reaches it when f' < f), a prefix of
-// the depth's sorted top-K logits found by binary search; its position is r plus those counts.
-// After the last layer, a candidate's place in the global order (key desc, depth asc, parent's
-// position asc, rank asc) is its layer position plus, for every other layer, the number of
-// entries above its key there (at or above it for shallower layers), again by binary search;
-// the N first are the nodes, numbered in that order. Keys are the 64-bit fixed-point path
+// deep. Every layer is kept sorted by (key desc, parent's position asc, rank asc): a layer of at
+// most kEptSmallLayer candidates by counting, for each candidate, the ones before it (several
+// threads per candidate); a wider one by binary search: candidate (f, r) of layer d+1 has sum
+// Sx = Sx_f + x_{d,r}, the candidates of frontier entry f' that precede it are those whose logit
+// exceeds Sx - Sx_f' (or reaches it when f' < f), a prefix of the depth's sorted top-K logits,
+// and its position is r plus those counts.
+// After the last layer, one warp merges the sorted layers in the global order (key desc, depth
+// asc, parent's position asc, rank asc): the N first are the nodes, numbered in that order. Keys are the 64-bit fixed-point path
 // sums of the max-heap planner, so same-depth comparisons are exact and a frontier holding N
 // candidates gives the heap's tree bit for bit.
 constexpr int kEptThreads = 512;
-constexpr int kEptGroup = 8;  // layers searched in lockstep per candidate
+constexpr int kEptSmallLayer = 512;  // layers up to this size are ranked by counting
 
 struct EptArgs {
     int L, N, K, W;
@@ -655,34 +655,46 @@ __global__ void __launch_bounds__(kEptThreads) k_plan_ept(EptArgs a) {
         smeta[j] = j;
     }
     __syncthreads();
-    // 2. layers 2..L, each placed at its sorted positions: a layer of at most one candidate per
-    //    thread by counting the candidates before each (index order j = f*K + r is the order of
-    //    equal keys), a wider one by binary searches over the depth's sorted logits
-    __shared__ long long tkey[kEptThreads];
+    // 2. layers 2..L, each placed at its sorted positions: a layer of at most kEptSmallLayer
+    //    candidates by counting the candidates before each, a wider one by binary searches over
+    //    the depth's sorted logits
+    __shared__ long long tkey[kEptSmallLayer];
+    __shared__ int tpos[kEptSmallLayer];
     int kbits = 0;  // steps of the binary search over a depth's K logits
     while ((1 << kbits) <= K) ++kbits;
     for (int d = 1; d < L; ++d) {
         const int prev = lstart[d], nf = min(W, lstart[d + 1] - prev), base = lstart[d + 1];
         const long long cd = CL[d], cd1 = CL[d + 1];
         const long long *row = fx + d * K;  // logits of depth d+1, non-increasing in rank
-        if (nf * K <= kEptThreads) {  // uniform over the CTA
-            const int n = nf * K, j = threadIdx.x;
-            const int f = j / K, r = j - f * K;
-            long long key = 0;
-            if (j < n) {
-                key = skey[prev + f] + cd + row[r] - cd1;
-                tkey[j] = key;
+        if (nf * K <= kEptSmallLayer) {  // uniform over the CTA
+            const int n = nf * K;
+            for (int j = threadIdx.x; j < n; j += kEptThreads) {
+                const int f = j / K, r = j - f * K;
+                tkey[j] = skey[prev + f] + cd + row[r] - cd1;
+                tpos[j] = 0;
             }
             __syncthreads();
-            if (j < n) {
-                int pos = 0;
-#pragma unroll 8
-                for (int i2 = 0; i2 < n; ++i2) {  // independent loads, eight in flight
+            // candidate j's position = the candidates before it (larger key, or the same key and a
+            // smaller index: index order j = f*K + r is the order of equal keys), counted by
+            // S threads per candidate over slices of the layer
+            const int S = max(1, kEptThreads / n), per = (n + S - 1) / S;
+            for (int t = threadIdx.x; t < n * S; t += kEptThreads) {
+                const int j = t / S, part = t - j * S;
+                const long long key = tkey[j];
+                const int lo = part * per, hi = min(n, lo + per);
+                int cnt = 0;
+#pragma unroll 4
+                for (int i2 = lo; i2 < hi; ++i2) {
                     const long long k2 = tkey[i2];
-                    pos += (k2 > key || (k2 == key && i2 < j)) ? 1 : 0;
+                    cnt += (k2 > key || (k2 == key && i2 < j)) ? 1 : 0;
                 }
-                skey[base + pos] = key;
-                smeta[base + pos] = (f << 8) | r;
+                if (cnt) atomicAdd(&tpos[j], cnt);
+            }
+            __syncthreads();
+            for (int j = threadIdx.x; j < n; j += kEptThreads) {
+                const int f = j / K, r = j - f * K;
+                skey[base + tpos[j]] = tkey[j];
+                smeta[base + tpos[j]] = (f << 8) | r;
             }
             __syncthreads();  // before the next layer reads skey and rewrites tkey
             continue;
@@ -705,45 +717,54 @@ __global__ void __launch_bounds__(kEptThreads) k_plan_ept(EptArgs a) {
         }
         __syncthreads();
     }
-    // 3. places in the global order; the first N are the nodes
-    int lbits = 0;  // steps of a binary search over a layer
-    while ((1 << lbits) <= W * K || (1 << lbits) <= K) ++lbits;
-    for (int idx = threadIdx.x; idx < G; idx += kEptThreads) {
-        int d = 1;
-        while (lstart[d + 1] <= idx) ++d;
-        int g = idx - lstart[d];
-        if (g >= N) {  // N candidates of its own layer come first
-            node_of[idx] = 0;
-            continue;
-        }
-        const long long k = skey[idx];
-        for (int d0 = 1; d0 <= L && g < N; d0 += kEptGroup) {
-            int c[kEptGroup], lo[kEptGroup], len[kEptGroup];
-#pragma unroll
-            for (int q = 0; q < kEptGroup; ++q) {
-                const int d2 = d0 + q;
-                const bool live = d2 <= L && d2 != d;
-                c[q] = 0;
-                lo[q] = live ? lstart[d2] : 0;
-                len[q] = live ? lstart[d2 + 1] - lstart[d2] : 0;
+    // 3. the first N of the global order, merged from the sorted layers by one warp: lane l
+    //    holds the heads of layers l+1 and l+33; each step takes the largest head by (key desc,
+    //    depth asc), the 32-bit monotone image of the key first, the full key and the depth
+    //    only among lanes that tie on it
+    for (int idx = threadIdx.x; idx < G; idx += kEptThreads) node_of[idx] = 0;
+    __syncthreads();
+    if (warp == 0) {
+        const int lane = threadIdx.x & 31;
+        const int dA = lane + 1, dB = lane + 33;
+        const int sA = dA <= L ? lstart[dA] : 0, nA = dA <= L ? lstart[dA + 1] - sA : 0;
+        const int sB = dB <= L ? lstart[dB] : 0, nB = dB <= L ? lstart[dB + 1] - sB : 0;
+        int pA = 0, pB = 0;
+        unsigned long long kA = nA > 0 ? okey_of(skey[sA]) : 0ull;
+        unsigned long long kB = nB > 0 ? okey_of(skey[sB]) : 0ull;
+        for (int i = 1; i <= N; ++i) {
+            const bool useB = kB > kA;  // equal keys: the shallower layer A first
+            const unsigned long long kb = useB ? kB : kA;
+            const unsigned wd = 255u - (unsigned)(useB ? dB : dA);
+            const unsigned ck = coarse_of(kb);
+            const unsigned m0 = __reduce_max_sync(kFull, ck);
+            unsigned c = __ballot_sync(kFull, ck == m0);
+            if (__popc(c) > 1) {
+                const unsigned hk = (unsigned)(kb >> 32);
+                const unsigned m1 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? hk : 0u);
+                c &= __ballot_sync(kFull, hk == m1);
+                const unsigned lk = (unsigned)kb;
+                const unsigned m2 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? lk : 0u);
+                c &= __ballot_sync(kFull, lk == m2);
+                const unsigned m3 = __reduce_max_sync(kFull, ((c >> lane) & 1u) ? wd : 0u);
+                c &= __ballot_sync(kFull, wd == m3);
             }
-            for (int step = 1 << (lbits - 1); step > 0; step >>= 1) {
-                long long k2[kEptGroup];
-#pragma unroll
-                for (int q = 0; q < kEptGroup; ++q) {  // the group's loads issued together
-                    const bool in = c[q] + step <= len[q];
-                    k2[q] = skey[lo[q] + (in ? c[q] + step - 1 : 0)];
-                }
-#pragma unroll
-                for (int q = 0; q < kEptGroup; ++q) {
-                    const bool in = c[q] + step <= len[q];
-                    c[q] += (in && (d0 + q < d ? k2[q] >= k : k2[q] > k)) ? step : 0;
+            const int owner = __ffs(c) - 1;
+            if (__shfl_sync(kFull, kb, owner) == 0ull) {  // every layer used up (N > G: rejected on the host)
+                if (lane == 0) raise_status(a.status, kDevBadTree);
+                break;
+            }
+            if (lane == owner) {
+                if (useB) {
+                    node_of[sB + pB] = i;
+                    ++pB;
+                    kB = pB < nB ? okey_of(skey[sB + pB]) : 0ull;
+                } else {
+                    node_of[sA + pA] = i;
+                    ++pA;
+                    kA = pA < nA ? okey_of(skey[sA + pA]) : 0ull;
                 }
             }
-#pragma unroll
-            for (int q = 0; q < kEptGroup; ++q) g += c[q];
         }
-        node_of[idx] = g < N ? g + 1 : 0;
     }
     __syncthreads();
     bool bad = false;
