@@ -59,6 +59,7 @@ def parse():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-variants", action="store_true", help="skip the other sampling / verification schemes")
     ap.add_argument("--variant-steps", type=int, default=300)
+    ap.add_argument("--no-planners", action="store_true", help="skip the first-pass-only timings at N = 64 and 256")
     ap.add_argument("--workload", default="batched", choices=("batched", "batched128k"))
     args = ap.parse_args()
     if args.steps is None:
@@ -269,6 +270,36 @@ def run_variants(w, sets, device, steps=300, warmup=10):
     return out
 
 
+def run_planners(w, sets, device, steps=300, warmup=10, budgets=(64, 256), width=10):
+    """The first pass alone (draft statistics + top-K + expansion) at two budgets: the max-heap
+    planner against expand-then-prune with the given frontier width (App. B.3)."""
+    import torch
+
+    from paper_2609_33652_gb300 import tsb
+
+    B, L, S = w["B"], w["L"], len(sets)
+    out = {}
+    for N in budgets:
+        bufs = [tsb.TsbBuffers.allocate(B, L, N, w["K"], w["V"], w["T"], device=device) for _ in range(S)]
+        for name, wd in (("max_heap", None), (f"expand_prune_w{width}", width)):
+            prep = [tsb.PreparedStep(bufs[k % S], sets[k % S]["draft"], sets[k % S]["target"], 1, width=wd,
+                                     plan_only=True) for k in range(steps)]
+            for k in range(min(warmup, steps)):
+                prep[k].run()
+            torch.cuda.synchronize()
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record()
+            for p in prep:
+                p.run()
+            t1.record()
+            torch.cuda.synchronize()
+            for bf in bufs:
+                if tsb.tsb_device_status(bf.ws) != 0:
+                    raise RuntimeError(f"device status bits set in planner {name}, N={N}")
+            out[f"{name}_N{N}"] = round(t0.elapsed_time(t1) * 1e3 / steps, 3)
+    return out
+
+
 def max_over_ranks(value: float, dist, device) -> float:
     """The largest of the ranks' values (every rank gets it): a job's time is its slowest
     replica's. ``device`` is where the process group's backend reduces (cuda for nccl)."""
@@ -382,6 +413,8 @@ def run_tsb(args):
     # end to end through the C ABI with pinned host buffers
     e2e = run_e2e(args, w, sets, device) if args.e2e_steps > 0 else None
     variants = run_variants(w, sets, device, steps=args.variant_steps) if not args.no_variants else None
+    if variants is not None and not args.no_planners:
+        variants["first_pass_us_per_call"] = run_planners(w, sets, device, steps=args.variant_steps)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:

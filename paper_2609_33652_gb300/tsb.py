@@ -294,10 +294,11 @@ class PreparedStep:
     tsb_plan_rows (or, with ``width``, tsb_plan_rows_expand), tsb_replay (``replay="wor"``),
     tsb_replay_mixed (``"mixed"``) or nothing (``"plan"``: the first pass's tokens are
     verified), then tsb_verify in ``mode``. With ``fused=False`` the first pass is
-    tsb_row_stats + tsb_plan instead."""
+    tsb_row_stats + tsb_plan instead; with ``plan_only`` only the first pass runs."""
 
     def __init__(self, buf: TsbBuffers, draft: torch.Tensor, target: torch.Tensor, seed: int, mode=TSB_VERIFY_RRS,
-                 out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True, width=None, replay="wor"):
+                 out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True, width=None, replay="wor",
+                 plan_only=False):
         lib = load()
         self._keep = []
         s = _stream(stream)
@@ -342,6 +343,8 @@ class PreparedStep:
                                             ctypes.byref(tr), _ptr(tok), seed, _ptr(ot), _ptr(on), _ptr(ol),
                                             _ptr(buf.ws), wb, s)),
         ]
+        if plan_only:  # the first pass alone
+            self.calls = plan
 
     def run(self, events=None):
         """Launch the calls; with ``events`` (len(calls) + 1 torch.cuda.Event), record one
