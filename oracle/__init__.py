@@ -29,6 +29,12 @@ Parity status of each function (what pins it, see tests/test_oracle_*.py):
                      against q renormalised over the remaining tokens; m = 1 is the WoR draw.
   verify_naive     : chi-square of the emitted tokens against the target law; acceptance
                      frequency vs the closed form p(y) (Sec. 2.3); forced acceptances.
+  plan (pool=P)    : brute-force path enumeration with pooled normalisers; P = V is the
+                     full-vocabulary planner.
+  replay_pooled    : chi-square of ordered draws vs the WoR law of the pooled q; tokens stay
+                     in the pool; P = V is the flat sampler token for token.
+  verify_rrs(pool) : chi-square losslessness with pooled q; single-child acceptance
+                     sum min(p, q_pool); P = V is the full-vocabulary verifier.
 """
 from __future__ import annotations
 
@@ -96,6 +102,11 @@ def _load():
                                  _P]),
         "orc_replay_mixed": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, ctypes.c_uint64, _P, _P, _P]),
         "orc_verify_naive": (_I, [_P, ctypes.c_float, _I, _I, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _P]),
+        "orc_plan_pooled": (_I, [_P, ctypes.c_float, _I, _I, _I, _I, _P, _P, _P, _P, _P, _P, _P, ctypes.c_double, _P,
+                                 _P]),
+        "orc_replay_pooled": (_I, [_P, ctypes.c_float, _P, _I, _P, _P, _P, _P, _I, _I, ctypes.c_uint64, _P, _P, _P]),
+        "orc_verify_rrs_pooled": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _I,
+                                       _I, _P, _P, _P, _P]),
         "orc_verify_block": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P,
                                   _P, _P, _P]),
     }
@@ -168,7 +179,8 @@ def row_stats(rows: np.ndarray, temperature: float, K: int = 1):
             "topk_x": tx.reshape(B, R, K), "chunk_lse": clse.reshape(B, R, C)}
 
 
-def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps: float = 1e-6):
+def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps: float = 1e-6, pool: int = 0):
+    """First pass; ``pool`` = P > 0 normalises each depth's law over its P most probable tokens."""
     lib = _load()
     B = draft.shape[0]
     NN = N + 1
@@ -179,9 +191,15 @@ def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps:
     child_ids = np.zeros(B * N, dtype=np.int32)
     exempt = np.zeros(B, dtype=np.uint8)
     margin = np.zeros(B)
-    _check(lib.orc_plan(ctypes.byref(d), temperature, N, K, L, _ptr(out["parent"]), _ptr(out["depth"]),
-                        _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score), _ptr(child_off), _ptr(child_ids),
-                        key_eps, _ptr(exempt), _ptr(margin)), "plan")
+    if pool:
+        rc = lib.orc_plan_pooled(ctypes.byref(d), temperature, N, K, L, int(pool), _ptr(out["parent"]),
+                                 _ptr(out["depth"]), _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score),
+                                 _ptr(child_off), _ptr(child_ids), key_eps, _ptr(exempt), _ptr(margin))
+    else:
+        rc = lib.orc_plan(ctypes.byref(d), temperature, N, K, L, _ptr(out["parent"]), _ptr(out["depth"]),
+                          _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score), _ptr(child_off), _ptr(child_ids),
+                          key_eps, _ptr(exempt), _ptr(margin))
+    _check(rc, "plan")
     tree = {k: v.reshape(B, NN) for k, v in out.items()}
     tree["score"] = score.reshape(B, NN)
     tree["child_off"] = child_off.reshape(B, NN + 1)
@@ -273,8 +291,33 @@ def verify_naive(target: np.ndarray, temperature: float, tree, token, seed: int,
     return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool)}
 
 
+def pools(draft: np.ndarray, temperature: float, P: int):
+    """Per (tree, depth row) the P most probable tokens by (x desc, id asc): [B, R, P] int32."""
+    return np.ascontiguousarray(row_stats(draft, temperature, P)["topk_id"])
+
+
+def replay_pooled(q: np.ndarray, temperature: float, tree, seed: int, pool_ids: np.ndarray, qrow_of_node=None,
+                  batch_ids=None):
+    """WoR draws from the pooled draft laws; pool_ids [B, Lp, P]. Tokens [B, N+1] and near-tie flags."""
+    lib = _load()
+    bids = _i32(batch_ids)
+    B = q.shape[0]
+    NN = tree["depth"].shape[1]
+    d, keep = _logits(q)
+    depth, off, ids = _tree_ptrs(tree)
+    qr = _i32(qrow_of_node)
+    pl = _i32(pool_ids)
+    token = np.zeros(B * NN, dtype=np.int32)
+    exempt = np.zeros(B * NN, dtype=np.uint8)
+    _check(lib.orc_replay_pooled(ctypes.byref(d), temperature, _ptr(qr), NN - 1, _ptr(depth), _ptr(off), _ptr(ids),
+                                 _ptr(pl), pl.shape[2], pl.shape[1], int(seed), _ptr(bids), _ptr(token),
+                                 _ptr(exempt)), "replay_pooled")
+    return token.reshape(B, NN), exempt.reshape(B, NN).astype(bool)
+
+
 def verify_rrs(target: np.ndarray, q: np.ndarray, temperature: float, tree, token, seed: int, L: int,
-               qrow_of_node=None, batch_ids=None):
+               qrow_of_node=None, batch_ids=None, pool_ids=None):
+    """Recursive rejection sampling; with ``pool_ids`` [B, Lp, P] the draft laws are pooled."""
     lib = _load()
     bids = _i32(batch_ids)
     B = target.shape[0]
@@ -288,9 +331,16 @@ def verify_rrs(target: np.ndarray, q: np.ndarray, temperature: float, tree, toke
     onode = np.zeros(B * L, dtype=np.int32)
     olen = np.zeros(B, dtype=np.int32)
     ex = np.zeros(B, dtype=np.uint8)
-    _check(lib.orc_verify_rrs(ctypes.byref(dt), ctypes.byref(dq), temperature, _ptr(qr), NN - 1, L, _ptr(depth),
-                              _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(bids), _ptr(otok), _ptr(onode),
-                              _ptr(olen), _ptr(ex)), "verify_rrs")
+    if pool_ids is not None:
+        pl = _i32(pool_ids)
+        rc = lib.orc_verify_rrs_pooled(ctypes.byref(dt), ctypes.byref(dq), temperature, _ptr(qr), NN - 1, L,
+                                       _ptr(depth), _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(bids), _ptr(pl),
+                                       pl.shape[2], pl.shape[1], _ptr(otok), _ptr(onode), _ptr(olen), _ptr(ex))
+    else:
+        rc = lib.orc_verify_rrs(ctypes.byref(dt), ctypes.byref(dq), temperature, _ptr(qr), NN - 1, L, _ptr(depth),
+                                _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(bids), _ptr(otok), _ptr(onode),
+                                _ptr(olen), _ptr(ex))
+    _check(rc, "verify_rrs")
     return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool)}
 
 

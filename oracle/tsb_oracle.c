@@ -232,11 +232,15 @@ static int64_t max_nodes(int K, int L)
     return total;
 }
 
-int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L,
-             int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
-             int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+/* pool = 0: path scores use the full-vocabulary log-normaliser of each draft row; pool = P > 0:
+ * the log-normaliser of the row's P most probable tokens (the pooled draft law of Sec. 3.1),
+ * whose K most probable tokens are the candidates.                                        */
+static int plan_impl(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L, int32_t pool,
+                     int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
+                     int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
 {
     if (!draft || N < 1 || K < 1 || L < 1 || K > 64 || K > draft->V || draft->R < L) return -1;
+    if (pool != 0 && (pool < K || pool > draft->V)) return -1;
     if (!(temperature > 0.0f)) return -1;
     if ((int64_t)N > max_nodes(K, L)) return -2;
     const float invT = 1.0f / temperature;
@@ -249,7 +253,9 @@ int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, i
     double *sxn = (double *)malloc(sizeof(double) * NN);
     cand *front = (cand *)malloc(sizeof(cand) * (2 * (size_t)NN + 2));
     int32_t *nchild = (int32_t *)malloc(sizeof(int32_t) * NN);
-    if (!x || !lse || !CL || !tid || !tx || !sxn || !front || !nchild) return -3;
+    int32_t *pid = (int32_t *)malloc(sizeof(int32_t) * (pool > 0 ? pool : 1));
+    double *px = (double *)malloc(sizeof(double) * (pool > 0 ? pool : 1));
+    if (!x || !lse || !CL || !tid || !tx || !sxn || !front || !nchild || !pid || !px) return -3;
 
     for (int b = 0; b < draft->B; ++b) {
         int32_t *par = parent + (int64_t)b * NN, *dep = depth + (int64_t)b * NN;
@@ -258,7 +264,12 @@ int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, i
         /* per-depth candidate pools: top-K of draft row d (tokens of depth d+1) */
         for (int d = 0; d < L; ++d) {
             read_row(draft, b, d, invT, x);
-            lse[d] = logsumexp(x, V);
+            if (pool > 0) { /* the pooled law: normalised over the row's P most probable tokens */
+                topk_row(x, V, pool, pid, px);
+                lse[d] = logsumexp(px, pool);
+            } else {
+                lse[d] = logsumexp(x, V);
+            }
             topk_row(x, V, K, tid + d * K, tx + d * K);
         }
         CL[0] = 0.0;
@@ -328,8 +339,27 @@ int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, i
         for (int u = 0; u < NN; ++u) nchild[u] = 0;
         for (int i = 1; i <= N; ++i) ids[off[par[i]] + nchild[par[i]]++] = i;
     }
-    free(x); free(lse); free(CL); free(tid); free(tx); free(sxn); free(front); free(nchild);
+    free(x); free(lse); free(CL); free(tid); free(tx); free(sxn); free(front); free(nchild); free(pid); free(px);
     return 0;
+}
+
+int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L,
+             int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
+             int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+{
+    return plan_impl(draft, temperature, N, K, L, 0, parent, depth, rank, plan_token, score, child_off, child_ids,
+                     key_eps, exempt, min_margin);
+}
+
+/* First pass with pooled draft laws (Sec. 3.1, App. B.7): as orc_plan, with each depth's law
+ * normalised over its P most probable tokens. */
+int orc_plan_pooled(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L, int32_t P,
+                    int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
+                    int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+{
+    if (P < 1) return -1;
+    return plan_impl(draft, temperature, N, K, L, P, parent, depth, rank, plan_token, score, child_off, child_ids,
+                     key_eps, exempt, min_margin);
 }
 
 /* ------------------------------------------------------------------------------------ */
@@ -627,10 +657,28 @@ int orc_rrs_node_law(int32_t V, const double *P_in, const double *Q, int32_t m, 
     return degenerate;
 }
 
-int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperature, const int32_t *qrow_of_node,
-                   int32_t N, int32_t L, const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
-                   const int32_t *token, uint64_t seed, const int32_t *batch_ids, int32_t *out_tokens,
-                   int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
+/* The draft law of node u: softmax of its q row over the whole vocabulary, or, with pools
+ * (pool_ids [B][Lp][P], row depth[u] of tree b), over the P pool tokens only (zero elsewhere). */
+static void draft_law(const double *xq, int V, const int32_t *pool, int P, double *Q)
+{
+    if (!pool) {
+        softmax(xq, V, Q);
+        return;
+    }
+    double m = -INFINITY, s = 0.0;
+    for (int j = 0; j < P; ++j)
+        if (xq[pool[j]] > m) m = xq[pool[j]];
+    for (int j = 0; j < P; ++j) s += exp(xq[pool[j]] - m);
+    const double lse = m + log(s);
+    for (int v = 0; v < V; ++v) Q[v] = 0.0;
+    for (int j = 0; j < P; ++j) Q[pool[j]] = exp(xq[pool[j]] - lse);
+}
+
+static int verify_rrs_impl(const orc_logits *target, const orc_logits *q, float temperature,
+                           const int32_t *qrow_of_node, int32_t N, int32_t L, const int32_t *depth,
+                           const int32_t *child_off, const int32_t *child_ids, const int32_t *token, uint64_t seed,
+                           const int32_t *batch_ids, const int32_t *pool_ids, int32_t Pn, int32_t Lp,
+                           int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
 {
     if (!target || !q || N < 0 || L < 1 || !(temperature > 0.0f) || target->V != q->V || target->R < N + 1) return -1;
     const float invT = 1.0f / temperature;
@@ -660,7 +708,9 @@ int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperat
             if (r < 0 || r >= q->R) return -5;
             read_row(q, b, r, invT, xq);
             softmax(xt, V, P);
-            softmax(xq, V, Q);
+            const int pd = depth[nb + u];
+            if (pool_ids && (pd < 0 || pd >= Lp)) return -5;
+            draft_law(xq, V, pool_ids ? pool_ids + ((int64_t)b * Lp + pd) * Pn : NULL, Pn, Q);
             memset(drawn, 0, V);
             double t = 1.0;
             int accepted = -1;
@@ -697,6 +747,30 @@ int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperat
     }
     free(xt); free(xq); free(P); free(Q); free(R); free(drawn);
     return 0;
+}
+
+int orc_verify_rrs(const orc_logits *target, const orc_logits *q, float temperature, const int32_t *qrow_of_node,
+                   int32_t N, int32_t L, const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
+                   const int32_t *token, uint64_t seed, const int32_t *batch_ids, int32_t *out_tokens,
+                   int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
+{
+    return verify_rrs_impl(target, q, temperature, qrow_of_node, N, L, depth, child_off, child_ids, token, seed,
+                           batch_ids, NULL, 0, 0, out_tokens, out_nodes, out_len, exempt);
+}
+
+/* Recursive rejection sampling with pooled draft laws (Sec. 3.3: the probabilities of replayed
+ * candidates are normalised within the pool; the residual stays full-vocabulary, App. B.1
+ * on pools: the restriction applies to draft proposals only). pool_ids [B][Lp][P]: the pool of
+ * the tokens at depth d+1 in row d, used for the children of every node at depth d. */
+int orc_verify_rrs_pooled(const orc_logits *target, const orc_logits *q, float temperature,
+                          const int32_t *qrow_of_node, int32_t N, int32_t L, const int32_t *depth,
+                          const int32_t *child_off, const int32_t *child_ids, const int32_t *token, uint64_t seed,
+                          const int32_t *batch_ids, const int32_t *pool_ids, int32_t P, int32_t Lp,
+                          int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
+{
+    if (!pool_ids || P < 1 || P > q->V || Lp < 1) return -1;
+    return verify_rrs_impl(target, q, temperature, qrow_of_node, N, L, depth, child_off, child_ids, token, seed,
+                           batch_ids, pool_ids, P, Lp, out_tokens, out_nodes, out_len, exempt);
 }
 
 /* ------------------------------------------------------------------------------------ */
@@ -1125,5 +1199,57 @@ int orc_verify_naive(const orc_logits *target, float temperature, int32_t N, int
         if (exempt) exempt[b] = ex;
     }
     free(xt);
+    return 0;
+}
+
+/* ------------------------------------------------------------------------------------ */
+/* REPLAY with pooled draft laws (Sec. 3.2: q_u is restricted to the same sparse candidate
+ * pools as the first pass and normalised within them). For a parent u with m children, the
+ * pool is row depth[u] of pool_ids [B][Lp][P] (the P tokens of the children's position); the
+ * m ordered WoR draws from q_u restricted to the pool are the top-m Gumbel keys
+ * x_v + G(U[REPLAY_ELEM, u, v]) over the pool tokens (Gumbel-top-k over P tokens; the pool is
+ * small, so the keys are drawn flat, with the counters the flat sampler uses).            */
+int orc_replay_pooled(const orc_logits *q, float temperature, const int32_t *qrow_of_node, int32_t N,
+                      const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
+                      const int32_t *pool_ids, int32_t P, int32_t Lp, uint64_t seed, const int32_t *batch_ids,
+                      int32_t *token, uint8_t *exempt_node)
+{
+    if (!q || !pool_ids || N < 0 || P < 1 || P > q->V || Lp < 1 || !(temperature > 0.0f)) return -1;
+    const float invT = 1.0f / temperature;
+    const int V = q->V, NN = N + 1;
+    double *x = (double *)malloc(sizeof(double) * V);
+    elem_key *ek = (elem_key *)malloc(sizeof(elem_key) * (size_t)P);
+    if (!x || !ek) return -3;
+    for (int b = 0; b < q->B; ++b) {
+        const int32_t *off = child_off + (int64_t)b * (NN + 1), *ids = child_ids + (int64_t)b * N;
+        const int bid = batch_of(batch_ids, b);
+        token[(int64_t)b * NN] = -1;
+        for (int u = 0; u < NN; ++u) {
+            if (exempt_node) exempt_node[(int64_t)b * NN + u] = 0;
+            const int m = off[u + 1] - off[u];
+            if (m == 0) continue;
+            const int d = depth[(int64_t)b * NN + u];
+            const int r = replay_row_index(qrow_of_node, depth, (int64_t)b * NN + u);
+            if (m > P || d < 0 || d >= Lp || r < 0 || r >= q->R) return -5;
+            read_row(q, b, r, invT, x);
+            const int32_t *pool = pool_ids + ((int64_t)b * Lp + d) * P;
+            for (int j = 0; j < P; ++j) {
+                const int v = pool[j];
+                if (v < 0 || v >= V) return -6;
+                const double uv = orc_uniform(seed, PURPOSE_REPLAY_ELEM, bid, u, v);
+                ek[j].k = x[v] + gumbel_of(uv);
+                ek[j].v = v;
+                ek[j].sens = gumbel_slope(uv);
+            }
+            partial_sort(ek, P, m + 1 < P ? m + 1 : P);
+            uint8_t ex = 0;
+            for (int j = 0; j < m; ++j) {
+                if (j + 1 < P && near_tie(&ek[j], &ek[j + 1])) ex = 1;
+                token[(int64_t)b * NN + ids[off[u] + j]] = ek[j].v;
+            }
+            if (exempt_node) exempt_node[(int64_t)b * NN + u] = ex;
+        }
+    }
+    free(x); free(ek);
     return 0;
 }
