@@ -71,6 +71,7 @@ typedef enum {
 
 /* Limits (validated). */
 #define TSB_MAX_WIDTH 1024              /* frontier width of the expand-then-prune first pass */
+#define TSB_MAX_POOL 32                 /* tokens in a pooled draft law (one warp) */
 #define TSB_MAX_EXPAND_CANDIDATES 8192  /* candidates it may generate: K + (L-1) layers of <= W*K */
 #define TSB_CHUNK 256 /* fixed chunk of the chunk statistics and of the replay sampler */
 #define TSB_MAX_K 32
@@ -181,6 +182,35 @@ tsb_status tsb_plan_expand(const tsb_cfg *cfg, int32_t width, const tsb_logits *
 tsb_status tsb_plan_rows_expand(const tsb_cfg *cfg, int32_t width, const tsb_logits *draft, void *draft_stats,
                                 size_t stats_bytes, const tsb_tree *out, void *ws, size_t ws_bytes,
                                 tsb_stream stream);
+
+/* Pooled draft laws (Sec. 3.1: the draft law of a position is restricted to a pool of its P
+ * most probable tokens and normalised within it; Sec. 3.2: replay uses the same pools; Sec. 3.3:
+ * verification uses the pooled probabilities, the target law and the residual stay
+ * full-vocabulary). The pool of the tokens at depth d+1 is the P most probable tokens of draft
+ * row d by (x desc, id asc); it serves every node at depth d, whatever its q row.
+ *
+ * tsb_plan_pooled: tsb_plan with each depth's law normalised over its pool; the candidates are
+ *   the pool's first K tokens (K <= P <= TSB_MAX_POOL, P <= V, else TSB_ERR_SHAPE). Writes the
+ *   pools to pool_ids (device, caller-owned, [B, L, P] int32, sorted by (x desc, id asc)) and
+ *   *out as tsb_plan does. draft_stats: tsb_row_stats of the draft rows.
+ * tsb_replay_pooled: for every parent u with m_u children, the m_u ordered draws without
+ *   replacement from q_u restricted to pool row depth[u] and renormalised there: the top-m_u
+ *   Gumbel keys x_v + G(U[replay element, u, v]) over the P pool tokens. qrows / qrow_of_node
+ *   as in tsb_replay (no statistics needed).
+ * tsb_verify_pooled: recursive rejection sampling as tsb_verify's TSB_VERIFY_RRS with q_u the
+ *   pooled law; a child token outside the pool has draft probability 0 and is accepted.
+ * Other arguments, layouts and errors as in tsb_plan / tsb_replay / tsb_verify; a pool token
+ * out of range sets TSB_DEV_BAD_INDEX. */
+tsb_status tsb_plan_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *draft, const void *draft_stats,
+                           size_t stats_bytes, int32_t *pool_ids, const tsb_tree *out, void *ws, size_t ws_bytes,
+                           tsb_stream stream);
+tsb_status tsb_replay_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *qrows, const int32_t *qrow_of_node,
+                             const int32_t *pool_ids, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
+                             size_t ws_bytes, tsb_stream stream);
+tsb_status tsb_verify_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *target, const tsb_logits *qrows,
+                             const int32_t *qrow_of_node, const int32_t *pool_ids, const tsb_tree *tree,
+                             const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
+                             int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream);
 
 /* Size of the device scratch array behind tsb_plan_noalloc (1 MiB per device). */
 #define TSB_NOALLOC_SCRATCH_BYTES ((size_t)1 << 20)

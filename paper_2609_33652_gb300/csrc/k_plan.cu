@@ -198,7 +198,7 @@ __device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st, ui
             const int rk = rank_among(cand, n2, v);
             if (rk < K) {
                 a.topk_id[(int64_t)row * K + rk] = (int32_t)key_id(v);
-                a.topk_x[(int64_t)row * K + rk] = key_value(v);
+                if (a.topk_x) a.topk_x[(int64_t)row * K + rk] = key_value(v);
             }
         }
         return;
@@ -214,7 +214,7 @@ __device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st, ui
             const uint64_t best = warp_pop_max(t);
             if (lane == 0) {
                 a.topk_id[(int64_t)row * K + j] = (int32_t)key_id(best);
-                a.topk_x[(int64_t)row * K + j] = key_value(best);
+                if (a.topk_x) a.topk_x[(int64_t)row * K + j] = key_value(best);
             }
         }
     }
@@ -948,6 +948,27 @@ cudaError_t launch_plan_expand(const RowsDesc &draft, const float2 *stats, float
     ea.tree = tree;
     ea.status = static_cast<uint32_t *>(ws);
     return launch_ept(ea, draft.B, s);
+}
+
+// Pooled first pass: the per-row top-P pass writes the pools (ids only) to pool_ids, then
+// k_pool_finish turns each pool into the pooled log-normaliser and the K candidates, then the
+// max-heap expansion as in launch_plan.
+cudaError_t launch_plan_pooled(const RowsDesc &draft, const float2 *stats, int L, int N, int K, int P, float invT,
+                               int32_t *pool_ids, const TreeDesc &tree, void *ws, cudaStream_t s) {
+    const PlanScratch sc = plan_scratch(ws, draft.B, N, L, K);
+    TopkArgs t = topk_args(draft, stats, L, P, invT, sc);
+    t.topk_id = pool_ids;
+    t.topk_x = nullptr;
+    cudaError_t e;
+    if (draft.dtype == 1)
+        e = P <= 8 ? launch_topk_t<8, __nv_bfloat16>(t, s) : launch_topk_t<32, __nv_bfloat16>(t, s);
+    else
+        e = P <= 8 ? launch_topk_t<8, float>(t, s) : launch_topk_t<32, float>(t, s);
+    if (e != cudaSuccess) return e;
+    e = launch_pool_finish(draft, L, K, P, invT, pool_ids, sc.lse, sc.topk_x, sc.topk_id, static_cast<uint32_t *>(ws),
+                           s);
+    if (e != cudaSuccess) return e;
+    return launch_heap(heap_args(L, N, K, sc, tree, static_cast<uint32_t *>(ws)), draft.B, s);
 }
 
 }  // namespace tsb

@@ -116,6 +116,12 @@ tsb_status plan_expand_common(const tsb_cfg *cfg, int32_t width, const tsb_logit
                                                (cudaStream_t)stream));
 }
 
+// pooled draft laws: K <= P <= TSB_MAX_POOL, P <= V
+tsb_status check_pool(const tsb_cfg *c, int32_t P) {
+    if (P < c->K || P > TSB_MAX_POOL || P > c->V) return TSB_ERR_SHAPE;
+    return TSB_OK;
+}
+
 tsb_status replay_common(bool mixed, const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats,
                          size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed,
                          int32_t *token, void *ws, size_t ws_bytes, tsb_stream stream) {
@@ -148,6 +154,60 @@ tsb_status tsb_plan_rows_expand(const tsb_cfg *cfg, int32_t width, const tsb_log
                                 tsb_stream stream) {
     if (!draft_stats) return TSB_ERR_ARG;
     return plan_expand_common(cfg, width, draft, nullptr, draft_stats, stats_bytes, out, ws, ws_bytes, stream);
+}
+
+tsb_status tsb_plan_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *draft, const void *draft_stats,
+                           size_t stats_bytes, int32_t *pool_ids, const tsb_tree *out, void *ws, size_t ws_bytes,
+                           tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st == TSB_OK) st = check_pool(cfg, P);
+    if (st != TSB_OK) return st;
+    st = check_logits(draft, cfg->B, cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_stats(draft_stats, stats_bytes, cfg->B, draft->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!pool_ids || !out || !out->parent || !out->depth || !out->rank || !out->plan_token || !out->score ||
+        !out->child_off || !out->child_ids)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_plan_pooled(rows_of(draft), static_cast<const float2 *>(draft_stats), cfg->L,
+                                               cfg->N, cfg->K, P, inv_temperature(cfg->temperature), pool_ids,
+                                               tree_of(out), ws, (cudaStream_t)stream));
+}
+
+tsb_status tsb_replay_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *qrows, const int32_t *qrow_of_node,
+                             const int32_t *pool_ids, const tsb_tree *tree, uint64_t seed, int32_t *token, void *ws,
+                             size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st == TSB_OK) st = check_pool(cfg, P);
+    if (st != TSB_OK) return st;
+    st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!pool_ids || !tree || !tree->child_off || !tree->child_ids || !tree->depth || !token) return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_replay_pooled(rows_of(qrows), qrow_of_node, cfg->B, cfg->N, cfg->L, P,
+                                                 tree_of(tree), pool_ids, inv_temperature(cfg->temperature), seed,
+                                                 token, static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+}
+
+tsb_status tsb_verify_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *target, const tsb_logits *qrows,
+                             const int32_t *qrow_of_node, const int32_t *pool_ids, const tsb_tree *tree,
+                             const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
+                             int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st == TSB_OK) st = check_pool(cfg, P);
+    if (st != TSB_OK) return st;
+    st = check_logits(target, cfg->B, cfg->N + 1, cfg->V);
+    if (st == TSB_OK) st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
+    if (st == TSB_OK && target->dtype != qrows->dtype) st = TSB_ERR_DTYPE;
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!pool_ids || !tree || !tree->child_off || !tree->child_ids || !tree->depth || !token || !out_tokens ||
+        !out_nodes || !out_len)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_verify_pooled(rows_of(target), rows_of(qrows), qrow_of_node, cfg->B, cfg->N,
+                                                 cfg->L, P, tree_of(tree), pool_ids, token,
+                                                 inv_temperature(cfg->temperature), seed, out_tokens, out_nodes,
+                                                 out_len, static_cast<uint32_t *>(ws), (cudaStream_t)stream));
 }
 
 tsb_status tsb_replay_mixed(const tsb_cfg *cfg, const tsb_logits *qrows, const void *qstats, size_t stats_bytes,

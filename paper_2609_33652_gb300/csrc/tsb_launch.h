@@ -98,6 +98,18 @@ cudaError_t launch_plan_scratch(const RowsDesc &draft, const float2 *stats, int 
 cudaError_t launch_plan_expand(const RowsDesc &draft, const float2 *stats, float2 *stats_out, int L, int N, int K,
                                int W, float invT, const TreeDesc &tree, void *ws, cudaStream_t s);
 
+cudaError_t launch_plan_pooled(const RowsDesc &draft, const float2 *stats, int L, int N, int K, int P, float invT,
+                               int32_t *pool_ids, const TreeDesc &tree, void *ws, cudaStream_t s);
+cudaError_t launch_pool_finish(const RowsDesc &draft, int L, int K, int P, float invT, const int32_t *pool_ids,
+                               float2 *lse, float *topk_x, int32_t *topk_id, uint32_t *status, cudaStream_t s);
+cudaError_t launch_replay_pooled(const RowsDesc &q, const int32_t *qrow_of_node, int B, int N, int L, int P,
+                                 const TreeDesc &tree, const int32_t *pool_ids, float invT, uint64_t seed,
+                                 int32_t *token, uint32_t *status, cudaStream_t s);
+cudaError_t launch_verify_pooled(const RowsDesc &target, const RowsDesc &q, const int32_t *qrow_of_node, int B,
+                                 int N, int L, int P, const TreeDesc &tree, const int32_t *pool_ids,
+                                 const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                                 int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s);
+
 cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
                           int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token, uint32_t *status,
                           cudaStream_t s);

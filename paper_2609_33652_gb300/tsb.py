@@ -27,10 +27,12 @@ TSB_CHUNK = 256
 
 EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_bytes", "tsb_workspace_init",
            "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify", "tsb_plan_noalloc",
-           "tsb_plan_rows", "tsb_plan_expand", "tsb_plan_rows_expand", "tsb_replay_mixed")
+           "tsb_plan_rows", "tsb_plan_expand", "tsb_plan_rows_expand", "tsb_replay_mixed", "tsb_plan_pooled",
+           "tsb_replay_pooled", "tsb_verify_pooled")
 TSB_NOALLOC_SCRATCH_BYTES = 1 << 20
 TSB_MAX_WIDTH = 1024
 TSB_MAX_EXPAND_CANDIDATES = 8192
+TSB_MAX_POOL = 32
 
 
 class TsbError(RuntimeError):
@@ -88,6 +90,9 @@ def load():
         "tsb_replay_mixed": (_I32, [_P, _P, _P, _SZ, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
         "tsb_plan_expand": (_I32, [_P, _I32, _P, _P, _SZ, _P, _P, _SZ, _P]),
         "tsb_plan_rows_expand": (_I32, [_P, _I32, _P, _P, _SZ, _P, _P, _SZ, _P]),
+        "tsb_plan_pooled": (_I32, [_P, _I32, _P, _P, _SZ, _P, _P, _P, _SZ, _P]),
+        "tsb_replay_pooled": (_I32, [_P, _I32, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
+        "tsb_verify_pooled": (_I32, [_P, _I32, _P, _P, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
         "tsb_verify": (_I32, [_P, _I32, _P, _P, _P, _SZ, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
     }
     for name, (res, args) in sig.items():
@@ -209,6 +214,37 @@ def tsb_plan_rows_expand(cfg: Cfg, width: int, draft: torch.Tensor, stats: torch
     _check(load().tsb_plan_rows_expand(ctypes.byref(cfg), int(width), ctypes.byref(d), _ptr(stats),
                                        stats.numel() * stats.element_size(), ctypes.byref(t), _ptr(ws),
                                        ws.numel() * ws.element_size(), _stream(stream)), "tsb_plan_rows_expand")
+
+
+def tsb_plan_pooled(cfg: Cfg, P: int, draft: torch.Tensor, stats: torch.Tensor, pool_ids: torch.Tensor, tree: dict,
+                    ws: torch.Tensor, stream=None):
+    """First pass with pooled draft laws; writes the pools [B, L, P] int32 into ``pool_ids``."""
+    d = logits_desc(draft)
+    t = tree_struct(tree)
+    _check(load().tsb_plan_pooled(ctypes.byref(cfg), int(P), ctypes.byref(d), _ptr(stats),
+                                  stats.numel() * stats.element_size(), _ptr(pool_ids), ctypes.byref(t), _ptr(ws),
+                                  ws.numel() * ws.element_size(), _stream(stream)), "tsb_plan_pooled")
+
+
+def tsb_replay_pooled(cfg: Cfg, P: int, qrows: torch.Tensor, qrow_of_node, pool_ids: torch.Tensor, tree: dict,
+                      seed: int, token: torch.Tensor, ws: torch.Tensor, stream=None):
+    d = logits_desc(qrows)
+    t = tree_struct(tree)
+    _check(load().tsb_replay_pooled(ctypes.byref(cfg), int(P), ctypes.byref(d), _ptr(qrow_of_node), _ptr(pool_ids),
+                                    ctypes.byref(t), int(seed) & (2**64 - 1), _ptr(token), _ptr(ws),
+                                    ws.numel() * ws.element_size(), _stream(stream)), "tsb_replay_pooled")
+
+
+def tsb_verify_pooled(cfg: Cfg, P: int, target: torch.Tensor, qrows: torch.Tensor, qrow_of_node, pool_ids, tree: dict,
+                      token: torch.Tensor, seed: int, out_tokens: torch.Tensor, out_nodes: torch.Tensor,
+                      out_len: torch.Tensor, ws: torch.Tensor, stream=None):
+    dt = logits_desc(target)
+    dq = logits_desc(qrows)
+    t = tree_struct(tree)
+    _check(load().tsb_verify_pooled(ctypes.byref(cfg), int(P), ctypes.byref(dt), ctypes.byref(dq), _ptr(qrow_of_node),
+                                    _ptr(pool_ids), ctypes.byref(t), _ptr(token), int(seed) & (2**64 - 1),
+                                    _ptr(out_tokens), _ptr(out_nodes), _ptr(out_len), _ptr(ws),
+                                    ws.numel() * ws.element_size(), _stream(stream)), "tsb_verify_pooled")
 
 
 def tsb_plan_noalloc(cfg: Cfg, draft: torch.Tensor, stats: torch.Tensor, tree: dict, dev_status=None, stream=None):

@@ -188,6 +188,39 @@ def test_plan_expand_validation(lib):
         assert call(64, cfg=tsb.make_cfg(4, 16, 64, 32, 1024, 1.0), fused=fused) == SHAPE
 
 
+def test_pooled_validation(lib):
+    cfg = tsb.make_cfg(2, 4, 8, 4, 64, 1.0)
+    t = _tree()
+    d = _logits(2, 4, 64)
+
+    def plan(P, draft=d, pools=FAKE):
+        return lib.tsb_plan_pooled(ctypes.byref(cfg), P, ctypes.byref(draft), FAKE, 1 << 30, pools,
+                                   ctypes.byref(t), FAKE, 1 << 30, None)
+
+    assert plan(3) == SHAPE  # P < K
+    assert plan(tsb.TSB_MAX_POOL + 1) == SHAPE
+    assert plan(8, pools=None) == ARG
+    assert plan(8, draft=_logits(2, 3, 64)) == SHAPE
+
+    def replay(P, pools=FAKE, token=FAKE):
+        return lib.tsb_replay_pooled(ctypes.byref(cfg), P, ctypes.byref(d), None, pools, ctypes.byref(t), 1, token,
+                                     FAKE, 1 << 30, None)
+
+    assert replay(2) == SHAPE
+    assert replay(8, pools=None) == ARG
+    assert replay(8, token=None) == ARG
+
+    def verify(P, target=None, pools=FAKE):
+        tg = target if target is not None else _logits(2, 9, 64)
+        return lib.tsb_verify_pooled(ctypes.byref(cfg), P, ctypes.byref(tg), ctypes.byref(d), None, pools,
+                                     ctypes.byref(t), FAKE, 1, FAKE, FAKE, FAKE, FAKE, 1 << 30, None)
+
+    assert verify(65) == SHAPE  # P > V
+    assert verify(8, target=_logits(2, 8, 64)) == SHAPE
+    assert verify(8, target=_logits(2, 9, 64, dtype=1)) == DTYPE
+    assert verify(8, pools=None) == ARG
+
+
 def test_workspace_and_status_validation(lib):
     assert lib.tsb_workspace_init(None, 256, None) == ARG
     assert lib.tsb_workspace_init(FAKE, 100, None) == WS
