@@ -300,6 +300,67 @@ def run_planners(w, sets, device, steps=300, warmup=10, budgets=(64, 256), width
     return out
 
 
+def run_pooled(w, sets, device, steps=300, warmup=10, P=16):
+    """A step with pooled draft laws (pools of P tokens, as DFlash2's 16): tsb_row_stats +
+    tsb_plan_pooled, tsb_replay_pooled, tsb_verify_pooled, on the same inputs."""
+    import ctypes
+
+    import torch
+
+    from paper_2609_33652_gb300 import tsb
+
+    lib = tsb.load()
+    B, L, S = w["B"], w["L"], len(sets)
+    bufs = [tsb.TsbBuffers.allocate(B, L, w["N"], w["K"], w["V"], w["T"], device=device) for _ in range(S)]
+    pools = [torch.empty(B, L, P, dtype=torch.int32, device=device) for _ in range(S)]
+    s = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    keep, steps_calls = [], []
+    for k in range(steps):
+        st, bf, pl = sets[k % S], bufs[k % S], pools[k % S]
+        dd, dt, tr = tsb.logits_desc(st["draft"]), tsb.logits_desc(st["target"]), tsb.tree_struct(bf.tree)
+        keep += [dd, dt, tr]
+        sb, wb = bf.stats.numel() * 4, bf.ws.numel()
+        seed = 9_000_000 + k
+        steps_calls.append([
+            (lib.tsb_row_stats, (ctypes.byref(dd), ctypes.c_float(w["T"]), ctypes.c_void_p(bf.stats.data_ptr()), sb,
+                                 ctypes.c_void_p(bf.ws.data_ptr()), wb, s)),
+            (lib.tsb_plan_pooled, (ctypes.byref(bf.cfg), P, ctypes.byref(dd), ctypes.c_void_p(bf.stats.data_ptr()), sb,
+                                   ctypes.c_void_p(pl.data_ptr()), ctypes.byref(tr), ctypes.c_void_p(bf.ws.data_ptr()),
+                                   wb, s)),
+            (lib.tsb_replay_pooled, (ctypes.byref(bf.cfg), P, ctypes.byref(dd), None, ctypes.c_void_p(pl.data_ptr()),
+                                     ctypes.byref(tr), seed, ctypes.c_void_p(bf.token.data_ptr()),
+                                     ctypes.c_void_p(bf.ws.data_ptr()), wb, s)),
+            (lib.tsb_verify_pooled, (ctypes.byref(bf.cfg), P, ctypes.byref(dt), ctypes.byref(dd), None,
+                                     ctypes.c_void_p(pl.data_ptr()), ctypes.byref(tr),
+                                     ctypes.c_void_p(bf.token.data_ptr()), seed,
+                                     ctypes.c_void_p(bf.out_tokens.data_ptr()), ctypes.c_void_p(bf.out_nodes.data_ptr()),
+                                     ctypes.c_void_p(bf.out_len.data_ptr()), ctypes.c_void_p(bf.ws.data_ptr()), wb,
+                                     s)),
+        ])
+
+    def run(calls):
+        for fn, args in calls:
+            rc = fn(*args)
+            if rc != 0:
+                raise RuntimeError(f"pooled step failed with status {rc}")
+
+    for k in range(min(warmup, steps)):
+        run(steps_calls[k])
+    torch.cuda.synchronize()
+    t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t0.record()
+    for c in steps_calls:
+        run(c)
+    t1.record()
+    torch.cuda.synchronize()
+    for bf in bufs:
+        if tsb.tsb_device_status(bf.ws) != 0:
+            raise RuntimeError("device status bits set in the pooled step")
+    lens = torch.stack([bf.out_len for bf in bufs]).float().mean().item()
+    return {"us_per_step": round(t0.elapsed_time(t1) * 1e3 / steps, 3), "pool": P, "steps": steps,
+            "mean_emitted_len_last_steps": round(lens, 4)}
+
+
 def max_over_ranks(value: float, dist, device) -> float:
     """The largest of the ranks' values (every rank gets it): a job's time is its slowest
     replica's. ``device`` is where the process group's backend reduces (cuda for nccl)."""
@@ -415,6 +476,8 @@ def run_tsb(args):
     variants = run_variants(w, sets, device, steps=args.variant_steps) if not args.no_variants else None
     if variants is not None and not args.no_planners:
         variants["first_pass_us_per_call"] = run_planners(w, sets, device, steps=args.variant_steps)
+    if variants is not None:
+        variants["pooled16_wor_rrs"] = run_pooled(w, sets, device, steps=args.variant_steps)
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
