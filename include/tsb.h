@@ -10,8 +10,16 @@
  *   tsb_plan_rows   draft rows            -> their statistics + T, in one pass over the rows
  *   tsb_replay      q rows + stats + T    -> one fresh token per node (second pass, Sec. 3.2)
  *   tsb_verify      target rows + q rows + T + tokens -> accepted path and final token
- *                   (recursive rejection sampling, Sec. 2.3 and App. A; or block verification
- *                   of a sampled chain, Sun et al. 2025 as cited in Sec. 1 and App. A)
+ *                   (recursive rejection sampling, Sec. 2.3 and App. A; block verification
+ *                   of a sampled chain, Sun et al. 2025 as cited in Sec. 1 and App. A; or
+ *                   target-sample matching, Table 2)
+ *
+ * and the paper's other choices for each pass:
+ *
+ *   tsb_plan_expand, tsb_plan_rows_expand   expand-then-prune first pass (Sec. 3.1, App. B.3)
+ *   tsb_replay_mixed                        mixed sampling in the second pass (App. A)
+ *   tsb_plan_pooled, tsb_replay_pooled,     draft laws restricted to per-position pools of the
+ *   tsb_verify_pooled                       P most probable tokens (Sec. 3.1-3.3)
  *
  * Conventions
  *   - Every tensor pointer is a DEVICE pointer owned by the caller. The library never
