@@ -60,6 +60,7 @@ def parse():
     ap.add_argument("--no-variants", action="store_true", help="skip the other sampling / verification schemes")
     ap.add_argument("--variant-steps", type=int, default=300)
     ap.add_argument("--no-planners", action="store_true", help="skip the first-pass-only timings at N = 64 and 256")
+    ap.add_argument("--no-pooled", action="store_true", help="skip the pooled-law step")
     ap.add_argument("--workload", default="batched", choices=("batched", "batched128k"))
     args = ap.parse_args()
     if args.steps is None:
@@ -476,7 +477,7 @@ def run_tsb(args):
     variants = run_variants(w, sets, device, steps=args.variant_steps) if not args.no_variants else None
     if variants is not None and not args.no_planners:
         variants["first_pass_us_per_call"] = run_planners(w, sets, device, steps=args.variant_steps)
-    if variants is not None:
+    if variants is not None and not args.no_pooled:
         variants["pooled16_wor_rrs"] = run_pooled(w, sets, device, steps=args.variant_steps)
 
     cpu = None
