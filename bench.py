@@ -61,6 +61,10 @@ def parse():
     ap.add_argument("--variant-steps", type=int, default=300)
     ap.add_argument("--no-planners", action="store_true", help="skip the first-pass-only timings at N = 64 and 256")
     ap.add_argument("--no-pooled", action="store_true", help="skip the pooled-law step")
+    ap.add_argument("--sweep", action="store_true",
+                    help="instead of the headline step: the budget sweep at scale (B=64, V=151,936, L=16, "
+                         "N in --budgets, bf16 and fp32), one JSON line with us/step and HBM GB/s per (dtype, N)")
+    ap.add_argument("--budgets", default="16,32,64,128,256")
     ap.add_argument("--workload", default="batched", choices=("batched", "batched128k"))
     args = ap.parse_args()
     if args.steps is None:
@@ -660,10 +664,77 @@ def run_reference(args):
     del torch
 
 
+def run_sweep(args):
+    """Budget sweep at scale: B=64 trees, V=151,936, L=16, K=8, T=1, one plan + replay + verify
+    (RRS) step per batch, for each dtype and budget N; each (dtype, N) rotates two input sets and
+    is timed like the headline step (start and end events around K steps after W warm-up
+    steps). Algorithmic bytes: draft rows once + the visited target rows."""
+    import torch
+
+    from paper_2609_33652_gb300 import build as libbuild
+    from paper_2609_33652_gb300 import synth, tsb
+
+    device = torch.device("cuda", 0)
+    torch.cuda.set_device(device)
+    libbuild.build()
+    tsb.load()
+    B, V, L, K, T = 64, 151936, 16, 8, 1.0
+    peak, peak_kind = measured_peak_hbm()
+    out = {}
+    for dtype in ("bf16", "f32"):
+        es = 2 if dtype == "bf16" else 4
+        for N in [int(x) for x in args.budgets.split(",")]:
+            sets = []
+            for s_ in range(2):
+                seed = 1004 + 100 * s_
+                draft = synth.draft_logits(B, L, V, "planted", dtype, seed, device=device)
+                buf = tsb.TsbBuffers.allocate(B, L, N, K, V, T, device=device)
+                tsb.tsb_row_stats(draft, T, buf.stats, buf.ws)
+                tsb.tsb_plan(buf.cfg, draft, buf.stats, buf.tree, buf.ws)
+                target = synth.rows_from_depth(draft, buf.tree["depth"], 0.7, seed + 1)
+                sets.append((draft, target, buf))
+            torch.cuda.synchronize()
+            olen = torch.empty(args.steps, B, dtype=torch.int32, device=device)
+            prep = [tsb.PreparedStep(sets[k % 2][2], sets[k % 2][0], sets[k % 2][1], 1 + k, out_len=olen[k])
+                    for k in range(args.steps)]
+            warm = [tsb.PreparedStep(sets[k % 2][2], sets[k % 2][0], sets[k % 2][1], 500_000 + k)
+                    for k in range(args.warmup)]
+            for p_ in warm:
+                p_.run()
+            torch.cuda.synchronize()
+            t0, t1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t0.record()
+            for p_ in prep:
+                p_.run()
+            t1.record()
+            torch.cuda.synchronize()
+            for _, _, bf in sets:
+                if tsb.tsb_device_status(bf.ws) != 0:
+                    raise RuntimeError(f"device status bits set in the sweep at {dtype}, N={N}")
+            us = t0.elapsed_time(t1) * 1e3 / args.steps
+            visited = float(olen.float().sum(dim=1).mean().item())
+            nbytes = B * L * V * es + visited * V * es
+            out[f"{dtype}_N{N}"] = {"us_per_step": round(us, 3), "hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
+                                    "hbm_frac_of_measured": round(nbytes / (us * 1e-6) / 1e9 / peak, 4),
+                                    "algorithmic_bytes_per_step": round(nbytes),
+                                    "mean_emitted_len": round(float(olen.float().mean().item()), 4)}
+            del sets, prep, warm
+            torch.cuda.empty_cache()
+    print(json.dumps({"metric": "budget sweep: plan+replay+verify us/step and HBM GB/s per N", "n_gpus": 1,
+                      "steps": args.steps, "warmup": args.warmup, "higher_is_better": False,
+                      "config": {"workload": "budget sweep at scale: B=64, V=151936, L=16, K=8, T=1.0, depth cap 16, "
+                                             "target = depth row + N(0,0.7^2)", "B": B, "V": V, "L": L, "K": K,
+                                 "l2": "two input sets rotated (every set is above the L2 size)",
+                                 "peak_source": f"{peak_kind} (MEASURED_PEAKS hbm_gbs copy)"},
+                      "data": "synthetic", "sweep": out}), flush=True)
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         run_reference(args)
+    elif args.sweep:
+        run_sweep(args)
     else:
         run_tsb(args)
 
