@@ -591,9 +591,9 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
 // exceeds Sx - Sx_f' (or reaches it when f' < f), a prefix of the depth's sorted top-K logits,
 // and its position is r plus those counts.
 // After the last layer, one warp merges the sorted layers in the global order (key desc, depth
-// asc, parent's position asc, rank asc): the N first are the nodes, numbered in that order. Keys are the 64-bit fixed-point path
-// sums of the max-heap planner, so same-depth comparisons are exact and a frontier holding N
-// candidates gives the heap's tree bit for bit.
+// asc, parent's position asc, rank asc): the N first are the nodes, numbered in that order.
+// Keys are the 64-bit fixed-point path sums of the max-heap planner, so same-depth comparisons
+// are exact and a frontier holding N candidates gives the heap's tree bit for bit.
 constexpr int kEptThreads = 512;
 constexpr int kEptSmallLayer = 512;  // layers up to this size are ranked by counting
 
