@@ -596,7 +596,7 @@ def oracle_tree_step(w, draft_h, seed):
 
     t0 = time.perf_counter()
     ref = oracle.plan(draft_h, w["T"], w["N"], w["K"], w["L"])
-    tok, _ = oracle.replay(draft_h, w["T"], ref, seed)
+    tok, rex = oracle.replay(draft_h, w["T"], ref, seed)
     t1 = time.perf_counter()
     dt = torch.from_numpy(draft_h.view(np.int16)).view(torch.bfloat16) if draft_h.dtype == np.uint16 else \
         torch.from_numpy(draft_h)
@@ -604,7 +604,12 @@ def oracle_tree_step(w, draft_h, seed):
     t2 = time.perf_counter()
     out = oracle.verify_rrs(target, draft_h, w["T"], ref, tok, seed, w["L"])
     t3 = time.perf_counter()
-    return (t1 - t0) + (t3 - t2), out
+    # decisions the oracle flags as near ties (where a GPU result may differ, reading of the
+    # 1e-6 band): planner pops per tree, Gumbel selections per parent, walk decisions per tree
+    parents = int((np.diff(ref["child_off"], axis=1) > 0).sum())
+    flags = {"trees": int(draft_h.shape[0]), "plan": int(ref["exempt"].sum()), "replay_parents": parents,
+             "replay_flagged": int(rex.sum()), "verify": int(out["exempt"].sum())}
+    return (t1 - t0) + (t3 - t2), out, flags
 
 
 def cpu_baseline(w, sets, seconds=12.0):
@@ -613,19 +618,23 @@ def cpu_baseline(w, sets, seconds=12.0):
 
     oracle.build()
     times = []
+    flags = {"trees": 0, "plan": 0, "replay_parents": 0, "replay_flagged": 0, "verify": 0}
     k = 0
     t_start = time.perf_counter()
     while time.perf_counter() - t_start < seconds or k < 1:
         st = sets[k % len(sets)]
         b = k % w["B"]
         h = synth.to_host(st["draft"][b:b + 1])
-        t, _ = oracle_tree_step(w, h, 100 + k)
+        t, _, f = oracle_tree_step(w, h, 100 + k)
         times.append(t)
+        for key in flags:
+            flags[key] += f[key]
         k += 1
     per_tree = statistics.mean(times)
     return {"value": round(per_tree * w["B"] * 1e6, 1), "unit": "us/step", "cores": 1, "kind": "oracle",
             "sample": f"{k} single trees of the workload (plan + replay + verify, one thread), "
-                      f"mean per tree x B={w['B']}"}
+                      f"mean per tree x B={w['B']}",
+            "near_tie_flags": flags}
 
 
 def run_reference(args):
