@@ -37,6 +37,23 @@ def test_exports_every_declared_function(lib):
         assert hasattr(lib, n), n
 
 
+def test_header_is_plain_c(tmp_path):
+    """include/tsb.h is a C header: it compiles as strict C99 (and as C++) on its own."""
+    import shutil
+    import subprocess
+
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    src = tmp_path / "use_tsb.c"
+    src.write_text('#include "tsb.h"\nint main(void) { return (int)tsb_version(); }\n')
+    inc = os.path.join(ROOT, "include")
+    for cmd in ([gcc, "-std=c99", "-Wall", "-Wextra", "-pedantic", "-Werror", "-fsyntax-only", "-I", inc, str(src)],
+                [gcc, "-x", "c++", "-std=c++17", "-Wall", "-Werror", "-fsyntax-only", "-I", inc, str(src)]):
+        r = subprocess.run(cmd, capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr
+
+
 def test_host_queries(lib):
     assert tsb.tsb_version() >= 100
     for s in range(8):
