@@ -54,6 +54,45 @@ def test_header_is_plain_c(tmp_path):
         assert r.returncode == 0, r.stderr
 
 
+def test_c_program_links_and_validates(tmp_path, lib):
+    """A plain C program linked against libtsb.so (no Python, no torch) queries sizes and gets
+    host-validation errors back; nothing reaches a GPU."""
+    import shutil
+    import subprocess
+
+    gcc = shutil.which("gcc")
+    if gcc is None:
+        pytest.skip("no gcc")
+    libdir = os.path.dirname(tsb.library_path())
+    src = tmp_path / "abi.c"
+    src.write_text(r"""
+#include <stdio.h>
+#include "tsb.h"
+int main(void) {
+    tsb_cfg cfg = {16, 16, 64, 8, 151936, 1.0f};
+    size_t ws = tsb_workspace_bytes(&cfg);
+    if (ws != 256 + 16 * 65 * 32 + 16 * 16 * (8 + 8 * 8)) return 1;
+    if (tsb_stats_bytes(16, 16, 151936) != (size_t)16 * 16 * 594 * 8) return 2;
+    tsb_cfg bad = cfg;
+    bad.temperature = 0.0f;
+    if (tsb_workspace_bytes(&bad) != 0) return 3;
+    if (tsb_plan(&bad, 0, 0, 0, 0, 0, 0, 0) != TSB_ERR_ARG) return 4;
+    if (tsb_replay_mixed(0, 0, 0, 0, 0, 0, 1, 0, 0, 0, 0) != TSB_ERR_ARG) return 5;
+    printf("%s\n", tsb_status_str(TSB_ERR_SHAPE));
+    return 0;
+}
+""")
+    exe = tmp_path / "abi"
+    r = subprocess.run([gcc, "-std=c99", "-I", os.path.join(ROOT, "include"), str(src), "-L", libdir, "-ltsb",
+                        f"-Wl,-rpath,{libdir}", "-o", str(exe)], capture_output=True, text=True)
+    if r.returncode != 0 and "cannot find -ltsb" in r.stderr:
+        pytest.skip("libtsb.so not linkable here")
+    assert r.returncode == 0, r.stderr
+    r = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert r.returncode == 0, (r.returncode, r.stderr)
+    assert r.stdout.strip() == "shape out of range or inconsistent"
+
+
 def test_host_queries(lib):
     assert tsb.tsb_version() >= 100
     for s in range(8):
