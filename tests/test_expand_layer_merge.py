@@ -15,7 +15,7 @@ def _layer_merge_plan(topk_x, lse, K, L, N, W):
     """topk_x [L, K] (sorted desc), lse [L]; returns node list of (depth, parent position, rank)
     in node order, and the layers."""
     fx = _fixed(topk_x)
-    CL = np.concatenate([[0], np.cumsum(_fixed(lse))])  # the GPU rounds each prefix once
+    CL = np.concatenate([[0], _fixed(np.cumsum(lse.astype(np.float64)))])  # each prefix rounded once
     layers = []  # per depth: list of (key, f, r) sorted
     cur = [(int(fx[0, r] - CL[1]), 0, r) for r in range(K)]
     layers.append(cur)
