@@ -12,7 +12,8 @@ across every tree.
 
 Parity status of each function (what pins it, see tests/test_oracle_*.py):
   philox / uniform : published Philox4x32-10 known-answer vectors.
-  row_stats        : scipy logsumexp, numpy stable sort.
+  row_stats        : numpy max, scipy logsumexp on numpy slices (row and every chunk),
+                     numpy lexsort for the top-K (tests/test_oracle_row_stats.py).
   plan             : brute-force enumeration of every path + exact same-depth order;
                      exhaustive search for the maximum-probability prefix-closed set.
   replay           : chi-square against the closed-form ordered WoR law (flat and
@@ -20,6 +21,10 @@ Parity status of each function (what pins it, see tests/test_oracle_*.py):
   verify_rrs       : exact enumeration of the emitted-token law over all ordered child
                      tuples (= target law, Prop. 1); closed-form single-child acceptance
                      (Eq. rs-overlap); chi-square of the sampled path against the target.
+  verify_traversal : exact enumeration of the extended output law on several topologies
+                     (= target law); a chain gives block verification's law and a star
+                     gives recursive rejection sampling's; the sampler against the exact
+                     law (chi-square); sampled paths with path-keyed targets.
   verify_block     : exact enumeration of the extended output law (= target law);
                      gamma = 1 reduces to rejection sampling; E[tau] >= token-wise RS.
   plan_expand      : equals the heap planner once the frontier holds N; brute-force
@@ -51,6 +56,12 @@ _LIB_PATH = os.path.join(_HERE, "liboracle.so")
 _lib = None
 
 CHUNK = 256
+
+# Bound on another implementation's error in one draft row's log-normaliser (absolute, nats).
+# The planner's near-tie flag for a pop between candidates at depths da and db is
+# PLAN_LSE_ERR * |da - db| + 2^-30 * (da + db + 2) (see plan_band in tsb_oracle.c); the GPU
+# test test_gpu_accuracy.py holds the CUDA path's log-normalisers to this bound.
+PLAN_LSE_ERR = 2e-6
 (PURPOSE_REPLAY_CHUNK, PURPOSE_REPLAY_ELEM, PURPOSE_ACCEPT, PURPOSE_FINAL, PURPOSE_BLOCK_ETA,
  PURPOSE_FINAL_CHUNK) = 0, 1, 2, 3, 4, 5
 
@@ -109,6 +120,9 @@ def _load():
                                        _I, _P, _P, _P, _P]),
         "orc_verify_block": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P,
                                   _P, _P, _P]),
+        "orc_verify_traversal": (_I, [_P, _P, ctypes.c_float, _P, _I, _I, _P, _P, _P, _P, _P, ctypes.c_uint64, _P,
+                                      _P, _P, _P, _P]),
+        "orc_traversal_law": (_I, [_I, _I, _P, _P, _P, _P, _P, _P, _P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -179,7 +193,8 @@ def row_stats(rows: np.ndarray, temperature: float, K: int = 1):
             "topk_x": tx.reshape(B, R, K), "chunk_lse": clse.reshape(B, R, C)}
 
 
-def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps: float = 1e-6, pool: int = 0):
+def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, lse_err: float = PLAN_LSE_ERR,
+         pool: int = 0):
     """First pass; ``pool`` = P > 0 normalises each depth's law over its P most probable tokens."""
     lib = _load()
     B = draft.shape[0]
@@ -194,11 +209,11 @@ def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps:
     if pool:
         rc = lib.orc_plan_pooled(ctypes.byref(d), temperature, N, K, L, int(pool), _ptr(out["parent"]),
                                  _ptr(out["depth"]), _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score),
-                                 _ptr(child_off), _ptr(child_ids), key_eps, _ptr(exempt), _ptr(margin))
+                                 _ptr(child_off), _ptr(child_ids), lse_err, _ptr(exempt), _ptr(margin))
     else:
         rc = lib.orc_plan(ctypes.byref(d), temperature, N, K, L, _ptr(out["parent"]), _ptr(out["depth"]),
                           _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score), _ptr(child_off), _ptr(child_ids),
-                          key_eps, _ptr(exempt), _ptr(margin))
+                          lse_err, _ptr(exempt), _ptr(margin))
     _check(rc, "plan")
     tree = {k: v.reshape(B, NN) for k, v in out.items()}
     tree["score"] = score.reshape(B, NN)
@@ -209,7 +224,8 @@ def plan(draft: np.ndarray, temperature: float, N: int, K: int, L: int, key_eps:
     return tree
 
 
-def plan_expand(draft: np.ndarray, temperature: float, N: int, K: int, L: int, W: int, key_eps: float = 1e-6):
+def plan_expand(draft: np.ndarray, temperature: float, N: int, K: int, L: int, W: int,
+                lse_err: float = PLAN_LSE_ERR):
     """Expand-then-prune first pass with frontier width W; same outputs as ``plan``."""
     lib = _load()
     B = draft.shape[0]
@@ -222,7 +238,7 @@ def plan_expand(draft: np.ndarray, temperature: float, N: int, K: int, L: int, W
     exempt = np.zeros(B, dtype=np.uint8)
     _check(lib.orc_plan_expand(ctypes.byref(d), temperature, N, K, L, W, _ptr(out["parent"]), _ptr(out["depth"]),
                                _ptr(out["rank"]), _ptr(out["plan_token"]), _ptr(score), _ptr(child_off),
-                               _ptr(child_ids), key_eps, _ptr(exempt)), "plan_expand")
+                               _ptr(child_ids), lse_err, _ptr(exempt)), "plan_expand")
     tree = {k: v.reshape(B, NN) for k, v in out.items()}
     tree["score"] = score.reshape(B, NN)
     tree["child_off"] = child_off.reshape(B, NN + 1)
@@ -365,6 +381,46 @@ def verify_block(target: np.ndarray, q: np.ndarray, temperature: float, tree, to
                                 _ptr(olen), _ptr(ex), _ptr(tau)), "verify_block")
     return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool),
             "tau": tau}
+
+
+def verify_traversal(target: np.ndarray, q: np.ndarray, temperature: float, tree, token, seed: int, L: int,
+                     qrow_of_node=None, batch_ids=None):
+    """Traversal verification (sequence-level recursive rejection sampling); outputs as
+    ``verify_rrs``."""
+    lib = _load()
+    bids = _i32(batch_ids)
+    B = target.shape[0]
+    NN = tree["depth"].shape[1]
+    dt, keep_t = _logits(target)
+    dq, keep_q = _logits(q)
+    depth, off, ids = _tree_ptrs(tree)
+    parent = _i32(tree["parent"])
+    tok = _i32(token)
+    qr = _i32(qrow_of_node)
+    otok = np.zeros(B * (L + 1), dtype=np.int32)
+    onode = np.zeros(B * L, dtype=np.int32)
+    olen = np.zeros(B, dtype=np.int32)
+    ex = np.zeros(B, dtype=np.uint8)
+    _check(lib.orc_verify_traversal(ctypes.byref(dt), ctypes.byref(dq), temperature, _ptr(qr), NN - 1, L,
+                                    _ptr(parent), _ptr(depth), _ptr(off), _ptr(ids), _ptr(tok), int(seed), _ptr(bids),
+                                    _ptr(otok), _ptr(onode), _ptr(olen), _ptr(ex)), "verify_traversal")
+    return {"tokens": otok.reshape(B, L + 1), "nodes": onode.reshape(B, L), "len": olen, "exempt": ex.astype(bool)}
+
+
+def traversal_law(child_off, child_ids, token, P_rows, Q_rows):
+    """Exact law of traversal verification on one tree: (acc[NN], final_law[NN, V], degenerate)."""
+    lib = _load()
+    P_rows = np.ascontiguousarray(P_rows, dtype=np.float64)
+    Q_rows = np.ascontiguousarray(Q_rows, dtype=np.float64)
+    NN, V = P_rows.shape
+    off, ids, tok = _i32(child_off), _i32(child_ids), _i32(token)
+    acc = np.zeros(NN)
+    law = np.zeros(NN * V)
+    deg = lib.orc_traversal_law(NN, V, _ptr(off), _ptr(ids), _ptr(tok), _ptr(P_rows), _ptr(Q_rows), _ptr(acc),
+                                _ptr(law))
+    if deg < 0:
+        raise RuntimeError(f"oracle traversal_law failed with code {deg}")
+    return acc, law.reshape(NN, V), bool(deg)
 
 
 def rrs_node_law(P, Q, y):

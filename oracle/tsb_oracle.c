@@ -36,10 +36,25 @@ enum {
 
 /* Near ties. A decision taken from floating point is flagged when a uniform that decides it
  * lies within U_BAND of the value that would flip it (the parity contract's 1e-6 band), or
- * when the compared keys differ by less than KEY_BAND relative (fp32 key rounding on the
- * device side, a few ulp). */
+ * when the compared keys differ by less than KEY_BAND times max(1, |key|): an fp32 Gumbel key
+ * x + G(U) is formed with at most four roundings at its own magnitude (two logarithms of
+ * relative error <= 2^-24 each, the sum, and the shift to the chunk maximum), so a correct
+ * fp32 implementation is within 4 * 2^-24 = 2^-22 of it, relative.
+ *
+ * Planner pops: a candidate's key is Sx - CL[d] (Sx the path's sum of logits, CL[d] the sum of
+ * the first d draft rows' log-normalisers). Another implementation that holds Sx exactly and
+ * each row's log-normaliser within lse_err, rounding CL[d] and the logits onto a 2^-30 grid,
+ * can swap two candidates at depths da and db only when their keys differ by less than
+ *     lse_err * |da - db| + 2^-30 * (da + db + 2)
+ * (the rows da and db share contribute to both keys alike); plan_band() is that bound. */
 static const double U_BAND = 1e-6;
-static const double KEY_BAND = 1e-6;
+static const double KEY_BAND = 2.384185791015625e-07; /* 2^-22 */
+static const double FIX_GRID = 9.313225746154785e-10; /* 2^-30 */
+
+static double plan_band(int da, int db, double lse_err)
+{
+    return lse_err * (double)(da > db ? da - db : db - da) + FIX_GRID * (double)(da + db + 2);
+}
 
 /* ------------------------------------------------------------------------------------ */
 /* Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy as 1, 2, 3",
@@ -237,7 +252,7 @@ static int64_t max_nodes(int K, int L)
  * whose K most probable tokens are the candidates.                                        */
 static int plan_impl(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L, int32_t pool,
                      int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
-                     int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+                     int32_t *child_off, int32_t *child_ids, double lse_err, uint8_t *exempt, double *min_margin)
 {
     if (!draft || N < 1 || K < 1 || L < 1 || K > 64 || K > draft->V || draft->R < L) return -1;
     if (pool != 0 && (pool < K || pool > draft->V)) return -1;
@@ -290,16 +305,16 @@ static int plan_impl(const orc_logits *draft, float temperature, int32_t N, int3
             int best = 0;
             for (int f = 1; f < nf; ++f)
                 if (cand_before(&front[f], &front[best])) best = f;
-            /* Near-tie check. Keys of different depths depend on the log-normalisers, which
-             * another implementation rounds differently; same-depth keys with different Sx can
-             * only tie through the rounding of Sx - CL[d]. Same-depth candidates with equal Sx
-             * tie exactly everywhere and are not near ties. */
+            /* Near-tie check (plan_band). Keys of different depths depend on the
+             * log-normalisers, which another implementation computes with some error; same-depth
+             * keys differ only through their exact sums of logits. Same-depth candidates with
+             * equal Sx tie exactly everywhere and are not near ties. */
             for (int f = 0; f < nf; ++f) {
                 if (f == best) continue;
                 if (front[f].depth == front[best].depth && front[f].sx == front[best].sx) continue;
                 double margin = front[best].key - front[f].key;
                 if (front[f].depth != front[best].depth && margin < mm) mm = margin;
-                if (margin < key_eps * (1.0 + fabs(front[best].key))) ex = 1;
+                if (margin < plan_band(front[f].depth, front[best].depth, lse_err)) ex = 1;
             }
             cand c = front[best];
             front[best] = front[--nf];
@@ -345,21 +360,21 @@ static int plan_impl(const orc_logits *draft, float temperature, int32_t N, int3
 
 int orc_plan(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L,
              int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
-             int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+             int32_t *child_off, int32_t *child_ids, double lse_err, uint8_t *exempt, double *min_margin)
 {
     return plan_impl(draft, temperature, N, K, L, 0, parent, depth, rank, plan_token, score, child_off, child_ids,
-                     key_eps, exempt, min_margin);
+                     lse_err, exempt, min_margin);
 }
 
 /* First pass with pooled draft laws (Sec. 3.1, App. B.7): as orc_plan, with each depth's law
  * normalised over its P most probable tokens. */
 int orc_plan_pooled(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L, int32_t P,
                     int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
-                    int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt, double *min_margin)
+                    int32_t *child_off, int32_t *child_ids, double lse_err, uint8_t *exempt, double *min_margin)
 {
     if (P < 1) return -1;
     return plan_impl(draft, temperature, N, K, L, P, parent, depth, rank, plan_token, score, child_off, child_ids,
-                     key_eps, exempt, min_margin);
+                     lse_err, exempt, min_margin);
 }
 
 /* ------------------------------------------------------------------------------------ */
@@ -888,6 +903,259 @@ int orc_verify_block(const orc_logits *target, const orc_logits *q, float temper
 }
 
 /* ------------------------------------------------------------------------------------ */
+/* TRAVERSAL VERIFICATION (Weng et al. 2025, cited in Sec. 2.3, Table 2 ("RRS with
+ * sequence-level coupling", WoR candidates) and App. A; UniVer reduces to it under WoR).
+ * Recursive rejection sampling lifted from tokens to sequences: a node is accepted or
+ * rejected only after the whole subtree below it has been tried, deepest first.
+ *
+ * Every node u carries a sequence weight p_a(u), a target-side law Mb_u (initially its target
+ * row's softmax P_u) and its draft law Ms_u (Q_u with the tokens of rejected children removed
+ * and renormalised, t = the draft mass left). p_a(root) = 1. Entering child c of u (slot order)
+ *     p_a(c) = min(p_a(u) Mb_u(y_c) / Ms_u(y_c), 1),
+ * then c's children are tried first (depth first, in slot order). When every child of u has
+ * been tried and rejected (or u is a leaf), u is a leaf of the remaining tree and is accepted
+ * iff U[ACCEPT, u] < p_a(u); the root is accepted once its children are rejected. Accepting u
+ * emits the path from the root to u and a final token: the bonus from P_u if u had no
+ * children, else a draw from the last residual below. When the subtree of child c (token y) of
+ * u is rejected, u is updated (the block-verification step, for trees):
+ *     R(v) = max(p_a(u) Mb_u(v) - Ms_u(v), 0),  S = sum_v R(v),
+ *     p_a(u) <- S / (S + 1 - p_a(u)),  Mb_u <- R / S,  y leaves Ms_u.
+ * A rejected child has p_a(u) Mb_u(y) < Ms_u(y) (otherwise p_a(c) = 1 and c is accepted when
+ * tried), so R(y) = 0 before y leaves the draft law. S = 0 with p_a(u) < 1 leaves p_a(u) = 0
+ * (u and everything tried after it are rejected); S = 0 with p_a(u) = 1 cannot happen in exact
+ * arithmetic (it needs Mb_u = Ms_u, whose child is always accepted): should rounding produce
+ * it, u is accepted with its final token from its target row, as in the RRS walk.
+ * On a chain this is block verification (tau = the deepest accepted position); at the root it
+ * is the WoR recursive rejection sampling above.                                           */
+
+/* p_a of a child with token y of a node in state (pa, Mb, Q with t and drawn) */
+static double trav_weight(double pa, const double *Mb, const double *Q, double t, const uint8_t *drawn, int y)
+{
+    double qy = drawn[y] ? 0.0 : draft_ratio(Q[y], t);
+    double num = pa * Mb[y];
+    if (qy > 0.0) {
+        double r = num / qy;
+        return r < 1.0 ? r : 1.0;
+    }
+    return num > 0.0 ? 1.0 : 0.0;
+}
+
+/* The update after the subtree of the child with token y was rejected. R receives the
+ * unnormalised residual. Returns 1 in the degenerate case (no residual mass with pa = 1). */
+static int trav_reject(int V, double *pa, double *Mb, const double *Q, double *t, uint8_t *drawn, int y, double *R)
+{
+    double S = 0.0;
+    for (int v = 0; v < V; ++v) {
+        double qv = drawn[v] ? 0.0 : draft_ratio(Q[v], *t);
+        double r = *pa * Mb[v] - qv;
+        R[v] = r > 0.0 ? r : 0.0;
+        S += R[v];
+    }
+    int degenerate = 0;
+    if (S > 0.0) {
+        *pa = S / (S + 1.0 - *pa);
+        for (int v = 0; v < V; ++v) Mb[v] = R[v] / S;
+    } else if (*pa < 1.0) {
+        *pa = 0.0;
+    } else {
+        degenerate = 1;
+    }
+    drawn[y] = 1;
+    *t -= Q[y];
+    return degenerate;
+}
+
+typedef struct {
+    /* inputs of one tree */
+    const orc_logits *target, *q;
+    float invT;
+    const int32_t *qrow_of_node, *depth, *off, *ids, *token;
+    int64_t nb;
+    int b, bid, V;
+    uint64_t seed;
+    /* per stack level: Mb, Q (V doubles each), drawn (V bytes); scratch R, x */
+    double *Mb, *Q, *R, *x;
+    uint8_t *drawn;
+    int levels;
+    /* results */
+    uint8_t ex;
+    int err, accepted, final_tok;
+} trav_walk;
+
+/* Try node u (stack level lev) with sequence weight pa. Returns 1 if u or a node below it was
+ * accepted (the walk then stops), 0 if u's whole subtree was rejected. */
+static int trav_visit(trav_walk *w, int u, int lev, double pa)
+{
+    const int V = w->V;
+    if (lev >= w->levels) { w->err = -7; return 1; }
+    double *Mb = w->Mb + (int64_t)lev * V, *Q = w->Q + (int64_t)lev * V;
+    uint8_t *drawn = w->drawn + (int64_t)lev * V;
+    const int m = w->off[u + 1] - w->off[u];
+    read_row(w->target, w->b, u, w->invT, w->x);
+    softmax(w->x, V, Mb);
+    double t = 1.0;
+    int degenerate = 0, rejected_any = 0;
+    if (m > 0) {
+        const int r = replay_row_index(w->qrow_of_node, w->depth, w->nb + u);
+        if (r < 0 || r >= w->q->R) { w->err = -5; return 1; }
+        read_row(w->q, w->b, r, w->invT, w->x);
+        softmax(w->x, V, Q);
+        memset(drawn, 0, V);
+    }
+    for (int i = 0; i < m; ++i) {
+        const int c = w->ids[w->off[u] + i];
+        const int y = w->token[w->nb + c];
+        if (y < 0 || y >= V) { w->err = -6; return 1; }
+        if (trav_visit(w, c, lev + 1, trav_weight(pa, Mb, Q, t, drawn, y))) return 1;
+        rejected_any = 1;
+        if (trav_reject(V, &pa, Mb, Q, &t, drawn, y, w->R)) { degenerate = 1; break; }
+    }
+    int accept = 1;
+    if (u != 0 && !degenerate) {
+        double U = orc_uniform(w->seed, PURPOSE_ACCEPT, w->bid, u, 0);
+        if (fabs(U - pa) < U_BAND) w->ex = 1;
+        accept = U < pa;
+    }
+    if (!accept) return 0;
+    w->accepted = u;
+    if (!rejected_any || degenerate) { /* bonus token from the node's target row */
+        read_row(w->target, w->b, u, w->invT, w->x);
+        w->final_tok = sample_final(w->x, 1, V, w->seed, w->bid, u, &w->ex);
+    } else { /* from the last residual (R still holds it: nothing ran since the update) */
+        w->final_tok = sample_final(w->R, 0, V, w->seed, w->bid, u, &w->ex);
+    }
+    return 1;
+}
+
+int orc_verify_traversal(const orc_logits *target, const orc_logits *q, float temperature,
+                         const int32_t *qrow_of_node, int32_t N, int32_t L, const int32_t *parent,
+                         const int32_t *depth, const int32_t *child_off, const int32_t *child_ids,
+                         const int32_t *token, uint64_t seed, const int32_t *batch_ids, int32_t *out_tokens,
+                         int32_t *out_nodes, int32_t *out_len, uint8_t *exempt)
+{
+    if (!target || !q || N < 0 || L < 1 || !(temperature > 0.0f) || target->V != q->V || target->R < N + 1) return -1;
+    const int V = target->V, NN = N + 1, levels = L + 2;
+    trav_walk w;
+    memset(&w, 0, sizeof w);
+    w.target = target;
+    w.q = q;
+    w.invT = 1.0f / temperature;
+    w.qrow_of_node = qrow_of_node;
+    w.depth = depth;
+    w.token = token;
+    w.V = V;
+    w.seed = seed;
+    w.levels = levels;
+    w.Mb = (double *)malloc(sizeof(double) * (size_t)levels * V);
+    w.Q = (double *)malloc(sizeof(double) * (size_t)levels * V);
+    w.R = (double *)malloc(sizeof(double) * V);
+    w.x = (double *)malloc(sizeof(double) * V);
+    w.drawn = (uint8_t *)malloc((size_t)levels * V);
+    if (!w.Mb || !w.Q || !w.R || !w.x || !w.drawn) return -3;
+    int rc = 0;
+    for (int b = 0; b < target->B && rc == 0; ++b) {
+        w.b = b;
+        w.bid = batch_of(batch_ids, b);
+        w.nb = (int64_t)b * NN;
+        w.off = child_off + (int64_t)b * (NN + 1);
+        w.ids = child_ids + (int64_t)b * N;
+        w.ex = 0;
+        w.err = 0;
+        w.accepted = -1;
+        w.final_tok = -1;
+        trav_visit(&w, 0, 0, 1.0);
+        if (w.err) { rc = w.err; break; }
+        int32_t *otok = out_tokens + (int64_t)b * (L + 1), *onode = out_nodes + (int64_t)b * L;
+        for (int k = 0; k <= L; ++k) otok[k] = -1;
+        for (int k = 0; k < L; ++k) onode[k] = -1;
+        const int n = depth[w.nb + w.accepted];
+        if (n > L) { rc = -7; break; }
+        for (int a = w.accepted, k = n - 1; k >= 0; --k, a = parent[w.nb + a]) {
+            onode[k] = a;
+            otok[k] = token[w.nb + a];
+        }
+        otok[n] = w.final_tok;
+        out_len[b] = n + 1;
+        if (exempt) exempt[b] = w.ex;
+    }
+    free(w.Mb); free(w.Q); free(w.R); free(w.x); free(w.drawn);
+    return rc;
+}
+
+/* Exact law of traversal verification on one tree with explicit laws (for the enumeration
+ * pins), by the same weight and update steps as the sampler: P_rows / Q_rows [NN][V] (the
+ * target and draft law at every node), tokens [NN]. Writes acc[u] = P(u is the accepted node)
+ * and final_law[u][V] = the law of the final token when u is accepted. Returns 1 if a
+ * degenerate update was met, else 0. */
+typedef struct {
+    int V;
+    const int32_t *off, *ids, *token;
+    const double *P, *Q;
+    double *Mb, *Qs, *R;
+    uint8_t *drawn;
+    double *acc, *law;
+    int degenerate;
+} trav_law_ctx;
+
+/* Returns the probability that u's subtree is rejected, given it is entered with prob reach. */
+static double trav_law_visit(trav_law_ctx *c, int u, int lev, double pa, double reach)
+{
+    const int V = c->V;
+    double *Mb = c->Mb + (int64_t)lev * V, *Q = c->Qs + (int64_t)lev * V;
+    uint8_t *drawn = c->drawn + (int64_t)lev * V;
+    const int m = c->off[u + 1] - c->off[u];
+    memcpy(Mb, c->P + (int64_t)u * V, sizeof(double) * V);
+    memcpy(Q, c->Q + (int64_t)u * V, sizeof(double) * V);
+    memset(drawn, 0, V);
+    double t = 1.0, cont = reach;
+    int degenerate = 0, rejected_any = 0;
+    for (int i = 0; i < m; ++i) {
+        const int ch = c->ids[c->off[u] + i];
+        const int y = c->token[ch];
+        cont = trav_law_visit(c, ch, lev + 1, trav_weight(pa, Mb, Q, t, drawn, y), cont);
+        rejected_any = 1;
+        if (trav_reject(V, &pa, Mb, Q, &t, drawn, y, c->R)) { degenerate = 1; break; }
+    }
+    if (degenerate) c->degenerate = 1;
+    const double pacc = (u == 0 || degenerate) ? 1.0 : pa;
+    c->acc[u] += cont * pacc;
+    double *law = c->law + (int64_t)u * V;
+    if (!rejected_any || degenerate) {
+        memcpy(law, c->P + (int64_t)u * V, sizeof(double) * V);
+    } else {
+        double S = 0.0;
+        for (int v = 0; v < V; ++v) S += c->R[v];
+        for (int v = 0; v < V; ++v) law[v] = S > 0.0 ? c->R[v] / S : 0.0;
+    }
+    return cont * (1.0 - pacc);
+}
+
+int orc_traversal_law(int32_t NN, int32_t V, const int32_t *child_off, const int32_t *child_ids,
+                      const int32_t *token, const double *P_rows, const double *Q_rows, double *acc, double *final_law)
+{
+    trav_law_ctx c;
+    memset(&c, 0, sizeof c);
+    c.V = V;
+    c.off = child_off;
+    c.ids = child_ids;
+    c.token = token;
+    c.P = P_rows;
+    c.Q = Q_rows;
+    c.Mb = (double *)malloc(sizeof(double) * (size_t)NN * V);
+    c.Qs = (double *)malloc(sizeof(double) * (size_t)NN * V);
+    c.R = (double *)malloc(sizeof(double) * V);
+    c.drawn = (uint8_t *)malloc((size_t)NN * V);
+    c.acc = acc;
+    c.law = final_law;
+    if (!c.Mb || !c.Qs || !c.R || !c.drawn) return -3;
+    for (int u = 0; u < NN; ++u) acc[u] = 0.0;
+    memset(final_law, 0, sizeof(double) * (size_t)NN * V);
+    trav_law_visit(&c, 0, 0, 1.0, 1.0);
+    free(c.Mb); free(c.Qs); free(c.R); free(c.drawn);
+    return c.degenerate;
+}
+
+/* ------------------------------------------------------------------------------------ */
 /* PLAN, expand-then-prune (the EAGLE-2-style first pass of Sec. 3.1 and App. B.3).
  * Depth by depth, the W best candidates of the newest layer (its frontier) are expanded into
  * their K children each (a node at the depth cap L gets none). Once every layer exists, the N
@@ -920,16 +1188,16 @@ static int ept_cmp(const void *pa, const void *pb)
     return ept_before(a, b) ? -1 : (ept_before(b, a) ? 1 : 0);
 }
 
-/* adjacent entries in a sorted list whose order rounding could swap */
-static int ept_near(const ept_cand *a, const ept_cand *b, double key_eps)
+/* adjacent entries in a sorted list whose order rounding could swap (plan_band) */
+static int ept_near(const ept_cand *a, const ept_cand *b, double lse_err)
 {
     if (a->depth == b->depth && a->sx == b->sx) return 0; /* exact tie on every machine */
-    return a->key - b->key < key_eps * (1.0 + fabs(a->key));
+    return a->key - b->key < plan_band(a->depth, b->depth, lse_err);
 }
 
 int orc_plan_expand(const orc_logits *draft, float temperature, int32_t N, int32_t K, int32_t L, int32_t W,
                     int32_t *parent, int32_t *depth, int32_t *rank, int32_t *plan_token, double *score,
-                    int32_t *child_off, int32_t *child_ids, double key_eps, uint8_t *exempt)
+                    int32_t *child_off, int32_t *child_ids, double lse_err, uint8_t *exempt)
 {
     if (!draft || N < 1 || K < 1 || L < 1 || W < 1 || K > 64 || K > draft->V || draft->R < L) return -1;
     if (!(temperature > 0.0f)) return -1;
@@ -983,7 +1251,7 @@ int orc_plan_expand(const orc_logits *draft, float temperature, int32_t N, int32
                         cur[n].ppos = (int)f;
                         cur[n].rank = r;
                     }
-                if (np > W && ept_near(&par[W - 1], &par[W], key_eps)) ex = 1; /* frontier edge */
+                if (np > W && ept_near(&par[W - 1], &par[W], lse_err)) ex = 1; /* frontier edge */
             }
             for (int64_t i = 0; i < n; ++i) {
                 cur[i].depth = d;
@@ -1000,7 +1268,7 @@ int orc_plan_expand(const orc_logits *draft, float temperature, int32_t N, int32
         }
         qsort(all, (size_t)total, sizeof(ept_cand), ept_cmp);
         for (int64_t i = 0; i < N && i + 1 < total; ++i)
-            if (ept_near(&all[i], &all[i + 1], key_eps)) ex = 1; /* numbering and the budget edge */
+            if (ept_near(&all[i], &all[i + 1], lse_err)) ex = 1; /* numbering and the budget edge */
         int32_t *par = parent + (int64_t)b * NN, *dep = depth + (int64_t)b * NN;
         int32_t *rk = rank + (int64_t)b * NN, *tok = plan_token + (int64_t)b * NN;
         double *sc = score + (int64_t)b * NN;

@@ -62,6 +62,10 @@ def chi2_pvalue(counts: np.ndarray, probs: np.ndarray, min_expected: float = 20.
     """Chi-square goodness of fit; categories with small expectation are pooled."""
     counts = np.asarray(counts, dtype=np.float64)
     probs = np.asarray(probs, dtype=np.float64)
+    if (counts[probs <= 0.0] > 0).any():  # an outcome the law gives probability 0
+        return 0.0
+    keep = probs > 0.0
+    counts, probs = counts[keep], probs[keep]
     n = counts.sum()
     exp = probs * n
     big = exp >= min_expected
