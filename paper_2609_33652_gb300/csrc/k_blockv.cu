@@ -205,7 +205,6 @@ __global__ void __launch_bounds__(kThreads, 8) k_bv_rows(BvArgs a) {
     }
     const T *row = trow_ptr<T>(a, b, i);
     const uint32_t ub = (uint32_t)b, un = (uint32_t)i;
-    const float c2 = __fmul_rn(a.invT, kLog2e);
     const ChunkRange cr = chunk_range<U>(a.C, rank);
     MaxSum acc{-INFINITY, FF{0.f, 0.f}};  // normaliser of the chunks this lane keeps
     unsigned long long best = 0ull;       // best chunk key for the draw from Mb_i
@@ -228,9 +227,10 @@ __global__ void __launch_bounds__(kThreads, 8) k_bv_rows(BvArgs a) {
 #pragma unroll
             for (int e = 1; e < 8; ++e) zm = fmaxf(zm, z[e]);
             mcs[k] = __fmul_rn(warp_max(zm), a.invT);
-            const float offs = __fmul_rn(mcs[k], kLog2e);
+            const float2 offs = exp_offset(mcs[k]);
 #pragma unroll
-            for (int e = 0; e < 8; ++e) part[k] += fast_exp2(__fmaf_rn(z[e], c2, -offs));
+            for (int e = 0; e < 8; ++e) part[k] += chunk_term(z[e], a.invT, offs.x);
+            part[k] = chunk_sum_fix(part[k], offs.y);
         }
         // the U chunk sums at once; the lane holding a chunk's sum merges and keys that chunk
         const float sm = warp_multi_sum<U>(part);

@@ -63,7 +63,6 @@ __global__ void __launch_bounds__(kDrawThreads, 8) k_naive_draw(NaiveArgs a) {
     const int b = rid / NN, u = rid - (rid / NN) * NN;
     const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.bstride + (int64_t)u * a.rstride;
     const uint32_t ub = (uint32_t)b, un = (uint32_t)u;
-    const float c2 = __fmul_rn(a.invT, kLog2e);
     const int per = (a.C + kSplit - 1) / kSplit;
     const int c_lo = rank * per, c_hi = min(a.C, c_lo + per);
     const int units = c_hi > c_lo ? (c_hi - c_lo + U - 1) / U : 0;
@@ -87,9 +86,10 @@ __global__ void __launch_bounds__(kDrawThreads, 8) k_naive_draw(NaiveArgs a) {
 #pragma unroll
             for (int i = 1; i < 8; ++i) zm = fmaxf(zm, z[i]);
             mcs[k] = __fmul_rn(warp_max(zm), a.invT);
-            const float offs = __fmul_rn(mcs[k], kLog2e);
+            const float2 offs = exp_offset(mcs[k]);
 #pragma unroll
-            for (int i = 0; i < 8; ++i) part[k] += fast_exp2(__fmaf_rn(z[i], c2, -offs));
+            for (int i = 0; i < 8; ++i) part[k] += chunk_term(z[i], a.invT, offs.x);
+            part[k] = chunk_sum_fix(part[k], offs.y);
         }
         // the U chunk sums at once; the lane holding a chunk's sum keys that chunk
         const float tot = warp_multi_sum<U>(part);

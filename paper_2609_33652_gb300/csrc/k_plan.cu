@@ -262,7 +262,6 @@ __global__ void __launch_bounds__(kRowPlanThreads, KCAP <= 8 ? 2 : 1) k_row_stat
     const int C = a.C;
     const T *rp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
     float2 *gst = a.stats_out + ((int64_t)b * a.R + d) * C;
-    const float c2 = __fmul_rn(a.invT, kLog2e);
     const int units = (C + 3) / 4;  // four chunks (eight lanes each) per warp unit
     constexpr int kU = sizeof(T) == 2 ? 2 : 1;  // units in flight per warp (register budget)
     bool bad = false;
@@ -280,7 +279,7 @@ __global__ void __launch_bounds__(kRowPlanThreads, KCAP <= 8 ? 2 : 1) k_row_stat
             const int c = (u0 + e * NW) * 4 + q;
             const bool live = u0 + e * NW < units && c < C;
             float mc, sc;
-            chunk_stats8<T>(raw[e], live, a.invT, c2, &mc, &sc);
+            chunk_stats8<T>(raw[e], live, a.invT, &mc, &sc);
             if (live && g == 0) {
                 const float2 v = make_float2(mc, sc);
                 gst[c] = v;

@@ -234,7 +234,6 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
     extern __shared__ __align__(16) float2 cst[];  // [C] chunk statistics of the current target row
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
     const int b = blockIdx.x, NN = a.N + 1;
-    const float c2 = __fmul_rn(a.invT, kLog2e);
     const int32_t *off = a.child_off + (int64_t)b * (NN + 1), *ids = a.child_ids + (int64_t)b * a.N;
     int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1), *onode = a.out_nodes + (int64_t)b * a.L;
     int u = 0, nacc = 0, final_tok = -1;
@@ -260,9 +259,10 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
 #pragma unroll
                 for (int e = 1; e < 8; ++e) zm = fmaxf(zm, z[e]);
                 mcs[k] = __fmul_rn(warp_max(zm), a.invT);
-                const float offs = __fmul_rn(mcs[k], kLog2e);
+                const float2 offs = exp_offset(mcs[k]);
 #pragma unroll
-                for (int e = 0; e < 8; ++e) part[k] += fast_exp2(__fmaf_rn(z[e], c2, -offs));
+                for (int e = 0; e < 8; ++e) part[k] += chunk_term(z[e], a.invT, offs.x);
+                part[k] = chunk_sum_fix(part[k], offs.y);
             }
             const float sm = warp_multi_sum<U>(part);
             const int ch = multi_sum_index<U>(lane), c = cu + ch;

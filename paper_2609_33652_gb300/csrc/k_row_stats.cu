@@ -30,7 +30,6 @@ __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__
     pdl_begin();
     const int lane = threadIdx.x & 31, g = lane & 7, q = lane >> 3;
     const int upr = (C + kUnitChunks - 1) / kUnitChunks;  // units per row
-    const float c2 = __fmul_rn(invT, kLog2e);             // exp(x - m) = 2^(z invT log2e - m log2e)
     bool bad = false;
     const int64_t stride = (int64_t)gridDim.x * kWarps;
     for (int64_t u0 = (int64_t)blockIdx.x * kWarps + (threadIdx.x >> 5); u0 < units_total; u0 += stride * kUnits) {
@@ -58,7 +57,7 @@ __global__ void __launch_bounds__(kWarps * 32) k_row_stats(const T *__restrict__
         for (int e = 0; e < kUnits; ++e) {
             const int c = c_of[e];
             float mc, s;
-            chunk_stats8<T>(raw[e], c >= 0, invT, c2, &mc, &s);
+            chunk_stats8<T>(raw[e], c >= 0, invT, &mc, &s);
             if (c >= 0 && g == 0) {
                 stats[row_of[e] * C + c] = make_float2(mc, s);
                 bad |= !(s == s) || isinf(mc);

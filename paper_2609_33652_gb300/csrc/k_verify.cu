@@ -277,7 +277,6 @@ struct Walk {
         constexpr int kU = sizeof(T) == 2 ? 2 : 1;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int g = lane & 7, q = lane >> 3;
-        const float c2 = __fmul_rn(a.invT, kLog2e);
         const int units = (nch + 3) / 4;
         for (int u0 = warp; u0 < units; u0 += kU * kWarps) {  // uniform over the warp
             RawGroup<T> raw[kU][4];
@@ -293,7 +292,7 @@ struct Walk {
                 const int cl = (u0 + e * kWarps) * 4 + q;
                 const bool live = u0 + e * kWarps < units && cl < nch;
                 float mc, sc;
-                chunk_stats8<T>(raw[e], live, a.invT, c2, &mc, &sc);
+                chunk_stats8<T>(raw[e], live, a.invT, &mc, &sc);
                 if (live && g == 0) cst[cl] = make_float2(mc, sc);
                 if (dst && live) {
 #pragma unroll
@@ -520,7 +519,6 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     }
     const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)j * a.t_rstride;
     const int g = lane & 7, q = lane >> 3;
-    const float c2 = __fmul_rn(a.invT, kLog2e);
     const int C = a.C, units = (C + 3) / 4;
     const int ulo = half == 0 ? 0 : (units + 1) / 2, uhi = half == 0 ? (units + 1) / 2 : units;
     constexpr int kU = sizeof(T) == 2 ? 2 : 1;  // units in flight per warp (register budget)
@@ -538,7 +536,7 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
             const int c = (u0 + e * nwarps) * 4 + q;
             const bool live = u0 + e * nwarps < uhi && c < C;
             float mc, sc;
-            chunk_stats8<T>(raw[e], live, a.invT, c2, &mc, &sc);
+            chunk_stats8<T>(raw[e], live, a.invT, &mc, &sc);
             if (live && g == 0) pst[c] = make_float2(mc, sc);
         }
     }

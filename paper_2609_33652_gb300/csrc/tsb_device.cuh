@@ -545,9 +545,28 @@ __device__ __forceinline__ float fast_exp2(float x) {
 
 constexpr float kLog2e = 1.4426950408889634f;
 
+// Terms of a chunk sum s_c = sum_v e^(x_v - m_c), x_v = fp32(z_v * invT) (the contract's x,
+// one rounding). m_c log2 e is split into the head hi = fp32(m_c log2 e), which every term
+// subtracts inside one fma (x log2 e - hi, rounded once: an error relative to that small
+// exponent), and the exact remainder lo = m_c log2 e - hi, which would otherwise be an error
+// shared by every term of the chunk (up to 2^-24 |m_c log2 e|); it is applied to the sum once,
+// s * 2^-lo = s - s lo ln 2 (|lo| < 4e-6, so the omitted second-order term is below 1e-11).
+constexpr float kLn2 = 0.6931471805599453f;
+__device__ __forceinline__ float2 exp_offset(float mc) {
+    const float hi = __fmul_rn(mc, kLog2e);
+    const float lo = isfinite(hi) ? __fmaf_rn(mc, kLog2e, -hi) : 0.f;
+    return make_float2(hi, lo);
+}
+__device__ __forceinline__ float chunk_term(float z, float invT, float off_hi) {
+    return fast_exp2(__fmaf_rn(__fmul_rn(z, invT), kLog2e, -off_hi));
+}
+__device__ __forceinline__ float chunk_sum_fix(float s, float off_lo) {
+    return __fmaf_rn(s, __fmul_rn(-off_lo, kLn2), s);
+}
+
 // Statistics of one 256-logit chunk held by an 8-lane group (lane g holds logits 8g..8g+7 of
 // each 64-logit quarter, raw[k] = quarter k): the maximum m_c = fp32(max z * invT) and
-// s_c = sum 2^(z c2 - m_c log2 e) with c2 = invT log2 e, in a fixed order, then xor 4, 2, 1
+// s_c = sum e^(x - m_c) by the chunk_term form above, in a fixed order, then xor 4, 2, 1
 // inside the group. Every lane of the warp must call it (the shuffles are warp-wide); a group
 // with live == false contributes -inf / 0. Shared by the statistics kernels so that they
 // produce the same bits.
@@ -580,14 +599,14 @@ __device__ __forceinline__ float group_max32(const RawGroup<__nv_bfloat16> (&raw
 }
 
 template <typename T>
-__device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool live, float invT, float c2,
-                                             float *mc_out, float *s_out) {
+__device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool live, float invT, float *mc_out,
+                                             float *s_out) {
     float zm = live ? group_max32(raw) : -INFINITY;
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 1));
     const float mc = __fmul_rn(zm, invT);
-    const float off = __fmul_rn(mc, kLog2e);
+    const float2 off = exp_offset(mc);
     float s = 0.f;
     if (live) {
 #pragma unroll
@@ -595,8 +614,9 @@ __device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool l
             float z[8];
             raw[k].unpack(z);  // unpacked again rather than kept: fewer registers
 #pragma unroll
-            for (int i = 0; i < 8; ++i) s += fast_exp2(__fmaf_rn(z[i], c2, -off));
+            for (int i = 0; i < 8; ++i) s += chunk_term(z[i], invT, off.x);
         }
+        s = chunk_sum_fix(s, off.y);
     }
     s += __shfl_xor_sync(kFull, s, 4);
     s += __shfl_xor_sync(kFull, s, 2);
