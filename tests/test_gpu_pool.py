@@ -8,7 +8,7 @@ import torch
 
 import helpers
 import oracle
-from gpu_harness import Report, check_status, compare_plan, compare_tokens, compare_verify, host_tree
+from gpu_harness import Report, check_status, compare_plan, compare_tokens, compare_trials, compare_verify, host_tree
 from paper_2609_33652_gb300 import synth, tsb
 
 pytestmark = pytest.mark.gpu
@@ -68,13 +68,8 @@ def pooled_step(draft, L, N, K, P, T, seed, target_noise, qrows=None, qrow_of_no
     gout = {"len": buf.out_len.cpu().numpy(), "tokens": buf.out_tokens.cpu().numpy(),
             "nodes": buf.out_nodes.cpu().numpy()}
     compare_verify(gout, rout, same, rep, sel)
+    rep.check()
     return rep, buf, gout
-
-
-def _mostly_exact(rep, min_frac=0.9):
-    for stage, n in rep.compared.items():
-        if n:
-            assert rep.flagged_diff[stage] <= (1.0 - min_frac) * n, rep
 
 
 @pytest.mark.parametrize("wl,V,B,P,dtype", [("batched", 151936, 16, 16, "bf16"), ("batched", 128256, 16, 8, "bf16"),
@@ -83,7 +78,6 @@ def test_pooled_step(wl, V, B, P, dtype):
     w = synth.WORKLOADS[wl]
     draft = _draft(B, w["L"], V, "planted" if V > 100 else "normal2", dtype, 1401)
     rep, _, gout = pooled_step(draft, w["L"], w["N"], w["K"], P, w["T"], seed=29, target_noise=w["target_noise"])
-    _mostly_exact(rep, 0.98 if wl == "tiny" else 0.9)
     assert (gout["len"] >= 1).all()
 
 
@@ -101,16 +95,13 @@ def test_pooled_per_node_rows(T):
     qidx = torch.arange(w["N"] + 1, dtype=torch.int32, device=DEV).repeat(B, 1).contiguous()
     rep, _, _ = pooled_step(draft, w["L"], w["N"], w["K"], 16, T, seed=31, target_noise=w["target_noise"], qrows=qrows,
                             qrow_of_node=qidx)
-    _mostly_exact(rep, 0.9)
 
 
 def test_pooled_edges():
     # P = K (the pool is the candidate list), ragged V, fp32
     rep, _, _ = pooled_step(_draft(8, 4, 1001, "normal3", "f32", 1403), 4, 20, 4, 4, 0.8, seed=3, target_noise=0.7)
-    _mostly_exact(rep, 0.9)
     # P = V for a one-chunk vocabulary
     rep, _, _ = pooled_step(_draft(16, 3, 24, "normal2", "f32", 1404), 3, 12, 3, 24, 1.0, seed=4, target_noise=1.0)
-    _mostly_exact(rep, 0.9)
 
 
 def test_pooled_losslessness_on_gpu():
@@ -144,9 +135,4 @@ def test_pooled_losslessness_on_gpu():
     rtok, rex = oracle.replay_pooled(h_draft, T, ref, seed, ref_pools)
     rt = synth.path_keyed_rows(base, ref["parent"], ref["depth"], rtok, 1.0, seed=79)
     rout = oracle.verify_rrs(rt, h_draft, T, ref, rtok, seed, L, pool_ids=ref_pools)
-    ok = ~rex.any(axis=1)
-    assert np.array_equal(tok[ok], rtok[ok])
-    ok &= ~rout["exempt"]
-    assert ok.mean() > 0.995
-    assert np.array_equal(buf.out_len.cpu().numpy()[ok], rout["len"][ok])
-    assert np.array_equal(buf.out_tokens.cpu().numpy()[ok], rout["tokens"][ok])
+    compare_trials(buf, tok, rtok, rex, rout)

@@ -7,7 +7,7 @@ import torch
 
 import helpers
 import oracle
-from gpu_harness import Report, check_status, compare_plan, gpu_plan, run_step
+from gpu_harness import Report, check_status, compare_plan, compare_trials, gpu_plan, run_step
 from paper_2609_33652_gb300 import synth, tsb
 
 pytestmark = pytest.mark.gpu
@@ -30,10 +30,6 @@ def _draft(B, L, V, kind, dtype, seed):
     return synth.draft_logits(B, L, V, kind, dtype, seed, device=DEV)
 
 
-def _mostly_exact(rep, min_frac=0.9):
-    for stage, n in rep.compared.items():
-        if n:
-            assert rep.flagged_diff[stage] <= (1.0 - min_frac) * n, rep
 
 
 # --------------------------------------------------------------------------------------
@@ -46,7 +42,6 @@ def test_expand_step_matches_oracle(wl, V, B, width, dtype):
     draft = _draft(B, w["L"], V, "planted" if V > 100 else "normal2", dtype, 1203)
     rep, _, gout = run_step(draft, w["L"], w["N"], w["K"], w["T"], seed=7, target_noise=w["target_noise"],
                             width=width)
-    _mostly_exact(rep, 0.98 if wl == "tiny" else 0.9)
     assert (gout["len"] >= 1).all()
 
 
@@ -55,7 +50,6 @@ def test_expand_sweep_budget_256_sampled():
     draft = _draft(64, w["L"], w["V"], "planted", "bf16", 1204)
     rep, _, _ = run_step(draft, w["L"], 256, w["K"], w["T"], seed=3, target_noise=w["target_noise"], width=10,
                          trees=[0, 31, 63])
-    _mostly_exact(rep, 0.6)
 
 
 @pytest.mark.parametrize("B,L,N,K,V,kind,dtype", [
@@ -97,8 +91,8 @@ def test_expand_large_layers_and_edges():
         check_status(buf)
         ref = oracle.plan_expand(synth.to_host(draft), 1.0, N, K, L, W)
         rep = Report()
-        same = compare_plan(buf, ref, rep, list(range(B)))
-        assert sum(same.values()) >= 1 or all(ref["exempt"]), rep
+        compare_plan(buf, ref, rep, list(range(B)))
+        rep.check()
 
 
 def test_expand_rejects_bad_width():
@@ -121,7 +115,6 @@ def test_mixed_replay_naive_verify(wl, V, B):
     draft = _draft(B, w["L"], V, "planted" if V > 100 else "normal2", "bf16" if V > 100 else "f32", 1301)
     rep, _, gout = run_step(draft, w["L"], w["N"], w["K"], w["T"], seed=17, target_noise=w["target_noise"],
                             replay="mixed", mode=tsb.TSB_VERIFY_NAIVE)
-    _mostly_exact(rep, 0.98 if wl == "tiny" else 0.9)
     assert (gout["len"] >= 1).all()
 
 
@@ -134,7 +127,6 @@ def test_mixed_replay_per_node_rows_k32():
     qidx = torch.arange(N + 1, dtype=torch.int32, device=DEV).repeat(B, 1).contiguous()
     rep, _, _ = run_step(draft, L, N, K, 0.6, seed=19, target_noise=0.7, qrows=qrows, qrow_of_node=qidx,
                          replay="mixed", mode=tsb.TSB_VERIFY_NAIVE)
-    _mostly_exact(rep, 0.9)
 
 
 @pytest.mark.parametrize("wl,V,B,K", [("batched", 151936, 16, 8), ("tiny", 32, 256, 4), ("batched", 151936, 16, 1)])
@@ -145,7 +137,6 @@ def test_first_pass_tokens_naive_verify(wl, V, B, K):
     draft = _draft(B, w["L"], V, "planted" if V > 100 else "normal2", "bf16" if V > 100 else "f32", 1303)
     rep, _, _ = run_step(draft, w["L"], N, K, w["T"], seed=23, target_noise=w["target_noise"], replay="plan",
                          mode=tsb.TSB_VERIFY_NAIVE)
-    _mostly_exact(rep, 0.98 if wl == "tiny" else 0.9)
 
 
 def test_mixed_single_child_equals_wor():
@@ -187,12 +178,7 @@ def test_naive_losslessness_on_gpu():
     rtok, rex = oracle.replay_mixed(h_draft, T, ref, seed)
     rt = synth.path_keyed_rows(base, ref["parent"], ref["depth"], rtok, 1.0, seed=78)
     rout = oracle.verify_naive(rt, T, ref, rtok, seed, L)
-    ok = ~rex.any(axis=1)
-    assert np.array_equal(tok[ok], rtok[ok])
-    ok &= ~rout["exempt"]
-    assert ok.mean() > 0.995
-    assert np.array_equal(buf.out_len.cpu().numpy()[ok], rout["len"][ok])
-    assert np.array_equal(buf.out_tokens.cpu().numpy()[ok], rout["tokens"][ok])
+    compare_trials(buf, tok, rtok, rex, rout)
 
 
 def test_naive_flags_nonfinite_target():
