@@ -153,9 +153,11 @@ tsb_status tsb_row_stats(const tsb_logits *rows, float temperature, void *stats,
 
 /* First pass (Sec. 3.1, App. B.3): per draft row d the top-K tokens by (x desc, id asc),
  * then best-first (max-heap) expansion by cumulative draft path log-probability, popping N
- * nodes. Candidates pop in the order (path log-probability desc, depth asc, sum of x desc,
- * parent asc, rank asc); a node at depth d takes its token from draft row d-1; a node at
- * depth L gets no children. draft: [B, >=L, V]; draft_stats: tsb_row_stats of the same rows
+ * nodes. Candidates pop in the order (path log-probability desc, depth asc, parent asc,
+ * rank asc), where parent is the parent's node number; two candidates of the same depth
+ * compare their path log-probabilities exactly (they share the depth's log-normaliser
+ * prefix, so only their sums of x differ). A node at depth d takes its token from draft row
+ * d-1; a node at depth L gets no children. draft: [B, >=L, V]; draft_stats: tsb_row_stats of the same rows
  * and temperature. Writes every array of *out. */
 tsb_status tsb_plan(const tsb_cfg *cfg, const tsb_logits *draft, const void *draft_stats, size_t stats_bytes,
                     const tsb_tree *out, void *ws, size_t ws_bytes, tsb_stream stream);
@@ -239,9 +241,11 @@ tsb_status tsb_verify_pooled(const tsb_cfg *cfg, int32_t P, const tsb_logits *ta
  * GPU (different streams, or different host threads, without ordering between them) race
  * and give undefined outputs: order them on one stream or with events.
  *
- * Set-up: the first call on each device (with that device current) looks up the array's
- * device address and caches it; make that first call before any stream capture on the
- * device. The call allocates and frees nothing and calls no allocating library routine.
+ * Set-up: every call looks up the array's device address on the current device with
+ * cudaGetSymbolAddress (nothing is cached, so a cudaDeviceReset leaves no stale address);
+ * the first call on a device may load the library's module there, so make that first call
+ * before any stream capture on the device. The call allocates and frees nothing and calls
+ * no allocating library routine.
  *
  * dev_status: optional 4-byte aligned device word, owned by the caller, into which the
  * device status bits (TSB_DEV_*) are OR-ed; the caller clears it (it may be the status

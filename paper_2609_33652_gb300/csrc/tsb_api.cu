@@ -3,7 +3,6 @@
 #include <math.h>
 #include <stdint.h>
 
-#include <mutex>
 
 #include "../../include/tsb.h"
 #include "tsb_launch.h"
@@ -373,23 +372,17 @@ static_assert(kNoallocBytes % 256 == 0 && kNoallocBytes > kStatusBytes, "scratch
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocBytes];
 
-// In host code g_noalloc_scratch names a host-side shadow, not device memory: the device
-// address is looked up once per device and cached here.
-constexpr int kNoallocMaxDevices = 64;
-std::mutex g_noalloc_mu;
-void *g_noalloc_ptr[kNoallocMaxDevices];  // guarded by g_noalloc_mu
-
-// Device address of the scratch array on the current device (set-up on the first call there).
+// In host code g_noalloc_scratch names a host-side shadow, not device memory: its device
+// address on the current device is looked up with cudaGetSymbolAddress. The lookup is made
+// on every call rather than cached, so the address stays right after a cudaDeviceReset (which
+// unloads the module) or under another context on the same device; once the module is
+// loaded on the device the lookup is a table read in the runtime.
 tsb_status noalloc_scratch(unsigned char **out) {
     int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kNoallocMaxDevices) return TSB_ERR_CUDA;
-    std::lock_guard<std::mutex> lock(g_noalloc_mu);
-    if (!g_noalloc_ptr[dev]) {
-        void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return TSB_ERR_CUDA;
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = static_cast<unsigned char *>(g_noalloc_ptr[dev]);
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return TSB_ERR_CUDA;
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return TSB_ERR_CUDA;
+    *out = static_cast<unsigned char *>(p);
     return TSB_OK;
 }
 

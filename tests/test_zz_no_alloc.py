@@ -71,3 +71,37 @@ def test_noalloc_plan_matches_workspace_plan_twice(lib):
     assert tsb.tsb_device_status(r1.ws) == 0 and tsb.tsb_device_status(r2.ws) == 0
     _assert_same_tree(r1.tree, o1)
     _assert_same_tree(r2.tree, o2)
+
+    # the same two calls again, with the device's free memory (cudaMemGetInfo, which also
+    # sees allocations made outside torch's caching allocator) read on both sides: the
+    # module and its static array are loaded by now, so nothing may change it
+    for o in (o1, o2):
+        for v in o.values():
+            v.fill_(-7)
+    torch.cuda.synchronize()
+    free_before, _ = torch.cuda.mem_get_info(dev)
+    tsb.tsb_plan_noalloc(r1.cfg, d1, r1.stats, o1, dev_status=status)
+    tsb.tsb_plan_noalloc(r2.cfg, d2, r2.stats, o2, dev_status=None)
+    torch.cuda.synchronize()
+    free_after, _ = torch.cuda.mem_get_info(dev)
+    assert free_after == free_before
+    assert int(status.item()) == 0
+    _assert_same_tree(r1.tree, o1)
+    _assert_same_tree(r2.tree, o2)
+
+
+@pytest.mark.gpu
+def test_noalloc_plan_at_the_exact_scratch_limit(lib):
+    """The largest batch whose scratch fits (910 trees at L = 16, K = 8: 256 + 910*16*72 bytes
+    of the 1 MiB) runs, fills every tree like tsb_plan, and sets no status bit."""
+    dev = torch.device("cuda:0")
+    torch.cuda.set_device(dev)
+    B, L, N, K, V = 910, 16, 12, 8, 256
+    assert 256 + B * L * (8 + 8 * K) <= tsb.TSB_NOALLOC_SCRATCH_BYTES < 256 + (B + 1) * L * (8 + 8 * K)
+    d, r, o = _case(B, L, N, K, V, "bf16", seed=13, device=dev)
+    status = torch.zeros(1, dtype=torch.int32, device=dev)
+    tsb.tsb_plan_noalloc(r.cfg, d, r.stats, o, dev_status=status)
+    torch.cuda.synchronize()
+    assert int(status.item()) == 0
+    assert tsb.tsb_device_status(r.ws) == 0
+    _assert_same_tree(r.tree, o)
