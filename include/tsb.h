@@ -74,7 +74,8 @@ typedef enum { TSB_F32 = 0, TSB_BF16 = 1 } tsb_dtype;
 typedef enum {
     TSB_VERIFY_RRS = 0,   /* recursive rejection sampling, WoR candidates, any topology */
     TSB_VERIFY_BLOCK = 1, /* block verification; the topology must be the chain 0->1->...->N */
-    TSB_VERIFY_NAIVE = 2  /* target-sample matching: any topology, any way of filling it */
+    TSB_VERIFY_NAIVE = 2, /* target-sample matching: any topology, any way of filling it */
+    TSB_VERIFY_TRAVERSAL = 3 /* traversal verification, WoR candidates, any topology */
 } tsb_verify_mode;
 
 /* Limits (validated). */
@@ -284,6 +285,18 @@ tsb_status tsb_replay_mixed(const tsb_cfg *cfg, const tsb_logits *qrows, const v
  *   children are rejected the final token is drawn from the last residual; at a leaf the
  *   bonus token is drawn from the node's target row.
  * TSB_VERIFY_BLOCK: block verification of the chain 0->1->...->N (requires N <= L).
+ * TSB_VERIFY_TRAVERSAL: traversal verification (Sec. 2.3, Table 2 "Traversal" and App. A:
+ *   recursive rejection sampling lifted to sequences, for WoR candidates; UniVer reduces to it
+ *   under WoR). The tree is traversed depth first, children in slot order, and a node is tried
+ *   only once every child subtree below it has been rejected; it is accepted iff
+ *   U[accept, node] < p_a(node), the root always. Entering child c (token y) of u gives
+ *   p_a(c) = min(p_a(u) Mb_u(y) / Ms_u(y), 1) with p_a(root) = 1, Mb_u = softmax(target row u)
+ *   and Ms_u = q_u renormalised over tokens of u's children not yet rejected. After the subtree
+ *   of a child is rejected: R = max(p_a(u) Mb_u - Ms_u, 0), p_a(u) <- sum R / (sum R + 1 -
+ *   p_a(u)), Mb_u <- R / sum R. Accepting u emits the path to u and a final token: from the last
+ *   R if u had children, the bonus from u's target row otherwise. On a chain this is block
+ *   verification, at the root recursive rejection sampling. Every internal node's target row is
+ *   normalised (one parallel pass), so the call reads each internal node's row at least once.
  * TSB_VERIFY_NAIVE: target-sample matching (Sec. 2.3, "Naive" in Table 2): from the root, draw
  *   y from the node's target law (the two-level Gumbel-max of the bonus token); the first child
  *   carrying y is accepted and the walk continues there, otherwise y is the final token. Each

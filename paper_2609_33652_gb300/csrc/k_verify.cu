@@ -91,6 +91,7 @@ struct VerifyArgs {
     PreRow *pre;  // [B, N+1]
     int M;        // node ids below M with children are pre-computed
     int Lq;       // per-depth q rows whose normaliser the pre-pass computes (0 for per-node rows)
+    int qn;       // 1: the pre-pass computes each internal node's per-node q-row normaliser (slot u)
     int B;
 };
 
@@ -482,7 +483,105 @@ __device__ FF q_log_normaliser(const float2 *st, int C) {
 // (float-float) and whether it has one; topology (child_off [N+2], child_ids [N], token [N+1],
 // q row of node [N+1]); per child slot its parent, target logit, q logit and uniform.
 inline size_t topo_bytes(int N) {
-    return (size_t)(N + 1) * sizeof(float2) + (size_t)(6 * N + 6) * sizeof(int32_t) + (size_t)3 * N * sizeof(float);
+    return (size_t)2 * (N + 1) * sizeof(float2) + (size_t)(6 * N + 6) * sizeof(int32_t) +
+           (size_t)3 * N * sizeof(float);
+}
+
+// The tree's copy in shared memory, after the two row slices.
+struct TreeSmem {
+    FF *l2t;   // [N+1] pre-computed target normalisers (times log2 e)
+    FF *l2qn;  // [N+1] pre-computed per-node q-row normalisers (when a.qn)
+    int32_t *pre, *off, *kid, *tok, *row, *ps;
+    float *cxt, *cxq, *cu;
+};
+
+// Copy of tree b for a walk: topology, per child slot its parent, target and q logits and
+// acceptance uniform, the pre-pass results. Sets sh.cbad on inconsistent tree arrays. Every
+// thread of the CTA calls it; it ends with the CTA synchronised.
+template <typename T>
+__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
+    const int NN = a.N + 1;
+    TreeSmem ts;
+    ts.l2t = reinterpret_cast<FF *>(base);
+    ts.l2qn = ts.l2t + NN;
+    ts.pre = reinterpret_cast<int32_t *>(ts.l2qn + NN);
+    ts.off = ts.pre + NN;
+    ts.kid = ts.off + (NN + 1);
+    ts.tok = ts.kid + a.N;
+    ts.row = ts.tok + NN;
+    ts.ps = ts.row + NN;
+    ts.cxt = reinterpret_cast<float *>(ts.ps + a.N);
+    ts.cxq = ts.cxt + a.N;
+    ts.cu = ts.cxq + a.N;
+    {
+        const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+        const int32_t *kids = a.child_ids + (int64_t)b * a.N;
+        const int32_t *tok = a.token + (int64_t)b * NN;
+        const int32_t *row = per_depth ? a.depth + (int64_t)b * NN : a.qrow_of_node + (int64_t)b * NN;
+        for (int i = threadIdx.x; i <= NN; i += kThreads) ts.off[i] = __ldg(off + i);
+        for (int i = threadIdx.x; i < a.N; i += kThreads) {
+            ts.kid[i] = __ldg(kids + i);
+            ts.ps[i] = -1;
+        }
+        for (int i = threadIdx.x; i < NN; i += kThreads) {
+            ts.tok[i] = __ldg(tok + i);
+            ts.row[i] = __ldg(row + i);
+        }
+        for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
+            const float2 v = a.pre[(int64_t)b * NN + i].l2q;
+            sh.l2q[i] = FF{v.x, v.y};
+        }
+        if (threadIdx.x == 0) sh.cbad = 0;
+    }
+    __syncthreads();
+    {  // every valid internal node claims its child slots
+        bool bad_here = false;
+        for (int u = threadIdx.x; u < NN; u += kThreads) {
+            const int o = ts.off[u], m = ts.off[u + 1] - o;
+            if (m == 0) continue;
+            const int r = ts.row[u];
+            if (m < 0 || m > kMaxK || o < 0 || o + m > a.N || r < 0 || r >= a.q_R || (per_depth && r >= a.Lq)) {
+                bad_here = true;
+                continue;
+            }
+            for (int i = 0; i < m; ++i) ts.ps[o + i] = u;
+        }
+        if (bad_here) sh.cbad = 1;
+    }
+    __syncthreads();
+    for (int u = threadIdx.x; u < NN; u += kThreads) {  // the pre-computed set, as the pre-pass saw it
+        const bool p = u < a.M && ts.off[u + 1] - ts.off[u] > 0;
+        ts.pre[u] = p ? 1 : 0;
+        if (p) {
+            const float2 v = a.pre[(int64_t)b * NN + u].l2t;
+            ts.l2t[u] = FF{v.x, v.y};
+            if (a.qn) {
+                const float2 w = a.pre[(int64_t)b * NN + u].l2q;
+                ts.l2qn[u] = FF{w.x, w.y};
+            }
+        }
+    }
+    {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
+        bool bad_here = false;
+        for (int j = threadIdx.x; j < a.N; j += kThreads) {
+            const int u = ts.ps[j];
+            if (u < 0) continue;  // not a child slot of a valid node (never read by the walk)
+            const int c = ts.kid[j];
+            const int y = (c >= 1 && c <= a.N) ? ts.tok[c] : -1;
+            if (y < 0 || y >= a.V) {
+                bad_here = true;
+                continue;
+            }
+            const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
+            const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)ts.row[u] * a.q_rstride;
+            ts.cxt[j] = __fmul_rn(Logit<T>::load1(trow, y), a.invT);
+            ts.cxq[j] = __fmul_rn(Logit<T>::load1(qrow, y), a.invT);
+            ts.cu[j] = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
+        }
+        if (bad_here) sh.cbad = 1;
+    }
+    __syncthreads();
+    return ts;
 }
 
 // Pre-pass, in clusters of two CTAs. Clusters [0, B*M): cluster (b, j) streams target row j of
@@ -503,9 +602,17 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     const int ntarget = 2 * a.B * a.M;  // even: a cluster is all target or all q-row CTAs
     if ((int)blockIdx.x >= ntarget) {  // q-row log-normalisers, one warp each
         const int task = ((int)blockIdx.x - ntarget) * nwarps + warp;
-        if (task >= a.B * a.Lq) return;  // warp-uniform; no barrier in this branch
-        const int b = task / a.Lq, d = task - (task / a.Lq) * a.Lq;
-        const FF L2q = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + d) * a.C, a.C);
+        const int per = a.qn ? NN : a.Lq;  // per-node rows of internal nodes, or per-depth rows
+        if (task >= a.B * per) return;  // warp-uniform; no barrier in this branch
+        const int b = task / per, d = task - (task / per) * per;
+        int r = d;
+        if (a.qn) {
+            const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+            if (__ldg(off + d + 1) - __ldg(off + d) <= 0) return;  // a leaf needs no draft law
+            r = __ldg(a.qrow_of_node + (int64_t)b * NN + d);
+            if (r < 0 || r >= a.q_R) return;  // the walk flags the tree
+        }
+        const FF L2q = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
         if (lane == 0) a.pre[(int64_t)b * NN + d].l2q = make_float2(L2q.hi, L2q.lo);
         return;
     }
@@ -583,79 +690,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
 
     // the tree's copy in shared memory
-    FF *s_l2t = reinterpret_cast<FF *>(dyn + 2 * a.slice);  // [N+1] pre-computed normalisers
-    int32_t *s_pre = reinterpret_cast<int32_t *>(s_l2t + NN);  // [N+1] 1 if pre-computed
-    int32_t *s_off = s_pre + NN;
-    int32_t *s_kid = s_off + (NN + 1);
-    int32_t *s_tok = s_kid + a.N;
-    int32_t *s_row = s_tok + NN;
-    int32_t *s_ps = s_row + NN;                             // [N] parent of each child slot
-    float *s_cxt = reinterpret_cast<float *>(s_ps + a.N);  // [N] per child slot
-    float *s_cxq = s_cxt + a.N;
-    float *s_cu = s_cxq + a.N;
-    {
-        const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
-        const int32_t *kids = a.child_ids + (int64_t)b * a.N;
-        const int32_t *tok = a.token + (int64_t)b * NN;
-        const int32_t *row = per_depth ? a.depth + (int64_t)b * NN : a.qrow_of_node + (int64_t)b * NN;
-        for (int i = threadIdx.x; i <= NN; i += kThreads) s_off[i] = __ldg(off + i);
-        for (int i = threadIdx.x; i < a.N; i += kThreads) {
-            s_kid[i] = __ldg(kids + i);
-            s_ps[i] = -1;
-        }
-        for (int i = threadIdx.x; i < NN; i += kThreads) {
-            s_tok[i] = __ldg(tok + i);
-            s_row[i] = __ldg(row + i);
-        }
-        for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
-            const float2 v = a.pre[(int64_t)b * NN + i].l2q;
-            sh.l2q[i] = FF{v.x, v.y};
-        }
-        if (threadIdx.x == 0) sh.cbad = 0;
-    }
-    __syncthreads();
-    {  // every valid internal node claims its child slots
-        bool bad_here = false;
-        for (int u = threadIdx.x; u < NN; u += kThreads) {
-            const int o = s_off[u], m = s_off[u + 1] - o;
-            if (m == 0) continue;
-            const int r = s_row[u];
-            if (m < 0 || m > kMaxK || o < 0 || o + m > a.N || r < 0 || r >= a.q_R || (per_depth && r >= a.Lq)) {
-                bad_here = true;
-                continue;
-            }
-            for (int i = 0; i < m; ++i) s_ps[o + i] = u;
-        }
-        if (bad_here) sh.cbad = 1;
-    }
-    __syncthreads();
-    for (int u = threadIdx.x; u < NN; u += kThreads) {  // the pre-computed set, as the pre-pass saw it
-        const bool p = u < a.M && s_off[u + 1] - s_off[u] > 0;
-        s_pre[u] = p ? 1 : 0;
-        if (p) {
-            const float2 v = a.pre[(int64_t)b * NN + u].l2t;
-            s_l2t[u] = FF{v.x, v.y};
-        }
-    }
-    {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
-        bool bad_here = false;
-        for (int j = threadIdx.x; j < a.N; j += kThreads) {
-            const int u = s_ps[j];
-            if (u < 0) continue;  // not a child slot of a valid node (never read by the walk)
-            const int c = s_kid[j];
-            const int y = (c >= 1 && c <= a.N) ? s_tok[c] : -1;
-            if (y < 0 || y >= a.V) {
-                bad_here = true;
-                continue;
-            }
-            const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
-            const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)s_row[u] * a.q_rstride;
-            s_cxt[j] = __fmul_rn(Logit<T>::load1(trow, y), a.invT);
-            s_cxq[j] = __fmul_rn(Logit<T>::load1(qrow, y), a.invT);
-            s_cu[j] = uniform_of(draw_word(a.seed, kAccept, (uint32_t)b, (uint32_t)c, 0u));
-        }
-        if (bad_here) sh.cbad = 1;
-    }
+    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    const FF *s_l2t = ts.l2t;
+    const int32_t *s_pre = ts.pre, *s_off = ts.off, *s_kid = ts.kid, *s_tok = ts.tok, *s_row = ts.row;
+    const float *s_cxt = ts.cxt, *s_cxq = ts.cxq, *s_cu = ts.cu;
     int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
     int32_t *onode = a.out_nodes + (int64_t)b * a.L;
 
@@ -823,6 +861,237 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
+// Traversal verification (Weng et al. 2025 as cited in Sec. 2.3, Table 2 and App. A:
+// recursive rejection sampling lifted to sequences for WoR candidates). One cluster per tree,
+// the slice layout and cluster reductions of the RRS walk. The tree is traversed depth first,
+// children in slot order; a node is tried only after every child subtree below it has been
+// rejected, and is then accepted iff U[accept, node] < p_a(node) (the root always). Entering
+// child c (token y) of u gives p_a(c) = min(p_a(u) Mb_u(y) / Ms_u(y), 1). After k rejected
+// child subtrees, u's target-side law is Mb_k = max(P0 - A_k Q, 0) / D_k (A_0 = 0, D_0 = 1),
+// Ms_k = Q / t_k over the tokens not yet rejected, and the update after the next rejection is
+//     A_{k+1} = A_k + D_k / (p_a t_k),  D_{k+1} = sum_v max(P0(v) - A_{k+1} Q(v), 0),
+//     S = p_a D_{k+1} / D_k,  p_a <- S / (S + 1 - p_a),  t_{k+1} = t_k - Q(y):
+// the residual max(p_a Mb_k - Ms_k, 0) = (p_a / D_k) max(P0 - A_{k+1} Q, 0) (subtracting
+// non-negative multiples of Q and clamping compose, and a rejected token already has zero
+// residual). Each update is one pass over u's slices of P0 and Q that only sums; the slices
+// are staged again when the walk returns to u after staging another node. A child whose
+// weight is 0 is rejected without entering it (every node below it has weight 0). An accepted
+// node that had children draws its final token from max(P0 - A Q, 0), a leaf its bonus from
+// its target row. Every internal node's target log-normaliser (and per-node q-row normaliser)
+// comes from the pre-pass; per-depth q normalisers too.
+constexpr int kMaxStack = kMaxDepthRows + 2;
+
+struct TravStack {
+    int node[kMaxStack], next[kMaxStack], deg[kMaxStack];
+    float pa[kMaxStack], A[kMaxStack], D[kMaxStack], th[kMaxStack], tl[kMaxStack];
+};
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 1) k_verify_trav(VerifyArgs a) {
+    pdl_begin();
+    extern __shared__ __align__(16) float dyn[];
+    float *P = dyn;
+    float *Q = dyn + a.slice;
+    __shared__ Scratch sh;
+    __shared__ TravStack st;
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int CS = (int)cluster.num_blocks();
+    const int crank = (int)cluster.block_rank();
+    const int b = blockIdx.x / CS;
+    const int lo = crank * a.slice;
+    const int n = max(0, min(a.V - lo, a.slice));
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const bool writer = threadIdx.x == 0;  // one writer per CTA: every CTA keeps the same stack
+    const bool per_depth = a.qrow_of_node == nullptr;
+    int par = 0;
+    Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
+    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+
+    auto trow_of = [&](int u) {
+        return static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
+    };
+    auto qrow_of = [&](int u) {
+        return static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)ts.row[u] * a.q_rstride;
+    };
+    auto l2q_of = [&](int u) { return per_depth ? sh.l2q[ts.row[u]] : ts.l2qn[u]; };
+
+    if (writer) {
+        st.node[0] = 0;
+        st.next[0] = 0;
+        st.deg[0] = 0;
+        st.pa[0] = 1.f;
+        st.A[0] = 0.f;
+        st.D[0] = 1.f;
+        st.th[0] = 1.f;
+        st.tl[0] = 0.f;
+    }
+    cluster.sync();  // the copy is complete; every CTA of the cluster runs before any distributed access
+
+    bool bad = sh.cbad != 0;  // every CTA checked the same arrays
+    int lev = 0, accepted = -1, final_tok = -1;
+    int staged = -1, staged_rej = 0;  // node whose P0 / Q slices are in P / Q; its rejected tokens zeroed
+
+    // u (stack level lv) after the subtree of its child slot ci was rejected
+    auto update = [&](int lv, int ci) {
+        const int u = st.node[lv], o = ts.off[u];
+        const float pa = st.pa[lv];
+        const FF L2t = ts.l2t[u], L2q = l2q_of(u);
+        const float Qy = exp_shifted(ts.cxq[o + ci], L2q);
+        float npa = pa, nA = st.A[lv], nD = st.D[lv];
+        int ndeg = 0;
+        if (pa > 0.f) {
+            const float A1 = __fmaf_rn(st.D[lv], __frcp_rn(__fmul_rn(pa, st.th[lv])), st.A[lv]);
+            __syncthreads();  // earlier readers of P and Q are done
+            if (staged != u) {
+                W.template stage<true>(trow_of(u), P, kWarps, L2t);
+                W.template stage<true>(qrow_of(u), Q, kWarps, L2q);
+                staged = u;
+                staged_rej = 0;
+                __syncthreads();
+            }
+            for (int j = staged_rej + threadIdx.x; j <= ci; j += kThreads) {  // rejected tokens leave P0
+                const int y = ts.tok[ts.kid[o + j]];
+                if (y >= lo && y < lo + n) P[y - lo] = 0.f;
+            }
+            staged_rej = ci + 1;
+            __syncthreads();
+            KahanF zl;
+            for (int cl = warp; cl < W.nch; cl += kWarps) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const int j = Walk<T>::quad_at(cl, h, lane);
+                    const float4 x = ld4(P, j), q = ld4(Q, j);
+                    const float r0 = fmaxf(__fmaf_rn(-A1, q.x, x.x), 0.f), r1 = fmaxf(__fmaf_rn(-A1, q.y, x.y), 0.f);
+                    const float r2 = fmaxf(__fmaf_rn(-A1, q.z, x.z), 0.f), r3 = fmaxf(__fmaf_rn(-A1, q.w, x.w), 0.f);
+                    zl.add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
+                }
+            }
+            Slot mine = neutral_slot();
+            const FF z = zl.ff();
+            mine.zh = z.hi;
+            mine.zl = z.lo;
+            reduce_round<kRedSum>(sh, par, cluster, mine);
+            const float D1 = sh.res.zh;
+            if (D1 > 0.f) {
+                const float S = __fmul_rn(__fmul_rn(pa, D1), __frcp_rn(st.D[lv]));
+                npa = __fdiv_rn(S, __fadd_rn(S, __fsub_rn(1.f, pa)));
+                nA = A1;
+                nD = D1;
+            } else if (pa < 1.f) {
+                npa = 0.f;
+            } else {
+                ndeg = 1;  // no residual mass with p_a = 1 (rounding only)
+            }
+        }
+        const FF t = ff_add(FF{st.th[lv], st.tl[lv]}, FF{-Qy, 0.f});
+        __syncthreads();  // every thread has read the level's state
+        if (writer) {
+            st.pa[lv] = npa;
+            st.A[lv] = nA;
+            st.D[lv] = nD;
+            st.deg[lv] = ndeg;
+            st.th[lv] = t.hi;
+            st.tl[lv] = t.lo;
+        }
+        __syncthreads();
+    };
+
+    for (int iter = 0; !bad; ++iter) {
+        if (iter > 2 * (a.N + 1) + 2) {  // each node is entered and left once: cannot happen
+            bad = true;
+            break;
+        }
+        const int u = st.node[lev];
+        const int o = ts.off[u], m = ts.off[u + 1] - o;
+        const int i = st.next[lev];
+        if (st.deg[lev] == 0 && i < m) {  // the next child subtree
+            const int c = ts.kid[o + i];
+            const int y = ts.tok[c];
+            const float pa = st.pa[lev];
+            float w = 0.f;
+            bool drawn = false;  // a token repeated among rejected siblings: no residual mass left
+            for (int j = 0; j < i; ++j) drawn |= ts.tok[ts.kid[o + j]] == y;
+            if (pa > 0.f && !drawn) {
+                const float P0y = exp_shifted(ts.cxt[o + i], ts.l2t[u]);
+                const float Qy = exp_shifted(ts.cxq[o + i], l2q_of(u));
+                const float num = __fmul_rn(pa, __fmul_rn(fmaxf(__fmaf_rn(-st.A[lev], Qy, P0y), 0.f),
+                                                          __frcp_rn(st.D[lev])));
+                const float qp = __fmul_rn(Qy, __frcp_rn(st.th[lev]));
+                w = qp > 0.f ? fminf(__fdiv_rn(num, qp), 1.f) : (num > 0.f ? 1.f : 0.f);
+            }
+            if (w > 0.f && lev + 1 >= min(a.L + 1, kMaxStack)) {  // deeper than the depth cap
+                bad = true;
+                break;
+            }
+            __syncthreads();  // every thread has read the level's state
+            if (writer) {
+                st.next[lev] = i + 1;
+                if (w > 0.f) {
+                    st.node[lev + 1] = c;
+                    st.next[lev + 1] = 0;
+                    st.deg[lev + 1] = 0;
+                    st.pa[lev + 1] = w;
+                    st.A[lev + 1] = 0.f;
+                    st.D[lev + 1] = 1.f;
+                    st.th[lev + 1] = 1.f;
+                    st.tl[lev + 1] = 0.f;
+                }
+            }
+            __syncthreads();
+            if (w > 0.f)
+                ++lev;
+            else
+                update(lev, i);  // a weight-0 subtree is rejected without entering it
+            continue;
+        }
+        // u is a leaf of the remaining tree
+        bool acc = true;
+        if (lev > 0 && st.deg[lev] == 0) {
+            const int pu = st.node[lev - 1];
+            acc = ts.cu[ts.off[pu] + st.next[lev - 1] - 1] < st.pa[lev];
+        }
+        if (acc) {
+            accepted = lev;
+            if (m == 0 || st.deg[lev] != 0) {  // bonus from the node's target row
+                final_tok = W.draw_from_row(trow_of(u), u);
+            } else {  // every child rejected: from max(P0 - A Q, 0)
+                if (staged != u) {  // cannot happen: the last update staged u (p_a > 0)
+                    bad = true;
+                    break;
+                }
+                const float A = st.A[lev];
+                final_tok = W.template draw<false>(u, [&](int j, float *v) {
+                    const float4 x = ld4(P, j), q = ld4(Q, j);
+                    v[0] = fmaxf(__fmaf_rn(-A, q.x, x.x), 0.f);
+                    v[1] = fmaxf(__fmaf_rn(-A, q.y, x.y), 0.f);
+                    v[2] = fmaxf(__fmaf_rn(-A, q.z, x.z), 0.f);
+                    v[3] = fmaxf(__fmaf_rn(-A, q.w, x.w), 0.f);
+                });
+                if (final_tok < 0) final_tok = W.draw_from_row(trow_of(u), u);  // no mass (rounding)
+            }
+            break;
+        }
+        --lev;  // u's subtree is rejected: update its parent
+        update(lev, st.next[lev] - 1);
+    }
+    if (writer && crank == 0) {
+        int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
+        int32_t *onode = a.out_nodes + (int64_t)b * a.L;
+        const int nacc = bad ? 0 : accepted;
+        if (bad) raise_status(a.status, kDevBadTree);
+        for (int k = 0; k < nacc; ++k) {
+            otok[k] = ts.tok[st.node[k + 1]];
+            onode[k] = st.node[k + 1];
+        }
+        otok[nacc] = bad ? -1 : final_tok;
+        for (int k = nacc + 1; k <= a.L; ++k) otok[k] = -1;
+        for (int k = nacc; k < a.L; ++k) onode[k] = -1;
+        a.out_len[b] = bad ? 0 : nacc + 1;
+    }
+    cluster.sync();  // no CTA leaves while another may still read its shared memory
+}
+
 constexpr size_t kSmemLimit = 210 * 1024;
 
 // Chunk-aligned slice of each CTA and the dynamic shared memory it needs for cluster size cs
@@ -935,12 +1204,34 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
 
-}  // namespace
+template <typename T>
+cudaError_t launch_trav_t(VerifyArgs a, int B, cudaStream_t s) {
+    int slice = 0;
+    size_t smem = 0;
+    const int cs = choose_cluster<T>(a.V, a.N, B, &slice, &smem);  // same slices and shared memory
+    if (cs < 0) return cudaErrorInvalidValue;
+    a.slice = slice;
+    cudaError_t e = cudaFuncSetAttribute(k_verify_trav<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (cs > 8) {
+        e = cudaFuncSetAttribute(k_verify_trav<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+    }
+    const int per = a.qn ? a.N + 1 : a.Lq;
+    int64_t pre_blocks = 2 * (int64_t)B * a.M + ((int64_t)B * per + kPreThreads / 32 - 1) / (kPreThreads / 32);
+    pre_blocks += pre_blocks & 1;  // whole clusters of two (a spare q-row CTA finds no task)
+    if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    const size_t psmem = (size_t)a.C * sizeof(float2);
+    e = cudaFuncSetAttribute(k_verify_pre<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), psmem, s, 2, a);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_verify_trav<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
+}
 
-cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
-                              const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
-                              const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
-                              int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s) {
+VerifyArgs verify_args(const RowsDesc &target, const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node,
+                       int B, int N, int L, const TreeDesc &tree, const int32_t *token, float invT, uint64_t seed,
+                       int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, uint32_t *status) {
     VerifyArgs a;
     a.target = target.data;
     a.t_bstride = target.batch_stride;
@@ -970,7 +1261,31 @@ cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const f
     a.pre = reinterpret_cast<PreRow *>(reinterpret_cast<char *>(status) + kWsStatusBytes);
     a.M = N + 1 < kPreTop ? N + 1 : kPreTop;
     a.Lq = qrow_of_node ? 0 : (L < N + 1 ? L : N + 1);
+    a.qn = 0;
     a.B = B;
+    return a;
+}
+
+}  // namespace
+
+cudaError_t launch_verify_traversal(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
+                                    const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
+                                    const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                                    int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s) {
+    VerifyArgs a = verify_args(target, q, qstats, qrow_of_node, B, N, L, tree, token, invT, seed, out_tokens,
+                               out_nodes, out_len, status);
+    a.M = N + 1;                       // every internal node's target normaliser
+    a.qn = qrow_of_node ? 1 : 0;       // and, for per-node q rows, each internal node's q normaliser
+    if (target.dtype == 1) return launch_trav_t<__nv_bfloat16>(a, B, s);
+    return launch_trav_t<float>(a, B, s);
+}
+
+cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
+                              const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
+                              const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                              int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s) {
+    const VerifyArgs a = verify_args(target, q, qstats, qrow_of_node, B, N, L, tree, token, invT, seed, out_tokens,
+                                     out_nodes, out_len, status);
     if (target.dtype == 1) return launch_rrs_t<__nv_bfloat16>(a, B, s);
     return launch_rrs_t<float>(a, B, s);
 }

@@ -321,7 +321,9 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
                       int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream) {
     tsb_status st = check_cfg(cfg);
     if (st != TSB_OK) return st;
-    if (mode != TSB_VERIFY_RRS && mode != TSB_VERIFY_BLOCK && mode != TSB_VERIFY_NAIVE) return TSB_ERR_ARG;
+    if (mode != TSB_VERIFY_RRS && mode != TSB_VERIFY_BLOCK && mode != TSB_VERIFY_NAIVE &&
+        mode != TSB_VERIFY_TRAVERSAL)
+        return TSB_ERR_ARG;
     if (mode == TSB_VERIFY_BLOCK && cfg->N > cfg->L) return TSB_ERR_SHAPE;
     st = check_logits(target, cfg->B, cfg->N + 1, cfg->V);
     if (mode == TSB_VERIFY_NAIVE) {  // no draft rows: only the target and the tree
@@ -343,7 +345,12 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
         return TSB_ERR_ARG;
     const float invT = inv_temperature(cfg->temperature);
     cudaError_t e;
-    if (mode == TSB_VERIFY_RRS)
+    if (mode == TSB_VERIFY_TRAVERSAL)
+        e = tsb::launch_verify_traversal(rows_of(target), rows_of(qrows), static_cast<const float2 *>(qstats),
+                                         qrow_of_node, cfg->B, cfg->N, cfg->L, tree_of(tree), token, invT, seed,
+                                         out_tokens, out_nodes, out_len, static_cast<uint32_t *>(ws),
+                                         (cudaStream_t)stream);
+    else if (mode == TSB_VERIFY_RRS)
         e = tsb::launch_verify_rrs(rows_of(target), rows_of(qrows), static_cast<const float2 *>(qstats),
                                    qrow_of_node, cfg->B, cfg->N, cfg->L, tree_of(tree), token, invT, seed,
                                    out_tokens, out_nodes, out_len, static_cast<uint32_t *>(ws),

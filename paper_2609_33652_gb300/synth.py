@@ -162,3 +162,43 @@ def path_keyed_row(base: np.ndarray, path_tokens, noise_std: float, seed: int) -
         h = _mix64(h ^ _mix64(np.array([t], dtype=np.uint64) + np.uint64(1)))
     d = min(len(path_tokens), L - 1)
     return (base[d] + noise_std * prefix_noise(h, V)[0]).astype(np.float32)
+
+
+def _signed64(c: int) -> int:
+    return c - (1 << 64) if c >= 1 << 63 else c
+
+
+def _lsr_t(x: torch.Tensor, k: int) -> torch.Tensor:
+    """Logical right shift of int64 tensors holding uint64 bit patterns."""
+    return (x >> k) & ((1 << (64 - k)) - 1)
+
+
+def _mix64_t(x: torch.Tensor) -> torch.Tensor:
+    """_mix64 on int64 tensors (two's-complement wraparound gives the uint64 arithmetic)."""
+    z = x + _signed64(0x9E3779B97F4A7C15)
+    z = (z ^ _lsr_t(z, 30)) * _signed64(0xBF58476D1CE4E5B9)
+    z = (z ^ _lsr_t(z, 27)) * _signed64(0x94D049BB133111EB)
+    return z ^ _lsr_t(z, 31)
+
+
+def path_keyed_rows_device(base: torch.Tensor, parent: np.ndarray, depth: np.ndarray, token: np.ndarray,
+                           noise_std: float, seed: int, trees_per_batch: int = 8192) -> torch.Tensor:
+    """``path_keyed_rows`` generated on base's device (the same path hashes and noise formula),
+    for trial counts whose rows do not fit the host comfortably. base: [L, V] float32."""
+    L, V = base.shape
+    dev = base.device
+    h = torch.from_numpy(path_hashes(parent, token, seed).view(np.int64)).to(dev)
+    d = torch.from_numpy(np.minimum(depth, L - 1).astype(np.int64)).to(dev)
+    B, NN = h.shape
+    out = torch.empty(B, NN, V, dtype=torch.float32, device=dev)
+    v = torch.arange(V, dtype=torch.int64, device=dev)
+    for b0 in range(0, B, trees_per_batch):
+        hb = h[b0:b0 + trees_per_batch].unsqueeze(-1)
+        a = _mix64_t(hb ^ (2 * v + 1))
+        c = _mix64_t(hb ^ (2 * v + 2) ^ _signed64(0x5851F42D4C957F2D))
+        u1 = (_lsr_t(a, 11).to(torch.float64) + 0.5) * 2.0**-53
+        u2 = (_lsr_t(c, 11).to(torch.float64) + 0.5) * 2.0**-53
+        noise = torch.sqrt(-2.0 * torch.log(u1)) * torch.cos(2.0 * np.pi * u2)
+        rows = base.to(torch.float64)[d[b0:b0 + trees_per_batch]] + noise_std * noise
+        out[b0:b0 + trees_per_batch] = rows.to(torch.float32)
+    return out

@@ -21,7 +21,7 @@ TSB_OK = 0
 STATUS_NAMES = {0: "TSB_OK", 1: "TSB_ERR_ARG", 2: "TSB_ERR_SHAPE", 3: "TSB_ERR_DTYPE", 4: "TSB_ERR_ALIGN",
                 5: "TSB_ERR_WORKSPACE", 6: "TSB_ERR_CUDA", 7: "TSB_ERR_DEVICE"}
 TSB_F32, TSB_BF16 = 0, 1
-TSB_VERIFY_RRS, TSB_VERIFY_BLOCK, TSB_VERIFY_NAIVE = 0, 1, 2
+TSB_VERIFY_RRS, TSB_VERIFY_BLOCK, TSB_VERIFY_NAIVE, TSB_VERIFY_TRAVERSAL = 0, 1, 2, 3
 TSB_DEV_NONFINITE, TSB_DEV_BAD_INDEX, TSB_DEV_BAD_TREE = 0x1, 0x2, 0x4
 TSB_CHUNK = 256
 
@@ -330,11 +330,14 @@ class PreparedStep:
     tsb_plan_rows (or, with ``width``, tsb_plan_rows_expand), tsb_replay (``replay="wor"``),
     tsb_replay_mixed (``"mixed"``) or nothing (``"plan"``: the first pass's tokens are
     verified), then tsb_verify in ``mode``. With ``fused=False`` the first pass is
-    tsb_row_stats + tsb_plan instead; with ``plan_only`` only the first pass runs."""
+    tsb_row_stats + tsb_plan instead; with ``plan_only`` only the first pass runs. With
+    ``qrows`` (per-node draft rows [B, Rq, V]), ``qstats`` (their statistics buffer) and
+    ``qrow_of_node`` ([B, N+1]), the step also runs tsb_row_stats on the q rows, and replay and
+    verification draw from them (the corrected-drafter workload)."""
 
     def __init__(self, buf: TsbBuffers, draft: torch.Tensor, target: torch.Tensor, seed: int, mode=TSB_VERIFY_RRS,
                  out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True, width=None, replay="wor",
-                 plan_only=False):
+                 plan_only=False, qrows=None, qstats=None, qrow_of_node=None):
         lib = load()
         self._keep = []
         s = _stream(stream)
@@ -363,19 +366,29 @@ class PreparedStep:
                     ("tsb_plan", lib.tsb_plan, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb,
                                                 ctypes.byref(tr), _ptr(buf.ws), wb, s))]
         tok = buf.tree["plan_token"] if replay == "plan" else buf.token
+        qcalls = []
+        if qrows is not None:  # per-node draft rows: their statistics first
+            dq = logits_desc(qrows)
+            self._keep += [dq, qrows, qstats, qrow_of_node]
+            qsb_ = qstats.numel() * qstats.element_size()
+            qcalls = [("tsb_row_stats_q", lib.tsb_row_stats,
+                       (ctypes.byref(dq), ctypes.c_float(cfg.temperature), _ptr(qstats), qsb_, _ptr(buf.ws), wb, s))]
+            qref, qst, qstb, qidx = ctypes.byref(dq), _ptr(qstats), qsb_, _ptr(qrow_of_node)
+        else:
+            qref, qst, qstb, qidx = ctypes.byref(dd), _ptr(buf.stats), sb, None
         if replay == "plan":
             rep = []
         else:
             fn, name = (lib.tsb_replay_mixed, "tsb_replay_mixed") if replay == "mixed" else (lib.tsb_replay,
                                                                                               "tsb_replay")
-            rep = [(name, fn, (ctypes.byref(cfg), ctypes.byref(dd), _ptr(buf.stats), sb, None, ctypes.byref(tr),
-                               seed, _ptr(tok), _ptr(buf.ws), wb, s))]
+            rep = [(name, fn, (ctypes.byref(cfg), qref, qst, qstb, qidx, ctypes.byref(tr), seed, _ptr(tok),
+                               _ptr(buf.ws), wb, s))]
         if mode == TSB_VERIFY_NAIVE:
-            qd, qs, qsb = None, None, 0
+            qd, qs, qsb, qi = None, None, 0, None
         else:
-            qd, qs, qsb = ctypes.byref(dd), _ptr(buf.stats), sb
-        self.calls = plan + rep + [
-            ("tsb_verify", lib.tsb_verify, (ctypes.byref(cfg), int(mode), ctypes.byref(dt), qd, qs, qsb, None,
+            qd, qs, qsb, qi = qref, qst, qstb, qidx
+        self.calls = plan + qcalls + rep + [
+            ("tsb_verify", lib.tsb_verify, (ctypes.byref(cfg), int(mode), ctypes.byref(dt), qd, qs, qsb, qi,
                                             ctypes.byref(tr), _ptr(tok), seed, _ptr(ot), _ptr(on), _ptr(ol),
                                             _ptr(buf.ws), wb, s)),
         ]

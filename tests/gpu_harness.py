@@ -233,6 +233,8 @@ def run_step(draft, L, N, K, T, seed, target_noise=0.7, target_seed=2000, qrows=
     check_status(buf)
     if mode == tsb.TSB_VERIFY_RRS:
         rout = oracle.verify_rrs(h_target, h_q, T, ref, rtok, seed, L, qrow_of_node=h_qidx, batch_ids=bids)
+    elif mode == tsb.TSB_VERIFY_TRAVERSAL:
+        rout = oracle.verify_traversal(h_target, h_q, T, ref, rtok, seed, L, qrow_of_node=h_qidx, batch_ids=bids)
     elif mode == tsb.TSB_VERIFY_NAIVE:
         rout = oracle.verify_naive(h_target, T, ref, rtok, seed, L, batch_ids=bids)
     else:

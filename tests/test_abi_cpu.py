@@ -191,7 +191,7 @@ def test_replay_verify_validation(lib):
         return lib.tsb_verify(ctypes.byref(cfg), mode, ctypes.byref(tg), ctypes.byref(q), FAKE, 1 << 30, None,
                               ctypes.byref(t), FAKE, 1, out, FAKE, FAKE, FAKE, 1 << 30, None)
 
-    assert verify(mode=3) == ARG
+    assert verify(mode=4) == ARG
     assert verify(target=_logits(2, 8, 64)) == SHAPE  # needs N+1 target rows
     assert verify(target=_logits(2, 9, 64, dtype=1)) == DTYPE  # target / q dtypes differ
     assert verify(out=None) == ARG
