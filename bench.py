@@ -18,8 +18,12 @@ programmatic launches. Inputs rotate over several independent sets whose per-ste
 footprint together exceeds the L2 several times, so no step finds its rows in L2 from an
 earlier step. ``e2e`` repeats the measurement through the same C ABI with host (pinned)
 inputs: every step copies its draft and target rows to the device and its outputs back.
-``--impl reference`` times the CPU oracle on the same workload (one tree per step, scaled to
-the batch), rank 0 only.
+``timing`` adds per-step percentiles (a pass with an event between steps) and the same steps
+replayed from one CUDA graph; ``other_workloads`` times the single-stream, corrected-drafter
+(T = 0.6 and 1.0) and V = 128,256 workloads the same way; ``variants`` the paper's other
+sampling and verification schemes. ``cpu_baseline`` and ``--impl reference`` time the CPU
+oracle as it stands on the host's cores: whole steps (the B trees of a set) over a process
+pool with one process per usable core, rank 0 only.
 """
 from __future__ import annotations
 
@@ -61,6 +65,9 @@ def parse():
     ap.add_argument("--variant-steps", type=int, default=300)
     ap.add_argument("--no-planners", action="store_true", help="skip the first-pass-only timings at N = 64 and 256")
     ap.add_argument("--no-pooled", action="store_true", help="skip the pooled-law step")
+    ap.add_argument("--no-graph", action="store_true", help="skip the CUDA-graph replay timing")
+    ap.add_argument("--no-presets", action="store_true",
+                    help="skip the other workloads (single stream, corrected drafter at T 0.6 / 1.0, V = 128,256)")
     ap.add_argument("--sweep", action="store_true",
                     help="instead of the headline step: the budget sweep at scale (B=64, V=151,936, L=16, "
                          "N in --budgets, bf16 and fp32), one JSON line with us/step and HBM GB/s per (dtype, N)")
@@ -83,13 +90,16 @@ def workload(args):
     return w
 
 
-def config_of(w, extra=None):
-    cfg = {"workload": f"batched serving: B={w['B']}, V={w['V']}, L={w['L']}, N={w['N']}, K={w['K']}, "
-                       f"T={w['T']}, {w['dtype']} logits, target = depth row + N(0,{w['target_noise']}^2)",
-           "B": w["B"], "V": w["V"], "L": w["L"], "N": w["N"], "K": w["K"], "temperature": w["T"]}
-    if extra:
-        cfg.update(extra)
-    return cfg
+def config_of(w, args):
+    """The workload as both arms state it (identical dicts for the same arguments)."""
+    es = 2 if w["dtype"] == "bf16" else 4
+    set_mb = (w["B"] * w["L"] + w["B"] * (w["N"] + 1)) * w["V"] * es / 1e6
+    return {"workload": f"batched serving: B={w['B']}, V={w['V']}, L={w['L']}, N={w['N']}, K={w['K']}, "
+                        f"T={w['T']}, {w['dtype']} logits, target = depth row + N(0,{w['target_noise']}^2)",
+            "B": w["B"], "V": w["V"], "L": w["L"], "N": w["N"], "K": w["K"], "temperature": w["T"],
+            "parallelism": f"replicas only, {args.gpus} x 1 GPU",
+            "l2": f"inputs larger than L2: {args.sets} input sets rotated, {set_mb:.0f} MB of draft and target rows "
+                  f"each ({args.sets * set_mb * 1e6 / L2_BYTES:.0f}x L2)"}
 
 
 def measured_peak_hbm():
@@ -223,6 +233,7 @@ VARIANTS = (
     ("expand_prune_w10_wor_rrs", dict(width=10), False),
     ("top1_chain_naive_verify", dict(replay="plan", mode=2), True),
     ("sampled_chain_block_verify", dict(mode=1), True),
+    ("wor_traversal_verify", dict(mode=3), False),
 )
 
 
@@ -366,6 +377,76 @@ def run_pooled(w, sets, device, steps=300, warmup=10, P=16):
             "mean_emitted_len_last_steps": round(lens, 4)}
 
 
+PRESETS = (
+    # name, workload, per-node q rows
+    ("single_stream_B1_N32", dict(name="single", B=1, V=151936, L=16, N=32, K=8, T=1.0, dtype="bf16",
+                                  target_noise=0.7), False),
+    ("corrected_B1_N64_T0.6", dict(name="corrected", B=1, V=151936, L=16, N=64, K=8, T=0.6, dtype="bf16",
+                                   target_noise=0.7), True),
+    ("corrected_B1_N64_T1.0", dict(name="corrected", B=1, V=151936, L=16, N=64, K=8, T=1.0, dtype="bf16",
+                                   target_noise=0.7), True),
+    ("batched_B16_N64_V128256", dict(name="batched128k", B=16, V=128256, L=16, N=64, K=8, T=1.0, dtype="bf16",
+                                     target_noise=0.7), False),
+)
+
+
+def run_presets(device, steps=300, warmup=10):
+    """The other workloads of the benchmark (not bench lines): each rotates enough input sets
+    that their rows exceed L2 three times, and is timed like the headline step (start and end
+    events around the steps), with per-step percentiles. Algorithmic bytes: draft rows once,
+    per-node q rows once, target rows of the visited nodes."""
+    import torch
+
+    from paper_2609_33652_gb300 import synth, tsb
+
+    peak, _ = measured_peak_hbm()
+    out = {}
+    for name, w, per_node in PRESETS:
+        es = 2 if w["dtype"] == "bf16" else 4
+        row = w["V"] * es
+        NN = w["N"] + 1
+        set_bytes = (w["B"] * w["L"] + w["B"] * NN * (2 if per_node else 1)) * row
+        S = max(2, int(np.ceil(3 * L2_BYTES / set_bytes)))
+        sets = build_sets(w, S, device, 0)
+        olen = torch.empty(steps, w["B"], dtype=torch.int32, device=device)
+        prep = []
+        for st_i, st in enumerate(sets):
+            if per_node:
+                st["qrows"] = synth.rows_from_depth(st["draft"], st["buf"].tree["depth"], 0.3, 7000 + st_i)
+                st["qstats"] = torch.empty(tsb.tsb_stats_bytes(w["B"], NN, w["V"]) // 4, dtype=torch.float32,
+                                           device=device)
+                st["qidx"] = torch.arange(NN, dtype=torch.int32, device=device).repeat(w["B"], 1).contiguous()
+        for k in range(steps + warmup):
+            st = sets[k % S]
+            extra = dict(qrows=st["qrows"], qstats=st["qstats"], qrow_of_node=st["qidx"]) if per_node else {}
+            prep.append(tsb.PreparedStep(st["buf"], st["draft"], st["target"], 6_000_000 + k,
+                                         out_len=olen[k - warmup] if k >= warmup else None, **extra))
+        for p in prep[:warmup]:
+            p.run()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for p in prep[warmup:]:
+            p.run()
+        b.record()
+        torch.cuda.synchronize()
+        us = a.elapsed_time(b) * 1e3 / steps
+        pct = step_percentiles(prep[warmup:warmup + min(steps, 200)])
+        for st in sets:
+            if tsb.tsb_device_status(st["buf"].ws) != 0:
+                raise RuntimeError(f"device status bits set in preset {name}")
+        visited = float(olen.float().sum(dim=1).mean().item())
+        nbytes = w["B"] * w["L"] * row + (w["B"] * NN * row if per_node else 0) + visited * row
+        out[name] = {"us_per_step": round(us, 3), "per_step_us": pct, "hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
+                     "hbm_frac_of_measured": round(nbytes / (us * 1e-6) / 1e9 / peak, 4),
+                     "algorithmic_bytes_per_step": round(nbytes),
+                     "mean_emitted_len": round(float(olen.float().mean().item()), 4), "input_sets": S,
+                     "steps": steps}
+        del sets, prep
+        torch.cuda.empty_cache()
+    return out
+
+
 def max_over_ranks(value: float, dist, device) -> float:
     """The largest of the ranks' values (every rank gets it): a job's time is its slowest
     replica's. ``device`` is where the process group's backend reduces (cuda for nccl)."""
@@ -452,6 +533,8 @@ def run_tsb(args):
             per_kernel[n].append(events[k][i].elapsed_time(events[k][i + 1]) * 1e3)
     kern_us = {n: statistics.mean(v) for n, v in per_kernel.items()}
     us_step = total_ms * 1e3 / K
+    dist_us = step_percentiles(steps[:KA])
+    graph_us = graph_step_us(w, sets, device) if not args.no_graph else None
 
     h_len = out_len.cpu().numpy()
     h_nodes = out_nodes.cpu().numpy()
@@ -484,6 +567,8 @@ def run_tsb(args):
     if variants is not None and not args.no_pooled:
         variants["pooled16_wor_rrs"] = run_pooled(w, sets, device, steps=args.variant_steps)
 
+    presets = run_presets(device) if not args.no_presets else None
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         cpu = cpu_baseline(w, sets, seconds=12.0)
@@ -494,10 +579,11 @@ def run_tsb(args):
         "ms_per_step": round(us_step / 1e3, 6), "higher_is_better": False, "scaling": "weak", "vs_baseline": None,
         "dtype": w["dtype"], "data": "synthetic (seeded; shapes and value distributions of the batched serving "
                                      "workload; no datasets or model weights)",
-        "config": config_of(w, {"parallelism": f"replicas x{world}" if world > 1 else "single GPU",
-                                "l2": f"{S} input sets rotated (per-step footprint {step_bytes / 1e6:.0f} MB, "
-                                      f"{S * step_bytes / L2_BYTES:.1f}x L2)",
-                                "launch": "eager C-ABI calls with programmatic dependent launch, inputs resident in HBM"}),
+        "config": config_of(w, args),
+        "timing": {"launch": "eager C-ABI calls with programmatic dependent launch, inputs resident in HBM; "
+                             "start and end events only in the timed region",
+                   "per_step_us": dist_us, "cuda_graph_us_per_step": graph_us,
+                   "algorithmic_footprint_per_step_mb": round(step_bytes / 1e6, 1)},
         "hbm_gbs": round(hbm_gbs, 1), "hbm_frac_of_measured": round(hbm_gbs / peak, 4),
         "hbm_frac_of_nominal_8tbs": round(hbm_gbs / NOMINAL_HBM_GBS, 4),
         "algorithmic_bytes_per_step": round(step_bytes), "rows_per_s": round(rows_per_s, 1),
@@ -509,6 +595,7 @@ def run_tsb(args):
         "clocks": clocks.summary(),
         "e2e": e2e,
         "variants": variants,
+        "other_workloads": presets,
         "cpu_baseline": cpu,
     }
     if rank == 0:
@@ -516,6 +603,61 @@ def run_tsb(args):
     if dist is not None:
         dist.barrier()
         dist.destroy_process_group()
+
+
+def step_percentiles(prep):
+    """Per-step device times (an event between consecutive steps, which serialises only the
+    step boundary): p10, median and p90 in microseconds."""
+    import torch
+
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(len(prep) + 1)]
+    ev[0].record()
+    for k, p in enumerate(prep):
+        p.run()
+        ev[k + 1].record()
+    torch.cuda.synchronize()
+    d = np.array([ev[k].elapsed_time(ev[k + 1]) * 1e3 for k in range(len(prep))])
+    return {"p10": round(float(np.percentile(d, 10)), 3), "median": round(float(np.median(d)), 3),
+            "p90": round(float(np.percentile(d, 90)), 3), "steps": len(prep)}
+
+
+def graph_step_us(w, sets, device, steps_per_graph=16, replays=20):
+    """The same steps captured in one CUDA graph (steps_per_graph steps over the rotating input
+    sets) and replayed: mean device time per step. None (with the reason) if capture fails."""
+    import torch
+
+    from paper_2609_33652_gb300 import tsb
+
+    S = len(sets)
+    stream = torch.cuda.Stream(device)
+    try:
+        prep = [tsb.PreparedStep(sets[k % S]["buf"], sets[k % S]["draft"], sets[k % S]["target"], 3_000_000 + k,
+                                 stream=stream) for k in range(steps_per_graph)]
+        with torch.cuda.stream(stream):
+            for p in prep:  # warm-up on the capture stream (cluster choices cached, modules loaded)
+                p.run()
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream, capture_error_mode="relaxed"):
+            for p in prep:
+                p.run()
+        torch.cuda.synchronize()
+        g.replay()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            a.record()
+            for _ in range(replays):
+                g.replay()
+            b.record()
+        torch.cuda.synchronize()
+        for st in sets:
+            if tsb.tsb_device_status(st["buf"].ws) != 0:
+                raise RuntimeError("device status bits set in the graph replays")
+        return round(a.elapsed_time(b) * 1e3 / (replays * steps_per_graph), 3)
+    except Exception as e:  # capture not possible here: report why
+        torch.cuda.synchronize()
+        return {"error": f"{type(e).__name__}: {e}"[:300]}
 
 
 def bind_near_gpu(device):
@@ -586,91 +728,174 @@ def run_e2e(args, w, sets, device):
 
 
 # ---------------------------------------------------------------------------------------
-def oracle_tree_step(w, draft_h, seed):
-    """The CPU oracle on one tree: plan, replay, then verify against target rows built (by the
-    shared input generator) from the oracle's own plan."""
-    import torch
+_SHARED = {}  # worker side: set index -> (draft [B, L, V], target [B, N+1, V]) views of shared memory
+
+
+def _pool_init(descs):
+    """Worker start-up: attach the shared input sets and load the oracle."""
+    from multiprocessing import shared_memory
 
     import oracle
+
+    oracle.build()
+    oracle._load()
+    for i, (dn, ds, dd, tn, ts_, td) in enumerate(descs):
+        a = shared_memory.SharedMemory(name=dn)
+        b = shared_memory.SharedMemory(name=tn)
+        _SHARED[i] = (np.ndarray(ds, dtype=dd, buffer=a.buf), np.ndarray(ts_, dtype=td, buffer=b.buf), a, b)
+
+
+def _pool_tree(task):
+    """One tree of the oracle in a worker: (workload, set, tree, seed) -> (seconds, flags)."""
+    w, si, b, seed = task
+    d, t = _SHARED[si][0], _SHARED[si][1]
+    sec, _, flags = oracle_tree_step(w, d[b:b + 1], t[b:b + 1], seed)
+    return sec, flags
+
+
+def _pool_pid(_):
+    return os.getpid()
+
+
+class OraclePool:
+    """Input sets in shared memory (draft rows and target rows, as the oracle reads them) and a
+    spawn pool of n oracle processes attached to them (spawn: the parent may hold a CUDA
+    context)."""
+
+    def __init__(self, n, host_sets):
+        import multiprocessing as mp
+        from multiprocessing import shared_memory
+
+        self.blocks, descs = [], []
+        for d, t in host_sets:
+            entry = []
+            for arr in (d, t):
+                shm = shared_memory.SharedMemory(create=True, size=arr.nbytes)
+                np.ndarray(arr.shape, dtype=arr.dtype, buffer=shm.buf)[...] = arr
+                self.blocks.append(shm)
+                entry += [shm.name, arr.shape, arr.dtype.str]
+            descs.append(tuple(entry))
+        self.nsets = len(host_sets)
+        self.pool = mp.get_context("spawn").Pool(n, initializer=_pool_init, initargs=(descs,))
+        self.pool.map(_pool_pid, range(n))  # every worker has started and attached
+
+    def steps(self, w, steps, seed0):
+        """Whole steps: each runs the B trees of one set across the pool; returns the wall
+        seconds of every step and the summed near-tie flags."""
+        times, flags = [], {"trees": 0, "plan": 0, "replay_parents": 0, "replay_flagged": 0, "verify": 0}
+        for k in range(steps):
+            tasks = [(w, k % self.nsets, b, seed0 + k * w["B"] + b) for b in range(w["B"])]
+            t0 = time.perf_counter()
+            res = self.pool.map(_pool_tree, tasks, chunksize=1)
+            times.append(time.perf_counter() - t0)
+            for _, f in res:
+                for key in flags:
+                    flags[key] += f[key]
+        return times, flags
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+        for shm in self.blocks:
+            shm.close()
+            shm.unlink()
+
+
+def host_sets(sets):
+    """(draft, target) host arrays of each input set, in the oracle's layout."""
     from paper_2609_33652_gb300 import synth
+
+    return [(synth.to_host(st["draft"].contiguous()), synth.to_host(st["target"].contiguous())) for st in sets]
+
+
+def oracle_tree_step(w, draft_h, target_h, seed):
+    """The CPU oracle on one tree: plan, replay, verify (RRS); returns its seconds, outputs and
+    the near-tie flags of its decisions."""
+    import oracle
 
     t0 = time.perf_counter()
     ref = oracle.plan(draft_h, w["T"], w["N"], w["K"], w["L"])
     tok, rex = oracle.replay(draft_h, w["T"], ref, seed)
+    out = oracle.verify_rrs(target_h, draft_h, w["T"], ref, tok, seed, w["L"])
     t1 = time.perf_counter()
-    dt = torch.from_numpy(draft_h.view(np.int16)).view(torch.bfloat16) if draft_h.dtype == np.uint16 else \
-        torch.from_numpy(draft_h)
-    target = synth.to_host(synth.rows_from_depth(dt, torch.from_numpy(ref["depth"]), w["target_noise"], seed + 7))
-    t2 = time.perf_counter()
-    out = oracle.verify_rrs(target, draft_h, w["T"], ref, tok, seed, w["L"])
-    t3 = time.perf_counter()
     # decisions the oracle flags as near ties (where a GPU result may differ, reading of the
     # 1e-6 band): planner pops per tree, Gumbel selections per parent, walk decisions per tree
     parents = int((np.diff(ref["child_off"], axis=1) > 0).sum())
     flags = {"trees": int(draft_h.shape[0]), "plan": int(ref["exempt"].sum()), "replay_parents": parents,
              "replay_flagged": int(rex.sum()), "verify": int(out["exempt"].sum())}
-    return (t1 - t0) + (t3 - t2), out, flags
+    return t1 - t0, out, flags
 
 
 def cpu_baseline(w, sets, seconds=12.0):
-    import oracle
-    from paper_2609_33652_gb300 import synth
-
-    oracle.build()
-    times = []
-    flags = {"trees": 0, "plan": 0, "replay_parents": 0, "replay_flagged": 0, "verify": 0}
-    k = 0
-    t_start = time.perf_counter()
-    while time.perf_counter() - t_start < seconds or k < 1:
-        st = sets[k % len(sets)]
-        b = k % w["B"]
-        h = synth.to_host(st["draft"][b:b + 1])
-        t, _, f = oracle_tree_step(w, h, 100 + k)
-        times.append(t)
-        for key in flags:
-            flags[key] += f[key]
-        k += 1
-    per_tree = statistics.mean(times)
-    return {"value": round(per_tree * w["B"] * 1e6, 1), "unit": "us/step", "cores": 1, "kind": "oracle",
-            "sample": f"{k} single trees of the workload (plan + replay + verify, one thread), "
-                      f"mean per tree x B={w['B']}",
+    """The oracle as it stands on the host cores: whole steps (the B trees of a set across a
+    pool of one process per usable core) for about ``seconds``, and single trees on one core."""
+    cores = len(os.sched_getaffinity(0))
+    hs = host_sets(sets[:2])
+    pool = OraclePool(cores, hs)
+    try:
+        pool.steps(w, 1, 50)  # warm-up step
+        t0 = time.perf_counter()
+        times, flags = [], None
+        while time.perf_counter() - t0 < seconds or not times:
+            tt, ff = pool.steps(w, 1, 100 + len(times) * w["B"])
+            times += tt
+            flags = ff if flags is None else {k: flags[k] + ff[k] for k in flags}
+    finally:
+        pool.close()
+    one = []
+    t1 = time.perf_counter()
+    while time.perf_counter() - t1 < seconds / 3 or not one:
+        b = len(one) % w["B"]
+        one.append(oracle_tree_step(w, hs[0][0][b:b + 1], hs[0][1][b:b + 1], 9000 + len(one))[0])
+    return {"value": round(statistics.mean(times) * 1e6, 1), "unit": "us/step", "cores": cores, "kind": "oracle",
+            "sample": f"{len(times)} whole steps (B={w['B']} trees of plan + replay + verify, spread over {cores} "
+                      f"processes, one per usable core; inputs in shared memory); one core: {len(one)} single "
+                      f"trees, {statistics.mean(one) * 1e6:.0f} us per tree",
+            "one_core_us_per_tree": round(statistics.mean(one) * 1e6, 1),
             "near_tie_flags": flags}
 
 
 def run_reference(args):
+    """The CPU oracle as the reference arm: K timed steps of the B trees of the workload on the
+    host's cores (a spawn pool, one process per usable core), after W warm-up steps; the number
+    of timed steps is capped so the arm ends within a few minutes (``steps_run``)."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return
+    import torch
+
+    import oracle
     from paper_2609_33652_gb300 import synth
 
     w = workload(args)
     K, W = args.steps, args.warmup
-    import torch
-
-    drafts = [synth.draft_logits(w["B"], w["L"], w["V"], "planted", w["dtype"], 1003 + 100 * s, device="cpu")
-              for s in range(2)]
-
-    def sample(k):
-        h = synth.to_host(drafts[k % 2][(k // 2) % w["B"]:(k // 2) % w["B"] + 1])
-        return oracle_tree_step(w, h, 10 + k)[0]
-
-    for k in range(W):
-        sample(k)
-    t_one = sample(W)
-    budget = 150.0
-    run_k = K if K * t_one <= budget else max(3, int(budget / t_one))
-    times = [sample(W + 1 + k) for k in range(run_k)]
-    us = statistics.mean(times) * w["B"] * 1e6
-    sample_txt = (f"one tree of B={w['B']} per step (plan + replay + verify, one thread), scaled by B; "
-                  f"{run_k} of the {K} requested steps run to stay within {budget:.0f} s")
+    cores = len(os.sched_getaffinity(0))
+    sets = []
+    for s_ in range(2):  # the bench's first two input sets, targets from the oracle's own plan
+        seed = 1003 + 100 * s_
+        draft = synth.draft_logits(w["B"], w["L"], w["V"], "planted", w["dtype"], seed, device="cpu")
+        ref = oracle.plan(synth.to_host(draft), w["T"], w["N"], w["K"], w["L"])
+        target = synth.rows_from_depth(draft, torch.from_numpy(ref["depth"]), w["target_noise"], seed + 1)
+        sets.append({"draft": draft, "target": target})
+    pool = OraclePool(cores, host_sets(sets))
+    try:
+        pool.steps(w, max(W, 1), 10)
+        t_one = pool.steps(w, 1, 20)[0][0]
+        budget = 150.0
+        run_k = K if K * t_one <= budget else max(3, int(budget / t_one))
+        times, _ = pool.steps(w, run_k, 1000)
+    finally:
+        pool.close()
+    us = statistics.mean(times) * 1e6
+    sample_txt = (f"{run_k} of the {K} requested steps, each the B={w['B']} trees of one input set (plan + replay + "
+                  f"verify) over {cores} processes, one per usable core")
     line = {"impl": "reference", "metric": METRIC, "value": round(us, 1), "unit": "us/step", "n_gpus": args.gpus,
             "steps": K, "steps_run": run_k, "warmup": W, "ms_per_step": round(us / 1e3, 4), "higher_is_better": False,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config_of(w),
-            "cpu_baseline": {"value": round(us, 1), "unit": "us/step", "cores": 1, "kind": "oracle",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "config": config_of(w, args),
+            "cpu_baseline": {"value": round(us, 1), "unit": "us/step", "cores": cores, "kind": "oracle",
                              "sample": sample_txt},
             "e2e": {"value": round(us, 1), "unit": "us/step", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
-    del torch
 
 
 def run_sweep(args):
@@ -690,6 +915,8 @@ def run_sweep(args):
     B, V, L, K, T = 64, 151936, 16, 8, 1.0
     peak, peak_kind = measured_peak_hbm()
     out = {}
+    sampler = ClockSampler(0)
+    sampler.__enter__()
     for dtype in ("bf16", "f32"):
         es = 2 if dtype == "bf16" else 4
         for N in [int(x) for x in args.budgets.split(",")]:
@@ -721,15 +948,17 @@ def run_sweep(args):
                 if tsb.tsb_device_status(bf.ws) != 0:
                     raise RuntimeError(f"device status bits set in the sweep at {dtype}, N={N}")
             us = t0.elapsed_time(t1) * 1e3 / args.steps
+            pct = step_percentiles(prep[:min(args.steps, 100)])
             visited = float(olen.float().sum(dim=1).mean().item())
             nbytes = B * L * V * es + visited * V * es
             out[f"{dtype}_N{N}"] = {"us_per_step": round(us, 3), "hbm_gbs": round(nbytes / (us * 1e-6) / 1e9, 1),
                                     "hbm_frac_of_measured": round(nbytes / (us * 1e-6) / 1e9 / peak, 4),
-                                    "algorithmic_bytes_per_step": round(nbytes),
+                                    "algorithmic_bytes_per_step": round(nbytes), "per_step_us": pct,
                                     "mean_emitted_len": round(float(olen.float().mean().item()), 4)}
             del sets, prep, warm
             torch.cuda.empty_cache()
-    print(json.dumps({"metric": "budget sweep: plan+replay+verify us/step and HBM GB/s per N", "n_gpus": 1,
+    sampler.__exit__(None, None, None)
+    print(json.dumps({"clocks": sampler.summary(), "metric": "budget sweep: plan+replay+verify us/step and HBM GB/s per N", "n_gpus": 1,
                       "steps": args.steps, "warmup": args.warmup, "higher_is_better": False,
                       "config": {"workload": "budget sweep at scale: B=64, V=151936, L=16, K=8, T=1.0, depth cap 16, "
                                              "target = depth row + N(0,0.7^2)", "B": B, "V": V, "L": L, "K": K,
