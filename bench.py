@@ -565,7 +565,8 @@ def run_tsb(args):
     if variants is not None and not args.no_planners:
         variants["first_pass_us_per_call"] = run_planners(w, sets, device, steps=args.variant_steps)
     if variants is not None and not args.no_pooled:
-        variants["pooled16_wor_rrs"] = run_pooled(w, sets, device, steps=args.variant_steps)
+        for P in (16, 64):  # DFlash2's pools of 16 and Domino's sparse pools of 64 (App. B.7)
+            variants[f"pooled{P}_wor_rrs"] = run_pooled(w, sets, device, steps=args.variant_steps, P=P)
 
     presets = run_presets(device) if not args.no_presets else None
 

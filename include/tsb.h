@@ -80,7 +80,7 @@ typedef enum {
 
 /* Limits (validated). */
 #define TSB_MAX_WIDTH 1024              /* frontier width of the expand-then-prune first pass */
-#define TSB_MAX_POOL 32                 /* tokens in a pooled draft law (one warp) */
+#define TSB_MAX_POOL 64                 /* tokens in a pooled draft law (one warp, two per lane) */
 #define TSB_MAX_EXPAND_CANDIDATES 8192  /* candidates it may generate: K + (L-1) layers of <= W*K */
 #define TSB_CHUNK 256 /* fixed chunk of the chunk statistics and of the replay sampler */
 #define TSB_MAX_K 32

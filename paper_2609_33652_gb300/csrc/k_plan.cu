@@ -949,7 +949,8 @@ cudaError_t launch_plan_expand(const RowsDesc &draft, const float2 *stats, float
     return launch_ept(ea, draft.B, s);
 }
 
-// Pooled first pass: the per-row top-P pass writes the pools (ids only) to pool_ids, then
+// Pooled first pass: the per-row top-P pass (k_pool_select for P > 32) writes the pools (ids
+// only) to pool_ids, then
 // k_pool_finish turns each pool into the pooled log-normaliser and the K candidates, then the
 // max-heap expansion as in launch_plan.
 cudaError_t launch_plan_pooled(const RowsDesc &draft, const float2 *stats, int L, int N, int K, int P, float invT,
@@ -959,7 +960,9 @@ cudaError_t launch_plan_pooled(const RowsDesc &draft, const float2 *stats, int L
     t.topk_id = pool_ids;
     t.topk_x = nullptr;
     cudaError_t e;
-    if (draft.dtype == 1)
+    if (P > 32)  // pools above the top-K pass's 32: the exact selection kernel
+        e = launch_pool_select(draft, stats, L, P, invT, pool_ids, s);
+    else if (draft.dtype == 1)
         e = P <= 8 ? launch_topk_t<8, __nv_bfloat16>(t, s) : launch_topk_t<32, __nv_bfloat16>(t, s);
     else
         e = P <= 8 ? launch_topk_t<8, float>(t, s) : launch_topk_t<32, float>(t, s);

@@ -1,7 +1,7 @@
 // Pooled draft laws (Sec. 3.1 and 3.2: a position's draft law is restricted to its P most
 // probable tokens and normalised within them; Sec. 3.3: verification uses those pooled
-// probabilities, while the target law and the residual stay full-vocabulary). P <= 32, so a
-// pool is one warp, lane j holding pool token j.
+// probabilities, while the target law and the residual stay full-vocabulary). P <= 64, so a
+// pool is one warp, lane j holding pool tokens j and j + 32.
 //
 //   k_pool_finish     first pass: from the rows' top-P lists (the pools), the pooled
 //                     log-normaliser and the K candidates the max-heap expands.
@@ -21,7 +21,7 @@
 namespace tsb {
 namespace {
 
-constexpr int kMaxPool = 32;
+constexpr int kMaxPool = 64;
 
 // ---------------------------------------------------------------------------------------
 struct FinishArgs {
@@ -44,13 +44,15 @@ __global__ void __launch_bounds__(128) k_pool_finish(FinishArgs a) {
     if (row >= a.rows) return;  // uniform over the warp
     const int b = row / a.L, d = row - (row / a.L) * a.L;
     const T *rp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
-    float x = -INFINITY;
+    float x = -INFINITY, x1 = -INFINITY;
     int v = -1;
     if (lane < a.P) {
         v = a.pool_ids[(int64_t)row * a.P + lane];
         x = __fmul_rn(Logit<T>::load1(rp, v), a.invT);
     }
-    const MaxSum ms = warp_maxsum(MaxSum{x, FF{lane < a.P ? 1.f : 0.f, 0.f}});
+    if (lane + 32 < a.P) x1 = __fmul_rn(Logit<T>::load1(rp, a.pool_ids[(int64_t)row * a.P + lane + 32]), a.invT);
+    const MaxSum ms = warp_maxsum(maxsum_merge(MaxSum{x, FF{lane < a.P ? 1.f : 0.f, 0.f}},
+                                               MaxSum{x1, FF{lane + 32 < a.P ? 1.f : 0.f, 0.f}}));
     if (lane == 0) {
         const FF l = maxsum_lse(ms);
         a.lse[row] = make_float2(l.hi, l.lo);
@@ -92,21 +94,25 @@ __global__ void __launch_bounds__(128) k_replay_pooled(ReplayPoolArgs a) {
         return;
     }
     const T *row = static_cast<const T *>(a.q) + (int64_t)b * a.bstride + (int64_t)r * a.rstride;
-    uint64_t key = 0ull;
-    if (lane < a.P) {
-        const int v = a.pool_ids[((int64_t)b * a.L + d) * a.P + lane];
+    uint64_t key[2] = {0ull, 0ull};  // pool entries lane and lane + 32
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+        const int j = lane + 32 * h;
+        if (j >= a.P) continue;
+        const int v = a.pool_ids[((int64_t)b * a.L + d) * a.P + j];
         if (v >= 0 && v < a.V) {
             const float g = __fadd_rn(__fmul_rn(Logit<T>::load1(row, v), a.invT),
                                       gumbel_of(draw_word(a.seed, kReplayElem, (uint32_t)b, (uint32_t)u, (uint32_t)v)));
-            key = pack_key(g, (uint32_t)v);
+            key[h] = pack_key(g, (uint32_t)v);
         } else {
             raise_status(a.status, kDevBadIndex);
         }
     }
     const int32_t *kids = a.child_ids + (int64_t)b * a.N + o;
     for (int s = 0; s < m; ++s) {  // the s-th largest key fills child slot s
-        const uint64_t best = warp_max_u64(key);
-        if (key == best) key = 0ull;  // keys are distinct (token ids)
+        const uint64_t best = warp_max_u64(key[0] > key[1] ? key[0] : key[1]);
+        if (key[0] == best) key[0] = 0ull;  // keys are distinct (token ids)
+        if (key[1] == best) key[1] = 0ull;
         if (lane == 0) {
             const int child = kids[s];
             if (best != 0ull && child > 0 && child < NN)
@@ -304,28 +310,33 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
             final_tok = -1;
             break;
         }
-        float P0 = 0.f, Q = 0.f;  // warp 0, lane j: pool entry j
+        float P0[2] = {0.f, 0.f}, Q[2] = {0.f, 0.f};  // warp 0, lane j: pool entries j and j + 32
         if (warp == 0) {
             const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
-            int v = -1;
-            float xt = -INFINITY, xq = -INFINITY;
-            if (lane < a.P) {
-                v = a.pool_ids[((int64_t)b * a.L + d) * a.P + lane];
+            float xt[2] = {-INFINITY, -INFINITY}, xq[2] = {-INFINITY, -INFINITY};
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                const int j = lane + 32 * h;
+                if (j >= a.P) continue;
+                int v = a.pool_ids[((int64_t)b * a.L + d) * a.P + j];
                 if (v < 0 || v >= a.V) {
                     raise_status(a.status, kDevBadIndex);
                     v = 0;
                 }
-                xt = __fmul_rn(Logit<T>::load1(trow, v), a.invT);
-                xq = __fmul_rn(Logit<T>::load1(qrow, v), a.invT);
-                sh.pool[lane] = v;
+                xt[h] = __fmul_rn(Logit<T>::load1(trow, v), a.invT);
+                xq[h] = __fmul_rn(Logit<T>::load1(qrow, v), a.invT);
+                sh.pool[j] = v;
             }
             __syncwarp();  // sh.pool is read by lane 0 below
-            const MaxSum mq = warp_maxsum(MaxSum{xq, FF{lane < a.P ? 1.f : 0.f, 0.f}});
+            const MaxSum mq = warp_maxsum(maxsum_merge(MaxSum{xq[0], FF{lane < a.P ? 1.f : 0.f, 0.f}},
+                                                       MaxSum{xq[1], FF{lane + 32 < a.P ? 1.f : 0.f, 0.f}}));
             const FF L2q = ff_times_log2e(maxsum_lse(mq));
-            if (lane < a.P) {
-                P0 = exp_shifted(xt, sh.L2t);
-                Q = exp_shifted(xq, L2q);
-            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h)
+                if (lane + 32 * h < a.P) {
+                    P0[h] = exp_shifted(xt[h], sh.L2t);
+                    Q[h] = exp_shifted(xq[h], L2q);
+                }
             if (lane == 0) {  // distinct chunks of the pool tokens
                 int n = 0;
                 for (int j = 0; j < a.P; ++j) {
@@ -374,8 +385,8 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
         // 5. the sibling tests on the pool entries (warp 0): lane j holds the current law on
         //    pool entry j; outside the pool the law is the target's times out / mout
         if (warp == 0) {
-            float cur = lane < a.P ? P0 : 0.f, out = sh.mout, t = 1.f;
-            bool drawn = false;
+            float cur[2] = {lane < a.P ? P0[0] : 0.f, lane + 32 < a.P ? P0[1] : 0.f}, out = sh.mout, t = 1.f;
+            bool drawn[2] = {false, false};
             int mode = 0, next = -1;
             for (int i = 0; i < m; ++i) {
                 const int c = ids[o + i];
@@ -385,13 +396,16 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
                     break;
                 }
                 const int y = a.token[(int64_t)b * NN + c];
-                const unsigned hit = __ballot_sync(kFull, lane < a.P && sh.pool[lane] == y);
-                const int k = hit ? __ffs(hit) - 1 : -1;
+                const unsigned hit0 = __ballot_sync(kFull, lane < a.P && sh.pool[lane] == y);
+                const unsigned hit1 = __ballot_sync(kFull, lane + 32 < a.P && sh.pool[lane + 32] == y);
+                const int k = hit0 ? __ffs(hit0) - 1 : (hit1 ? 32 + __ffs(hit1) - 1 : -1);
                 // (k is uniform over the warp: every lane takes the same branch)
                 float qk = 0.f, pk = 0.f;
                 if (k >= 0) {
-                    qk = __shfl_sync(kFull, Q, k);
-                    pk = __shfl_sync(kFull, cur, k);
+                    const float q0 = __shfl_sync(kFull, Q[0], k & 31), q1 = __shfl_sync(kFull, Q[1], k & 31);
+                    const float c0 = __shfl_sync(kFull, cur[0], k & 31), c1 = __shfl_sync(kFull, cur[1], k & 31);
+                    qk = k < 32 ? q0 : q1;
+                    pk = k < 32 ? c0 : c1;
                 } else if (y >= 0 && y < a.V && sh.mout > 0.f) {  // outside the pool: q = 0
                     const float py = exp_shifted(__fmul_rn(Logit<T>::load1(trow, y), a.invT), sh.L2t);
                     pk = __fmul_rn(__fdiv_rn(out, sh.mout), py);
@@ -403,22 +417,31 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
                     break;
                 }
                 // reject: R = max(cur - [not drawn] Q / t, 0) on the pool, unchanged outside
-                const float qt = t > 0.f ? __fdiv_rn(Q, t) : 0.f;
-                const float R = lane < a.P ? fmaxf(__fsub_rn(cur, drawn ? 0.f : qt), 0.f) : 0.f;
-                const float Z = __fadd_rn(warp_sum(R), out);
+                float Rr[2];
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    const float qt = t > 0.f ? __fdiv_rn(Q[h], t) : 0.f;
+                    Rr[h] = lane + 32 * h < a.P ? fmaxf(__fsub_rn(cur[h], drawn[h] ? 0.f : qt), 0.f) : 0.f;
+                }
+                const float Z = __fadd_rn(warp_sum(__fadd_rn(Rr[0], Rr[1])), out);
                 if (!(Z > 0.f)) {  // no residual mass (rounding only): draw from the target row
                     mode = 2;
                     break;
                 }
                 if (i == m - 1) {  // every slot rejected: draw from the residual R
-                    if (lane < a.P) sh.rj[lane] = R;
+#pragma unroll
+                    for (int h = 0; h < 2; ++h)
+                        if (lane + 32 * h < a.P) sh.rj[lane + 32 * h] = Rr[h];
                     if (lane == 0) sh.scale = sh.mout > 0.f ? __fdiv_rn(out, sh.mout) : 0.f;
                     mode = 1;
                     break;
                 }
-                cur = __fdiv_rn(R, Z);
+#pragma unroll
+                for (int h = 0; h < 2; ++h) {
+                    cur[h] = __fdiv_rn(Rr[h], Z);
+                    drawn[h] |= lane + 32 * h == k;
+                }
                 out = __fdiv_rn(out, Z);
-                drawn |= lane == k;
                 t = __fsub_rn(t, qk);
             }
             if (lane == 0) {
@@ -450,6 +473,156 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
     }
 }
 
+// ---------------------------------------------------------------------------------------
+// Pools of P = 33..64 tokens (the first pass's per-row top-P above the 32 the top-K pass of
+// the first pass keeps): one CTA per draft row, exact (x desc, id asc) through the unique
+// 64-bit keys pack_key(x, id). tau = the P-th largest chunk maximum (a bitonic sort of the
+// row's chunk keys from its statistics) bounds the P-th largest logit from below, so the
+// pool is among the logits >= tau of the chunks whose maximum reaches tau. Those keys are
+// collected into shared memory and sorted; when more than kSelCap of them reach tau (flat
+// rows, heavy ties), a most-significant-digit radix pass over the keys (8 bits at a time,
+// counting only keys above the current threshold) first raises the threshold to the top of
+// the digit bucket that holds the P-th key, until at most kSelCap keys remain.
+constexpr int kSelThreads = 256;
+constexpr int kSelCap = 4096;  // candidate keys held in shared memory
+
+struct SelectArgs {
+    const void *draft;
+    int64_t bstride, rstride;
+    const float2 *stats;  // [B][R][C]
+    int R, L, C, V, P;
+    float invT;
+    int32_t *pool_ids;  // [B*L][P]
+};
+
+// Bitonic sort of keys[0, m) into descending order (m a power of two, empty slots hold 0).
+__device__ void bitonic_desc(uint64_t *keys, int m) {
+    for (int k = 2; k <= m; k <<= 1)
+        for (int j = k >> 1; j > 0; j >>= 1) {
+            for (int i = threadIdx.x; i < m; i += kSelThreads) {
+                const int ixj = i ^ j;
+                if (ixj > i) {
+                    const uint64_t x = keys[i], y = keys[ixj];
+                    if ((i & k) == 0 ? x < y : x > y) {
+                        keys[i] = y;
+                        keys[ixj] = x;
+                    }
+                }
+            }
+            __syncthreads();
+        }
+}
+
+struct SelShared {
+    int n, nch, sel;
+    unsigned long long prefix, mask, above, cnt;
+    int hist[256];
+};
+
+// Calls f(key) for every logit of the row whose key is >= thr (one warp per chunk whose
+// maximum reaches the threshold's value). All threads call it; ends with a barrier.
+template <typename T, typename F>
+__device__ void for_keys_above(const SelectArgs &a, const T *row, const float2 *st, int *chunks, SelShared &sh,
+                               uint64_t thr, F f) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    constexpr int NW = kSelThreads / 32;
+    if (threadIdx.x == 0) sh.nch = 0;
+    __syncthreads();
+    const uint32_t hi = (uint32_t)(thr >> 32);
+    for (int c = threadIdx.x; c < a.C; c += kSelThreads)
+        if (ord_f32(st[c].x) >= hi) chunks[atomicAdd(&sh.nch, 1)] = c;
+    __syncthreads();
+    const int nch = sh.nch;
+    for (int i = warp; i < nch; i += NW) {
+        const int v0 = chunks[i] * kChunk + lane * 8;
+        float x[8];
+        Logit<T>::load8(row, v0, a.V, x);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            if (v0 + e >= a.V) continue;
+            const uint64_t key = pack_key(__fmul_rn(x[e], a.invT), (uint32_t)(v0 + e));
+            if (key >= thr) f(key);
+        }
+    }
+    __syncthreads();
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kSelThreads) k_pool_select(SelectArgs a) {
+    pdl_begin();
+    extern __shared__ __align__(16) unsigned char smem[];
+    uint64_t *keys = reinterpret_cast<uint64_t *>(smem);           // [kSelCap]
+    float2 *st = reinterpret_cast<float2 *>(keys + kSelCap);        // [C]
+    int *chunks = reinterpret_cast<int *>(st + a.C);                // [C]
+    __shared__ SelShared sh;
+    const int row = blockIdx.x;
+    const int b = row / a.L, d = row - (row / a.L) * a.L;
+    const T *rp = static_cast<const T *>(a.draft) + (int64_t)b * a.bstride + (int64_t)d * a.rstride;
+    const float2 *gst = a.stats + ((int64_t)b * a.R + d) * a.C;
+    for (int c = threadIdx.x; c < a.C; c += kSelThreads) st[c] = __ldg(&gst[c]);
+    int mc = 1;
+    while (mc < a.C) mc <<= 1;  // <= kSelCap: C <= TSB_MAX_V / 256 = 1600
+    __syncthreads();
+    // 1. tau from the P-th largest chunk key
+    for (int i = threadIdx.x; i < mc; i += kSelThreads) keys[i] = i < a.C ? pack_key(st[i].x, (uint32_t)i) : 0ull;
+    __syncthreads();
+    bitonic_desc(keys, mc);
+    uint64_t thr = a.C >= a.P ? (keys[a.P - 1] >> 32) << 32 : 0ull;  // every key of x >= tau
+    __syncthreads();
+    // 2. the keys above the threshold, raising it first if more than kSelCap reach it
+    for (int round = 0; round < 2; ++round) {
+        if (threadIdx.x == 0) sh.n = 0;
+        __syncthreads();
+        for_keys_above<T>(a, rp, st, chunks, sh, thr, [&](uint64_t k) {
+            const int i = atomicAdd(&sh.n, 1);
+            if (i < kSelCap) keys[i] = k;
+        });
+        if (sh.n <= kSelCap) break;  // uniform: read after the barrier that ends the scan
+        if (threadIdx.x == 0) {
+            sh.prefix = 0ull;
+            sh.mask = 0ull;
+            sh.above = 0ull;
+            sh.cnt = ~0ull;
+        }
+        for (int shift = 56; shift >= 0; shift -= 8) {
+            for (int i = threadIdx.x; i < 256; i += kSelThreads) sh.hist[i] = 0;
+            __syncthreads();
+            const uint64_t pre = sh.prefix, msk = sh.mask;
+            for_keys_above<T>(a, rp, st, chunks, sh, thr, [&](uint64_t k) {
+                if ((k & msk) == pre) atomicAdd(&sh.hist[(int)((k >> shift) & 255ull)], 1);
+            });
+            if (threadIdx.x == 0) {
+                unsigned long long cum = 0ull;
+                int bin = 0;
+                for (int j = 255; j >= 0; --j) {
+                    if (sh.above + cum + (unsigned long long)sh.hist[j] >= (unsigned long long)a.P) {
+                        bin = j;
+                        break;
+                    }
+                    cum += (unsigned long long)sh.hist[j];
+                }
+                sh.above += cum;
+                sh.prefix |= (unsigned long long)bin << shift;
+                sh.mask |= 0xFFull << shift;
+                sh.cnt = sh.above + (unsigned long long)sh.hist[bin];
+            }
+            __syncthreads();
+            if (sh.cnt <= (unsigned long long)kSelCap) break;  // uniform
+        }
+        thr = sh.prefix > thr ? sh.prefix : thr;
+        __syncthreads();
+    }
+    // 3. the top P by (x desc, id asc)
+    const int n = min(sh.n, kSelCap);
+    int m = 1;
+    while (m < n) m <<= 1;
+    for (int i = n + threadIdx.x; i < m; i += kSelThreads) keys[i] = 0ull;
+    __syncthreads();
+    bitonic_desc(keys, m);
+    for (int j = threadIdx.x; j < a.P; j += kSelThreads)
+        a.pool_ids[(int64_t)row * a.P + j] = j < n ? (int32_t)key_id(keys[j]) : -1;
+}
+
 }  // namespace
 
 cudaError_t launch_pool_finish(const RowsDesc &draft, int L, int K, int P, float invT, const int32_t *pool_ids,
@@ -471,6 +644,34 @@ cudaError_t launch_pool_finish(const RowsDesc &draft, int L, int K, int P, float
     const dim3 grid((unsigned)((a.rows + 3) / 4));
     return draft.dtype == 1 ? launch_pdl(k_pool_finish<__nv_bfloat16>, grid, dim3(128), 0, s, 0, a)
                             : launch_pdl(k_pool_finish<float>, grid, dim3(128), 0, s, 0, a);
+}
+
+cudaError_t launch_pool_select(const RowsDesc &draft, const float2 *stats, int L, int P, float invT,
+                               int32_t *pool_ids, cudaStream_t s) {
+    SelectArgs a;
+    a.draft = draft.data;
+    a.bstride = draft.batch_stride;
+    a.rstride = draft.row_stride;
+    a.stats = stats;
+    a.R = draft.R;
+    a.L = L;
+    a.C = num_chunks(draft.V);
+    a.V = draft.V;
+    a.P = P;
+    a.invT = invT;
+    a.pool_ids = pool_ids;
+    if (a.C > kSelCap || P > kSelCap) return cudaErrorInvalidValue;
+    const size_t smem = (size_t)kSelCap * sizeof(uint64_t) + (size_t)a.C * (sizeof(float2) + sizeof(int));
+    const dim3 grid((unsigned)(draft.B * L));
+    if (draft.dtype == 1) {
+        cudaError_t e = cudaFuncSetAttribute(k_pool_select<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
+        return launch_pdl(k_pool_select<__nv_bfloat16>, grid, dim3(kSelThreads), smem, s, 0, a);
+    }
+    cudaError_t e = cudaFuncSetAttribute(k_pool_select<float>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_pool_select<float>, grid, dim3(kSelThreads), smem, s, 0, a);
 }
 
 cudaError_t launch_replay_pooled(const RowsDesc &q, const int32_t *qrow_of_node, int B, int N, int L, int P,

@@ -102,6 +102,9 @@ cudaError_t launch_plan_pooled(const RowsDesc &draft, const float2 *stats, int L
                                int32_t *pool_ids, const TreeDesc &tree, void *ws, cudaStream_t s);
 cudaError_t launch_pool_finish(const RowsDesc &draft, int L, int K, int P, float invT, const int32_t *pool_ids,
                                float2 *lse, float *topk_x, int32_t *topk_id, uint32_t *status, cudaStream_t s);
+cudaError_t launch_pool_select(const RowsDesc &draft, const float2 *stats, int L, int P, float invT,
+                               int32_t *pool_ids, cudaStream_t s);
+
 cudaError_t launch_replay_pooled(const RowsDesc &q, const int32_t *qrow_of_node, int B, int N, int L, int P,
                                  const TreeDesc &tree, const int32_t *pool_ids, float invT, uint64_t seed,
                                  int32_t *token, uint32_t *status, cudaStream_t s);

@@ -32,7 +32,7 @@ EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_by
 TSB_NOALLOC_SCRATCH_BYTES = 1 << 20
 TSB_MAX_WIDTH = 1024
 TSB_MAX_EXPAND_CANDIDATES = 8192
-TSB_MAX_POOL = 32
+TSB_MAX_POOL = 64
 
 
 class TsbError(RuntimeError):

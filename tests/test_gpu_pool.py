@@ -73,7 +73,8 @@ def pooled_step(draft, L, N, K, P, T, seed, target_noise, qrows=None, qrow_of_no
 
 
 @pytest.mark.parametrize("wl,V,B,P,dtype", [("batched", 151936, 16, 16, "bf16"), ("batched", 128256, 16, 8, "bf16"),
-                                            ("tiny", 32, 256, 6, "f32"), ("single", 151936, 4, 32, "bf16")])
+                                            ("tiny", 32, 256, 6, "f32"), ("single", 151936, 4, 32, "bf16"),
+                                            ("batched", 151936, 16, 64, "bf16"), ("single", 151936, 4, 33, "bf16")])
 def test_pooled_step(wl, V, B, P, dtype):
     w = synth.WORKLOADS[wl]
     draft = _draft(B, w["L"], V, "planted" if V > 100 else "normal2", dtype, 1401)
@@ -104,13 +105,45 @@ def test_pooled_edges():
     rep, _, _ = pooled_step(_draft(16, 3, 24, "normal2", "f32", 1404), 3, 12, 3, 24, 1.0, seed=4, target_noise=1.0)
 
 
-def test_pooled_losslessness_on_gpu():
-    """1e5 trees share the tiny workload's rows, target rows keyed by the token path: the first
-    emitted token follows the root's target law, and the GPU matches the oracle where it flags
-    no near tie."""
+@pytest.mark.parametrize("V,P", [(5003, 64), (700, 40), (151936, 48)])
+def test_pool_selection_degenerate_rows(V, P):
+    """Pools above 32 tokens on rows that defeat the chunk bound: a flat row (every logit ties,
+    so every chunk reaches tau), a maximum repeated 300 times, a vocabulary with fewer chunks
+    than P (every logit is a candidate), and random rows; bit-exact against the host's stable
+    sort by (x desc, id asc)."""
+    B, L, K, N = 2, 4, 4, 12
+    g = torch.Generator().manual_seed(V + P)
+    z = torch.randn(B, L, V, generator=g) * 3
+    z[0, 0] = 0.25  # flat
+    pos = torch.randperm(V, generator=g)[:min(300, V)]
+    z[0, 1, pos] = z[0, 1].max() + 1.0  # repeated maximum
+    z[1, 2, :V // 2] = 1.5  # half the row tied
+    stride = (V + 7) // 8 * 8
+    store = torch.zeros(B, L, stride, dtype=torch.float32)
+    store[..., :V] = z
+    draft = store.to(DEV)[..., :V]
+    buf = tsb.TsbBuffers.allocate(B, L, N, K, V, 1.0, device=DEV)
+    pools = torch.empty(B, L, P, dtype=torch.int32, device=DEV)
+    tsb.tsb_row_stats(draft, 1.0, buf.stats, buf.ws)
+    tsb.tsb_plan_pooled(buf.cfg, P, draft, buf.stats, pools, buf.tree, buf.ws)
+    check_status(buf)
+    got = pools.cpu().numpy()
+    x = z.numpy().astype(np.float32)
+    for b in range(B):
+        for d in range(L):
+            want = np.lexsort((np.arange(V), -x[b, d]))[:P]
+            assert np.array_equal(got[b, d], want), (b, d)
+
+
+@pytest.mark.parametrize("V,P", [(32, 8), (1000, 64)])
+def test_pooled_losslessness_on_gpu(V, P):
+    """1e5 trees share one set of draft rows, target rows keyed by the token path: the first
+    emitted token follows the root's target law (and the second token, extended by a target
+    draw, the law after the first), and a sample of the trees matches the oracle. At V = 1000
+    the pools hold 64 tokens (two per lane) across four chunks."""
     w = synth.WORKLOADS["tiny"]
-    B, L, N, K, V, T, P = 100_000, w["L"], w["N"], w["K"], w["V"], w["T"], 8
-    base1 = _draft(1, L, V, "normal2", "f32", 1000)
+    B, L, N, K, T = 100_000, w["L"], w["N"], w["K"], w["T"]
+    base1 = _draft(1, L, V, "normal2", "f32", 1000 + V)
     draft = base1.expand(B, -1, -1)
     buf = tsb.TsbBuffers.allocate(B, L, N, K, V, T, device=DEV)
     pools = torch.empty(B, L, P, dtype=torch.int32, device=DEV)
@@ -122,17 +155,39 @@ def test_pooled_losslessness_on_gpu():
     tree = {k: v.cpu().numpy() for k, v in buf.tree.items()}
     tok = buf.token.cpu().numpy()
     base = synth.to_host(base1)[0]
-    target = torch.from_numpy(synth.path_keyed_rows(base, tree["parent"], tree["depth"], tok, 1.0, seed=79)).to(DEV)
+    target = synth.path_keyed_rows_device(base1[0].contiguous(), tree["parent"], tree["depth"], tok, 1.0, seed=79)
     tsb.tsb_verify_pooled(buf.cfg, P, target, draft, None, pools, buf.tree, buf.token, seed, buf.out_tokens,
                           buf.out_nodes, buf.out_len, buf.ws)
     check_status(buf)
-    first = buf.out_tokens[:, 0].cpu().numpy()
+    out = {"len": buf.out_len.cpu().numpy(), "tokens": buf.out_tokens.cpu().numpy(),
+           "nodes": buf.out_nodes.cpu().numpy()}
+    first = out["tokens"][:, 0]
     p_root = helpers.softmax64(synth.path_keyed_row(base, [], 1.0, 79))
     assert helpers.chi2_pvalue(np.bincount(first, minlength=V), p_root) > 1e-4
-    h_draft = np.ascontiguousarray(np.broadcast_to(base[None], (B, L, V)))
-    ref = oracle.plan(h_draft, T, N, K, L, pool=P)
-    ref_pools = np.ascontiguousarray(oracle.pools(h_draft[:1], T, P)[:, :L].repeat(B, axis=0))
-    rtok, rex = oracle.replay_pooled(h_draft, T, ref, seed, ref_pools)
-    rt = synth.path_keyed_rows(base, ref["parent"], ref["depth"], rtok, 1.0, seed=79)
-    rout = oracle.verify_rrs(rt, h_draft, T, ref, rtok, seed, L, pool_ids=ref_pools)
-    compare_trials(buf, tok, rtok, rex, rout)
+    second = out["tokens"][:, 1].copy()
+    ext = np.random.default_rng(P)
+    vals, cnt = np.unique(first, return_counts=True)
+    for a in vals[np.argsort(-cnt)][:2]:
+        sel = first == a
+        pa = helpers.softmax64(synth.path_keyed_row(base, [int(a)], 1.0, 79))
+        short = sel & (out["len"] == 1)
+        second[short] = ext.choice(V, size=int(short.sum()), p=pa)
+        assert helpers.chi2_pvalue(np.bincount(second[sel], minlength=V), pa) > 1e-4
+    # the oracle on a sample of the trees, with their own batch indices
+    sel = list(range(0, B, B // 1500))[:1500]
+    bids = np.array(sel, dtype=np.int32)
+    h1 = synth.to_host(base1)
+    ref1 = oracle.plan(h1, T, N, K, L, pool=P)
+    for k in ("parent", "child_off", "child_ids"):
+        assert np.array_equal(ref1[k][0], tree[k][0]), k
+    ref = helpers.repeat_tree({k: v for k, v in ref1.items() if k not in ("exempt", "min_margin")}, len(sel))
+    hq = np.ascontiguousarray(np.broadcast_to(h1, (len(sel),) + h1.shape[1:]))
+    ref_pools = np.ascontiguousarray(oracle.pools(h1, T, P)[:, :L].repeat(len(sel), axis=0))
+    assert np.array_equal(pools.cpu().numpy()[0], ref_pools[0])
+    rtok, rex = oracle.replay_pooled(hq, T, ref, seed, ref_pools, batch_ids=bids)
+    rep = Report()
+    same = compare_tokens(tok, rtok, rex, tree, dict.fromkeys(sel, True), rep, sel)
+    rout = oracle.verify_rrs(synth.to_host(target[sel].contiguous()), hq, T, ref, rtok, seed, L, batch_ids=bids,
+                             pool_ids=ref_pools)
+    compare_verify(out, rout, same, rep, sel)
+    rep.check()
