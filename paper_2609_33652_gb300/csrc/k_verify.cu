@@ -26,21 +26,24 @@
 // with the two-level Gumbel-max of the randomness contract: chunk keys log(chunk mass) + G
 // over chunks of 256 tokens, then the best token of the winning chunk.
 //
-// Scheduling. A pre-pass kernel (all SMs, bandwidth-bound) computes the target
-// log-normaliser of the M highest-scoring nodes (ids below M, pop order) and, for per-depth
-// q rows, every q row's log-normaliser. The walk kernel copies the tree's topology, the
-// children's target and q logits and their acceptance uniforms to shared memory once. At a
-// node below M it needs no staging and no cluster round: every CTA takes the same decisions
-// from the same inputs, and the slice is staged only if a rejection needs the residual. At
-// any other node every warp stages the target slice in the chunk-statistics layout (x into
-// shared memory, each chunk's statistics beside it), every CTA gathers all chunk statistics
-// of the row through distributed shared memory and computes its log-normaliser, while warp
-// kQWarp computes a per-node q row's log-normaliser from its chunk statistics. 12 warps per
-// CTA: 160 registers a thread without spills (16 warps at 128 spilled in the walk's
-// hot paths and ran slower). Element passes give lane l the elements
-// 4l..4l+3 and 128+4l..128+4l+3 of each 256-token chunk, so every shared-memory access is a
-// conflict-free 16-byte vector. Which path computes a node's normaliser depends only on its
-// id, so results do not depend on timing.
+// Scheduling. A pre-pass kernel (all SMs) computes the target log-normalisers of the nodes a
+// walk is most likely to visit, the first kPreChain internal nodes of the first-child chain
+// from the root (slot 0 is accepted at most visits), and the q rows' log-normalisers (per
+// depth, or per internal node for per-node rows). The walk kernel copies the tree's topology,
+// the children's target and q logits and their acceptance uniforms to shared memory once. At
+// a node with a known normaliser it needs no staging and no cluster round: every CTA takes
+// the same decisions from the same inputs, and the slices are staged only if a rejection needs
+// the residual. At any other node the walk runs a staging round over that node and up to
+// kLook - 1 of its first-child descendants without a value: every warp streams the rows'
+// slices in the chunk-statistics layout (the node's x into shared memory, each chunk's
+// statistics beside it), every CTA gathers all chunk statistics of the rows through
+// distributed shared memory and computes their log-normalisers, one group of four warps per
+// row. 12 warps per CTA: 160 registers a thread without spills (16 warps at 128 spilled in
+// the walk's hot paths and ran slower). Element passes give lane l the elements 4l..4l+3 and
+// 128+4l..128+4l+3 of each 256-token chunk, so every shared-memory access is a conflict-free
+// 16-byte vector. Every normaliser comes from the same two functions over the row's chunk
+// statistics, whichever kernel computes it, and which nodes are pre-computed depends only on
+// the topology, so results do not depend on timing.
 #include <cooperative_groups.h>
 
 #include <mutex>
@@ -55,18 +58,25 @@ namespace {
 
 constexpr int kThreads = 384;
 constexpr int kWarps = kThreads / 32;
-constexpr int kQWarp = 10;            // q-row log-normaliser
 constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
-constexpr int kPreTop = 8;            // highest-scoring node ids the pre-pass covers
 constexpr int kMaxDepthRows = 64;     // per-depth q rows (depth cap L <= 64)
 constexpr int kPreThreads = 512;
+// Rows per staging round of the RRS walk: the node being visited and up to kLook - 1 of its
+// first-child descendants (the children a walk most often accepts next), whose target
+// log-normalisers the same round computes with the loads of all rows in flight together.
+constexpr int kLook = 3;
+// Internal nodes of the first-child chain from the root whose target normalisers the RRS
+// pre-pass computes on the whole GPU (the walk starts on that chain; nodes a walk reaches off it
+// are staged by the walk's own rounds).
+constexpr int kPreChain = 8;
+static_assert(kWarps % 4 == 0 && kLook <= kWarps, "groups of four warps per normaliser");
 
 // Pre-pass results, one 32-byte workspace slot per (tree, node) (the slots block
 // verification uses for its own per-position scalars): l2t = target log-normaliser of node u
-// (u in the pre-computed set), l2q = log-normaliser of per-depth q row u; both float-float,
-// times log2(e). Pre-computed set of a tree: its internal nodes with ids below kPreTop (the
-// highest-scoring nodes in pop order; the root is visited by every walk). Measured on the
-// batched workload, covering the first-child chain as well cost more bandwidth than it saved.
+// (u in the pre-computed set), l2q = log-normaliser of per-depth q row u, or of node u's own q
+// row for per-node rows; both float-float, times log2(e). Pre-computed set of a tree: for
+// recursive rejection sampling the first kPreChain internal nodes of the first-child chain,
+// for traversal verification every internal node.
 struct alignas(16) PreRow {
     float2 l2t, l2q;
     float pad[4];
@@ -89,7 +99,9 @@ struct VerifyArgs {
     int32_t *out_tokens, *out_nodes, *out_len;
     uint32_t *status;
     PreRow *pre;  // [B, N+1]
-    int M;        // node ids below M with children are pre-computed
+    int M;        // node ids below M with children are pre-computed (pre_chain == 0), or
+                  // the first M internal nodes of the first-child chain (pre_chain == 1)
+    int pre_chain;
     int Lq;       // per-depth q rows whose normaliser the pre-pass computes (0 for per-node rows)
     int qn;       // 1: the pre-pass computes each internal node's per-node q-row normaliser (slot u)
     int B;
@@ -152,7 +164,10 @@ struct Scratch {
     int path[kMaxDepthRows];      // accepted node ids (written out after the walk)
     float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
     FF l2q[kMaxDepthRows];        // per-depth q log-normalisers (times log2 e)
-    float2 cst[2][kMaxSliceChunks];  // chunk statistics of the slice, alternating per staged node
+    float2 cst[2][kLook][kMaxSliceChunks];  // chunk statistics of the slice's rows, alternating per round
+    Slot lpart[kLook][4];                   // per-warp partials of the round's normalisers
+    int look[kLook];                        // nodes of the current staging round
+    int nlook;
 };
 
 // One cluster-wide reduction: warp reductions, the CTA's warp partials in warp 0, the
@@ -191,17 +206,17 @@ __device__ __forceinline__ void st4(float *p, int j, float a, float b, float c, 
 }
 
 // A row's log-normaliser from its chunk statistics (m_c, s_c) in shared memory, over a fixed
-// partition: thread t < 128 takes chunks t, t + 128, ... (their maximum, then a Kahan sum of
+// partition: thread t < 128 of a group of four warps takes chunks t, t + 128, ... (their maximum, then a Kahan sum of
 // s_c e^(m_c - m)), each of warps 0..3 merges its lanes (lse_part), and warp 0 merges the
 // four warps in order (lse_final, result times log2 e). Every kernel that needs a target
 // row's normaliser calls these two functions, kept out of line, so the value does not depend
 // on which kernel or CTA computed it.
-__device__ __noinline__ Slot lse_part(const float2 *pst, int C) {
+__device__ __noinline__ Slot lse_part(const float2 *pst, int C, int t) {
     float m = -INFINITY;
-    for (int c = threadIdx.x; c < C; c += 128) m = fmaxf(m, pst[c].x);
+    for (int c = t; c < C; c += 128) m = fmaxf(m, pst[c].x);
     KahanF acc;
     if (m != -INFINITY)
-        for (int c = threadIdx.x; c < C; c += 128) acc.add(__fmul_rn(pst[c].y, expf(__fsub_rn(pst[c].x, m))));
+        for (int c = t; c < C; c += 128) acc.add(__fmul_rn(pst[c].y, expf(__fsub_rn(pst[c].x, m))));
     Slot mine = neutral_slot();
     const FF sv = acc.ff();
     mine.m = m;
@@ -269,41 +284,48 @@ struct Walk {
         }
     }
 
-    // Stage this CTA's slice of `row` in the chunk-statistics layout (eight lanes per 256-logit
-    // chunk, lane g holding logits 8g..8g+7 of each 64-logit quarter; four chunks per warp and
-    // unit, two units in flight for bf16): the statistics of every chunk of the slice into
-    // cst[] (the per-chunk code of the statistics kernels) and, with dst, x = fp32(z) * invT
-    // into dst (logits past the vocabulary become -inf). Every warp takes part.
-    __device__ void stage_chunks(const T *row, float *dst, float2 *cst) {
+    // One staging round over the rows of nodes sh.look[0..J-1] (target rows), in the
+    // chunk-statistics layout (eight lanes per 256-logit chunk, lane g holding logits
+    // 8g..8g+7 of each 64-logit quarter; four chunks per warp and unit): the statistics of
+    // every chunk of this CTA's slice of row j into cst[j] (the per-chunk code of the
+    // statistics kernels) and x = fp32(z) * invT of row 0 into dst (logits past the vocabulary
+    // become -inf). The (row, unit) pairs are dealt to the warps in one sequence, kU pairs in
+    // flight per warp, so the loads of all J rows are issued together. Every warp takes part.
+    __device__ void stage_look(int J, float *dst, float2 (*cst)[kMaxSliceChunks]) {
         constexpr int kU = sizeof(T) == 2 ? 2 : 1;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int g = lane & 7, q = lane >> 3;
-        const int units = (nch + 3) / 4;
-        for (int u0 = warp; u0 < units; u0 += kU * kWarps) {  // uniform over the warp
+        const int units = (nch + 3) / 4, total = J * units;
+        for (int i0 = warp; i0 < total; i0 += kU * kWarps) {  // uniform over the warp
             RawGroup<T> raw[kU][4];
 #pragma unroll
             for (int e = 0; e < kU; ++e) {
-                const int cl = (u0 + e * kWarps) * 4 + q;
-                if (u0 + e * kWarps < units && cl < nch)
+                const int idx = i0 + e * kWarps;
+                const int j = idx / units, cl = (idx - j * units) * 4 + q;
+                if (idx < total && cl < nch) {
+                    const T *row =
+                        static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)sh.look[j] * a.t_rstride;
 #pragma unroll
                     for (int k = 0; k < 4; ++k) raw[e][k].load(row, lo + cl * kChunk + k * 64 + g * 8, a.V);
+                }
             }
 #pragma unroll
             for (int e = 0; e < kU; ++e) {
-                const int cl = (u0 + e * kWarps) * 4 + q;
-                const bool live = u0 + e * kWarps < units && cl < nch;
+                const int idx = i0 + e * kWarps;
+                const int j = idx / units, cl = (idx - j * units) * 4 + q;
+                const bool live = idx < total && cl < nch;
                 float mc, sc;
                 chunk_stats8<T>(raw[e], live, a.invT, &mc, &sc);
-                if (live && g == 0) cst[cl] = make_float2(mc, sc);
-                if (dst && live) {
+                if (live && g == 0) cst[j][cl] = make_float2(mc, sc);
+                if (live && j == 0) {
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
                         float z[8];
                         raw[e][k].unpack(z);
-                        const int j = cl * kChunk + k * 64 + g * 8;
-                        st4(dst, j, __fmul_rn(z[0], a.invT), __fmul_rn(z[1], a.invT), __fmul_rn(z[2], a.invT),
+                        const int i = cl * kChunk + k * 64 + g * 8;
+                        st4(dst, i, __fmul_rn(z[0], a.invT), __fmul_rn(z[1], a.invT), __fmul_rn(z[2], a.invT),
                             __fmul_rn(z[3], a.invT));
-                        st4(dst, j + 4, __fmul_rn(z[4], a.invT), __fmul_rn(z[5], a.invT), __fmul_rn(z[6], a.invT),
+                        st4(dst, i + 4, __fmul_rn(z[4], a.invT), __fmul_rn(z[5], a.invT), __fmul_rn(z[6], a.invT),
                             __fmul_rn(z[7], a.invT));
                     }
                 }
@@ -311,30 +333,43 @@ struct Walk {
         }
     }
 
-    // The log-normaliser of a row whose chunk statistics every CTA of the cluster has staged
-    // into its cst[] (slice / 256 chunks per CTA): each CTA gathers all of them into `tmp`
-    // through distributed shared memory and computes the value itself (identical in every
-    // CTA); warp kQWarp meanwhile runs `side`. Ends with the value in sh.L2t.
-    template <typename F>
-    __device__ void gather_lse(const float2 *cst, float2 *tmp, F side) {
+    // The log-normalisers of the round's J rows, whose chunk statistics every CTA of the
+    // cluster has staged into its cst[0..J-1] (slice / 256 chunks per CTA and row): each CTA
+    // gathers all of them into `tmp` through distributed shared memory and computes the values
+    // itself, one group of four warps per row over the fixed partition of lse_part, so every
+    // CTA holds identical values. Ends with row j's value (times log2 e) in l2t[sh.look[j]]
+    // and the node marked as known.
+    __device__ void gather_look(int J, float2 (*cst)[kMaxSliceChunks], float2 *tmp, FF *l2t, int32_t *known) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         cluster.sync();  // every CTA's chunk statistics are written
-        const int per = a.slice / kChunk;
-        for (int c = threadIdx.x; c < a.C; c += kThreads) {
-            const int r = c / per;
-            tmp[c] = *cluster.map_shared_rank(&cst[c - r * per], r);
+        const int per = a.slice / kChunk, C = a.C;
+        for (int i0 = threadIdx.x; i0 < J * C; i0 += 4 * kThreads) {  // four remote loads in flight
+            float2 v[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int i = i0 + e * kThreads;
+                if (i < J * C) {
+                    const int j = i / C, c = i - j * C, r = c / per;
+                    v[e] = *cluster.map_shared_rank(&cst[j][c - r * per], r);
+                }
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                if (i0 + e * kThreads < J * C) tmp[i0 + e * kThreads] = v[e];
         }
         __syncthreads();
-        if (warp < 4) {
-            const Slot w = lse_part(tmp, a.C);
-            if (lane == 0) sh.wpart[warp] = w;
-        } else if (warp == kQWarp) {
-            side();
+        const int grp = warp >> 2;
+        for (int j = grp; j < J; j += kWarps / 4) {  // uniform over the warp
+            const Slot w = lse_part(tmp + (size_t)j * C, C, threadIdx.x - 128 * grp);
+            if (lane == 0) sh.lpart[j][warp & 3] = w;
         }
         __syncthreads();
-        if (warp == 0) {
-            const FF L2 = lse_final(sh.wpart);
-            if (lane == 0) sh.L2t = L2;
+        if (warp < J) {
+            const FF L2 = lse_final(sh.lpart[warp]);
+            if (lane == 0) {
+                l2t[sh.look[warp]] = L2;
+                known[sh.look[warp]] = 1;
+            }
         }
         __syncthreads();
     }
@@ -354,32 +389,50 @@ struct Walk {
     template <bool LOGITS, typename F>
     __device__ int draw(int node, F wt) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-        // 1. chunk log-masses, one warp per chunk
-        for (int cl = warp; cl < nch; cl += kWarps) {
-            float v[8];
-            wt(quad_at(cl, 0, lane), v);
-            wt(quad_at(cl, 1, lane), v + 4);
-            float A = -INFINITY;
-            if (LOGITS) {
-                float mx = v[0];
+        // 1. chunk log-masses: eight lanes per chunk (lane g of the group takes quads g, g + 8,
+        //    ..., g + 56), four chunks per warp and iteration
+        {
+            const int g = lane & 7, grp = lane >> 3;
+            for (int c0 = warp * 4; c0 < nch; c0 += kWarps * 4) {  // uniform over the warp
+                const int cl = c0 + grp;
+                const bool live = cl < nch;
+                float v[32];
 #pragma unroll
-                for (int k = 1; k < 8; ++k) mx = fmaxf(mx, v[k]);
-                mx = warp_max(mx);
-                float sm = 0.f;
-                if (mx != -INFINITY) {
-#pragma unroll
-                    for (int k = 0; k < 8; ++k) sm += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
+                for (int k = 0; k < 8; ++k) {
+                    if (live) {
+                        wt(cl * kChunk + 4 * (g + 8 * k), v + 4 * k);
+                    } else {
+                        v[4 * k] = v[4 * k + 1] = v[4 * k + 2] = v[4 * k + 3] = LOGITS ? -INFINITY : 0.f;
+                    }
                 }
-                sm = warp_sum(sm);
-                if (mx != -INFINITY) A = __fadd_rn(mx, logf(sm));
-            } else {
-                float sm = 0.f;
+                float A = -INFINITY;
+                if (LOGITS) {
+                    float mx = v[0];
 #pragma unroll
-                for (int k = 0; k < 8; ++k) sm += v[k];
-                sm = warp_sum(sm);
-                if (sm > 0.f) A = logf(sm);
+                    for (int k = 1; k < 32; ++k) mx = fmaxf(mx, v[k]);
+                    mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 4));
+                    mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
+                    mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
+                    float sm = 0.f;
+                    if (mx != -INFINITY) {
+#pragma unroll
+                        for (int k = 0; k < 32; ++k) sm += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
+                    }
+                    sm += __shfl_xor_sync(kFull, sm, 4);
+                    sm += __shfl_xor_sync(kFull, sm, 2);
+                    sm += __shfl_xor_sync(kFull, sm, 1);
+                    if (mx != -INFINITY) A = __fadd_rn(mx, logf(sm));
+                } else {
+                    float sm = 0.f;
+#pragma unroll
+                    for (int k = 0; k < 32; ++k) sm += v[k];
+                    sm += __shfl_xor_sync(kFull, sm, 4);
+                    sm += __shfl_xor_sync(kFull, sm, 2);
+                    sm += __shfl_xor_sync(kFull, sm, 1);
+                    if (sm > 0.f) A = logf(sm);
+                }
+                if (live && g == 0) sh.clog[cl] = A;
             }
-            if (lane == 0) sh.clog[cl] = A;
         }
         __syncthreads();
         // 2. chunk keys, one thread per chunk, and the CTA's best chunk
@@ -479,6 +532,22 @@ __device__ FF q_log_normaliser(const float2 *st, int C) {
     return S.hi > 0.f ? ff_times_log2e(maxsum_lse(MaxSum{m, S})) : FF{0.f, 0.f};
 }
 
+// Node j of the first-child chain (j = 0 the root): from the root, each step moves to the
+// node's first child while that child has children itself; -1 past the chain's end (or on
+// inconsistent arrays). off / kid: the tree's child lists. The pre-pass and the walk select
+// the chain's nodes with this one function.
+__device__ __forceinline__ int chain_node(const int32_t *off, const int32_t *kid, int N, int j) {
+    int v = 0;
+    for (int k = 0; k < j; ++k) {
+        const int o = off[v];
+        if (o < 0 || o >= N) return -1;
+        const int c = kid[o];
+        if (c < 1 || c > N || off[c + 1] - off[c] <= 0) return -1;
+        v = c;
+    }
+    return off[v + 1] - off[v] > 0 ? v : -1;
+}
+
 // Shared-memory bytes of the tree's copy: per node its pre-computed target log-normaliser
 // (float-float) and whether it has one; topology (child_off [N+2], child_ids [N], token [N+1],
 // q row of node [N+1]); per child slot its parent, target logit, q logit and uniform.
@@ -499,7 +568,7 @@ struct TreeSmem {
 // acceptance uniform, the pre-pass results. Sets sh.cbad on inconsistent tree arrays. Every
 // thread of the CTA calls it; it ends with the CTA synchronised.
 template <typename T>
-__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
+__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth, bool pre_q) {
     const int NN = a.N + 1;
     TreeSmem ts;
     ts.l2t = reinterpret_cast<FF *>(base);
@@ -527,10 +596,17 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
             ts.tok[i] = __ldg(tok + i);
             ts.row[i] = __ldg(row + i);
         }
-        for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
-            const float2 v = a.pre[(int64_t)b * NN + i].l2q;
-            sh.l2q[i] = FF{v.x, v.y};
-        }
+        if (pre_q)
+            for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
+                const float2 v = a.pre[(int64_t)b * NN + i].l2q;
+                sh.l2q[i] = FF{v.x, v.y};
+            }
+        if (a.M > 0 || a.qn)  // every node's slot, in this same round of loads (used for the set below)
+            for (int i = threadIdx.x; i < NN; i += kThreads) {
+                const float4 pr = __ldg(reinterpret_cast<const float4 *>(&a.pre[(int64_t)b * NN + i]));
+                ts.l2t[i] = FF{pr.x, pr.y};
+                ts.l2qn[i] = FF{pr.z, pr.w};
+            }
         if (threadIdx.x == 0) sh.cbad = 0;
     }
     __syncthreads();
@@ -549,16 +625,13 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
         if (bad_here) sh.cbad = 1;
     }
     __syncthreads();
-    for (int u = threadIdx.x; u < NN; u += kThreads) {  // the pre-computed set, as the pre-pass saw it
-        const bool p = u < a.M && ts.off[u + 1] - ts.off[u] > 0;
-        ts.pre[u] = p ? 1 : 0;
-        if (p) {
-            const float2 v = a.pre[(int64_t)b * NN + u].l2t;
-            ts.l2t[u] = FF{v.x, v.y};
-            if (a.qn) {
-                const float2 w = a.pre[(int64_t)b * NN + u].l2q;
-                ts.l2qn[u] = FF{w.x, w.y};
-            }
+    for (int u = threadIdx.x; u < NN; u += kThreads)  // the pre-computed set, as the pre-pass saw it
+        ts.pre[u] = !a.pre_chain && u < a.M && ts.off[u + 1] - ts.off[u] > 0 ? 1 : 0;
+    if (a.pre_chain) {
+        __syncthreads();
+        if (threadIdx.x < a.M) {
+            const int v = chain_node(ts.off, ts.kid, a.N, threadIdx.x);
+            if (v >= 0) ts.pre[v] = 1;
         }
     }
     {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
@@ -619,10 +692,20 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     cg::cluster_group cluster = cg::this_cluster();
     const int half = (int)cluster.block_rank();
     const int pair = (int)blockIdx.x >> 1;
-    const int b = pair / a.M, j = pair - (pair / a.M) * a.M;
-    {  // leaves need no normaliser (both CTAs of the cluster return)
-        const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
-        if (__ldg(off + j + 1) - __ldg(off + j) <= 0) return;
+    const int b = pair / a.M;
+    int j = pair - (pair / a.M) * a.M;
+    const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+    if (a.pre_chain) {  // slot j: node j of the first-child chain (both CTAs find the same node)
+        int32_t *s_off = reinterpret_cast<int32_t *>(pst + a.C);
+        int32_t *s_kid = s_off + NN + 1;
+        for (int i = threadIdx.x; i <= NN; i += kPreThreads) s_off[i] = __ldg(off + i);
+        const int32_t *kids = a.child_ids + (int64_t)b * a.N;
+        for (int i = threadIdx.x; i < a.N; i += kPreThreads) s_kid[i] = __ldg(kids + i);
+        __syncthreads();
+        j = chain_node(s_off, s_kid, a.N, j);
+        if (j < 0) return;
+    } else if (__ldg(off + j + 1) - __ldg(off + j) <= 0) {
+        return;  // leaves need no normaliser (both CTAs of the cluster return)
     }
     const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)j * a.t_rstride;
     const int g = lane & 7, q = lane >> 3;
@@ -658,7 +741,7 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     }
     cluster.sync();  // rank 1 may leave; rank 0's copy is complete (the barrier also orders the CTA)
     if (warp < 4) {  // the log-normaliser over threads 0..127, then warps 0..3 in order
-        const Slot w = lse_part(pst, C);
+        const Slot w = lse_part(pst, C, threadIdx.x);
         if (lane == 0) part[warp] = w;
     }
     __syncthreads();
@@ -689,10 +772,10 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     int par = 0;
     Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
 
-    // the tree's copy in shared memory
-    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    // the tree's copy in shared memory with the pre-pass results
+    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth, true);
     const FF *s_l2t = ts.l2t;
-    const int32_t *s_pre = ts.pre, *s_off = ts.off, *s_kid = ts.kid, *s_tok = ts.tok, *s_row = ts.row;
+    const int32_t *s_known = ts.pre, *s_off = ts.off, *s_kid = ts.kid, *s_tok = ts.tok, *s_row = ts.row;
     const float *s_cxt = ts.cxt, *s_cxq = ts.cxq, *s_cu = ts.cu;
     int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
     int32_t *onode = a.out_nodes + (int64_t)b * a.L;
@@ -710,44 +793,32 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
         }
         const int r = s_row[u];
         const T *qrow = static_cast<const T *>(a.q) + (int64_t)b * a.q_bstride + (int64_t)r * a.q_rstride;
-        const bool pre = s_pre[u] != 0;
-        bool staged = !pre;  // P holds this node's x
-        FF L2t, L2q;
-        if (pre) {
-            L2t = s_l2t[u];
-            if (per_depth) {
-                L2q = sh.l2q[r];
-            } else {
-                __syncthreads();
-                if (warp == kQWarp) {
-                    const FF v = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
-                    if (lane == 0) sh.L2q = v;
+        bool staged = s_known[u] == 0;  // P holds this node's x after its staging round
+        if (staged) {
+            W.prefetch_slice(qrow);  // likely next read: this node's q row (a first rejection)
+            __syncthreads();         // earlier readers of P, Q and the round's node list are done
+            if (threadIdx.x == 0) {  // u, then first children while they have children and no value
+                int J = 0, v = u;
+                for (;;) {
+                    sh.look[J++] = v;
+                    if (J == kLook) break;
+                    const int c = s_kid[s_off[v]];
+                    if (s_off[c + 1] - s_off[c] <= 0 || s_known[c] != 0) break;
+                    v = c;
                 }
-                __syncthreads();
-                L2q = sh.L2q;
+                sh.nlook = J;
             }
-        } else {
-            {  // likely next reads: this node's q row (first rejection), the first child's target row
-                W.prefetch_slice(qrow);
-                W.prefetch_slice(static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride +
-                                 (int64_t)s_kid[o] * a.t_rstride);
-            }
-            __syncthreads();  // earlier readers of P and Q are done
-            // x into P with the slice's chunk statistics, then the row's log-normaliser from all
-            // chunks of the cluster (gathered into Q, free until the node's first rejection);
-            // a per-node q row's normaliser on warp kQWarp meanwhile
-            float2 *cst = sh.cst[ncst];
-            ncst ^= 1;  // a CTA may stage its next node while another still reads this one
-            W.stage_chunks(trow, P, cst);
-            W.gather_lse(cst, reinterpret_cast<float2 *>(Q), [&] {
-                if (!per_depth) {
-                    const FF v = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
-                    if (lane == 0) sh.L2q = v;
-                }
-            });
-            L2t = sh.L2t;
-            L2q = per_depth ? sh.l2q[r] : sh.L2q;
+            __syncthreads();
+            const int J = sh.nlook;
+            float2(*cst)[kMaxSliceChunks] = sh.cst[ncst];
+            ncst ^= 1;  // a CTA may stage its next round while another still reads this one
+            // x of u into P with the chunk statistics of all J rows, then their log-normalisers
+            // from all chunks of the cluster (gathered into Q, free until u's first rejection)
+            W.stage_look(J, P, cst);
+            W.gather_look(J, cst, reinterpret_cast<float2 *>(Q), ts.l2t, ts.pre);
         }
+        const FF L2t = s_l2t[u];
+        const FF L2q = per_depth ? sh.l2q[r] : ts.l2qn[u];
         // After i rejections p_i(v) = max(P0(v) - A_i Q(v), 0) / D_i with A_0 = 0, D_0 = 1,
         // A_{i+1} = A_i + D_i / t_i and D_{i+1} = sum_v max(P0(v) - A_{i+1} Q(v), 0): the
         // recursive residual max(p_i - Q/t_i, 0), renormalised, in closed form. A pass over the
@@ -801,7 +872,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
                 break;
             }
             // residual pass: the mass of R_{i+1} (storing P0 the first time P holds x)
-            KahanF zl;
+            KahanF zl[2];  // one per half chunk: two independent chains
             for (int cl = warp; cl < W.nch; cl += kWarps) {
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
@@ -817,12 +888,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
                     const float4 q = ld4(Q, j);
                     const float r0 = fmaxf(__fmaf_rn(-A1, q.x, x.x), 0.f), r1 = fmaxf(__fmaf_rn(-A1, q.y, x.y), 0.f);
                     const float r2 = fmaxf(__fmaf_rn(-A1, q.z, x.z), 0.f), r3 = fmaxf(__fmaf_rn(-A1, q.w, x.w), 0.f);
-                    zl.add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
+                    zl[h].add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
                 }
             }
             {
                 Slot mine = neutral_slot();
-                const FF z = zl.ff();
+                const FF z = ff_add(zl[0].ff(), zl[1].ff());
                 mine.zh = z.hi;
                 mine.zl = z.lo;
                 reduce_round<kRedSum>(sh, par, cluster, mine);
@@ -906,7 +977,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_trav(VerifyArgs a) {
     const bool per_depth = a.qrow_of_node == nullptr;
     int par = 0;
     Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
-    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth, true);
 
     auto trow_of = [&](int u) {
         return static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
@@ -956,7 +1027,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_trav(VerifyArgs a) {
             }
             staged_rej = ci + 1;
             __syncthreads();
-            KahanF zl;
+            KahanF zl[2];  // one per half chunk: two independent chains
             for (int cl = warp; cl < W.nch; cl += kWarps) {
 #pragma unroll
                 for (int h = 0; h < 2; ++h) {
@@ -964,11 +1035,11 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_trav(VerifyArgs a) {
                     const float4 x = ld4(P, j), q = ld4(Q, j);
                     const float r0 = fmaxf(__fmaf_rn(-A1, q.x, x.x), 0.f), r1 = fmaxf(__fmaf_rn(-A1, q.y, x.y), 0.f);
                     const float r2 = fmaxf(__fmaf_rn(-A1, q.z, x.z), 0.f), r3 = fmaxf(__fmaf_rn(-A1, q.w, x.w), 0.f);
-                    zl.add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
+                    zl[h].add(__fadd_rn(__fadd_rn(r0, r1), __fadd_rn(r2, r3)));
                 }
             }
             Slot mine = neutral_slot();
-            const FF z = zl.ff();
+            const FF z = ff_add(zl[0].ff(), zl[1].ff());
             mine.zh = z.hi;
             mine.zl = z.lo;
             reduce_round<kRedSum>(sh, par, cluster, mine);
@@ -1178,6 +1249,21 @@ int choose_cluster(int V, int N, int B, int *slice_out, size_t *smem_out) {
     return chosen;
 }
 
+// The pre-pass kernel for a's pre-computed set (target rows of M nodes per tree, q-row
+// normalisers), launched ahead of a walk.
+template <typename T>
+cudaError_t launch_pre_t(const VerifyArgs &a, int B, cudaStream_t s) {
+    const int per = a.qn ? a.N + 1 : a.Lq;
+    int64_t pre_blocks = 2 * (int64_t)B * a.M + ((int64_t)B * per + kPreThreads / 32 - 1) / (kPreThreads / 32);
+    pre_blocks += pre_blocks & 1;  // whole clusters of two (a spare q-row CTA finds no task)
+    if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    if (pre_blocks == 0) return cudaSuccess;
+    const size_t psmem = (size_t)a.C * sizeof(float2) + (a.pre_chain ? (size_t)(2 * a.N + 2) * sizeof(int32_t) : 0);
+    cudaError_t e = cudaFuncSetAttribute(k_verify_pre<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), psmem, s, 2, a);
+}
+
 template <typename T>
 cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     int slice = 0;
@@ -1191,16 +1277,8 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
         e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
     }
-    int64_t pre_blocks = 2 * (int64_t)B * a.M + ((int64_t)B * a.Lq + kPreThreads / 32 - 1) / (kPreThreads / 32);
-    pre_blocks += pre_blocks & 1;  // whole clusters of two (a spare q-row CTA finds no task)
-    if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    if (pre_blocks > 0) {
-        const size_t psmem = (size_t)a.C * sizeof(float2);
-        e = cudaFuncSetAttribute(k_verify_pre<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
-        if (e != cudaSuccess) return e;
-        e = launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), psmem, s, 2, a);
-        if (e != cudaSuccess) return e;
-    }
+    e = launch_pre_t<T>(a, B, s);
+    if (e != cudaSuccess) return e;
     return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
 
@@ -1217,14 +1295,7 @@ cudaError_t launch_trav_t(VerifyArgs a, int B, cudaStream_t s) {
         e = cudaFuncSetAttribute(k_verify_trav<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
     }
-    const int per = a.qn ? a.N + 1 : a.Lq;
-    int64_t pre_blocks = 2 * (int64_t)B * a.M + ((int64_t)B * per + kPreThreads / 32 - 1) / (kPreThreads / 32);
-    pre_blocks += pre_blocks & 1;  // whole clusters of two (a spare q-row CTA finds no task)
-    if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
-    const size_t psmem = (size_t)a.C * sizeof(float2);
-    e = cudaFuncSetAttribute(k_verify_pre<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
-    if (e != cudaSuccess) return e;
-    e = launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), psmem, s, 2, a);
+    e = launch_pre_t<T>(a, B, s);
     if (e != cudaSuccess) return e;
     return launch_pdl(k_verify_trav<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
@@ -1259,7 +1330,8 @@ VerifyArgs verify_args(const RowsDesc &target, const RowsDesc &q, const float2 *
     a.status = status;
     // the pre-pass results use the workspace's per-(tree, node) slots (status word is ws[0])
     a.pre = reinterpret_cast<PreRow *>(reinterpret_cast<char *>(status) + kWsStatusBytes);
-    a.M = N + 1 < kPreTop ? N + 1 : kPreTop;
+    a.M = 0;
+    a.pre_chain = 0;
     a.Lq = qrow_of_node ? 0 : (L < N + 1 ? L : N + 1);
     a.qn = 0;
     a.B = B;
@@ -1284,8 +1356,11 @@ cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const f
                               const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
                               const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
                               int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s) {
-    const VerifyArgs a = verify_args(target, q, qstats, qrow_of_node, B, N, L, tree, token, invT, seed, out_tokens,
-                                     out_nodes, out_len, status);
+    VerifyArgs a = verify_args(target, q, qstats, qrow_of_node, B, N, L, tree, token, invT, seed, out_tokens,
+                               out_nodes, out_len, status);
+    a.M = kPreChain;  // the first-child chain's first internal nodes from the pre-pass
+    a.pre_chain = 1;
+    a.qn = qrow_of_node ? 1 : 0;  // per-node q rows: every internal node's normaliser
     if (target.dtype == 1) return launch_rrs_t<__nv_bfloat16>(a, B, s);
     return launch_rrs_t<float>(a, B, s);
 }
