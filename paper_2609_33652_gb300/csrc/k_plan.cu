@@ -7,13 +7,15 @@
 //   tau are re-read, spread over the warps; their logits >= tau go through per-lane sorted
 //   lists, and warp then CTA merges yield the top-K by (x desc, id asc). Results go to the
 //   workspace.
-// k_plan_heap, one CTA per tree: best-first expansion, popping N candidates. A candidate at
-//   depth d holds the sum Sx of its path's logits (exact, in 64-bit fixed point) and the key
+// k_plan_select, one CTA per tree: the best-first expansion's N nodes. A candidate at depth d
+//   holds the sum Sx of its path's logits (exact, in 64-bit fixed point) and the key
 //   Sx - CL[d], CL[d] = LSE_1 + ... + LSE_d (its draft path log-probability). Pop order:
 //   (key desc, depth asc, parent asc, rank asc), compared as integers. Popping (p, r) at depth d
-//   pushes the next sibling (p, r+1) and, below the depth cap, the first child (i, 0).
-//   Siblings are popped in rank order, so the children of u occupy
-//   child_ids[child_off[u] + rank] directly.
+//   pushes the next sibling (p, r+1) and, below the depth cap, the first child (i, 0). Keys never
+//   increase along these links, so the N pops are the N first paths of that order: the kernel
+//   bounds the N-th key, enumerates the paths that reach the bound and numbers them by counting
+//   (the serial pops remain as the fallback). Siblings are popped in rank order, so the children
+//   of u occupy child_ids[child_off[u] + rank] directly.
 //
 // Both are latency-bound: the draft rows were streamed once by the statistics kernel and only
 // the few candidate chunks per row are read again.
@@ -25,7 +27,7 @@ namespace {
 
 constexpr int kTopkThreads = 128;
 constexpr int kRowPlanThreads = 512;
-constexpr int kHeapThreads = 128;
+constexpr int kHeapThreads = 256;
 
 struct TopkArgs {
     const void *draft;
@@ -457,15 +459,110 @@ struct Slots {
     }
 };
 
-// Best-first expansion for one tree with one warp. Each pop: a warp maximum of the lanes'
-// best keys, one __reduce_max_sync on a 32-bit monotone image of the key, refined on the
-// full key (high word, low word, tie word) only among lanes whose images tie; the popped
-// candidate's slot takes its next sibling; its first child goes to the next round-robin
-// slot (children are numbered in creation order, lane = c % 32, slot = c / 32).
+// ---------------------------------------------------------------------------------------
+// Best-first expansion by selection. Keys never increase along a path's links: a first child's
+// key is its parent's plus x - (CL[d] - CL[d-1]) <= 0 (checked per tree), a sibling's is at
+// most its left neighbour's (the top-K lists are sorted). Then every candidate's predecessor
+// precedes it in the global order (key desc, depth asc, parent asc, rank asc), so the max-heap's
+// N pops are exactly the N first paths of that order, and the kernel finds them in parallel:
+//   1. a lower bound tau on the N-th key: the top-1 chain of each length and every path that
+//      leaves it once (rank r >= 1 at depth i, then rank 0 down to depth d) are real paths, so
+//      the N-th largest key among them (family F0) is at most the N-th largest overall; two
+//      histogram rounds over their keys (64 power-of-two bins of hi - key, then 64 sub-bins of
+//      the bin holding the N-th) give a bin edge with at least N keys of F0 at or above it;
+//   2. every path with key >= tau, as chains: the top-1 chain as far as it reaches tau, then
+//      level by level every rank >= 1 child (reaching tau) of a node found in the level before
+//      (first the root and the top-1 chain), each with its rank-0 continuation as far as it
+//      reaches tau (a binary search over the chain keys). More than `cap` paths: the N-th
+//      largest key among `cap` of them is a tighter bound, and the enumeration restarts;
+//   3. each path's position by counting the paths before it. Parents' positions decide only
+//      between equal keys at equal depths (frequent with bf16 logits): there the ancestors' keys
+//      are compared upwards, then the ranks below the common ancestor. Positions 0..N-1 are
+//      nodes 1..N.
+// Trees whose first-child keys would rise (a rounding of the normaliser prefix above a logit),
+// or whose bound does not tighten, take the serial expansion below (one warp popping the
+// frontier), which gives the same tree by definition.
+constexpr int kSelLevels = 64;   // chain levels (deviations from the top-1 chain) per enumeration
+constexpr int kMaxDepth = 64;    // depth cap L <= 64
+constexpr int kSelAttempts = 4;  // enumerations before the serial expansion takes over
+
+__device__ __forceinline__ int sel_cap(int N) { return 4 * N + 64; }
+
+size_t select_smem_bytes(int L, int N, int K) {
+    const size_t NN = (size_t)N + 1, cap = (size_t)4 * N + 64;
+    return (size_t)(L + 1) * 8 + NN * 8 + (size_t)L * K * 8 + 6 * NN * 4 + (size_t)L * K * 4 + 8 +  // heap layout
+           (size_t)(L + 1) * 8 + (size_t)(L + 1) * K * 8 + cap * 8 + 3 * cap * 4;
+}
+
+struct SelShared {
+    long long tau, lo;
+    int hist[64];
+    int nent, ovf, alo, ahi, root, mono, fast, jstar, cum, kstar;
+};
+
+// A bin edge t <= the N-th largest of a set of keys (all in [lo, hi], at least N of them) with
+// at least N of them >= t: 64 power-of-two bins of hi - key, then 64 sub-bins of the bin holding
+// the N-th. fill(s1, s2, jb, hist) adds every key's bin to hist: (hi - key) >> s1 for jb < 0,
+// else, for the keys with (hi - key) >> s1 == jb, ((hi - key) >> s2) - (jb << (s1 - s2)).
+// Every thread of the CTA calls it; ends synchronised.
+template <typename F>
+__device__ long long nth_bound(SelShared &ss, int N, long long hi, long long lo, F fill) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int bits = 64 - __clzll(hi - lo);  // hi - lo >= 0
+    const int s1 = bits > 6 ? bits - 6 : 0;  // (hi - lo) >> s1 < 64
+    const int s2 = s1 > 6 ? s1 - 6 : 0;
+    for (int round = 0; round < 2; ++round) {
+        if (threadIdx.x < 64) ss.hist[threadIdx.x] = 0;
+        __syncthreads();
+        fill(s1, s2, round == 0 ? -1 : ss.jstar, ss.hist);
+        __syncthreads();
+        if (warp == 0) {  // the first bin whose inclusive prefix reaches N (two bins per lane)
+            const int base = round == 0 ? 0 : ss.cum;
+            const int h0 = ss.hist[2 * lane], h1 = ss.hist[2 * lane + 1];
+            int incl = h0 + h1;
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const int y = __shfl_up_sync(kFull, incl, o);
+                if (lane >= o) incl += y;
+            }
+            const int excl = base + incl - h0 - h1;
+            const bool in0 = excl + h0 >= N, in1 = excl + h0 + h1 >= N;
+            const unsigned m = __ballot_sync(kFull, in1);
+            const int first = m ? __ffs(m) - 1 : 31;
+            if (lane == first) {
+                const int j = in0 ? 2 * lane : 2 * lane + 1;
+                if (round == 0) {
+                    ss.jstar = j;
+                    ss.cum = in0 ? excl : excl + h0;
+                } else {
+                    ss.kstar = j;
+                }
+            }
+        }
+        __syncthreads();
+    }
+    const long long idx = ((long long)ss.jstar << (s1 - s2)) + ss.kstar;
+    return hi - ((idx + 1) << s2) + 1;
+}
+
+// The bin of key k in a round of nth_bound (-1: outside the round's bin).
+__device__ __forceinline__ int bound_bin(long long hi, long long k, int s1, int s2, int jb) {
+    const unsigned long long dv = (unsigned long long)(hi - k);
+    if (jb < 0) return (int)(dv >> s1);
+    return (int)(dv >> s1) == jb ? (int)((dv >> s2) - ((unsigned long long)jb << (s1 - s2))) : -1;
+}
+
+// Max-heap expansion by selection (steps 1-3 above), with the serial expansion as fallback.
+// Each pop of the serial expansion: a warp maximum of the lanes' best keys, one
+// __reduce_max_sync on a 32-bit monotone image of the key, refined on the full key (high word,
+// low word, tie word) only among lanes whose images tie; the popped candidate's slot takes its
+// next sibling; its first child goes to the next round-robin slot (children are numbered in
+// creation order, lane = c % 32, slot = c / 32).
 template <int S>
-__global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
+__global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
     pdl_begin();
     extern __shared__ __align__(16) unsigned char smem[];
+    __shared__ SelShared ss;
     const int L = a.L, N = a.N, K = a.K, NN = N + 1;
     long long *CL = reinterpret_cast<long long *>(smem);           // [L+1] fixed point
     long long *n_sx = CL + (L + 1);                                // [NN] raw pop keys
@@ -477,6 +574,14 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     int32_t *n_count = n_token + NN;                               // [NN]
     float *n_score = reinterpret_cast<float *>(n_count + NN);      // [NN]
     int32_t *tk_id = reinterpret_cast<int32_t *>(n_score + NN);    // [L*K]
+    const int cap = sel_cap(N);
+    long long *Bk = reinterpret_cast<long long *>(smem + ((size_t)(L + 1) * 8 + (size_t)NN * 8 + (size_t)L * K * 8 +
+                                                          6 * (size_t)NN * 4 + (size_t)L * K * 4 + 7) / 8 * 8);
+    long long *dl = Bk + (L + 1);             // [(L+1)*K] key step of rank r at depth d: dl[d*K + r]
+    long long *ekey = dl + (size_t)(L + 1) * K;  // [cap] enumerated paths
+    int32_t *einfo = reinterpret_cast<int32_t *>(ekey + cap);  // depth | rank << 8
+    int32_t *epar = einfo + cap;                               // parent entry (-1: the root)
+    int32_t *epos = epar + cap;                                // position in the global order
 
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -496,6 +601,238 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_heap(HeapArgs a) {
     if (warp == 0) depth_prefix_fixed(a.lse + (int64_t)b * L, L, CL);
     __syncthreads();
 
+    // ---- 1. key steps, the top-1 chain keys Bk[d], monotonicity, the bound from F0
+    for (int i = threadIdx.x; i < L * K; i += kHeapThreads) {
+        const int d = i / K + 1;
+        dl[d * K + i % K] = fx[i] - (CL[d] - CL[d - 1]);
+    }
+    __syncthreads();
+    if (warp == 0) {  // Bk[d] = dl[1][0] + ... + dl[d][0] by a warp scan (depths lane + 1, lane + 33)
+        const long long a0 = lane < L ? dl[(lane + 1) * K] : 0, a1 = lane + 32 < L ? dl[(lane + 33) * K] : 0;
+        long long c0 = lane < L ? dl[(lane + 1) * K] - dl[(lane + 1) * K + K - 1] : 0;
+        const long long c1 = lane + 32 < L ? dl[(lane + 33) * K] - dl[(lane + 33) * K + K - 1] : 0;
+        long long s0 = a0, s1 = a1;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const long long y0 = __shfl_up_sync(kFull, s0, o), y1 = __shfl_up_sync(kFull, s1, o);
+            if (lane >= o) {
+                s0 += y0;
+                s1 += y1;
+            }
+        }
+        s1 += __shfl_sync(kFull, s0, 31);
+        if (lane < L) Bk[lane + 1] = s0;
+        if (lane + 32 < L) Bk[lane + 33] = s1;
+        c0 = c0 > c1 ? c0 : c1;  // the largest step off the chain at any depth: lo = Bk[L] - that
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            const long long y = __shfl_xor_sync(kFull, c0, o);
+            c0 = y > c0 ? y : c0;
+        }
+        const int bad = __ballot_sync(kFull, a0 > 0 || a1 > 0) != 0u;
+        const long long bkl = __shfl_sync(kFull, L <= 32 ? s0 : s1, (L - 1) & 31);
+        if (lane == 0) {
+            Bk[0] = 0;
+            ss.mono = !bad;
+            ss.fast = !bad;
+            ss.lo = bkl - c0;
+        }
+    }
+    __syncthreads();
+    long long tau = -(1ll << 62);
+    const long long hi = Bk[1];
+    if (ss.fast) {
+        const long long nF0 = (long long)L + (long long)(K - 1) * L * (L + 1) / 2;
+        if (nF0 >= N) {
+            const long long lo = ss.lo;
+            // F0 as sorted sequences: q = 0 the top-1 chain Bk[1..L]; q = 1 + (i - 1) (K - 1) + r - 1
+            // the paths leaving it at depth i with rank r, Bk[d] - c (d = i..L). Bins grow along a
+            // sequence, so each thread adds runs of equal bins.
+            const int nq = 1 + L * (K - 1);
+            tau = nth_bound(ss, N, hi, lo, [&](int s1, int s2, int jb, int *hist) {
+                for (int q = threadIdx.x; q < nq; q += kHeapThreads) {
+                    int d0 = 1;
+                    long long c = 0;
+                    if (q > 0) {
+                        const int i = 1 + (q - 1) / (K - 1), r = 1 + (q - 1) % (K - 1);
+                        d0 = i;
+                        c = dl[i * K] - dl[i * K + r];
+                    }
+                    int run_bin = -1, run = 0;
+                    for (int d = d0; d <= L; ++d) {
+                        const int bin = bound_bin(hi, Bk[d] - c, s1, s2, jb);
+                        if (bin != run_bin) {
+                            if (run_bin >= 0) atomicAdd(&hist[run_bin], run);
+                            run_bin = bin;
+                            run = 0;
+                        }
+                        ++run;
+                    }
+                    if (run_bin >= 0) atomicAdd(&hist[run_bin], run);
+                }
+            });
+        }
+    }
+
+    // ---- 2. every path with key >= tau, as chains
+    bool fast = ss.fast != 0;
+    int M = 0;
+    for (int attempt = 0; fast && attempt < kSelAttempts; ++attempt) {
+        if (threadIdx.x == 0) {  // the top-1 chain: a prefix of depths (Bk decreases)
+            int l0 = 0, h0 = L;  // the last depth whose chain key reaches tau
+            while (l0 < h0) {
+                const int mid = (l0 + h0 + 1) >> 1;
+                if (Bk[mid] >= tau)
+                    l0 = mid;
+                else
+                    h0 = mid - 1;
+            }
+            ss.nent = min(l0, cap);
+            ss.ovf = l0 > cap;
+            ss.alo = 0;
+            ss.ahi = min(l0, cap);
+            ss.root = 1;
+        }
+        __syncthreads();
+        for (int e = threadIdx.x; e < ss.ahi; e += kHeapThreads) {
+            ekey[e] = Bk[e + 1];
+            einfo[e] = e + 1;
+            epar[e] = e - 1;
+        }
+        __syncthreads();
+        for (int lev = 0; lev < kSelLevels && !ss.ovf; ++lev) {  // uniform: read after a barrier
+            const int alo = ss.alo, ahi = ss.ahi, root = ss.root;
+            const int na = root + (ahi - alo);
+            if (na == 0) break;
+            const int nc = na * (K - 1);
+            for (int c = threadIdx.x; c < nc; c += kHeapThreads) {
+                const int ai = c / (K - 1), r = 1 + c % (K - 1);
+                int ae = -1, da = 0;
+                long long ka = 0;
+                if (!(root && ai == 0)) {
+                    ae = alo + ai - root;
+                    da = einfo[ae] & 255;
+                    ka = ekey[ae];
+                }
+                const int d = da + 1;
+                if (d > L) continue;
+                const long long key = ka + dl[d * K + r];
+                if (key < tau) continue;
+                int lo2 = d, hi2 = L;  // the last depth whose rank-0 continuation reaches tau
+                while (lo2 < hi2) {
+                    const int mid = (lo2 + hi2 + 1) >> 1;
+                    if (key + Bk[mid] - Bk[d] >= tau)
+                        lo2 = mid;
+                    else
+                        hi2 = mid - 1;
+                }
+                const int n = 1 + lo2 - d;
+                const int base = atomicAdd(&ss.nent, n);
+                if (base + n > cap) ss.ovf = 1;
+                for (int j = 0; j < n && base + j < cap; ++j) {
+                    ekey[base + j] = j == 0 ? key : key + Bk[d + j] - Bk[d];
+                    einfo[base + j] = (d + j) | ((j == 0 ? r : 0) << 8);
+                    epar[base + j] = j == 0 ? ae : base + j - 1;
+                }
+            }
+            __syncthreads();
+            if (threadIdx.x == 0) {
+                ss.alo = ahi;
+                ss.ahi = min(ss.nent, cap);
+                ss.root = 0;
+            }
+            __syncthreads();
+        }
+        M = min(ss.nent, cap);
+        if (!ss.ovf) break;
+        const long long t2 = nth_bound(ss, N, hi, tau, [&](int s1, int s2, int jb, int *hist) {
+            for (int f = threadIdx.x; f < cap; f += kHeapThreads) {
+                const int bin = bound_bin(hi, ekey[f], s1, s2, jb);
+                if (bin >= 0) atomicAdd(&hist[bin], 1);
+            }
+        });
+        if (t2 <= tau || attempt + 1 == kSelAttempts) {
+            fast = false;
+            break;
+        }
+        tau = t2;
+        __syncthreads();
+    }
+    if (fast && M < N) fast = false;
+
+    if (fast) {
+        // ---- 3. positions by counting. Between equal keys at equal depths with different parents
+        //      the order is that of the parents, recursively: ancestors' keys compared upwards
+        //      until they differ, else (equal up to the common ancestor) the ranks of its two
+        //      children on the paths.
+        for (int x0 = warp * 8; x0 < M; x0 += kHeapThreads / 4) {  // uniform over the warp; four lanes per path
+            const int x = x0 + (lane >> 2), sub = lane & 3;
+            int n = 0;
+            if (x < M) {
+                const long long kx = ekey[x];
+                const int dx = einfo[x] & 255, rx = einfo[x] >> 8, px = epar[x];
+                for (int y = sub; y < M; y += 4) {
+                    const long long ky = ekey[y];
+                    int add = ky > kx ? 1 : 0;
+                    if (ky == kx && y != x) {
+                        const int iy = einfo[y], dy = iy & 255;
+                        if (dy < dx) {
+                            add = 1;
+                        } else if (dy == dx) {
+                            const int py = epar[y];
+                            if (py == px) {
+                                add = (iy >> 8) < rx ? 1 : 0;
+                            } else {  // both at depth >= 2: walk up to the first difference
+                                int cx = x, cy = y, ax = px, ay = py, before = -1;
+                                for (int up = 0; up < kMaxDepth && before < 0; ++up) {
+                                    if (ax == ay) {
+                                        before = (einfo[cy] >> 8) < (einfo[cx] >> 8) ? 1 : 0;
+                                    } else if (ekey[ax] != ekey[ay]) {
+                                        before = ekey[ay] > ekey[ax] ? 1 : 0;
+                                    } else {
+                                        cx = ax;
+                                        cy = ay;
+                                        ax = epar[ax];
+                                        ay = epar[ay];
+                                    }
+                                }
+                                add = before > 0 ? 1 : 0;
+                            }
+                        }
+                    }
+                    n += add;
+                }
+            }
+            n += __shfl_xor_sync(kFull, n, 1);
+            n += __shfl_xor_sync(kFull, n, 2);
+            if (x < M && sub == 0) epos[x] = n;
+        }
+        __syncthreads();
+        bool bad = false;
+        for (int x = threadIdx.x; x < M; x += kHeapThreads) {
+            const int pos = epos[x];
+            if (pos < 0 || pos >= N) continue;
+            const int i = pos + 1, d = einfo[x] & 255, r = einfo[x] >> 8;
+            const int par = epar[x] < 0 ? 0 : epos[epar[x]] + 1;
+            if (par >= i) bad = true;
+            n_parent[i] = par;
+            n_depth[i] = d;
+            n_rank[i] = r;
+            n_token[i] = tk_id[(d - 1) * K + r];
+            n_score[i] = __fmul_rn(__ll2float_rn(ekey[x]), kFixInv);
+        }
+        if (bad) raise_status(a.status, kDevBadTree);
+        if (threadIdx.x == 0) {
+            n_parent[0] = -1;
+            n_depth[0] = 0;
+            n_rank[0] = -1;
+            n_token[0] = -1;
+            n_score[0] = 0.f;
+        }
+        __syncthreads();
+        emit_tree<kHeapThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
+        return;
+    }
     // The expansion (warp 0). Per pop the critical path is the warp maximum, three shuffles,
     // the decode, independent shared loads of the candidate logits and depth normalisers, and
     // predicated slot updates: no dependent load of the parent's path sum (each slot carries
@@ -789,17 +1126,12 @@ __global__ void __launch_bounds__(kEptThreads) k_plan_ept(EptArgs a) {
     emit_tree<kEptThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
 }
 
-size_t heap_smem_bytes(int L, int N, int K) {
-    const size_t NN = (size_t)N + 1;
-    return (size_t)(L + 1) * 8 + NN * 8 + (size_t)L * K * 8 + 6 * NN * 4 + (size_t)L * K * 4;
-}
-
 template <int S>
 cudaError_t launch_heap_t(const HeapArgs &h, int B, cudaStream_t s) {
-    const size_t smem = heap_smem_bytes(h.L, h.N, h.K);
-    cudaError_t e = cudaFuncSetAttribute(k_plan_heap<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    const size_t smem = select_smem_bytes(h.L, h.N, h.K);
+    cudaError_t e = cudaFuncSetAttribute(k_plan_select<S>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
-    return launch_pdl(k_plan_heap<S>, dim3((unsigned)B), dim3(kHeapThreads), smem, s, 0, h);
+    return launch_pdl(k_plan_select<S>, dim3((unsigned)B), dim3(kHeapThreads), smem, s, 0, h);
 }
 
 template <int KCAP, typename T>
