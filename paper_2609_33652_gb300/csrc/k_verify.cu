@@ -33,13 +33,12 @@
 // the children's target and q logits and their acceptance uniforms to shared memory once. At
 // a node with a known normaliser it needs no staging and no cluster round: every CTA takes
 // the same decisions from the same inputs, and the slices are staged only if a rejection needs
-// the residual. At any other node the walk runs a staging round over that node and up to
-// kLook - 1 of its first-child descendants without a value: every warp streams the rows'
-// slices in the chunk-statistics layout (the node's x into shared memory, each chunk's
-// statistics beside it), every CTA gathers all chunk statistics of the rows through
-// distributed shared memory and computes their log-normalisers, one group of four warps per
-// row. 12 warps per CTA: 160 registers a thread without spills (16 warps at 128 spilled in
-// the walk's hot paths and ran slower). Element passes give lane l the elements 4l..4l+3 and
+// the residual. At any other node the walk runs a staging round over that node and up to two
+// (bf16; one for fp32) of its first-child descendants without a value: the rows' slices are
+// copied to shared memory with cp.async, all in flight together, their chunk statistics
+// computed there (the node's x kept in P), and each row's log-normaliser merged from one
+// partial per CTA through distributed shared memory. 12 warps per CTA: 160 registers a thread
+// without spills (16 warps at 128 spilled in the walk's hot paths and ran slower). Element passes give lane l the elements 4l..4l+3 and
 // 128+4l..128+4l+3 of each 256-token chunk, so every shared-memory access is a conflict-free
 // 16-byte vector. Every normaliser comes from the same two functions over the row's chunk
 // statistics, whichever kernel computes it, and which nodes are pre-computed depends only on
@@ -61,9 +60,9 @@ constexpr int kWarps = kThreads / 32;
 constexpr int kMaxSliceChunks = 128;  // slice <= 32768 tokens
 constexpr int kMaxDepthRows = 64;     // per-depth q rows (depth cap L <= 64)
 constexpr int kPreThreads = 512;
-// Rows per staging round of the RRS walk: the node being visited and up to kLook - 1 of its
+// Rows per staging round of the RRS walk, at most: the node being visited and up to two of its
 // first-child descendants (the children a walk most often accepts next), whose target
-// log-normalisers the same round computes with the loads of all rows in flight together.
+// log-normalisers the same round computes with the copies of all rows in flight together.
 constexpr int kLook = 3;
 // Internal nodes of the first-child chain from the root whose target normalisers the RRS
 // pre-pass computes on the whole GPU (the walk starts on that chain; nodes a walk reaches off it
@@ -164,8 +163,8 @@ struct Scratch {
     int path[kMaxDepthRows];      // accepted node ids (written out after the walk)
     float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
     FF l2q[kMaxDepthRows];        // per-depth q log-normalisers (times log2 e)
-    float2 cst[2][kLook][kMaxSliceChunks];  // chunk statistics of the slice's rows, alternating per round
-    Slot lpart[kLook][4];                   // per-warp partials of the round's normalisers
+    float2 cst[kLook][kMaxSliceChunks];  // chunk statistics of the slice's rows in a staging round
+    Slot lpart[2][kLook];                // this CTA's partials of the round's normalisers, alternating
     int look[kLook];                        // nodes of the current staging round
     int nlook;
 };
@@ -284,90 +283,106 @@ struct Walk {
         }
     }
 
-    // One staging round over the rows of nodes sh.look[0..J-1] (target rows), in the
-    // chunk-statistics layout (eight lanes per 256-logit chunk, lane g holding logits
-    // 8g..8g+7 of each 64-logit quarter; four chunks per warp and unit): the statistics of
-    // every chunk of this CTA's slice of row j into cst[j] (the per-chunk code of the
-    // statistics kernels) and x = fp32(z) * invT of row 0 into dst (logits past the vocabulary
-    // become -inf). The (row, unit) pairs are dealt to the warps in one sequence, kU pairs in
-    // flight per warp, so the loads of all J rows are issued together. Every warp takes part.
+    // One staging round over the target rows of nodes sh.look[0..J-1] (J <= kLookMax).
+    // Every thread copies 16-byte pieces of this CTA's slice of each row into shared memory
+    // with cp.async (all rows in flight at once, no registers held): row 0 into the lower half
+    // of Q, row 1 into the upper half of Q (bf16) or into P (fp32), row 2 into the upper half
+    // of P (bf16); the slice's tail past the vocabulary becomes -inf. Then, in the
+    // chunk-statistics layout (eight lanes per 256-logit chunk, lane g holding logits 8g..8g+7
+    // of each 64-logit quarter), every chunk's statistics into cst[j] (the per-chunk code of the
+    // statistics kernels): rows 1..J-1 first, then row 0 with x = fp32(z) * invT into P (which
+    // held the other rows' copies). Every thread takes part; ends synchronised.
+    static constexpr int kLookMax = sizeof(T) == 2 ? 3 : 2;
+    __device__ unsigned char *landing(int j) const {
+        if (j == 0) return reinterpret_cast<unsigned char *>(Q);
+        if (sizeof(T) == 4) return reinterpret_cast<unsigned char *>(P);
+        return j == 1 ? reinterpret_cast<unsigned char *>(Q) + (size_t)a.slice * 2
+                      : reinterpret_cast<unsigned char *>(P) + (size_t)a.slice * 2;
+    }
     __device__ void stage_look(int J, float *dst, float2 (*cst)[kMaxSliceChunks]) {
-        constexpr int kU = sizeof(T) == 2 ? 2 : 1;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int g = lane & 7, q = lane >> 3;
-        const int units = (nch + 3) / 4, total = J * units;
-        for (int i0 = warp; i0 < total; i0 += kU * kWarps) {  // uniform over the warp
-            RawGroup<T> raw[kU][4];
-#pragma unroll
-            for (int e = 0; e < kU; ++e) {
-                const int idx = i0 + e * kWarps;
-                const int j = idx / units, cl = (idx - j * units) * 4 + q;
-                if (idx < total && cl < nch) {
-                    const T *row =
-                        static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)sh.look[j] * a.t_rstride;
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) raw[e][k].load(row, lo + cl * kChunk + k * 64 + g * 8, a.V);
-                }
+        const int bytes = n * (int)sizeof(T), pieces = bytes >> 4;
+        for (int j = 0; j < J; ++j) {
+            const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)sh.look[j] * a.t_rstride;
+            const unsigned char *src = reinterpret_cast<const unsigned char *>(row + lo);
+            unsigned char *dstj = landing(j);
+            for (int i = threadIdx.x; i < pieces; i += kThreads) {
+                const unsigned sa = (unsigned)__cvta_generic_to_shared(dstj + 16 * i);
+                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(src + 16 * i) : "memory");
             }
+            // the ragged tail (fewer than 16 bytes) and the padding up to the last chunk's end
+            T *lt = reinterpret_cast<T *>(dstj);
+            for (int e = (pieces << 4) / (int)sizeof(T) + threadIdx.x; e < nch * kChunk; e += kThreads)
+                lt[e] = e < n ? row[lo + e] : Logit<T>::neg_inf();
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        __syncthreads();
+        const int units = (nch + 3) / 4;
+        for (int pass = 0; pass < 2; ++pass) {  // rows 1..J-1, then row 0 (its x overwrites P)
+            const int j0 = pass == 0 ? 1 : 0, nj = pass == 0 ? J - 1 : 1;
+            const int total = nj * units;
+            for (int i0 = warp; i0 < total; i0 += kWarps) {  // uniform over the warp
+                const int j = j0 + i0 / units, cl = (i0 - (i0 / units) * units) * 4 + q;
+                const bool live = cl < nch;
+                const unsigned char *zone = landing(j);
+                RawGroup<T> raw[4];
+                if (live)
 #pragma unroll
-            for (int e = 0; e < kU; ++e) {
-                const int idx = i0 + e * kWarps;
-                const int j = idx / units, cl = (idx - j * units) * 4 + q;
-                const bool live = idx < total && cl < nch;
+                    for (int k = 0; k < 4; ++k) raw[k].load_shared(zone, cl * kChunk + k * 64 + g * 8);
                 float mc, sc;
-                chunk_stats8<T>(raw[e], live, a.invT, &mc, &sc);
+                chunk_stats8<T>(raw, live, a.invT, &mc, &sc);
                 if (live && g == 0) cst[j][cl] = make_float2(mc, sc);
                 if (live && j == 0) {
 #pragma unroll
                     for (int k = 0; k < 4; ++k) {
                         float z[8];
-                        raw[e][k].unpack(z);
-                        const int i = cl * kChunk + k * 64 + g * 8;
-                        st4(dst, i, __fmul_rn(z[0], a.invT), __fmul_rn(z[1], a.invT), __fmul_rn(z[2], a.invT),
+                        raw[k].unpack(z);
+                        const int e = cl * kChunk + k * 64 + g * 8;
+                        st4(dst, e, __fmul_rn(z[0], a.invT), __fmul_rn(z[1], a.invT), __fmul_rn(z[2], a.invT),
                             __fmul_rn(z[3], a.invT));
-                        st4(dst, i + 4, __fmul_rn(z[4], a.invT), __fmul_rn(z[5], a.invT), __fmul_rn(z[6], a.invT),
+                        st4(dst, e + 4, __fmul_rn(z[4], a.invT), __fmul_rn(z[5], a.invT), __fmul_rn(z[6], a.invT),
                             __fmul_rn(z[7], a.invT));
                     }
                 }
             }
+            __syncthreads();
         }
     }
 
-    // The log-normalisers of the round's J rows, whose chunk statistics every CTA of the
-    // cluster has staged into its cst[0..J-1] (slice / 256 chunks per CTA and row): each CTA
-    // gathers all of them into `tmp` through distributed shared memory and computes the values
-    // itself, one group of four warps per row over the fixed partition of lse_part, so every
-    // CTA holds identical values. Ends with row j's value (times log2 e) in l2t[sh.look[j]]
-    // and the node marked as known.
-    __device__ void gather_look(int J, float2 (*cst)[kMaxSliceChunks], float2 *tmp, FF *l2t, int32_t *known) {
+    // The log-normalisers of the round's J rows: each CTA merges the statistics of its own
+    // chunks of row j (warp j: the maximum, then a float-float sum of s_c e^(m_c - m) over a
+    // fixed lane partition), publishes that partial, and after the cluster barrier every CTA
+    // merges the CS partials in rank order with the same warp reduction, so all CTAs hold
+    // identical values. Ends with row j's value (times log2 e) in l2t[sh.look[j]] and the node
+    // marked as known. `slot` alternates between rounds (a CTA may publish the next round's
+    // partials while another still reads these).
+    __device__ void gather_look(int J, const float2 (*cst)[kMaxSliceChunks], int slot, FF *l2t, int32_t *known) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-        cluster.sync();  // every CTA's chunk statistics are written
-        const int per = a.slice / kChunk, C = a.C;
-        for (int i0 = threadIdx.x; i0 < J * C; i0 += 4 * kThreads) {  // four remote loads in flight
-            float2 v[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int i = i0 + e * kThreads;
-                if (i < J * C) {
-                    const int j = i / C, c = i - j * C, r = c / per;
-                    v[e] = *cluster.map_shared_rank(&cst[j][c - r * per], r);
-                }
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-                if (i0 + e * kThreads < J * C) tmp[i0 + e * kThreads] = v[e];
-        }
-        __syncthreads();
-        const int grp = warp >> 2;
-        for (int j = grp; j < J; j += kWarps / 4) {  // uniform over the warp
-            const Slot w = lse_part(tmp + (size_t)j * C, C, threadIdx.x - 128 * grp);
-            if (lane == 0) sh.lpart[j][warp & 3] = w;
-        }
-        __syncthreads();
         if (warp < J) {
-            const FF L2 = lse_final(sh.lpart[warp]);
+            const float2 *c = cst[warp];
+            float m = -INFINITY;
+            for (int cl = lane; cl < nch; cl += 32) m = fmaxf(m, c[cl].x);
+            KahanF acc;
+            if (m != -INFINITY)
+                for (int cl = lane; cl < nch; cl += 32) acc.add(__fmul_rn(c[cl].y, expf(__fsub_rn(c[cl].x, m))));
+            Slot mine = neutral_slot();
+            const FF sv = acc.ff();
+            mine.m = m;
+            mine.sh = sv.hi;
+            mine.sl = sv.lo;
+            const Slot w = warp_reduce_slot<kRedLse>(mine);
+            if (lane == 0) sh.lpart[slot][warp] = w;
+        }
+        cluster.sync();  // every CTA's partials are published
+        if (warp < J) {
+            const int CS = (int)cluster.num_blocks();
+            const Slot v = warp_reduce_slot<kRedLse>(lane < CS ? *cluster.map_shared_rank(&sh.lpart[slot][warp], lane)
+                                                               : neutral_slot());
             if (lane == 0) {
-                l2t[sh.look[warp]] = L2;
+                const FF l = v.sh > 0.f ? maxsum_lse(MaxSum{v.m, FF{v.sh, v.sl}}) : FF{0.f, 0.f};
+                l2t[sh.look[warp]] = ff_times_log2e(l);
                 known[sh.look[warp]] = 1;
             }
         }
@@ -801,7 +816,7 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
                 int J = 0, v = u;
                 for (;;) {
                     sh.look[J++] = v;
-                    if (J == kLook) break;
+                    if (J == Walk<T>::kLookMax) break;
                     const int c = s_kid[s_off[v]];
                     if (s_off[c + 1] - s_off[c] <= 0 || s_known[c] != 0) break;
                     v = c;
@@ -810,12 +825,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             }
             __syncthreads();
             const int J = sh.nlook;
-            float2(*cst)[kMaxSliceChunks] = sh.cst[ncst];
-            ncst ^= 1;  // a CTA may stage its next round while another still reads this one
+            float2(*cst)[kMaxSliceChunks] = sh.cst;
             // x of u into P with the chunk statistics of all J rows, then their log-normalisers
             // from all chunks of the cluster (gathered into Q, free until u's first rejection)
             W.stage_look(J, P, cst);
-            W.gather_look(J, cst, reinterpret_cast<float2 *>(Q), ts.l2t, ts.pre);
+            W.gather_look(J, cst, ncst, ts.l2t, ts.pre);
+            ncst ^= 1;
         }
         const FF L2t = s_l2t[u];
         const FF L2q = per_depth ? sh.l2q[r] : ts.l2qn[u];

@@ -405,6 +405,7 @@ struct Logit<float> {
         }
     }
     __device__ __forceinline__ static float load1(const float *row, int v) { return __ldg(row + v); }
+    __device__ __forceinline__ static float neg_inf() { return -INFINITY; }
 };
 
 __device__ __forceinline__ float bf16_bits_to_f32(uint32_t bits16) { return __uint_as_float(bits16 << 16); }
@@ -429,6 +430,7 @@ struct Logit<__nv_bfloat16> {
     __device__ __forceinline__ static float load1(const __nv_bfloat16 *row, int v) {
         return bf16_bits_to_f32(__ldg(reinterpret_cast<const unsigned short *>(row) + v));
     }
+    __device__ __forceinline__ static __nv_bfloat16 neg_inf() { return __ushort_as_bfloat16((unsigned short)0xff80u); }
 };
 
 template <typename T>
@@ -449,6 +451,10 @@ struct RawGroup<__nv_bfloat16> {
             w.z = h[4] | ((uint32_t)h[5] << 16);
             w.w = h[6] | ((uint32_t)h[7] << 16);
         }
+    }
+    // logits v0..v0+7 of a copy in shared memory (v0 a multiple of 8)
+    __device__ __forceinline__ void load_shared(const unsigned char *zone, int v0) {
+        w = *reinterpret_cast<const uint4 *>(zone + 2 * v0);
     }
     __device__ __forceinline__ void unpack(float z[8]) const {
         const uint32_t u[4] = {w.x, w.y, w.z, w.w};
@@ -473,6 +479,10 @@ struct RawGroup<float> {
             a = make_float4(z[0], z[1], z[2], z[3]);
             b = make_float4(z[4], z[5], z[6], z[7]);
         }
+    }
+    __device__ __forceinline__ void load_shared(const unsigned char *zone, int v0) {
+        a = *reinterpret_cast<const float4 *>(zone + 4 * v0);
+        b = *reinterpret_cast<const float4 *>(zone + 4 * v0 + 16);
     }
     __device__ __forceinline__ void unpack(float z[8]) const {
         z[0] = a.x; z[1] = a.y; z[2] = a.z; z[3] = a.w;
