@@ -101,6 +101,7 @@ struct VerifyArgs {
     int M;        // node ids below M with children are pre-computed (pre_chain == 0), or
                   // the first M internal nodes of the first-child chain (pre_chain == 1)
     int pre_chain;
+    int copy_early;  // the pre-pass runs just before the walk: the walk copies its tree before waiting
     int Lq;       // per-depth q rows whose normaliser the pre-pass computes (0 for per-node rows)
     int qn;       // 1: the pre-pass computes each internal node's per-node q-row normaliser (slot u)
     int B;
@@ -580,10 +581,12 @@ struct TreeSmem {
 };
 
 // Copy of tree b for a walk: topology, per child slot its parent, target and q logits and
-// acceptance uniform, the pre-pass results. Sets sh.cbad on inconsistent tree arrays. Every
-// thread of the CTA calls it; it ends with the CTA synchronised.
+// acceptance uniform. It reads only the tree, the tokens and the logits (written before the
+// pre-pass began), so a walk may run it before waiting for the pre-pass. Sets sh.cbad on
+// inconsistent tree arrays. Every thread of the CTA calls it; it ends with the CTA
+// synchronised.
 template <typename T>
-__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth, bool pre_q) {
+__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
     const int NN = a.N + 1;
     TreeSmem ts;
     ts.l2t = reinterpret_cast<FF *>(base);
@@ -611,17 +614,6 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
             ts.tok[i] = __ldg(tok + i);
             ts.row[i] = __ldg(row + i);
         }
-        if (pre_q)
-            for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
-                const float2 v = a.pre[(int64_t)b * NN + i].l2q;
-                sh.l2q[i] = FF{v.x, v.y};
-            }
-        if (a.M > 0 || a.qn)  // every node's slot, in this same round of loads (used for the set below)
-            for (int i = threadIdx.x; i < NN; i += kThreads) {
-                const float4 pr = __ldg(reinterpret_cast<const float4 *>(&a.pre[(int64_t)b * NN + i]));
-                ts.l2t[i] = FF{pr.x, pr.y};
-                ts.l2qn[i] = FF{pr.z, pr.w};
-            }
         if (threadIdx.x == 0) sh.cbad = 0;
     }
     __syncthreads();
@@ -640,15 +632,6 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
         if (bad_here) sh.cbad = 1;
     }
     __syncthreads();
-    for (int u = threadIdx.x; u < NN; u += kThreads)  // the pre-computed set, as the pre-pass saw it
-        ts.pre[u] = !a.pre_chain && u < a.M && ts.off[u + 1] - ts.off[u] > 0 ? 1 : 0;
-    if (a.pre_chain) {
-        __syncthreads();
-        if (threadIdx.x < a.M) {
-            const int v = chain_node(ts.off, ts.kid, a.N, threadIdx.x);
-            if (v >= 0) ts.pre[v] = 1;
-        }
-    }
     {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
         bool bad_here = false;
         for (int j = threadIdx.x; j < a.N; j += kThreads) {
@@ -670,6 +653,34 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
     }
     __syncthreads();
     return ts;
+}
+
+// The pre-pass results for tree b (after the walk waited for the pre-pass): the pre-computed
+// set as the pre-pass chose it, its target normalisers, and the q-row normalisers (per depth
+// with pre_q, per node with a.qn). Every thread of the CTA calls it; ends synchronised.
+__device__ void load_pre(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, int b, bool pre_q) {
+    const int NN = a.N + 1;
+    if (pre_q)
+        for (int i = threadIdx.x; i < a.Lq; i += kThreads) {
+            const float2 v = a.pre[(int64_t)b * NN + i].l2q;
+            sh.l2q[i] = FF{v.x, v.y};
+        }
+    if (a.M > 0 || a.qn)  // every node's slot in one round of loads (only the set's are used)
+        for (int i = threadIdx.x; i < NN; i += kThreads) {
+            const float4 pr = *reinterpret_cast<const float4 *>(&a.pre[(int64_t)b * NN + i]);
+            ts.l2t[i] = FF{pr.x, pr.y};
+            ts.l2qn[i] = FF{pr.z, pr.w};
+        }
+    for (int u = threadIdx.x; u < NN; u += kThreads)
+        ts.pre[u] = !a.pre_chain && u < a.M && ts.off[u + 1] - ts.off[u] > 0 ? 1 : 0;
+    if (a.pre_chain) {
+        __syncthreads();
+        if (threadIdx.x < a.M) {
+            const int v = chain_node(ts.off, ts.kid, a.N, threadIdx.x);
+            if (v >= 0) ts.pre[v] = 1;
+        }
+    }
+    __syncthreads();
 }
 
 // Pre-pass, in clusters of two CTAs. Clusters [0, B*M): cluster (b, j) streams target row j of
@@ -768,7 +779,7 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
 
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
-    pdl_begin();
+    if (!a.copy_early) pdl_begin();
     extern __shared__ __align__(16) float dyn[];
     float *P = dyn;
     float *Q = dyn + a.slice;
@@ -787,8 +798,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     int par = 0;
     Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
 
-    // the tree's copy in shared memory with the pre-pass results
-    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth, true);
+    // the tree's copy in shared memory; with the pre-pass launched just before this kernel it
+    // overlaps the pre-pass's tail (it reads nothing the pre-pass writes), then the wait for
+    // the pre-pass and its results
+    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    if (a.copy_early) pdl_begin();
+    load_pre(a, sh, ts, b, true);
     const FF *s_l2t = ts.l2t;
     const int32_t *s_known = ts.pre, *s_off = ts.off, *s_kid = ts.kid, *s_tok = ts.tok, *s_row = ts.row;
     const float *s_cxt = ts.cxt, *s_cxq = ts.cxq, *s_cu = ts.cu;
@@ -992,7 +1007,8 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_trav(VerifyArgs a) {
     const bool per_depth = a.qrow_of_node == nullptr;
     int par = 0;
     Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
-    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth, true);
+    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    load_pre(a, sh, ts, b, true);
 
     auto trow_of = [&](int u) {
         return static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
@@ -1266,11 +1282,16 @@ int choose_cluster(int V, int N, int B, int *slice_out, size_t *smem_out) {
 
 // The pre-pass kernel for a's pre-computed set (target rows of M nodes per tree, q-row
 // normalisers), launched ahead of a walk.
-template <typename T>
-cudaError_t launch_pre_t(const VerifyArgs &a, int B, cudaStream_t s) {
+int64_t pre_blocks_of(const VerifyArgs &a, int B) {
     const int per = a.qn ? a.N + 1 : a.Lq;
     int64_t pre_blocks = 2 * (int64_t)B * a.M + ((int64_t)B * per + kPreThreads / 32 - 1) / (kPreThreads / 32);
-    pre_blocks += pre_blocks & 1;  // whole clusters of two (a spare q-row CTA finds no task)
+    return pre_blocks + (pre_blocks & 1);  // whole clusters of two (a spare q-row CTA finds no task)
+}
+bool pre_launched(const VerifyArgs &a, int B) { return pre_blocks_of(a, B) > 0; }
+
+template <typename T>
+cudaError_t launch_pre_t(const VerifyArgs &a, int B, cudaStream_t s) {
+    const int64_t pre_blocks = pre_blocks_of(a, B);
     if (pre_blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
     if (pre_blocks == 0) return cudaSuccess;
     const size_t psmem = (size_t)a.C * sizeof(float2) + (a.pre_chain ? (size_t)(2 * a.N + 2) * sizeof(int32_t) : 0);
@@ -1294,6 +1315,7 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
     }
     e = launch_pre_t<T>(a, B, s);
     if (e != cudaSuccess) return e;
+    a.copy_early = pre_launched(a, B) ? 1 : 0;
     return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
 
@@ -1347,6 +1369,7 @@ VerifyArgs verify_args(const RowsDesc &target, const RowsDesc &q, const float2 *
     a.pre = reinterpret_cast<PreRow *>(reinterpret_cast<char *>(status) + kWsStatusBytes);
     a.M = 0;
     a.pre_chain = 0;
+    a.copy_early = 0;
     a.Lq = qrow_of_node ? 0 : (L < N + 1 ? L : N + 1);
     a.qn = 0;
     a.B = B;

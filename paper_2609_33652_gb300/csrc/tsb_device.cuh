@@ -539,9 +539,12 @@ struct RawQuad<float> {
 // Programmatic dependent launch. Every kernel of the library starts with pdl_begin(): it
 // waits until the kernel launched before it on the stream has completed and its memory is
 // visible (griddepcontrol.wait; immediate when there is no programmatic dependency), then
-// lets the next kernel on the stream be launched (griddepcontrol.launch_dependents). No
-// global memory is touched before the wait, so launches with the programmatic-serialisation
-// attribute only overlap a kernel's launch and CTA scheduling with its predecessor's tail.
+// lets the next kernel on the stream be launched (griddepcontrol.launch_dependents). Before
+// the wait a kernel touches no global memory, with one exception: the RRS walk, launched right
+// after its own pre-pass, first copies its tree, tokens and logits, which were complete before
+// the pre-pass passed its own wait (and so before the walk could launch), and none of which the
+// pre-pass writes. Launches with the programmatic-serialisation attribute otherwise only
+// overlap a kernel's launch and CTA scheduling with its predecessor's tail.
 __device__ __forceinline__ void pdl_begin() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
