@@ -158,11 +158,9 @@ struct Scratch {
     Slot wpart[kWarps];  // per-warp partials of the current round
     Slot res;            // combined result
     FF L2t, L2q;         // log-normalisers of the target and q rows, times log2(e)
-    unsigned long long wbest[kWarps];
-    unsigned long long cbest, tbest;
+    unsigned long long wbest[kWarps], wtok[kWarps];
     int cbad;
     int path[kMaxDepthRows];      // accepted node ids (written out after the walk)
-    float clog[kMaxSliceChunks];  // per-chunk log-masses of a draw
     FF l2q[kMaxDepthRows];        // per-depth q log-normalisers (times log2 e)
     float2 cst[kLook][kMaxSliceChunks];  // chunk statistics of the slice's rows in a staging round
     Slot lpart[2][kLook];                // this CTA's partials of the round's normalisers, alternating
@@ -406,7 +404,9 @@ struct Walk {
     __device__ int draw(int node, F wt) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         // 1. chunk log-masses: eight lanes per chunk (lane g of the group takes quads g, g + 8,
-        //    ..., g + 56), four chunks per warp and iteration
+        //    ..., g + 56), four chunks per warp and iteration; 2. each chunk's key by its group's
+        //    first lane
+        unsigned long long best = 0ull;
         {
             const int g = lane & 7, grp = lane >> 3;
             for (int c0 = warp * 4; c0 < nch; c0 += kWarps * 4) {  // uniform over the warp
@@ -447,22 +447,15 @@ struct Walk {
                     sm += __shfl_xor_sync(kFull, sm, 1);
                     if (sm > 0.f) A = logf(sm);
                 }
-                if (live && g == 0) sh.clog[cl] = A;
+                if (live && g == 0 && A != -INFINITY) {  // 2. the chunk's key; the lane's best
+                    const int c = (lo >> 8) + cl;
+                    const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
+                    const unsigned long long pk = pack_key(__fadd_rn(A, gumbel_of(w)), (uint32_t)c);
+                    best = pk > best ? pk : best;
+                }
             }
         }
-        __syncthreads();
-        // 2. chunk keys, one thread per chunk, and the CTA's best chunk
-        unsigned long long best = 0ull;
-        for (int cl = threadIdx.x; cl < nch; cl += kThreads) {
-            const float A = sh.clog[cl];
-            if (A != -INFINITY) {
-                const int c = (lo >> 8) + cl;
-                const uint32_t w = draw_word(a.seed, kFinalChunk, (uint32_t)b, (uint32_t)node, (uint32_t)c);
-                const unsigned long long pk = pack_key(__fadd_rn(A, gumbel_of(w)), (uint32_t)c);
-                best = pk > best ? pk : best;
-            }
-        }
-        best = warp_max_u64(best);
+        best = warp_max_u64(best);  // the CTA's best chunk
         if (lane == 0) sh.wbest[warp] = best;
         __syncthreads();
         // 3. the best token inside this CTA's best chunk: one element per thread (threads
@@ -483,21 +476,15 @@ struct Walk {
             }
         }
         tb = warp_max_u64(tb);
-        __syncthreads();  // every warp has read sh.wbest
-        if (lane == 0) sh.wbest[warp] = tb;
+        if (lane == 0) sh.wtok[warp] = tb;
         __syncthreads();
+        Slot mine = neutral_slot();  // the CTA's pair (best chunk key, its best token), from thread 0
         if (warp == 0) {
-            const unsigned long long t = warp_max_u64(lane < kWarps ? sh.wbest[lane] : 0ull);
-            if (lane == 0) {
-                sh.cbest = cb;
-                sh.tbest = t;
+            const unsigned long long t = warp_max_u64(lane < kWarps ? sh.wtok[lane] : 0ull);
+            if (lane == 0 && cb != 0ull) {
+                mine.key = cb;
+                mine.tok = (int)key_id(t);
             }
-        }
-        __syncthreads();
-        Slot mine = neutral_slot();
-        if (threadIdx.x == 0 && sh.cbest != 0ull) {
-            mine.key = sh.cbest;
-            mine.tok = (int)key_id(sh.tbest);
         }
         reduce_round<kRedArg>(sh, par, cluster, mine);
         return sh.res.key == 0ull ? -1 : sh.res.tok;
