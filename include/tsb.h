@@ -303,7 +303,8 @@ tsb_status tsb_replay_mixed(const tsb_cfg *cfg, const tsb_logits *qrows, const v
  *   emitted token is a draw from the target law, whatever the children hold, so it verifies the
  *   first-pass tokens (plan_token) as well as WoR or mixed replays; a child with token v is
  *   accepted with probability p(v). qrows, qstats and qrow_of_node are not used and may be
- *   NULL. Every node's draw is computed in one parallel pass over all N+1 target rows.
+ *   NULL. Only the visited nodes' target rows are read (one cluster of CTAs walks each tree);
+ *   a visited row holding a NaN or +inf logit sets TSB_DEV_NONFINITE.
  * target: [B, N+1, V], row u = target logits after the path to node u. qrows / qstats /
  * qrow_of_node as in tsb_replay. Outputs: out_tokens [B, L+1] (accepted tokens then the
  * final token, -1 after), out_nodes [B, L] (accepted node ids, -1 after), out_len [B]

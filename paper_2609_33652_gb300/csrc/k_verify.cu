@@ -246,10 +246,11 @@ struct Walk {
     // past the vocabulary become -inf), or store exp(x - L) instead of x (the normalised
     // law). Loads are issued in batches of kB chunks per warp before any is used, so a slice
     // costs one memory round trip per batch.
-    template <bool NORMALISE>
+    template <bool NORMALISE, bool CHECK = false>
     __device__ void stage(const T *row, float *dst, int nw, FF L2) {
         constexpr int kB = sizeof(T) == 2 ? 9 : 5;
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        bool bad = false;  // CHECK: a NaN or +inf logit
         if (warp >= nw) return;
         const int end = lo + n;
         for (int c0 = warp; c0 < nch; c0 += nw * kB) {
@@ -272,6 +273,10 @@ struct Walk {
                     raw[e][h].unpack(x);
 #pragma unroll
                     for (int k = 0; k < 4; ++k) x[k] = __fmul_rn(x[k], a.invT);  // padding stays -inf
+                    if (CHECK) {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) bad |= !(x[k] <= FLT_MAX) && x[k] != -INFINITY;
+                    }
                     if (NORMALISE) {
 #pragma unroll
                         for (int k = 0; k < 4; ++k) x[k] = exp_shifted(x[k], L2);
@@ -280,6 +285,7 @@ struct Walk {
                 }
             }
         }
+        if (CHECK && __any_sync(kFull, bad) && lane == 0) raise_status(a.status, kDevNonFinite);
     }
 
     // One staging round over the target rows of nodes sh.look[0..J-1] (J <= kLookMax).
@@ -491,9 +497,10 @@ struct Walk {
     }
 
     // Bonus draw from the logits of `row` (a leaf, or a residual without mass).
+    template <bool CHECK = false>
     __device__ int draw_from_row(const T *row, int node) {
         __syncthreads();
-        stage<false>(row, P, kWarps, FF{0.f, 0.f});
+        stage<false, CHECK>(row, P, kWarps, FF{0.f, 0.f});
         __syncthreads();
         return draw<true>(node, [&](int j, float *v) {
             const float4 x = ld4(P, j);
@@ -1181,6 +1188,243 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_trav(VerifyArgs a) {
     cluster.sync();  // no CTA leaves while another may still read its shared memory
 }
 
+// Target-sample matching's pre-pass: the draw of each of the first kNaiveChain nodes of every
+// tree's first-child chain (the nodes a walk most likely visits; the chain's first leaf
+// included), all rows at once over the GPU, one cluster of kNaiveSplit CTAs per (tree, chain
+// position): CTA r takes the r-th quarter of the row's chunks, chunk log-masses with one warp per
+// chunk (lane l holds logits 8l..8l+7) and U chunks per warp iteration (all loads issued first,
+// the U sums reduced together), the chunk keys; the CTAs' best keys meet in CTA 0 through
+// distributed shared memory and one of its warps draws the token inside the best chunk. The
+// token goes to the node's workspace slot.
+constexpr int kNaiveChain = 10;
+constexpr int kNaiveSplit = 4;
+constexpr int kNaiveWarps = 4;
+
+// Node j of the first-child chain from the root, leaves included (the chain ends at its first
+// leaf); -1 past the end or on inconsistent arrays.
+__device__ __forceinline__ int chain_node_to_leaf(const int32_t *off, const int32_t *kid, int N, int j) {
+    int v = 0;
+    for (int k = 0; k < j; ++k) {
+        const int o = off[v];
+        if (off[v + 1] - o <= 0 || o < 0 || o >= N) return -1;
+        const int c = kid[o];
+        if (c < 1 || c > N) return -1;
+        v = c;
+    }
+    return v;
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kNaiveWarps * 32, 8) k_naive_pre(VerifyArgs a) {
+    pdl_begin();
+    constexpr int U = sizeof(T) == 2 ? 8 : 4;  // chunks per warp iteration (16-byte loads in flight per lane)
+    __shared__ uint64_t s_best[kNaiveWarps];
+    __shared__ uint64_t s_part;  // this CTA's best chunk key
+    __shared__ int s_node;
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank();
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int NN = a.N + 1;
+    const int rid = blockIdx.x / kNaiveSplit;
+    const int b = rid / a.M, j = rid - (rid / a.M) * a.M;
+    if (threadIdx.x == 0) {  // the chain's j-th node (every CTA of the cluster finds the same)
+        const int32_t *off = a.child_off + (int64_t)b * (NN + 1), *kids = a.child_ids + (int64_t)b * a.N;
+        int v = 0;
+        for (int k = 0; k < j && v >= 0; ++k) {
+            const int o = __ldg(off + v);
+            if (__ldg(off + v + 1) - o <= 0 || o < 0 || o >= a.N) {
+                v = -1;
+                break;
+            }
+            const int c = __ldg(kids + o);
+            v = c >= 1 && c <= a.N ? c : -1;
+        }
+        s_node = v;
+    }
+    __syncthreads();
+    const int u = s_node;
+    if (u < 0) return;  // past the chain's end (the whole cluster returns)
+    const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
+    const uint32_t ub = (uint32_t)b, un = (uint32_t)u;
+    const int per = (a.C + kNaiveSplit - 1) / kNaiveSplit;
+    const int c_lo = rank * per, c_hi = min(a.C, c_lo + per);
+    const int units = c_hi > c_lo ? (c_hi - c_lo + U - 1) / U : 0;
+    uint64_t best = 0ull;
+    bool bad = false;
+    for (int un0 = warp; un0 < units; un0 += kNaiveWarps) {  // uniform over the warp
+        const int cu = c_lo + un0 * U;
+        RawGroup<T> raw[U];
+#pragma unroll
+        for (int k = 0; k < U; ++k)
+            if (cu + k < c_hi) raw[k].load(row, (cu + k) * kChunk + lane * 8, a.V);
+        float mcs[U], part[U];
+#pragma unroll
+        for (int k = 0; k < U; ++k) {
+            mcs[k] = -INFINITY;
+            part[k] = 0.f;
+            if (cu + k >= c_hi) continue;  // uniform over the warp
+            float z[8];
+            raw[k].unpack(z);  // padding past V is -inf
+            float zm = z[0];
+#pragma unroll
+            for (int i = 1; i < 8; ++i) zm = fmaxf(zm, z[i]);
+            mcs[k] = __fmul_rn(warp_max(zm), a.invT);
+            const float2 offs = exp_offset(mcs[k]);
+#pragma unroll
+            for (int i = 0; i < 8; ++i) part[k] += chunk_term(z[i], a.invT, offs.x);
+            part[k] = chunk_sum_fix(part[k], offs.y);
+        }
+        // the U chunk sums at once; the lane holding a chunk's sum keys that chunk
+        const float tot = warp_multi_sum<U>(part);
+        const int ch = multi_sum_index<U>(lane), c = cu + ch;
+        if (lane % (32 / U) == 0 && c < c_hi) {
+            float mc = mcs[0];
+#pragma unroll
+            for (int k = 1; k < U; ++k) mc = ch == k ? mcs[k] : mc;
+            bad |= !(tot == tot) || isinf(mc);
+            const uint32_t w = draw_word(a.seed, kFinalChunk, ub, un, (uint32_t)c);
+            const uint64_t k = pack_key(__fadd_rn(__fadd_rn(mc, logf(tot)), gumbel_of(w)), (uint32_t)c);
+            best = k > best ? k : best;
+        }
+    }
+    if (__any_sync(kFull, bad) && lane == 0) raise_status(a.status, kDevNonFinite);
+    best = warp_max_u64(best);
+    if (lane == 0) s_best[warp] = best;
+    __syncthreads();
+    if (warp == 0) {
+        const uint64_t v = warp_max_u64(lane < kNaiveWarps ? s_best[lane] : 0ull);
+        if (lane == 0) s_part = v;
+    }
+    cluster.sync();  // every CTA's best chunk key is published
+    uint64_t cb = 0ull;
+    if (rank == 0 && warp == 0) cb = warp_max_u64(lane < kNaiveSplit ? *cluster.map_shared_rank(&s_part, lane) : 0ull);
+    cluster.sync();  // CTA 0 has read the others; they may leave
+    if (rank != 0 || warp != 0) return;
+    int32_t *slot = reinterpret_cast<int32_t *>(&a.pre[(int64_t)b * NN + u].pad[0]);
+    if (cb == 0ull) {  // no finite logit (status already raised)
+        if (lane == 0) *slot = -1;
+        return;
+    }
+    const int c = (int)key_id(cb);
+    const int v0 = c * kChunk + lane * 8;
+    float x[8];
+    Logit<T>::load8(row, v0, a.V, x);
+    const Words4 w0 = draw_block(a.seed, kFinal, ub, un, (uint32_t)(v0 >> 2));
+    const Words4 w1 = draw_block(a.seed, kFinal, ub, un, (uint32_t)(v0 >> 2) + 1u);
+    uint64_t tk = 0ull;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        if (v0 + i < a.V) {
+            const uint32_t wi = i < 4 ? w0.w[i] : w1.w[i - 4];
+            const uint64_t k = pack_key(__fadd_rn(__fmul_rn(x[i], a.invT), gumbel_of(wi)), (uint32_t)(v0 + i));
+            tk = k > tk ? k : tk;
+        }
+    }
+    tk = warp_max_u64(tk);
+    if (lane == 0) *slot = tk == 0ull ? -1 : (int32_t)key_id(tk);
+}
+
+// Target-sample matching ("Naive" in Table 2; Sec. 2.3) by walking: at the current node u a
+// token y is drawn from the target law p_u with the two-level Gumbel-max of the bonus token
+// (chunk keys log(chunk mass) + G(U[final chunk, u, c]), then x_v + G(U[final, u, v]) inside
+// the best chunk); the first child of u carrying y is accepted and the walk continues there,
+// otherwise y is the final token (at a leaf: the bonus token). One cluster per tree with the
+// RRS walk's slices; the first kNaiveChain nodes of the first-child chain come drawn from the
+// pre-pass, any other visit stages the node's target row (its x into P) and draws, so only the
+// chain's rows and the visited ones are read. A row holding a NaN or +inf logit sets the
+// non-finite status bit. Which kernel draws a node depends only on the topology.
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 1) k_verify_naive(VerifyArgs a) {
+    extern __shared__ __align__(16) float dyn[];
+    float *P = dyn;
+    float *Q = dyn + a.slice;
+    __shared__ Scratch sh;
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int CS = (int)cluster.num_blocks();
+    const int crank = (int)cluster.block_rank();
+    const int b = blockIdx.x / CS;
+    const int NN = a.N + 1;
+    const int lo = crank * a.slice;
+    const int n = max(0, min(a.V - lo, a.slice));
+    const bool writer = crank == 0 && threadIdx.x == 0;
+    int par = 0;
+    Walk<T> W{a, sh, cluster, P, Q, par, b, lo, n, (n + kChunk - 1) / kChunk};
+
+    int32_t *s_off = reinterpret_cast<int32_t *>(dyn + 2 * a.slice);  // [N+2]
+    int32_t *s_kid = s_off + (NN + 1);                                // [N]
+    int32_t *s_tok = s_kid + a.N;                                     // [N+1]
+    int32_t *s_pre = s_tok + NN;                                      // [N+1] pre-drawn token, -2 none
+    // the tree and tokens (complete before the pre-pass passed its own wait, and not written by
+    // it) before waiting for the pre-pass, then the pre-drawn tokens of the chain's nodes
+    for (int i = threadIdx.x; i <= NN; i += kThreads) s_off[i] = __ldg(a.child_off + (int64_t)b * (NN + 1) + i);
+    for (int i = threadIdx.x; i < a.N; i += kThreads) s_kid[i] = __ldg(a.child_ids + (int64_t)b * a.N + i);
+    for (int i = threadIdx.x; i < NN; i += kThreads) {
+        s_tok[i] = __ldg(a.token + (int64_t)b * NN + i);
+        s_pre[i] = -2;
+    }
+    pdl_begin();
+    __syncthreads();
+    if (threadIdx.x < a.M) {
+        const int v = chain_node_to_leaf(s_off, s_kid, a.N, threadIdx.x);
+        if (v >= 0) s_pre[v] = *reinterpret_cast<const int32_t *>(&a.pre[(int64_t)b * NN + v].pad[0]);
+    }
+    __syncthreads();
+    cluster.sync();  // every CTA of the cluster runs before any distributed access
+
+    int u = 0, nacc = 0, final_tok = -1;
+    bool bad = false;
+    for (int step = 0; step <= a.L; ++step) {
+        const T *trow = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)u * a.t_rstride;
+        // every CTA holds the same y: pre-drawn, or drawn here from the node's staged row
+        const int y = s_pre[u] != -2 ? s_pre[u] : W.template draw_from_row<true>(trow, u);
+        const int o = s_off[u], m = s_off[u + 1] - o;
+        if (o < 0 || m < 0 || m > kMaxK || o + m > a.N) {
+            bad = true;
+            break;
+        }
+        int next = -1;
+        for (int i = 0; i < m && y >= 0; ++i) {
+            const int c = s_kid[o + i];
+            if (c < 1 || c > a.N) {
+                bad = true;
+                break;
+            }
+            if (s_tok[c] == y) {
+                next = c;
+                break;
+            }
+        }
+        if (bad || next < 0) {
+            final_tok = y;
+            break;
+        }
+        if (nacc >= a.L) {  // deeper than the depth cap: the tree arrays are inconsistent
+            bad = true;
+            break;
+        }
+        if (writer) sh.path[nacc] = next;  // no global store while cluster barriers follow
+        ++nacc;
+        u = next;
+    }
+    if (writer) {
+        int32_t *otok = a.out_tokens + (int64_t)b * (a.L + 1);
+        int32_t *onode = a.out_nodes + (int64_t)b * a.L;
+        if (bad) raise_status(a.status, kDevBadTree);
+        if (!bad && final_tok < 0) raise_status(a.status, kDevNonFinite);  // no finite logit to draw
+        const int k_acc = bad ? 0 : nacc;
+        for (int k = 0; k < k_acc; ++k) {
+            otok[k] = s_tok[sh.path[k]];
+            onode[k] = sh.path[k];
+        }
+        otok[k_acc] = bad ? -1 : final_tok;
+        for (int k = k_acc + 1; k <= a.L; ++k) otok[k] = -1;
+        for (int k = k_acc; k < a.L; ++k) onode[k] = -1;
+        a.out_len[b] = bad ? 0 : k_acc + 1;
+    }
+    cluster.sync();  // no CTA leaves while another may still read its shared memory
+}
+
 constexpr size_t kSmemLimit = 210 * 1024;
 
 // Chunk-aligned slice of each CTA and the dynamic shared memory it needs for cluster size cs
@@ -1324,6 +1568,25 @@ cudaError_t launch_trav_t(VerifyArgs a, int B, cudaStream_t s) {
     return launch_pdl(k_verify_trav<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
 
+template <typename T>
+cudaError_t launch_naive_walk_t(VerifyArgs a, int B, cudaStream_t s) {
+    int slice = 0;
+    size_t smem = 0;
+    const int cs = choose_cluster<T>(a.V, a.N, B, &slice, &smem);  // the RRS walk's slices
+    if (cs < 0) return cudaErrorInvalidValue;
+    a.slice = slice;
+    cudaError_t e = cudaFuncSetAttribute(k_verify_naive<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+    if (e != cudaSuccess) return e;
+    if (cs > 8) {
+        e = cudaFuncSetAttribute(k_verify_naive<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        if (e != cudaSuccess) return e;
+    }
+    e = launch_pdl(k_naive_pre<T>, dim3((unsigned)(B * a.M * kNaiveSplit)), dim3(kNaiveWarps * 32), 0, s,
+                   kNaiveSplit, a);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(k_verify_naive<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
+}
+
 VerifyArgs verify_args(const RowsDesc &target, const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node,
                        int B, int N, int L, const TreeDesc &tree, const int32_t *token, float invT, uint64_t seed,
                        int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, uint32_t *status) {
@@ -1388,6 +1651,19 @@ cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const f
     a.qn = qrow_of_node ? 1 : 0;  // per-node q rows: every internal node's normaliser
     if (target.dtype == 1) return launch_rrs_t<__nv_bfloat16>(a, B, s);
     return launch_rrs_t<float>(a, B, s);
+}
+
+cudaError_t launch_verify_naive(const RowsDesc &target, int B, int N, int L, const TreeDesc &tree,
+                                const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
+                                int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s) {
+    VerifyArgs a = verify_args(target, target, nullptr, nullptr, B, N, L, tree, token, invT, seed, out_tokens,
+                               out_nodes, out_len, status);
+    a.q = nullptr;
+    a.q_R = 0;
+    a.Lq = 0;
+    a.M = N + 1 < kNaiveChain ? N + 1 : kNaiveChain;  // chain positions drawn by the pre-pass
+    if (target.dtype == 1) return launch_naive_walk_t<__nv_bfloat16>(a, B, s);
+    return launch_naive_walk_t<float>(a, B, s);
 }
 
 }  // namespace tsb

@@ -333,7 +333,8 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
             return TSB_ERR_ARG;
         return cuda_status(tsb::launch_verify_naive(rows_of(target), cfg->B, cfg->N, cfg->L, tree_of(tree), token,
                                                     inv_temperature(cfg->temperature), seed, out_tokens,
-                                                    out_nodes, out_len, ws, (cudaStream_t)stream));
+                                                    out_nodes, out_len, static_cast<uint32_t *>(ws),
+                                                    (cudaStream_t)stream));
     }
     if (st == TSB_OK) st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
     if (st == TSB_OK && target->dtype != qrows->dtype) st = TSB_ERR_DTYPE;

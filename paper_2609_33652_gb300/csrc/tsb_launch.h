@@ -123,7 +123,7 @@ cudaError_t launch_replay_mixed(const RowsDesc &q, const float2 *qstats, const i
 
 cudaError_t launch_verify_naive(const RowsDesc &target, int B, int N, int L, const TreeDesc &tree,
                                 const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,
-                                int32_t *out_nodes, int32_t *out_len, void *ws, cudaStream_t s);
+                                int32_t *out_nodes, int32_t *out_len, uint32_t *status, cudaStream_t s);
 
 cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
                               const int32_t *qrow_of_node, int B, int N, int L, const TreeDesc &tree,
