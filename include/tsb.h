@@ -68,6 +68,7 @@ typedef enum {
 #define TSB_DEV_NONFINITE 0x1u /* a logit was NaN or infinite after the temperature multiply */
 #define TSB_DEV_BAD_INDEX 0x2u /* a token, row index or child index was out of range */
 #define TSB_DEV_BAD_TREE 0x4u  /* tree arrays inconsistent (e.g. block verification on a non-chain) */
+#define TSB_DEV_CHECK 0x8u     /* libtsb_checked.so: a bounds check of a data-dependent index failed */
 
 typedef enum { TSB_F32 = 0, TSB_BF16 = 1 } tsb_dtype;
 

@@ -1,4 +1,6 @@
-"""Builds libtsb.so in-tree: every csrc/*.cu compiled in parallel for sm_103a, then linked.
+"""Builds libtsb.so in-tree: every csrc/*.cu compiled in parallel for sm_103a, then linked; and
+libtsb_checked.so, the same sources with TSB_CHECKED (every data-dependent shared-memory fill
+position and index bounds-checked, a failed check setting TSB_DEV_CHECK in the status word).
 
     python -m paper_2609_33652_gb300.build [--force]
 """
@@ -16,6 +18,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libtsb.so")
+BUILD_CHECKED = os.path.join(HERE, "_build_checked")
+LIB_CHECKED = os.path.join(HERE, "libtsb_checked.so")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-I", os.path.join(ROOT, "include")]
 
@@ -36,22 +40,27 @@ def _deps():
         os.path.join(ROOT, "include", "tsb.h"), os.path.abspath(__file__)]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIB):
+def up_to_date(lib: str = LIB) -> bool:
+    if not os.path.exists(lib):
         return False
-    t = os.path.getmtime(LIB)
+    t = os.path.getmtime(lib)
     return all(os.path.getmtime(p) <= t for p in _deps())
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
-    if not force and up_to_date():
+    """Both libraries; their translation units compile in one pool."""
+    variants = [(LIB, BUILD, []), (LIB_CHECKED, BUILD_CHECKED, ["-DTSB_CHECKED"])]
+    todo = [v for v in variants if force or not up_to_date(v[0])]
+    if not todo:
         return LIB
-    os.makedirs(BUILD, exist_ok=True)
     cc = nvcc()
+    srcs = _sources()
 
-    def compile_one(src):
-        obj = os.path.join(BUILD, os.path.basename(src)[:-3] + ".o")
-        cmd = [cc, *ARCH, *FLAGS, "-c", src, "-o", obj]
+    def compile_one(job):
+        src, out_dir, extra = job
+        os.makedirs(out_dir, exist_ok=True)
+        obj = os.path.join(out_dir, os.path.basename(src)[:-3] + ".o")
+        cmd = [cc, *ARCH, *FLAGS, *extra, "-c", src, "-o", obj]
         r = subprocess.run(cmd, capture_output=True, text=True)
         if r.returncode != 0:
             raise RuntimeError(f"nvcc failed on {src}:\n{r.stdout}\n{r.stderr}")
@@ -59,14 +68,16 @@ def build(force: bool = False, verbose: bool = False) -> str:
             print(r.stdout, r.stderr, file=sys.stderr)
         return obj
 
-    srcs = _sources()
-    with cf.ThreadPoolExecutor(max_workers=max(1, min(len(srcs), os.cpu_count() or 4))) as ex:
-        objs = list(ex.map(compile_one, srcs))
-    tmp = LIB + f".tmp{os.getpid()}"
-    r = subprocess.run([cc, *ARCH, "-shared", "-o", tmp, *objs], capture_output=True, text=True)
-    if r.returncode != 0:
-        raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB)
+    jobs = [(src, out_dir, extra) for (_, out_dir, extra) in todo for src in srcs]
+    with cf.ThreadPoolExecutor(max_workers=max(1, min(len(jobs), os.cpu_count() or 4))) as ex:
+        objs = list(ex.map(compile_one, jobs))
+    for k, (lib, _, _) in enumerate(todo):
+        mine = objs[k * len(srcs):(k + 1) * len(srcs)]
+        tmp = lib + f".tmp{os.getpid()}"
+        r = subprocess.run([cc, *ARCH, "-shared", "-o", tmp, *mine], capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
+        os.replace(tmp, lib)
     return LIB
 
 

@@ -138,7 +138,10 @@ __device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st, ui
     const uint64_t lb = s_lb;
     for (int c = threadIdx.x; c < C; c += NT) {
         const uint64_t k = pack_key(st[c].x, (uint32_t)c);
-        if (k >= lb) cand[atomicAdd(&s_n, 1)] = k;
+        if (k >= lb) {
+            const int pos = atomicAdd(&s_n, 1);
+            if (in_bounds(pos, C, a.status)) cand[pos] = k;
+        }
     }
     __syncthreads();
     if (C >= K) {
@@ -358,10 +361,12 @@ __device__ __forceinline__ void depth_prefix_fixed(const float2 *lse, int L, lon
 // reused for the child-list starts. All NT threads of the CTA call it after a barrier.
 template <int NT>
 __device__ void emit_tree(int b, int N, const int32_t *n_parent, const int32_t *n_depth, const int32_t *n_rank,
-                          const int32_t *n_token, int32_t *n_count, const float *n_score, const TreeDesc &tree) {
+                          const int32_t *n_token, int32_t *n_count, const float *n_score, const TreeDesc &tree,
+                          uint32_t *status) {
     const int NN = N + 1;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    for (int i = 1 + threadIdx.x; i <= N; i += NT) atomicAdd(&n_count[n_parent[i]], 1);
+    for (int i = 1 + threadIdx.x; i <= N; i += NT)
+        if (in_bounds(n_parent[i], NN, status)) atomicAdd(&n_count[n_parent[i]], 1);
     __syncthreads();
     int32_t *off = tree.child_off + (int64_t)b * (NN + 1);
     if (warp == 0) {
@@ -813,6 +818,8 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
             const int pos = epos[x];
             if (pos < 0 || pos >= N) continue;
             const int i = pos + 1, d = einfo[x] & 255, r = einfo[x] >> 8;
+            if (epar[x] >= 0 && !in_bounds(epar[x], M, a.status)) continue;
+            if (!in_bounds(d - 1, L, a.status) || !in_bounds(r, K, a.status)) continue;
             const int par = epar[x] < 0 ? 0 : epos[epar[x]] + 1;
             if (par >= i) bad = true;
             n_parent[i] = par;
@@ -830,7 +837,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
             n_score[0] = 0.f;
         }
         __syncthreads();
-        emit_tree<kHeapThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
+        emit_tree<kHeapThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree, a.status);
         return;
     }
     // The expansion (warp 0). Per pop the critical path is the warp maximum, three shuffles,
@@ -913,7 +920,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
     }
     __syncthreads();
 
-    emit_tree<kHeapThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
+    emit_tree<kHeapThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree, a.status);
 }
 
 // ---------------------------------------------------------------------------------------
@@ -1123,7 +1130,7 @@ __global__ void __launch_bounds__(kEptThreads) k_plan_ept(EptArgs a) {
     }
     if (bad) raise_status(a.status, kDevBadTree);
     __syncthreads();
-    emit_tree<kEptThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree);
+    emit_tree<kEptThreads>(b, N, n_parent, n_depth, n_rank, n_token, n_count, n_score, a.tree, a.status);
 }
 
 template <int S>

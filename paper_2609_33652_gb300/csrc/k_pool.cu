@@ -530,7 +530,10 @@ __device__ void for_keys_above(const SelectArgs &a, const T *row, const float2 *
     __syncthreads();
     const uint32_t hi = (uint32_t)(thr >> 32);
     for (int c = threadIdx.x; c < a.C; c += kSelThreads)
-        if (ord_f32(st[c].x) >= hi) chunks[atomicAdd(&sh.nch, 1)] = c;
+        if (ord_f32(st[c].x) >= hi) {
+            const int pos = atomicAdd(&sh.nch, 1);
+            if (in_bounds(pos, a.C, nullptr)) chunks[pos] = c;
+        }
     __syncthreads();
     const int nch = sh.nch;
     for (int i = warp; i < nch; i += NW) {

@@ -173,7 +173,10 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
         if (!single) {  // the chunk keys that reach the bound, then the top msel by rank
             const uint64_t lb = s_lb;
             for (int c = threadIdx.x; c < a.C; c += kThreads)
-                if (ckeys[c] >= lb) ebuf[atomicAdd(&s_n, 1)] = ckeys[c];
+                if (ckeys[c] >= lb) {
+                    const int pos = atomicAdd(&s_n, 1);
+                    if (in_bounds(pos, ecap, a.status)) ebuf[pos] = ckeys[c];
+                }
             __syncthreads();
             const int n = s_n;
             for (int i = threadIdx.x; i < n; i += kThreads) {

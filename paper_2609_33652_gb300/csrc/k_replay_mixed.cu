@@ -123,7 +123,10 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? 8 : 2) k_replay_mixed(Mi
         const float tau = tk == 0ull ? -INFINITY : key_value(tk);
         // 2b. the chunks whose maximum reaches tau
         for (int c = threadIdx.x; c < a.C; c += kThreads)
-            if (st[c].x >= tau) clist[atomicAdd(&s_ncand, 1)] = c;
+            if (st[c].x >= tau) {
+                const int pos = atomicAdd(&s_ncand, 1);
+                if (in_bounds(pos, a.C, a.status)) clist[pos] = c;
+            }
         __syncthreads();
         // 2c. their logits >= tau, one warp per chunk, into per-lane lists
         const int nc = s_ncand;

@@ -14,9 +14,26 @@ constexpr unsigned kFull = 0xffffffffu;
 
 enum Purpose : uint32_t { kReplayChunk = 0, kReplayElem = 1, kAccept = 2, kFinal = 3, kBlockEta = 4, kFinalChunk = 5 };
 
-constexpr uint32_t kDevNonFinite = 1u, kDevBadIndex = 2u, kDevBadTree = 4u;
+constexpr uint32_t kDevNonFinite = 1u, kDevBadIndex = 2u, kDevBadTree = 4u, kDevCheck = 8u;
 
 __device__ __forceinline__ void raise_status(uint32_t *status, uint32_t bits) { atomicOr(status, bits); }
+
+// Bounds check of a data-dependent index (a shared-memory fill position from an atomic counter,
+// a node, token or row index read from the caller's arrays). In the checked build (TSB_CHECKED)
+// an index outside [0, n) sets kDevCheck in the status word (when there is one) and the caller
+// skips the access; otherwise it returns true and compiles to nothing.
+__device__ __forceinline__ bool in_bounds(long long i, long long n, uint32_t *status) {
+#ifdef TSB_CHECKED
+    if (i >= 0 && i < n) return true;
+    if (status) raise_status(status, kDevCheck);
+    return false;
+#else
+    (void)i;
+    (void)n;
+    (void)status;
+    return true;
+#endif
+}
 
 // ---------------------------------------------------------------------------------------
 // Philox4x32-10 (Salmon, Moraes, Dror & Shaw, SC 2011): ten rounds of two 32x32->64

@@ -8,6 +8,7 @@ every output and scratch buffer one configuration needs.
 """
 from __future__ import annotations
 
+import contextlib
 import ctypes
 import os
 from dataclasses import dataclass
@@ -16,13 +17,14 @@ import torch
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(_HERE, "libtsb.so")
+LIB_CHECKED_PATH = os.path.join(_HERE, "libtsb_checked.so")
 
 TSB_OK = 0
 STATUS_NAMES = {0: "TSB_OK", 1: "TSB_ERR_ARG", 2: "TSB_ERR_SHAPE", 3: "TSB_ERR_DTYPE", 4: "TSB_ERR_ALIGN",
                 5: "TSB_ERR_WORKSPACE", 6: "TSB_ERR_CUDA", 7: "TSB_ERR_DEVICE"}
 TSB_F32, TSB_BF16 = 0, 1
 TSB_VERIFY_RRS, TSB_VERIFY_BLOCK, TSB_VERIFY_NAIVE, TSB_VERIFY_TRAVERSAL = 0, 1, 2, 3
-TSB_DEV_NONFINITE, TSB_DEV_BAD_INDEX, TSB_DEV_BAD_TREE = 0x1, 0x2, 0x4
+TSB_DEV_NONFINITE, TSB_DEV_BAD_INDEX, TSB_DEV_BAD_TREE, TSB_DEV_CHECK = 0x1, 0x2, 0x4, 0x8
 TSB_CHUNK = 256
 
 EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_bytes", "tsb_workspace_init",
@@ -71,10 +73,27 @@ def load():
     global _lib
     if _lib is not None:
         return _lib
-    if not os.path.exists(LIB_PATH):
-        raise RuntimeError(f"libtsb.so not found at {LIB_PATH}; build it with "
+    _lib = _open(LIB_PATH)
+    return _lib
+
+
+@contextlib.contextmanager
+def checked_library():
+    """Within the block every call goes to libtsb_checked.so (the TSB_CHECKED build)."""
+    global _lib
+    saved = load()
+    _lib = _open(LIB_CHECKED_PATH)
+    try:
+        yield _lib
+    finally:
+        _lib = saved
+
+
+def _open(path):
+    if not os.path.exists(path):
+        raise RuntimeError(f"{os.path.basename(path)} not found at {path}; build it with "
                            "`python -m paper_2609_33652_gb300.build` (or __graft_entry__.build())")
-    lib = ctypes.CDLL(LIB_PATH)
+    lib = ctypes.CDLL(path)
     sig = {
         "tsb_version": (_I32, []),
         "tsb_status_str": (ctypes.c_char_p, [_I32]),
@@ -99,7 +118,6 @@ def load():
         fn = getattr(lib, name)
         fn.restype = res
         fn.argtypes = args
-    _lib = lib
     return lib
 
 

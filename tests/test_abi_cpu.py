@@ -37,6 +37,17 @@ def test_exports_every_declared_function(lib):
         assert hasattr(lib, n), n
 
 
+def test_checked_build_exports_the_same_functions(lib):
+    """libtsb_checked.so (the TSB_CHECKED build) loads and exports every declared function;
+    the binding switches to it inside tsb.checked_library() and back afterwards."""
+    with tsb.checked_library() as checked:
+        for n in _declared():
+            assert hasattr(checked, n), n
+        assert tsb.load() is checked
+        assert tsb.tsb_version() >= 100
+    assert tsb.load() is lib
+
+
 def test_header_is_plain_c(tmp_path):
     """include/tsb.h is a C header: it compiles as strict C99 (and as C++) on its own."""
     import shutil
