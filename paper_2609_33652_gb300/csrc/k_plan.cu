@@ -108,6 +108,7 @@ __device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st, ui
     if (warp == 0) {
         // 3. lower bound of tau (= the K-th largest chunk key): the K-th largest of the warps'
         //    keys (K distinct chunk keys reach it), or 0 when they hold fewer than K keys
+        __syncwarp();  // converged before the shuffles (the warp reductions' note)
         const uint64_t v = lane < NW * r ? wl[lane / r][lane - (lane / r) * r] : 0ull;
         int rk = 0, nz = 0;
         for (int j = 0; j < 32; ++j) {
@@ -160,6 +161,7 @@ __device__ void topk_from_stats(const TopkArgs &a, int row, const float2 *st, ui
     el.clear();
     for (int cb = warp * 32; cb < C; cb += NT) {
         const int c = cb + lane;
+        __syncwarp();
         unsigned mask = __ballot_sync(kFull, c < C && st[c].x >= tau);
         while (mask) {
             int cs[4];
@@ -335,6 +337,7 @@ __device__ __forceinline__ long long fix_of(float x) { return __float2ll_rn(__fm
 // depth order and rounded onto the fixed grid once per depth. Called by one whole warp; lane 0
 // writes CL[0..L].
 __device__ __forceinline__ void depth_prefix_fixed(const float2 *lse, int L, long long *CL) {
+    __syncwarp();
     const int lane = threadIdx.x & 31;
     FF l0 = FF{0.f, 0.f}, l1 = FF{0.f, 0.f};
     if (lane < L) {
@@ -370,6 +373,7 @@ __device__ void emit_tree(int b, int N, const int32_t *n_parent, const int32_t *
     __syncthreads();
     int32_t *off = tree.child_off + (int64_t)b * (NN + 1);
     if (warp == 0) {
+        __syncwarp();
         const int per = (NN + 31) / 32;
         const int lo = min(NN, lane * per), hi = min(NN, lo + per);
         int s = 0;
@@ -522,6 +526,7 @@ __device__ long long nth_bound(SelShared &ss, int N, long long hi, long long lo,
         fill(s1, s2, round == 0 ? -1 : ss.jstar, ss.hist);
         __syncthreads();
         if (warp == 0) {  // the first bin whose inclusive prefix reaches N (two bins per lane)
+            __syncwarp();
             const int base = round == 0 ? 0 : ss.cum;
             const int h0 = ss.hist[2 * lane], h1 = ss.hist[2 * lane + 1];
             int incl = h0 + h1;
@@ -613,6 +618,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
     }
     __syncthreads();
     if (warp == 0) {  // Bk[d] = dl[1][0] + ... + dl[d][0] by a warp scan (depths lane + 1, lane + 33)
+        __syncwarp();
         const long long a0 = lane < L ? dl[(lane + 1) * K] : 0, a1 = lane + 32 < L ? dl[(lane + 33) * K] : 0;
         long long c0 = lane < L ? dl[(lane + 1) * K] - dl[(lane + 1) * K + K - 1] : 0;
         const long long c1 = lane + 32 < L ? dl[(lane + 33) * K] - dl[(lane + 33) * K + K - 1] : 0;
@@ -808,6 +814,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
                     n += add;
                 }
             }
+            __syncwarp();  // after the lanes' ancestor walks
             n += __shfl_xor_sync(kFull, n, 1);
             n += __shfl_xor_sync(kFull, n, 2);
             if (x < M && sub == 0) epos[x] = n;
@@ -855,6 +862,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
         fr.rescan();
         int nchild = 1;
         for (int i = 1; i <= N; ++i) {
+            __syncwarp();
             const unsigned ck = coarse_of(fr.bk);
             const unsigned m0 = __reduce_max_sync(kFull, ck);
             unsigned c = __ballot_sync(kFull, ck == m0);
@@ -1075,6 +1083,7 @@ __global__ void __launch_bounds__(kEptThreads) k_plan_ept(EptArgs a) {
         unsigned long long kA = nA > 0 ? okey_of(skey[sA]) : 0ull;
         unsigned long long kB = nB > 0 ? okey_of(skey[sB]) : 0ull;
         for (int i = 1; i <= N; ++i) {
+            __syncwarp();
             const bool useB = kB > kA;  // equal keys: the shallower layer A first
             const unsigned long long kb = useB ? kB : kA;
             const unsigned wd = 255u - (unsigned)(useB ? dB : dA);

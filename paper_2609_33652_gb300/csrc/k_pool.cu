@@ -396,6 +396,7 @@ __global__ void __launch_bounds__(kVpThreads) k_verify_pooled(VerifyPoolArgs a) 
                     break;
                 }
                 const int y = a.token[(int64_t)b * NN + c];
+                __syncwarp();
                 const unsigned hit0 = __ballot_sync(kFull, lane < a.P && sh.pool[lane] == y);
                 const unsigned hit1 = __ballot_sync(kFull, lane + 32 < a.P && sh.pool[lane + 32] == y);
                 const int k = hit0 ? __ffs(hit0) - 1 : (hit1 ? 32 + __ffs(hit1) - 1 : -1);

@@ -151,6 +151,7 @@ __global__ void __launch_bounds__(kThreads, KCAP <= 8 ? kMinBlocks : 2) k_replay
                 const uint64_t v = warp_max_u64(lane < kWarps ? cand[lane][0] : 0ull);
                 if (lane == 0) sel[0] = v;
             } else {
+                __syncwarp();  // converged before the shuffles (the warp reductions' note)
                 const uint64_t v = lane < kWarps * rr ? cand[lane / rr][lane - (lane / rr) * rr] : 0ull;
                 int rk = 0, nz = 0;
                 for (int j = 0; j < kWarps * rr; ++j) {

@@ -133,6 +133,7 @@ __device__ __forceinline__ FF rescale_to(float m, FF s, float M) {
 
 template <int KIND>
 __device__ __forceinline__ Slot warp_reduce_slot(Slot v) {
+    __syncwarp();
     if (KIND & kRedLse) {  // maximum first, then every lane rescales once, then a plain sum
         const float M = warp_max(v.m);
         const FF a = warp_sum_ff(rescale_to(v.m, FF{v.sh, v.sl}, M));
@@ -304,22 +305,80 @@ struct Walk {
         return j == 1 ? reinterpret_cast<unsigned char *>(Q) + (size_t)a.slice * 2
                       : reinterpret_cast<unsigned char *>(P) + (size_t)a.slice * 2;
     }
+    // This CTA's slice of `row`, raw, to shared memory at dst with cp.async (16-byte pieces);
+    // the ragged tail (fewer than 16 bytes) by plain loads and the padding up to the last
+    // chunk's end as -inf. The caller commits and waits.
+    __device__ void copy_slice_async(const T *row, unsigned char *dst) {
+        const int bytes = n * (int)sizeof(T), pieces = bytes >> 4;
+        const unsigned char *src = reinterpret_cast<const unsigned char *>(row + lo);
+        for (int i = threadIdx.x; i < pieces; i += kThreads) {
+            const unsigned sa = (unsigned)__cvta_generic_to_shared(dst + 16 * i);
+            asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(src + 16 * i) : "memory");
+        }
+        T *lt = reinterpret_cast<T *>(dst);
+        for (int e = (pieces << 4) / (int)sizeof(T) + threadIdx.x; e < nch * kChunk; e += kThreads)
+            lt[e] = e < n ? row[lo + e] : Logit<T>::neg_inf();
+    }
+
+    // The normalised law exp(fp32(z) * invT - L) of 8 raw bf16 logits at element e of zone
+    // into dst[e..e+7] (the arithmetic of stage<true>).
+    __device__ __forceinline__ void law8(const uint4 w, FF L2, float *dst, int e) {
+        RawGroup<T> r;
+        r.w = w;
+        float z[8];
+        r.unpack(z);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) z[k] = exp_shifted(__fmul_rn(z[k], a.invT), L2);
+        st4(dst, e, z[0], z[1], z[2], z[3]);
+        st4(dst, e + 4, z[4], z[5], z[6], z[7]);
+    }
+
+    // P0 into P (from trow; skipped when trow is null) and the normalised q law into Q, for bf16
+    // rows: both slices are copied raw with cp.async first (one memory round trip, no registers
+    // held), the target into the lower half of Q and the q row into its upper half; then P from
+    // the lower half; then Q in place: elements below slice/2 directly (their fp32 values land
+    // in the consumed lower half), the others held in registers across a barrier (their fp32
+    // values overwrite raw q values). Same values as stage<true>. Every thread takes part;
+    // ends synchronised.
+    __device__ void stage_pair(const T *trow, const T *qrow, FF L2t, FF L2q) {
+        static_assert(sizeof(T) == 2, "raw bf16 slices fit the halves of Q");
+        constexpr int kHold = (kMaxSliceChunks * kChunk / 2 / 8 + kThreads - 1) / kThreads;
+        unsigned char *zt = reinterpret_cast<unsigned char *>(Q);
+        unsigned char *zq = zt + (size_t)a.slice * 2;
+        if (trow) copy_slice_async(trow, zt);
+        copy_slice_async(qrow, zq);
+        asm volatile("cp.async.commit_group;" ::: "memory");
+        asm volatile("cp.async.wait_group 0;" ::: "memory");
+        __syncthreads();
+        const int g8 = nch * kChunk / 8, half8 = a.slice / 16;  // groups of 8 elements
+        if (trow) {
+            for (int e8 = threadIdx.x; e8 < g8; e8 += kThreads)
+                law8(*reinterpret_cast<const uint4 *>(zt + 16 * e8), L2t, P, 8 * e8);
+            __syncthreads();  // the lower half is consumed
+        }
+        uint4 hold[kHold];
+#pragma unroll
+        for (int h = 0; h < kHold; ++h) {
+            const int e8 = half8 + threadIdx.x + h * kThreads;
+            if (e8 < g8) hold[h] = *reinterpret_cast<const uint4 *>(zq + 16 * e8);
+        }
+        for (int e8 = threadIdx.x; e8 < min(half8, g8); e8 += kThreads)
+            law8(*reinterpret_cast<const uint4 *>(zq + 16 * e8), L2q, Q, 8 * e8);
+        __syncthreads();  // every raw q value has been read
+#pragma unroll
+        for (int h = 0; h < kHold; ++h) {
+            const int e8 = half8 + threadIdx.x + h * kThreads;
+            if (e8 < g8) law8(hold[h], L2q, Q, 8 * e8);
+        }
+        __syncthreads();
+    }
+
     __device__ void stage_look(int J, float *dst, float2 (*cst)[kMaxSliceChunks]) {
         const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
         const int g = lane & 7, q = lane >> 3;
-        const int bytes = n * (int)sizeof(T), pieces = bytes >> 4;
         for (int j = 0; j < J; ++j) {
             const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)sh.look[j] * a.t_rstride;
-            const unsigned char *src = reinterpret_cast<const unsigned char *>(row + lo);
-            unsigned char *dstj = landing(j);
-            for (int i = threadIdx.x; i < pieces; i += kThreads) {
-                const unsigned sa = (unsigned)__cvta_generic_to_shared(dstj + 16 * i);
-                asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(sa), "l"(src + 16 * i) : "memory");
-            }
-            // the ragged tail (fewer than 16 bytes) and the padding up to the last chunk's end
-            T *lt = reinterpret_cast<T *>(dstj);
-            for (int e = (pieces << 4) / (int)sizeof(T) + threadIdx.x; e < nch * kChunk; e += kThreads)
-                lt[e] = e < n ? row[lo + e] : Logit<T>::neg_inf();
+            copy_slice_async(row, landing(j));
         }
         asm volatile("cp.async.commit_group;" ::: "memory");
         asm volatile("cp.async.wait_group 0;" ::: "memory");
@@ -432,6 +491,7 @@ struct Walk {
                     float mx = v[0];
 #pragma unroll
                     for (int k = 1; k < 32; ++k) mx = fmaxf(mx, v[k]);
+                    __syncwarp();  // converged before the group shuffles
                     mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 4));
                     mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 2));
                     mx = fmaxf(mx, __shfl_xor_sync(kFull, mx, 1));
@@ -440,6 +500,7 @@ struct Walk {
 #pragma unroll
                         for (int k = 0; k < 32; ++k) sm += fast_exp2(__fmul_rn(__fsub_rn(v[k], mx), kLog2e));
                     }
+                    __syncwarp();
                     sm += __shfl_xor_sync(kFull, sm, 4);
                     sm += __shfl_xor_sync(kFull, sm, 2);
                     sm += __shfl_xor_sync(kFull, sm, 1);
@@ -448,6 +509,7 @@ struct Walk {
                     float sm = 0.f;
 #pragma unroll
                     for (int k = 0; k < 32; ++k) sm += v[k];
+                    __syncwarp();
                     sm += __shfl_xor_sync(kFull, sm, 4);
                     sm += __shfl_xor_sync(kFull, sm, 2);
                     sm += __shfl_xor_sync(kFull, sm, 1);
@@ -864,8 +926,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
             }
             __syncthreads();  // earlier readers of P and Q are done
             if (!staged || !q_staged) {  // the slices a rejection needs, once per node
-                if (!staged) W.template stage<true>(trow, P, kWarps, L2t);  // P0 directly
-                W.template stage<true>(qrow, Q, kWarps, L2q);
+                if constexpr (sizeof(T) == 2) {
+                    W.stage_pair(staged ? nullptr : trow, qrow, L2t, L2q);  // P0 directly when not staged
+                } else {
+                    if (!staged) W.template stage<true>(trow, P, kWarps, L2t);
+                    W.template stage<true>(qrow, Q, kWarps, L2q);
+                }
                 staged = q_staged = true;
                 __syncthreads();
             }

@@ -124,25 +124,33 @@ __device__ __forceinline__ uint32_t key_id(uint64_t k) { return ~(uint32_t)k; }
 __device__ __forceinline__ float key_value(uint64_t k) { return f32_of_ord((uint32_t)(k >> 32)); }
 
 // ---------------------------------------------------------------------------------------
-// Warp reductions (butterfly: every lane ends with the result).
+// Warp reductions (butterfly: every lane ends with the result). Each starts with __syncwarp():
+// a warp that reaches a full-mask shuffle still split from earlier divergent code (a lane-0
+// store, a loop with lane-dependent trip counts; a CTA barrier does not merge it) pays a
+// synchronisation at every shuffle, measured at ~500 cycles each on GB300 against ~16 once
+// the warp is converged.
 // Warp maximum of a float in one instruction (redux.sync.max.f32, sm_100a family); like
 // fmaxf, NaN inputs are ignored unless every input is NaN.
 __device__ __forceinline__ float warp_max(float v) {
+    __syncwarp();
     float r;
     asm volatile("redux.sync.max.f32 %0, %1, 0xffffffff;" : "=f"(r) : "f"(v));
     return r;
 }
 __device__ __forceinline__ float warp_sum(float v) {
+    __syncwarp();
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
     return v;
 }
 __device__ __forceinline__ double warp_sum_d(double v) {
+    __syncwarp();
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
     return v;
 }
 __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+    __syncwarp();
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const uint64_t w = __shfl_xor_sync(kFull, v, o);
@@ -164,6 +172,7 @@ __device__ __forceinline__ int multi_sum_index(int lane) {
 }
 template <int U>
 __device__ __forceinline__ float warp_multi_sum(const float (&v)[U]) {
+    __syncwarp();
     const int lane = threadIdx.x & 31;
     float c8[8];
 #pragma unroll
@@ -234,6 +243,7 @@ __device__ __forceinline__ FF ff_shfl_xor(FF v, int o) {
 }
 
 __device__ __forceinline__ FF warp_sum_ff(FF v) {
+    __syncwarp();
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v = ff_add(v, ff_shfl_xor(v, o));
     return v;
@@ -255,6 +265,7 @@ __device__ __forceinline__ MaxSum maxsum_merge(MaxSum a, MaxSum b) {
 }
 
 __device__ __forceinline__ MaxSum warp_maxsum(MaxSum v) {
+    __syncwarp();
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         MaxSum w{__shfl_xor_sync(kFull, v.m, o), ff_shfl_xor(v.s, o)};
@@ -380,6 +391,7 @@ __device__ __forceinline__ int rank_among(const uint64_t *keys, int n, uint64_t 
 // high words, then over the low words only among the lanes that tie. Returns the value to
 // every lane and the lane that holds it in *owner.
 __device__ __forceinline__ uint64_t warp_max_u64_owner(uint64_t v, int *owner) {
+    __syncwarp();
     const int lane = threadIdx.x & 31;
     const unsigned hi = (unsigned)(v >> 32);
     const unsigned m1 = __reduce_max_sync(kFull, hi);
@@ -631,6 +643,7 @@ __device__ __forceinline__ float group_max32(const RawGroup<__nv_bfloat16> (&raw
 template <typename T>
 __device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool live, float invT, float *mc_out,
                                              float *s_out) {
+    __syncwarp();
     float zm = live ? group_max32(raw) : -INFINITY;
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 4));
     zm = fmaxf(zm, __shfl_xor_sync(kFull, zm, 2));
@@ -648,6 +661,7 @@ __device__ __forceinline__ void chunk_stats8(const RawGroup<T> (&raw)[4], bool l
         }
         s = chunk_sum_fix(s, off.y);
     }
+    __syncwarp();
     s += __shfl_xor_sync(kFull, s, 4);
     s += __shfl_xor_sync(kFull, s, 2);
     s += __shfl_xor_sync(kFull, s, 1);
