@@ -3,9 +3,11 @@
 
 Workload (batched serving): B=16 trees, V=151,936, draft block L=16, N=64 planned nodes,
 top-k 8, T=1, bf16 logits; target rows [16, 65, V] = the node's depth row + N(0, 0.7^2).
-A step = tsb_plan_rows + tsb_replay + tsb_verify on one batch (5 kernel launches: the planner
+A step = tsb_plan_rows + tsb_replay_verify on one batch (4 kernel launches: the planner
 streams each draft row once for its chunk statistics and top-K, then runs the frontier
-kernel; the verifier runs its pre-pass and its walk).
+kernel; then one grid holds the replay draws beside the verifier's target-row pre-pass, and
+the verifier's walk follows). The same step as three calls (tsb_replay, then tsb_verify with
+its own pre-pass) is timed among the ``variants``.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl tsb|reference]
 
@@ -47,9 +49,9 @@ PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
 FALLBACK_HBM_GBS = 6800.0
 NOMINAL_HBM_GBS = 8000.0
 L2_BYTES = 129 * 1024 * 1024
-KERNELS = ("tsb_plan_rows", "tsb_replay", "tsb_verify")
-LAUNCHES_PER_STEP = {"tsb_plan_rows": 2, "tsb_replay": 1, "tsb_verify": 2}
-KERNEL_SOURCES = {"tsb_plan_rows": "k_plan.cu", "tsb_replay": "k_replay.cu", "tsb_verify": "k_verify.cu"}
+KERNELS = ("tsb_plan_rows", "tsb_replay_verify")
+LAUNCHES_PER_STEP = {"tsb_plan_rows": 2, "tsb_replay_verify": 2}
+KERNEL_SOURCES = {"tsb_plan_rows": ("k_plan.cu",), "tsb_replay_verify": ("k_verify.cu", "replay_body.cuh")}
 
 
 def parse():
@@ -110,9 +112,12 @@ def measured_peak_hbm():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def source_hash(name):
-    with open(os.path.join(ROOT, "paper_2609_33652_gb300", "csrc", name), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+def source_hash(names):
+    h = hashlib.sha256()
+    for name in names:
+        with open(os.path.join(ROOT, "paper_2609_33652_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
 
 
 def profiled_traffic(kernel, workload_name):
@@ -228,6 +233,7 @@ def algorithmic_bytes(w, sets, out_len, out_nodes):
 # 3.1): each runs eagerly like the headline step and is timed the same way (start and end
 # events only), followed by an event-separated pass for its per-call times.
 VARIANTS = (
+    ("wor_rrs_three_calls", dict(together=False), False),
     ("mixed_replay_naive_verify", dict(replay="mixed", mode=2), False),
     ("first_pass_tokens_naive_verify", dict(replay="plan", mode=2), False),
     ("expand_prune_w10_wor_rrs", dict(width=10), False),
@@ -549,8 +555,7 @@ def run_tsb(args):
     es = 2 if w["dtype"] == "bf16" else 4
     kernel_bytes = {
         "tsb_plan_rows": B * L * w["V"] * es + B * L * C * 8,
-        "tsb_verify": float(target_bytes.mean()),
-        "tsb_replay": B * w["N"] * (C * 8),
+        "tsb_replay_verify": B * w["N"] * (C * 8) + float(target_bytes.mean()),
     }
     achieved = kernel_bytes[dom] / (kern_us[dom] * 1e-6) / 1e9
     roofline = {"bound": "hbm", "kernel": dom, "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",

@@ -13,6 +13,8 @@
  *                   (recursive rejection sampling, Sec. 2.3 and App. A; block verification
  *                   of a sampled chain, Sun et al. 2025 as cited in Sec. 1 and App. A; or
  *                   target-sample matching, Table 2)
+ *   tsb_replay_verify  tsb_replay + tsb_verify (recursive rejection sampling) in one call, the
+ *                   verifier's target-row pre-pass running beside the replay draws
  *
  * and the paper's other choices for each pass:
  *
@@ -131,9 +133,10 @@ const char *tsb_status_str(tsb_status status);
 size_t tsb_stats_bytes(int32_t B, int32_t R, int32_t V);
 
 /* Bytes of the workspace for a configuration: a status word (256 bytes), per-(tree, node)
- * scalars of block verification (B*(N+1)*32) and the first pass's per-draft-row results
- * (B*L*(8 + 8*K)). The workspace must be 256-byte aligned; tsb_row_stats needs only the first
- * 256 bytes. 0 if the configuration is invalid. */
+ * scalars of the verifiers (B*(N+1)*32), the partial row normalisers of the recursive
+ * rejection pre-pass (B*1024) and the first pass's per-draft-row results (B*L*(8 + 8*K)). The
+ * workspace must be 256-byte aligned; tsb_row_stats needs only the first 256 bytes. 0 if the
+ * configuration is invalid. */
 size_t tsb_workspace_bytes(const tsb_cfg *cfg);
 
 /* Zero the workspace's status word on the stream. Call once before first use. */
@@ -314,6 +317,17 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
                       const void *qstats, size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree,
                       const int32_t *token, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
                       int32_t *out_len, void *ws, size_t ws_bytes, tsb_stream stream);
+
+/* tsb_replay followed by tsb_verify with TSB_VERIFY_RRS, same seed, in one call: the same
+ * tokens and outputs bit for bit. The verifier's pass over the target rows that it normalises
+ * ahead of the walk (the first internal nodes of each tree's first-child chain) reads only the
+ * tree and the target rows, so it runs in the same grid as the replay draws instead of after
+ * them. token [B, N+1] is written as by tsb_replay; the other arguments, layouts and errors are
+ * those of tsb_replay and tsb_verify. */
+tsb_status tsb_replay_verify(const tsb_cfg *cfg, const tsb_logits *target, const tsb_logits *qrows, const void *qstats,
+                             size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed,
+                             int32_t *token, int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, void *ws,
+                             size_t ws_bytes, tsb_stream stream);
 
 #ifdef __cplusplus
 }

@@ -1227,7 +1227,7 @@ HeapArgs heap_args(int L, int N, int K, const PlanScratch &sc, const TreeDesc &t
 }  // namespace
 
 PlanScratch plan_scratch(void *ws, int B, int N, int L, int K) {
-    unsigned char *p = static_cast<unsigned char *>(ws) + kWsStatusBytes + (size_t)B * (N + 1) * kWsBvRowBytes;
+    unsigned char *p = static_cast<unsigned char *>(ws) + ws_plan_offset(B, N);
     PlanScratch s;
     s.lse = reinterpret_cast<float2 *>(p);
     s.topk_x = reinterpret_cast<float *>(p + (size_t)B * L * sizeof(float2));

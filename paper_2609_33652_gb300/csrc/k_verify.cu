@@ -49,6 +49,7 @@
 
 #include "tsb_device.cuh"
 #include "tsb_launch.h"
+#include "replay_body.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -68,6 +69,9 @@ constexpr int kLook = 3;
 // pre-pass computes on the whole GPU (the walk starts on that chain; nodes a walk reaches off it
 // are staged by the walk's own rounds).
 constexpr int kPreChain = 8;
+constexpr int kPreSplit = 8;           // CTAs per pre-computed target row (equal parts of its chunks)
+constexpr int kPreSplitThreads = kRpThreads;  // shares a grid with the replay CTAs
+static_assert((size_t)kPreChain * kPreSplit * 16 == kWsPrePartBytes, "pre-pass partials per tree");
 static_assert(kWarps % 4 == 0 && kLook <= kWarps, "groups of four warps per normaliser");
 
 // Pre-pass results, one 32-byte workspace slot per (tree, node) (the slots block
@@ -105,6 +109,8 @@ struct VerifyArgs {
     int Lq;       // per-depth q rows whose normaliser the pre-pass computes (0 for per-node rows)
     int qn;       // 1: the pre-pass computes each internal node's per-node q-row normaliser (slot u)
     int B;
+    float4 *part;    // [B, kPreChain, kPreSplit] partial normalisers (max, float-float sum) of the chain rows
+    int tokens_late; // the tokens come from the launch just before the walk: read them after the wait
 };
 
 // A partial of one cluster-wide reduction: a softmax normaliser (max, float-float sum), a
@@ -636,13 +642,12 @@ struct TreeSmem {
     float *cxt, *cxq, *cu;
 };
 
-// Copy of tree b for a walk: topology, per child slot its parent, target and q logits and
-// acceptance uniform. It reads only the tree, the tokens and the logits (written before the
-// pre-pass began), so a walk may run it before waiting for the pre-pass. Sets sh.cbad on
-// inconsistent tree arrays. Every thread of the CTA calls it; it ends with the CTA
-// synchronised.
+// Copy of tree b's topology for a walk: child lists, q row per node, and each child slot's
+// parent. It reads only the tree (written before the pre-pass and the replay began), so a walk
+// may run it before waiting for the launch before it. Sets sh.cbad on inconsistent tree
+// arrays. Every thread of the CTA calls it; it ends with the CTA synchronised.
 template <typename T>
-__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
+__device__ TreeSmem copy_topo(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
     const int NN = a.N + 1;
     TreeSmem ts;
     ts.l2t = reinterpret_cast<FF *>(base);
@@ -659,17 +664,13 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
     {
         const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
         const int32_t *kids = a.child_ids + (int64_t)b * a.N;
-        const int32_t *tok = a.token + (int64_t)b * NN;
         const int32_t *row = per_depth ? a.depth + (int64_t)b * NN : a.qrow_of_node + (int64_t)b * NN;
         for (int i = threadIdx.x; i <= NN; i += kThreads) ts.off[i] = __ldg(off + i);
         for (int i = threadIdx.x; i < a.N; i += kThreads) {
             ts.kid[i] = __ldg(kids + i);
             ts.ps[i] = -1;
         }
-        for (int i = threadIdx.x; i < NN; i += kThreads) {
-            ts.tok[i] = __ldg(tok + i);
-            ts.row[i] = __ldg(row + i);
-        }
+        for (int i = threadIdx.x; i < NN; i += kThreads) ts.row[i] = __ldg(row + i);
         if (threadIdx.x == 0) sh.cbad = 0;
     }
     __syncthreads();
@@ -687,6 +688,19 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
         }
         if (bad_here) sh.cbad = 1;
     }
+    __syncthreads();
+    return ts;
+}
+
+// The tokens of tree b and, per child slot, its token's target and q logits (from the parent's
+// rows) and acceptance uniform, after copy_topo. The tokens are read with plain loads: they may
+// come from the launch just before the walk. Every thread of the CTA calls it; it ends with the
+// CTA synchronised.
+template <typename T>
+__device__ void copy_slots(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, int b) {
+    const int NN = a.N + 1;
+    const int32_t *tok = a.token + (int64_t)b * NN;
+    for (int i = threadIdx.x; i < NN; i += kThreads) ts.tok[i] = tok[i];
     __syncthreads();
     {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
         bool bad_here = false;
@@ -708,6 +722,13 @@ __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int
         if (bad_here) sh.cbad = 1;
     }
     __syncthreads();
+}
+
+// Both parts, for walks whose tokens were written before the launch before them.
+template <typename T>
+__device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
+    const TreeSmem ts = copy_topo<T>(a, sh, base, b, per_depth);
+    copy_slots<T>(a, sh, ts, b);
     return ts;
 }
 
@@ -729,18 +750,29 @@ __device__ void load_pre(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, i
         }
     for (int u = threadIdx.x; u < NN; u += kThreads)
         ts.pre[u] = !a.pre_chain && u < a.M && ts.off[u + 1] - ts.off[u] > 0 ? 1 : 0;
-    if (a.pre_chain) {
+    if (a.pre_chain) {  // chain node j's normaliser from the pre-pass's kPreSplit partials, in order
         __syncthreads();
         if (threadIdx.x < a.M) {
             const int v = chain_node(ts.off, ts.kid, a.N, threadIdx.x);
-            if (v >= 0) ts.pre[v] = 1;
+            if (v >= 0) {
+                const float4 *pp = a.part + ((int64_t)b * kPreChain + threadIdx.x) * kPreSplit;
+                MaxSum acc{-INFINITY, FF{0.f, 0.f}};
+#pragma unroll
+                for (int k = 0; k < kPreSplit; ++k) {
+                    const float4 p = pp[k];
+                    acc = maxsum_merge(acc, MaxSum{p.x, FF{p.y, p.z}});
+                }
+                ts.l2t[v] = acc.s.hi > 0.f ? ff_times_log2e(maxsum_lse(acc)) : FF{0.f, 0.f};
+                ts.pre[v] = 1;
+            }
         }
     }
     __syncthreads();
 }
 
-// Pre-pass, in clusters of two CTAs. Clusters [0, B*M): cluster (b, j) streams target row j of
-// tree b (if node j has children), each CTA half of its four-chunk units: the chunk statistics
+// Pre-pass of traversal verification, in clusters of two CTAs. Clusters [0, B*M): cluster (b, j)
+// streams target row j of tree b (if node j has children), each CTA half of its four-chunk
+// units: the chunk statistics
 // of every 256-logit chunk (eight lanes per chunk, two units in flight per warp, the same
 // per-chunk code as the row statistics kernel) into shared memory; rank 0 gathers rank 1's
 // half through distributed shared memory and computes the row's log-normaliser over a fixed
@@ -777,18 +809,7 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     const int b = pair / a.M;
     int j = pair - (pair / a.M) * a.M;
     const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
-    if (a.pre_chain) {  // slot j: node j of the first-child chain (both CTAs find the same node)
-        int32_t *s_off = reinterpret_cast<int32_t *>(pst + a.C);
-        int32_t *s_kid = s_off + NN + 1;
-        for (int i = threadIdx.x; i <= NN; i += kPreThreads) s_off[i] = __ldg(off + i);
-        const int32_t *kids = a.child_ids + (int64_t)b * a.N;
-        for (int i = threadIdx.x; i < a.N; i += kPreThreads) s_kid[i] = __ldg(kids + i);
-        __syncthreads();
-        j = chain_node(s_off, s_kid, a.N, j);
-        if (j < 0) return;
-    } else if (__ldg(off + j + 1) - __ldg(off + j) <= 0) {
-        return;  // leaves need no normaliser (both CTAs of the cluster return)
-    }
+    if (__ldg(off + j + 1) - __ldg(off + j) <= 0) return;  // leaves need no normaliser (both CTAs return)
     const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)j * a.t_rstride;
     const int g = lane & 7, q = lane >> 3;
     const int C = a.C, units = (C + 3) / 4;
@@ -833,6 +854,115 @@ __global__ void __launch_bounds__(kPreThreads, 2) k_verify_pre(VerifyArgs a) {
     }
 }
 
+// Chunks of one part of the split pre-pass (parts are equal runs of four-chunk units).
+__host__ __device__ inline int pre_part_chunks(int C) { return ((C + 3) / 4 + kPreSplit - 1) / kPreSplit * 4; }
+inline size_t pre_split_smem(int C, int N) {
+    return (size_t)pre_part_chunks(C) * sizeof(float2) + (size_t)(2 * N + 2) * sizeof(int32_t);
+}
+
+// Pre-pass of recursive rejection sampling, CTA blk of kPreSplitThreads threads (dynamic shared
+// memory: pre_split_smem). CTAs [0, B*kPreChain*kPreSplit): CTA (b, j, k) streams the k-th of
+// kPreSplit equal parts (four-chunk units) of the target row of node j of tree b's first-child
+// chain: chunk statistics (eight lanes per chunk, two units in flight per warp, the per-chunk
+// code of the statistics kernels) into shared memory, then warp 0 merges them into one partial
+// normaliser (maximum, float-float sum) at a.part[b][j][k]; the walk merges the kPreSplit
+// partials in order. It reads only the tree and the target rows, so it may run beside the
+// replay. Later CTAs: one warp per q-row normaliser (per-depth rows, or each internal node's
+// per-node row). Every thread calls it; it may return early.
+template <typename T>
+__device__ __forceinline__ void pre_split_cta(const VerifyArgs &a, int blk, float2 *pst) {
+    constexpr int nwarps = kPreSplitThreads / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int NN = a.N + 1;
+    const int ntarget = a.B * kPreChain * kPreSplit;
+    if (blk >= ntarget) {  // q-row log-normalisers, one warp each
+        const int task = (blk - ntarget) * nwarps + warp;
+        const int per = a.qn ? NN : a.Lq;
+        if (task >= a.B * per) return;  // warp-uniform; no barrier in this branch
+        const int b = task / per, d = task - (task / per) * per;
+        int r = d;
+        if (a.qn) {
+            const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+            if (__ldg(off + d + 1) - __ldg(off + d) <= 0) return;  // a leaf needs no draft law
+            r = __ldg(a.qrow_of_node + (int64_t)b * NN + d);
+            if (r < 0 || r >= a.q_R) return;  // the walk flags the tree
+        }
+        const FF L2q = q_log_normaliser(a.qstats + ((int64_t)b * a.q_R + r) * a.C, a.C);
+        if (lane == 0) a.pre[(int64_t)b * NN + d].l2q = make_float2(L2q.hi, L2q.lo);
+        return;
+    }
+    const int k = blk % kPreSplit, bj = blk / kPreSplit;
+    const int b = bj / kPreChain, j = bj - (bj / kPreChain) * kPreChain;
+    const int C = a.C, units = (C + 3) / 4, pc = pre_part_chunks(C);
+    int32_t *s_off = reinterpret_cast<int32_t *>(pst + pc);
+    int32_t *s_kid = s_off + NN + 1;
+    {
+        const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
+        const int32_t *kids = a.child_ids + (int64_t)b * a.N;
+        for (int i = threadIdx.x; i <= NN; i += kPreSplitThreads) s_off[i] = __ldg(off + i);
+        for (int i = threadIdx.x; i < a.N; i += kPreSplitThreads) s_kid[i] = __ldg(kids + i);
+    }
+    __syncthreads();
+    const int v = chain_node(s_off, s_kid, a.N, j);  // the walk finds the same node
+    if (v < 0) return;                               // uniform over the CTA
+    const T *row = static_cast<const T *>(a.target) + (int64_t)b * a.t_bstride + (int64_t)v * a.t_rstride;
+    const int g = lane & 7, q = lane >> 3;
+    const int ulo = k * (pc / 4), uhi = min(units, ulo + pc / 4), clo = 4 * ulo;
+    constexpr int kU = sizeof(T) == 2 ? 2 : 1;  // units in flight per warp (register budget)
+    for (int u0 = ulo + warp; u0 < uhi; u0 += kU * nwarps) {  // uniform over the warp
+        RawGroup<T> raw[kU][4];
+#pragma unroll
+        for (int e = 0; e < kU; ++e) {
+            const int c = (u0 + e * nwarps) * 4 + q;
+            if (u0 + e * nwarps < uhi && c < C)
+#pragma unroll
+                for (int kk = 0; kk < 4; ++kk) raw[e][kk].load(row, c * kChunk + kk * 64 + g * 8, a.V);
+        }
+#pragma unroll
+        for (int e = 0; e < kU; ++e) {
+            const int c = (u0 + e * nwarps) * 4 + q;
+            const bool live = u0 + e * nwarps < uhi && c < C;
+            float mc, sc;
+            chunk_stats8<T>(raw[e], live, a.invT, &mc, &sc);
+            if (live && g == 0) pst[c - clo] = make_float2(mc, sc);
+        }
+    }
+    __syncthreads();
+    if (warp == 0) {
+        const int n = max(0, min(4 * uhi, C) - clo);
+        float m = -INFINITY;
+        for (int c = lane; c < n; c += 32) m = fmaxf(m, pst[c].x);
+        m = warp_max(m);
+        KahanF acc;
+        if (m != -INFINITY)
+            for (int c = lane; c < n; c += 32) acc.add(__fmul_rn(pst[c].y, expf(__fsub_rn(pst[c].x, m))));
+        const FF sv = warp_sum_ff(acc.ff());
+        if (lane == 0) a.part[(int64_t)bj * kPreSplit + k] = make_float4(m, sv.hi, sv.lo, 0.f);
+    }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kPreSplitThreads, 8) k_pre_split(VerifyArgs a) {
+    pdl_begin();
+    extern __shared__ __align__(16) float2 pst[];
+    pre_split_cta<T>(a, (int)blockIdx.x, pst);
+}
+
+// The replay CTAs and the split pre-pass CTAs in one grid: blocks [0, nrep) draw the tokens,
+// the rest run the pre-pass (which reads neither the tokens nor anything else the replay
+// writes).
+template <int KCAP, typename T>
+__global__ void __launch_bounds__(kRpThreads, KCAP <= 8 ? kRpMinBlocks : 2)
+    k_replay_pre(ReplayArgs ra, VerifyArgs va, int nrep) {
+    pdl_begin();
+    if ((int)blockIdx.x < nrep) {
+        replay_node<KCAP, T>(ra, (int)blockIdx.x);
+        return;
+    }
+    extern __shared__ __align__(16) float2 pst[];
+    pre_split_cta<T>(va, (int)blockIdx.x - nrep, pst);
+}
+
 template <typename T>
 __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     if (!a.copy_early) pdl_begin();
@@ -856,9 +986,12 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
 
     // the tree's copy in shared memory; with the pre-pass launched just before this kernel it
     // overlaps the pre-pass's tail (it reads nothing the pre-pass writes), then the wait for
-    // the pre-pass and its results
-    const TreeSmem ts = copy_tree<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    // the pre-pass and its results; tokens written by that launch (replay beside the
+    // pre-pass) are read after the wait
+    const TreeSmem ts = copy_topo<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
+    if (!a.tokens_late) copy_slots<T>(a, sh, ts, b);
     if (a.copy_early) pdl_begin();
+    if (a.tokens_late) copy_slots<T>(a, sh, ts, b);
     load_pre(a, sh, ts, b, true);
     const FF *s_l2t = ts.l2t;
     const int32_t *s_known = ts.pre, *s_off = ts.off, *s_kid = ts.kid, *s_tok = ts.tok, *s_row = ts.row;
@@ -1597,8 +1730,15 @@ cudaError_t launch_pre_t(const VerifyArgs &a, int B, cudaStream_t s) {
     return launch_pdl(k_verify_pre<T>, dim3((unsigned)pre_blocks), dim3(kPreThreads), psmem, s, 2, a);
 }
 
+// The split pre-pass's grid: kPreSplit CTAs per chain row, then the q-row normaliser warps.
+int64_t pre_split_blocks(const VerifyArgs &a, int B) {
+    const int per = a.qn ? a.N + 1 : a.Lq;
+    return (int64_t)B * kPreChain * kPreSplit + ((int64_t)B * per + kPreSplitThreads / 32 - 1) / (kPreSplitThreads / 32);
+}
+
+// The RRS walk's cluster shape and shared memory, set on the kernel before any launch.
 template <typename T>
-cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
+cudaError_t prepare_rrs_walk(VerifyArgs &a, int B, int *cs_out, size_t *smem_out) {
     int slice = 0;
     size_t smem = 0;
     const int cs = choose_cluster<T>(a.V, a.N, B, &slice, &smem);
@@ -1610,9 +1750,45 @@ cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
         e = cudaFuncSetAttribute(k_verify_rrs<T>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         if (e != cudaSuccess) return e;
     }
-    e = launch_pre_t<T>(a, B, s);
+    *cs_out = cs;
+    *smem_out = smem;
+    return cudaSuccess;
+}
+
+template <typename T>
+cudaError_t launch_rrs_t(VerifyArgs a, int B, cudaStream_t s) {
+    int cs = 0;
+    size_t smem = 0;
+    cudaError_t e = prepare_rrs_walk<T>(a, B, &cs, &smem);
     if (e != cudaSuccess) return e;
-    a.copy_early = pre_launched(a, B) ? 1 : 0;
+    const int64_t blocks = pre_split_blocks(a, B);
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    const size_t psmem = pre_split_smem(a.C, a.N);
+    e = cudaFuncSetAttribute(k_pre_split<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)psmem);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(k_pre_split<T>, dim3((unsigned)blocks), dim3(kPreSplitThreads), psmem, s, 0, a);
+    if (e != cudaSuccess) return e;
+    a.copy_early = 1;  // the walk copies its tree and tokens while the pre-pass runs
+    return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
+}
+
+template <int KCAP, typename T>
+cudaError_t launch_replay_verify_t(const ReplayArgs &ra, VerifyArgs a, int B, cudaStream_t s) {
+    int cs = 0;
+    size_t smem = 0;
+    cudaError_t e = prepare_rrs_walk<T>(a, B, &cs, &smem);
+    if (e != cudaSuccess) return e;
+    const int64_t nrep = (int64_t)B * (a.N + 1), npre = pre_split_blocks(a, B);
+    if (nrep + npre > 0x7fffffffLL) return cudaErrorInvalidConfiguration;
+    const size_t rsmem = (size_t)key_buf_len(a.C) * sizeof(uint64_t), psmem = pre_split_smem(a.C, a.N);
+    const size_t smem1 = rsmem > psmem ? rsmem : psmem;
+    e = cudaFuncSetAttribute(k_replay_pre<KCAP, T>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem1);
+    if (e != cudaSuccess) return e;
+    e = launch_pdl(k_replay_pre<KCAP, T>, dim3((unsigned)(nrep + npre)), dim3(kRpThreads), smem1, s, 0, ra, a,
+                   (int)nrep);
+    if (e != cudaSuccess) return e;
+    a.copy_early = 1;  // the topology before the wait,
+    a.tokens_late = 1; // the tokens after it
     return launch_pdl(k_verify_rrs<T>, dim3((unsigned)(B * cs)), dim3(kThreads), smem, s, cs, a);
 }
 
@@ -1689,6 +1865,8 @@ VerifyArgs verify_args(const RowsDesc &target, const RowsDesc &q, const float2 *
     a.Lq = qrow_of_node ? 0 : (L < N + 1 ? L : N + 1);
     a.qn = 0;
     a.B = B;
+    a.part = reinterpret_cast<float4 *>(reinterpret_cast<char *>(status) + ws_pre_part_offset(B, N));
+    a.tokens_late = 0;
     return a;
 }
 
@@ -1717,6 +1895,23 @@ cudaError_t launch_verify_rrs(const RowsDesc &target, const RowsDesc &q, const f
     a.qn = qrow_of_node ? 1 : 0;  // per-node q rows: every internal node's normaliser
     if (target.dtype == 1) return launch_rrs_t<__nv_bfloat16>(a, B, s);
     return launch_rrs_t<float>(a, B, s);
+}
+
+cudaError_t launch_replay_verify(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
+                                 const int32_t *qrow_of_node, int B, int N, int L, int K, const TreeDesc &tree,
+                                 int32_t *token, float invT, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
+                                 int32_t *out_len, uint32_t *status, cudaStream_t s) {
+    VerifyArgs a = verify_args(target, q, qstats, qrow_of_node, B, N, L, tree, token, invT, seed, out_tokens,
+                               out_nodes, out_len, status);
+    a.M = kPreChain;
+    a.pre_chain = 1;
+    a.qn = qrow_of_node ? 1 : 0;
+    const ReplayArgs ra = replay_args(q, qstats, qrow_of_node, B, N, tree, invT, seed, token, status);
+    // sibling groups have at most K members: a list of 8 covers K <= 8 (as in launch_replay)
+    if (target.dtype == 1)
+        return K <= 8 ? launch_replay_verify_t<8, __nv_bfloat16>(ra, a, B, s)
+                      : launch_replay_verify_t<32, __nv_bfloat16>(ra, a, B, s);
+    return K <= 8 ? launch_replay_verify_t<8, float>(ra, a, B, s) : launch_replay_verify_t<32, float>(ra, a, B, s);
 }
 
 cudaError_t launch_verify_naive(const RowsDesc &target, int B, int N, int L, const TreeDesc &tree,

@@ -364,6 +364,27 @@ tsb_status tsb_verify(const tsb_cfg *cfg, int32_t mode, const tsb_logits *target
     return cuda_status(e);
 }
 
+tsb_status tsb_replay_verify(const tsb_cfg *cfg, const tsb_logits *target, const tsb_logits *qrows, const void *qstats,
+                             size_t stats_bytes, const int32_t *qrow_of_node, const tsb_tree *tree, uint64_t seed,
+                             int32_t *token, int32_t *out_tokens, int32_t *out_nodes, int32_t *out_len, void *ws,
+                             size_t ws_bytes, tsb_stream stream) {
+    tsb_status st = check_cfg(cfg);
+    if (st != TSB_OK) return st;
+    st = check_logits(target, cfg->B, cfg->N + 1, cfg->V);
+    if (st == TSB_OK) st = check_logits(qrows, cfg->B, qrow_of_node ? 1 : cfg->L, cfg->V);
+    if (st == TSB_OK && target->dtype != qrows->dtype) st = TSB_ERR_DTYPE;
+    if (st == TSB_OK) st = check_stats(qstats, stats_bytes, cfg->B, qrows->R, cfg->V);
+    if (st == TSB_OK) st = check_ws(ws, ws_bytes, ws_bytes_for(cfg));
+    if (st != TSB_OK) return st;
+    if (!tree || !tree->child_off || !tree->child_ids || (!qrow_of_node && !tree->depth) || !token ||
+        !out_tokens || !out_nodes || !out_len)
+        return TSB_ERR_ARG;
+    return cuda_status(tsb::launch_replay_verify(rows_of(target), rows_of(qrows), static_cast<const float2 *>(qstats),
+                                                 qrow_of_node, cfg->B, cfg->N, cfg->L, cfg->K, tree_of(tree), token,
+                                                 inv_temperature(cfg->temperature), seed, out_tokens, out_nodes,
+                                                 out_len, static_cast<uint32_t *>(ws), (cudaStream_t)stream));
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------------------------------

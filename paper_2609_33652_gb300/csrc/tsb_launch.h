@@ -54,14 +54,19 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 //   [0, 256)                       sticky status word
 //   B*(N+1) x 32 bytes             per-(tree, node) scalars: block verification's per-position
 //                                  values, or the verifier pre-pass's log-normalisers
+//   B x 1024 bytes                 per tree, the recursive-rejection pre-pass's partial
+//                                  normalisers (8 chain nodes x 8 row parts x 16 bytes)
 //   B*L float2, B*L*K floats,      per-draft-row log-normaliser (float-float) and top-K
 //   B*L*K int32                    (x, id) of the first pass
 constexpr size_t kWsStatusBytes = 256;
 constexpr size_t kWsBvRowBytes = 32;
+constexpr size_t kWsPrePartBytes = 1024;
+
+inline size_t ws_pre_part_offset(int B, int N) { return kWsStatusBytes + (size_t)B * ((size_t)N + 1) * kWsBvRowBytes; }
+inline size_t ws_plan_offset(int B, int N) { return ws_pre_part_offset(B, N) + (size_t)B * kWsPrePartBytes; }
 
 inline size_t workspace_bytes(int B, int N, int L, int K) {
-    return kWsStatusBytes + (size_t)B * ((size_t)N + 1) * kWsBvRowBytes + (size_t)B * L * 2 * sizeof(float) +
-           (size_t)B * L * K * (sizeof(float) + sizeof(int32_t));
+    return ws_plan_offset(B, N) + (size_t)B * L * 2 * sizeof(float) + (size_t)B * L * K * (sizeof(float) + sizeof(int32_t));
 }
 
 // Expand-then-prune first pass: layer d holds n_d candidates, n_1 = K and
@@ -120,6 +125,14 @@ cudaError_t launch_replay(const RowsDesc &q, const float2 *qstats, const int32_t
 cudaError_t launch_replay_mixed(const RowsDesc &q, const float2 *qstats, const int32_t *qrow_of_node, int B, int N,
                                 int K, const TreeDesc &tree, float invT, uint64_t seed, int32_t *token,
                                 uint32_t *status, cudaStream_t s);
+
+// tsb_replay followed by tsb_verify (recursive rejection sampling) in two launches: the replay
+// CTAs and the verifier's pre-pass CTAs in one grid (the pre-pass reads only the tree and the
+// target rows), then the walk.
+cudaError_t launch_replay_verify(const RowsDesc &target, const RowsDesc &q, const float2 *qstats,
+                                 const int32_t *qrow_of_node, int B, int N, int L, int K, const TreeDesc &tree,
+                                 int32_t *token, float invT, uint64_t seed, int32_t *out_tokens, int32_t *out_nodes,
+                                 int32_t *out_len, uint32_t *status, cudaStream_t s);
 
 cudaError_t launch_verify_naive(const RowsDesc &target, int B, int N, int L, const TreeDesc &tree,
                                 const int32_t *token, float invT, uint64_t seed, int32_t *out_tokens,

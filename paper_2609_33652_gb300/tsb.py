@@ -30,7 +30,7 @@ TSB_CHUNK = 256
 EXPORTS = ("tsb_version", "tsb_status_str", "tsb_stats_bytes", "tsb_workspace_bytes", "tsb_workspace_init",
            "tsb_device_status", "tsb_row_stats", "tsb_plan", "tsb_replay", "tsb_verify", "tsb_plan_noalloc",
            "tsb_plan_rows", "tsb_plan_expand", "tsb_plan_rows_expand", "tsb_replay_mixed", "tsb_plan_pooled",
-           "tsb_replay_pooled", "tsb_verify_pooled")
+           "tsb_replay_pooled", "tsb_verify_pooled", "tsb_replay_verify")
 TSB_NOALLOC_SCRATCH_BYTES = 1 << 20
 TSB_MAX_WIDTH = 1024
 TSB_MAX_EXPAND_CANDIDATES = 8192
@@ -113,6 +113,7 @@ def _open(path):
         "tsb_replay_pooled": (_I32, [_P, _I32, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _SZ, _P]),
         "tsb_verify_pooled": (_I32, [_P, _I32, _P, _P, _P, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
         "tsb_verify": (_I32, [_P, _I32, _P, _P, _P, _SZ, _P, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _SZ, _P]),
+        "tsb_replay_verify": (_I32, [_P, _P, _P, _P, _SZ, _P, _P, ctypes.c_uint64, _P, _P, _P, _P, _P, _SZ, _P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(lib, name)
@@ -310,6 +311,20 @@ def tsb_verify(cfg: Cfg, mode: int, target: torch.Tensor, qrows, qstats, qrow_of
                              ws.numel() * ws.element_size(), _stream(stream)), "tsb_verify")
 
 
+def tsb_replay_verify(cfg: Cfg, target: torch.Tensor, qrows: torch.Tensor, qstats: torch.Tensor, qrow_of_node,
+                      tree: dict, seed: int, token: torch.Tensor, out_tokens: torch.Tensor, out_nodes: torch.Tensor,
+                      out_len: torch.Tensor, ws: torch.Tensor, stream=None):
+    """tsb_replay then tsb_verify (recursive rejection sampling) in one call."""
+    dt = logits_desc(target)
+    dq = logits_desc(qrows)
+    t = tree_struct(tree)
+    _check(load().tsb_replay_verify(ctypes.byref(cfg), ctypes.byref(dt), ctypes.byref(dq), _ptr(qstats),
+                                    qstats.numel() * qstats.element_size(), _ptr(qrow_of_node), ctypes.byref(t),
+                                    int(seed) & (2**64 - 1), _ptr(token), _ptr(out_tokens), _ptr(out_nodes),
+                                    _ptr(out_len), _ptr(ws), ws.numel() * ws.element_size(), _stream(stream)),
+           "tsb_replay_verify")
+
+
 # ---------------------------------------------------------------------------------------
 @dataclass
 class TsbBuffers:
@@ -351,11 +366,12 @@ class PreparedStep:
     tsb_row_stats + tsb_plan instead; with ``plan_only`` only the first pass runs. With
     ``qrows`` (per-node draft rows [B, Rq, V]), ``qstats`` (their statistics buffer) and
     ``qrow_of_node`` ([B, N+1]), the step also runs tsb_row_stats on the q rows, and replay and
-    verification draw from them (the corrected-drafter workload)."""
+    verification draw from them (the corrected-drafter workload). With ``together`` (the default;
+    WoR replay and recursive rejection sampling only) the two are one tsb_replay_verify call."""
 
     def __init__(self, buf: TsbBuffers, draft: torch.Tensor, target: torch.Tensor, seed: int, mode=TSB_VERIFY_RRS,
                  out_tokens=None, out_nodes=None, out_len=None, stream=None, fused=True, width=None, replay="wor",
-                 plan_only=False, qrows=None, qstats=None, qrow_of_node=None):
+                 plan_only=False, qrows=None, qstats=None, qrow_of_node=None, together=True):
         lib = load()
         self._keep = []
         s = _stream(stream)
@@ -410,6 +426,12 @@ class PreparedStep:
                                             ctypes.byref(tr), _ptr(tok), seed, _ptr(ot), _ptr(on), _ptr(ol),
                                             _ptr(buf.ws), wb, s)),
         ]
+        if together and replay == "wor" and mode == TSB_VERIFY_RRS:  # replay and verification in one call
+            self.calls = plan + qcalls + [
+                ("tsb_replay_verify", lib.tsb_replay_verify,
+                 (ctypes.byref(cfg), ctypes.byref(dt), qref, qst, qstb, qidx, ctypes.byref(tr), seed, _ptr(tok),
+                  _ptr(ot), _ptr(on), _ptr(ol), _ptr(buf.ws), wb, s)),
+            ]
         if plan_only:  # the first pass alone
             self.calls = plan
 

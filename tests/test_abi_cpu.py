@@ -82,7 +82,7 @@ def test_c_program_links_and_validates(tmp_path, lib):
 int main(void) {
     tsb_cfg cfg = {16, 16, 64, 8, 151936, 1.0f};
     size_t ws = tsb_workspace_bytes(&cfg);
-    if (ws != 256 + 16 * 65 * 32 + 16 * 16 * (8 + 8 * 8)) return 1;
+    if (ws != 256 + 16 * 65 * 32 + 16 * 1024 + 16 * 16 * (8 + 8 * 8)) return 1;
     if (tsb_stats_bytes(16, 16, 151936) != (size_t)16 * 16 * 594 * 8) return 2;
     tsb_cfg bad = cfg;
     bad.temperature = 0.0f;
@@ -113,7 +113,7 @@ def test_host_queries(lib):
     assert tsb.tsb_stats_bytes(1, 1, 257) == 2 * 8
     assert tsb.tsb_stats_bytes(0, 1, 10) == 0
     cfg = tsb.make_cfg(16, 16, 64, 8, 151936, 1.0)
-    assert tsb.tsb_workspace_bytes(cfg) == 256 + 16 * 65 * 32 + 16 * 16 * (8 + 8 * 8)
+    assert tsb.tsb_workspace_bytes(cfg) == 256 + 16 * 65 * 32 + 16 * 1024 + 16 * 16 * (8 + 8 * 8)
     assert tsb.tsb_workspace_bytes(tsb.make_cfg(1, 2, 7, 2, 8, 1.0)) == 0  # N above K + K^2
 
 
@@ -160,7 +160,7 @@ def test_plan_validation(lib):
     assert _plan(lib, good, d, tree=t) == ARG
     # broadcast rows (batch stride 0) are accepted by validation
     cfg1 = tsb.make_cfg(4, 2, 6, 2, 8, 1.0)
-    assert lib.tsb_workspace_bytes(ctypes.byref(cfg1)) == 256 + 4 * 7 * 32 + 4 * 2 * (8 + 8 * 2)
+    assert lib.tsb_workspace_bytes(ctypes.byref(cfg1)) == 256 + 4 * 7 * 32 + 4 * 1024 + 4 * 2 * (8 + 8 * 2)
 
 
 def test_plan_rows_validation(lib):

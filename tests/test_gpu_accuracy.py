@@ -33,8 +33,9 @@ def _built():
 
 def _gpu_row_lse(buf, B, L, N):
     """The first pass's per-draft-row log-normaliser (float-float) from the workspace: after
-    the 256-byte header and B*(N+1) 32-byte slots come B*L float2 values."""
-    off = 256 + B * (N + 1) * 32
+    the 256-byte header, B*(N+1) 32-byte slots and B 1024-byte pre-pass partials come B*L
+    float2 values."""
+    off = 256 + B * (N + 1) * 32 + B * 1024
     v = buf.ws[off:off + B * L * 8].view(torch.float32).view(B, L, 2).cpu().numpy().astype(np.float64)
     return v[..., 0] + v[..., 1]
 

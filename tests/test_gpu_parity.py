@@ -207,9 +207,10 @@ def test_plan_large_budgets(B, L, N, K, V, kind, dtype):
 
 
 def _topk_scratch(buf, B, L, N, K):
-    """The first pass's per-row top-K (x, id) from the workspace: after the 256-byte header and
-    B*(N+1) 32-byte slots come B*L float2 log-normalisers, B*L*K x, B*L*K ids."""
-    off = 256 + B * (N + 1) * 32 + B * L * 8
+    """The first pass's per-row top-K (x, id) from the workspace: after the 256-byte header,
+    B*(N+1) 32-byte slots and B 1024-byte pre-pass partials come B*L float2 log-normalisers,
+    B*L*K x, B*L*K ids."""
+    off = 256 + B * (N + 1) * 32 + B * 1024 + B * L * 8
     x = buf.ws[off:off + B * L * K * 4].view(torch.float32).view(B * L, K).cpu().numpy()
     ids = buf.ws[off + B * L * K * 4:off + B * L * K * 8].view(torch.int32).view(B * L, K).cpu().numpy()
     return x, ids
