@@ -688,20 +688,26 @@ __device__ TreeSmem copy_topo(const VerifyArgs &a, Scratch &sh, float *base, int
         }
         if (bad_here) sh.cbad = 1;
     }
+    // the pre-computed set by node id (the chain's nodes are marked by load_pre)
+    for (int u = threadIdx.x; u < NN; u += kThreads)
+        ts.pre[u] = !a.pre_chain && u < a.M && ts.off[u + 1] - ts.off[u] > 0 ? 1 : 0;
     __syncthreads();
     return ts;
 }
 
-// The tokens of tree b and, per child slot, its token's target and q logits (from the parent's
-// rows) and acceptance uniform, after copy_topo. The tokens are read with plain loads: they may
-// come from the launch just before the walk. Every thread of the CTA calls it; it ends with the
-// CTA synchronised.
-template <typename T>
-__device__ void copy_slots(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, int b) {
+// The tokens of tree b (plain loads: they may come from the launch just before the walk); a
+// barrier must follow before they are read.
+__device__ __forceinline__ void copy_tokens(const VerifyArgs &a, const TreeSmem &ts, int b) {
     const int NN = a.N + 1;
     const int32_t *tok = a.token + (int64_t)b * NN;
     for (int i = threadIdx.x; i < NN; i += kThreads) ts.tok[i] = tok[i];
-    __syncthreads();
+}
+
+// Per child slot, after copy_topo and copy_tokens and a barrier: its token's target and q
+// logits (from the parent's rows) and acceptance uniform. Every thread of the CTA calls it; it
+// ends with the CTA synchronised.
+template <typename T>
+__device__ void slot_values(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, int b) {
     {  // every child slot: its token's target and q logits (from the parent's rows) and uniform
         bool bad_here = false;
         for (int j = threadIdx.x; j < a.N; j += kThreads) {
@@ -724,17 +730,20 @@ __device__ void copy_slots(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts,
     __syncthreads();
 }
 
-// Both parts, for walks whose tokens were written before the launch before them.
+// The whole copy, for walks whose tokens were written before the launch before them.
 template <typename T>
 __device__ TreeSmem copy_tree(const VerifyArgs &a, Scratch &sh, float *base, int b, bool per_depth) {
     const TreeSmem ts = copy_topo<T>(a, sh, base, b, per_depth);
-    copy_slots<T>(a, sh, ts, b);
+    copy_tokens(a, ts, b);
+    __syncthreads();
+    slot_values<T>(a, sh, ts, b);
     return ts;
 }
 
-// The pre-pass results for tree b (after the walk waited for the pre-pass): the pre-computed
-// set as the pre-pass chose it, its target normalisers, and the q-row normalisers (per depth
-// with pre_q, per node with a.qn). Every thread of the CTA calls it; ends synchronised.
+// The pre-pass results for tree b (after the walk waited for the pre-pass), after copy_topo:
+// the target normalisers of the pre-computed set (for the chain, merged from the partials and
+// the chain's nodes marked), and the q-row normalisers (per depth with pre_q, per node with
+// a.qn). All its loads form one round. Every thread of the CTA calls it; ends synchronised.
 __device__ void load_pre(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, int b, bool pre_q) {
     const int NN = a.N + 1;
     if (pre_q)
@@ -745,13 +754,10 @@ __device__ void load_pre(const VerifyArgs &a, Scratch &sh, const TreeSmem &ts, i
     if (a.M > 0 || a.qn)  // every node's slot in one round of loads (only the set's are used)
         for (int i = threadIdx.x; i < NN; i += kThreads) {
             const float4 pr = *reinterpret_cast<const float4 *>(&a.pre[(int64_t)b * NN + i]);
-            ts.l2t[i] = FF{pr.x, pr.y};
+            if (!a.pre_chain) ts.l2t[i] = FF{pr.x, pr.y};
             ts.l2qn[i] = FF{pr.z, pr.w};
         }
-    for (int u = threadIdx.x; u < NN; u += kThreads)
-        ts.pre[u] = !a.pre_chain && u < a.M && ts.off[u + 1] - ts.off[u] > 0 ? 1 : 0;
     if (a.pre_chain) {  // chain node j's normaliser from the pre-pass's kPreSplit partials, in order
-        __syncthreads();
         if (threadIdx.x < a.M) {
             const int v = chain_node(ts.off, ts.kid, a.N, threadIdx.x);
             if (v >= 0) {
@@ -989,10 +995,15 @@ __global__ void __launch_bounds__(kThreads, 1) k_verify_rrs(VerifyArgs a) {
     // the pre-pass and its results; tokens written by that launch (replay beside the
     // pre-pass) are read after the wait
     const TreeSmem ts = copy_topo<T>(a, sh, dyn + 2 * a.slice, b, per_depth);
-    if (!a.tokens_late) copy_slots<T>(a, sh, ts, b);
+    if (!a.tokens_late) {
+        copy_tokens(a, ts, b);
+        __syncthreads();
+        slot_values<T>(a, sh, ts, b);
+    }
     if (a.copy_early) pdl_begin();
-    if (a.tokens_late) copy_slots<T>(a, sh, ts, b);
+    if (a.tokens_late) copy_tokens(a, ts, b);  // in the round of load_pre's loads
     load_pre(a, sh, ts, b, true);
+    if (a.tokens_late) slot_values<T>(a, sh, ts, b);
     const FF *s_l2t = ts.l2t;
     const int32_t *s_known = ts.pre, *s_off = ts.off, *s_kid = ts.kid, *s_tok = ts.tok, *s_row = ts.row;
     const float *s_cxt = ts.cxt, *s_cxq = ts.cxq, *s_cu = ts.cu;

@@ -67,13 +67,15 @@ __device__ __forceinline__ void replay_node(const ReplayArgs &a, int blk) {
     const int b = blk / NN, u = blk - (blk / NN) * NN;
     if (u == 0 && threadIdx.x == 0) a.token[(int64_t)b * NN] = -1;
     const int32_t *off = a.child_off + (int64_t)b * (NN + 1);
-    const int o = off[u], m = off[u + 1] - o;
+    // the child count and the q row index in one round of loads (a leaf reads its row index too)
+    const int o = off[u], o1 = off[u + 1];
+    const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
+    const int m = o1 - o;
     if (m <= 0) return;  // uniform over the CTA
     if (m > KCAP || o < 0 || o + m > a.N) {
         if (threadIdx.x == 0) raise_status(a.status, kDevBadTree);
         return;
     }
-    const int r = a.qrow_of_node ? a.qrow_of_node[(int64_t)b * NN + u] : a.depth[(int64_t)b * NN + u];
     if (r < 0 || r >= a.R) {
         if (threadIdx.x == 0) raise_status(a.status, kDevBadIndex);
         return;
