@@ -500,13 +500,13 @@ __device__ __forceinline__ int sel_cap(int N) { return 4 * N + 64; }
 size_t select_smem_bytes(int L, int N, int K) {
     const size_t NN = (size_t)N + 1, cap = (size_t)4 * N + 64;
     return (size_t)(L + 1) * 8 + NN * 8 + (size_t)L * K * 8 + 6 * NN * 4 + (size_t)L * K * 4 + 8 +  // heap layout
-           (size_t)(L + 1) * 8 + (size_t)(L + 1) * K * 8 + cap * 8 + 3 * cap * 4;
+           (size_t)(L + 1) * 8 + (size_t)(L + 1) * K * 8 + cap * 8 + 4 * cap * 4;
 }
 
 struct SelShared {
     long long tau, lo;
     int hist[64];
-    int nent, ovf, alo, ahi, root, mono, fast, jstar, cum, kstar;
+    int nent, ovf, alo, ahi, root, mono, fast, jstar, cum, kstar, nkept;
 };
 
 // A bin edge t <= the N-th largest of a set of keys (all in [lo, hi], at least N of them) with
@@ -592,6 +592,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
     int32_t *einfo = reinterpret_cast<int32_t *>(ekey + cap);  // depth | rank << 8
     int32_t *epar = einfo + cap;                               // parent entry (-1: the root)
     int32_t *epos = epar + cap;                                // position in the global order
+    int32_t *ekept = epos + cap;                               // the entries that get a position
 
     const int b = blockIdx.x;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -772,17 +773,42 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
     if (fast && M < N) fast = false;
 
     if (fast) {
-        // ---- 3. positions by counting. Between equal keys at equal depths with different parents
-        //      the order is that of the parents, recursively: ancestors' keys compared upwards
-        //      until they differ, else (equal up to the common ancestor) the ranks of its two
-        //      children on the paths.
-        for (int x0 = warp * 8; x0 < M; x0 += kHeapThreads / 4) {  // uniform over the warp; four lanes per path
-            const int x = x0 + (lane >> 2), sub = lane & 3;
+        // ---- 3. positions by counting, among the paths whose key reaches t: with many more
+        //      paths than N, t is a second bound from the enumerated keys (at least N of them reach
+        //      it); a path's predecessors in the order all have keys >= its own, so they all
+        //      reach t and the counts among these paths are the global positions, and a parent
+        //      (key >= its child's) reaches t with its child. Between equal keys at equal depths
+        //      with different parents the order is that of the parents, recursively: ancestors'
+        //      keys compared upwards until they differ, else (equal up to the common ancestor)
+        //      the ranks of its two children on the paths.
+        long long t = tau;
+        if (M > N + (N >> 3))  // uniform: M from shared memory after a barrier
+            t = nth_bound(ss, N, hi, tau, [&](int s1, int s2, int jb, int *hist) {
+                for (int f = threadIdx.x; f < M; f += kHeapThreads) {
+                    const int bin = bound_bin(hi, ekey[f], s1, s2, jb);
+                    if (bin >= 0) atomicAdd(&hist[bin], 1);
+                }
+            });
+        if (threadIdx.x == 0) ss.nkept = 0;
+        __syncthreads();
+        for (int x = threadIdx.x; x < M; x += kHeapThreads) {
+            epos[x] = -1;
+            if (ekey[x] >= t) {
+                const int p = atomicAdd(&ss.nkept, 1);
+                if (in_bounds(p, cap, a.status)) ekept[p] = x;
+            }
+        }
+        __syncthreads();
+        const int MK = min(ss.nkept, cap);
+        for (int x0 = warp * 8; x0 < MK; x0 += kHeapThreads / 4) {  // uniform over the warp; four lanes per path
+            const int xi = x0 + (lane >> 2), sub = lane & 3;
+            const int x = xi < MK ? ekept[xi] : 0;
             int n = 0;
-            if (x < M) {
+            if (xi < MK) {
                 const long long kx = ekey[x];
                 const int dx = einfo[x] & 255, rx = einfo[x] >> 8, px = epar[x];
-                for (int y = sub; y < M; y += 4) {
+                for (int yi = sub; yi < MK; yi += 4) {
+                    const int y = ekept[yi];
                     const long long ky = ekey[y];
                     int add = ky > kx ? 1 : 0;
                     if (ky == kx && y != x) {
@@ -817,7 +843,7 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
             __syncwarp();  // after the lanes' ancestor walks
             n += __shfl_xor_sync(kFull, n, 1);
             n += __shfl_xor_sync(kFull, n, 2);
-            if (x < M && sub == 0) epos[x] = n;
+            if (xi < MK && sub == 0) epos[x] = n;
         }
         __syncthreads();
         bool bad = false;

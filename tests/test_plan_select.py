@@ -28,10 +28,10 @@ def _fixed(x):
     return np.rint(x.astype(np.float64) * 2.0**30).astype(np.int64)
 
 
-def nth_bound(keys, N, hi):
-    """A bin edge t <= the N-th largest of keys (all <= hi) with at least N keys >= t: 64
+def nth_bound(keys, N, hi, lo=None):
+    """A bin edge t <= the N-th largest of keys (all in [lo, hi]) with at least N keys >= t: 64
     power-of-two bins of hi - key, then 64 sub-bins of the bin holding the N-th."""
-    lo = min(keys)
+    lo = min(keys) if lo is None else lo
     s1 = 0
     while ((hi - lo) >> s1) >= 64:
         s1 += 1
@@ -139,9 +139,15 @@ def select_plan(topk_x, lse, K, L, N, cap=None):
                 return ent[ay][0] > ent[ax][0]
             cx, cy, ax, ay = ax, ay, ent[ax][3], ent[ay][3]
         return ent[cy][2] < ent[cx][2]
-    pos = [sum(1 for y in range(M) if before(y, x)) for x in range(M)]
+    # with many more paths than N, only those reaching a second bound get positions (their
+    # predecessors and parents all reach it)
+    kept = list(range(M))
+    if M > N + N // 8:
+        t = nth_bound([e[0] for e in ent], N, B[1], tau)
+        kept = [x for x in range(M) if ent[x][0] >= t]
+    pos = {x: sum(1 for y in kept if before(y, x)) for x in kept}
     nodes = [None] * N
-    for x in range(M):
+    for x in kept:
         if pos[x] < N:
             kx, dx, rx, px = ent[x]
             nodes[pos[x]] = (dx, 0 if px < 0 else pos[px] + 1, rx)
