@@ -562,6 +562,62 @@ __device__ __forceinline__ int bound_bin(long long hi, long long k, int s1, int 
     return (int)(dv >> s1) == jb ? (int)((dv >> s2) - ((unsigned long long)jb << (s1 - s2))) : -1;
 }
 
+// Positions in the global order (key desc, depth asc, parent's position asc, rank asc) of the
+// MK enumerated paths ekept[0..MK) (with COMPACT; else paths 0..MK), by counting the paths
+// before each one, four lanes per path: between equal keys at equal depths with different
+// parents, the ancestors' keys compared upwards until they differ, else (equal up to the common
+// ancestor) the ranks of its two children on the paths. All threads of the CTA call it.
+template <bool COMPACT>
+__device__ __forceinline__ void count_positions(const long long *ekey, const int32_t *einfo, const int32_t *epar,
+                                                const int32_t *ekept, int MK, int32_t *epos) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int x0 = warp * 8; x0 < MK; x0 += kHeapThreads / 4) {  // uniform over the warp; four lanes per path
+        const int xi = x0 + (lane >> 2), sub = lane & 3;
+        const int x = xi < MK ? (COMPACT ? ekept[xi] : xi) : 0;
+        int n = 0;
+        if (xi < MK) {
+            const long long kx = ekey[x];
+            const int dx = einfo[x] & 255, rx = einfo[x] >> 8, px = epar[x];
+            for (int yi = sub; yi < MK; yi += 4) {
+                const int y = COMPACT ? ekept[yi] : yi;
+                const long long ky = ekey[y];
+                int add = ky > kx ? 1 : 0;
+                if (ky == kx && y != x) {
+                    const int iy = einfo[y], dy = iy & 255;
+                    if (dy < dx) {
+                        add = 1;
+                    } else if (dy == dx) {
+                        const int py = epar[y];
+                        if (py == px) {
+                            add = (iy >> 8) < rx ? 1 : 0;
+                        } else {  // both at depth >= 2: walk up to the first difference
+                            int cx = x, cy = y, ax = px, ay = py, before = -1;
+                            for (int up = 0; up < kMaxDepth && before < 0; ++up) {
+                                if (ax == ay) {
+                                    before = (einfo[cy] >> 8) < (einfo[cx] >> 8) ? 1 : 0;
+                                } else if (ekey[ax] != ekey[ay]) {
+                                    before = ekey[ay] > ekey[ax] ? 1 : 0;
+                                } else {
+                                    cx = ax;
+                                    cy = ay;
+                                    ax = epar[ax];
+                                    ay = epar[ay];
+                                }
+                            }
+                            add = before > 0 ? 1 : 0;
+                        }
+                    }
+                }
+                n += add;
+            }
+        }
+        __syncwarp();  // after the lanes' ancestor walks
+        n += __shfl_xor_sync(kFull, n, 1);
+        n += __shfl_xor_sync(kFull, n, 2);
+        if (xi < MK && sub == 0) epos[x] = n;
+    }
+}
+
 // Max-heap expansion by selection (steps 1-3 above), with the serial expansion as fallback.
 // Each pop of the serial expansion: a warp maximum of the lanes' best keys, one
 // __reduce_max_sync on a 32-bit monotone image of the key, refined on the full key (high word,
@@ -781,70 +837,31 @@ __global__ void __launch_bounds__(kHeapThreads) k_plan_select(HeapArgs a) {
         //      with different parents the order is that of the parents, recursively: ancestors'
         //      keys compared upwards until they differ, else (equal up to the common ancestor)
         //      the ranks of its two children on the paths.
-        long long t = tau;
-        if (M > N + (N >> 3))  // uniform: M from shared memory after a barrier
-            t = nth_bound(ss, N, hi, tau, [&](int s1, int s2, int jb, int *hist) {
+        const bool compact = M > N + (N >> 3);  // uniform: M from shared memory after a barrier
+        int MK = M;
+        if (compact) {
+            const long long t = nth_bound(ss, N, hi, tau, [&](int s1, int s2, int jb, int *hist) {
                 for (int f = threadIdx.x; f < M; f += kHeapThreads) {
                     const int bin = bound_bin(hi, ekey[f], s1, s2, jb);
                     if (bin >= 0) atomicAdd(&hist[bin], 1);
                 }
             });
-        if (threadIdx.x == 0) ss.nkept = 0;
-        __syncthreads();
-        for (int x = threadIdx.x; x < M; x += kHeapThreads) {
-            epos[x] = -1;
-            if (ekey[x] >= t) {
-                const int p = atomicAdd(&ss.nkept, 1);
-                if (in_bounds(p, cap, a.status)) ekept[p] = x;
-            }
-        }
-        __syncthreads();
-        const int MK = min(ss.nkept, cap);
-        for (int x0 = warp * 8; x0 < MK; x0 += kHeapThreads / 4) {  // uniform over the warp; four lanes per path
-            const int xi = x0 + (lane >> 2), sub = lane & 3;
-            const int x = xi < MK ? ekept[xi] : 0;
-            int n = 0;
-            if (xi < MK) {
-                const long long kx = ekey[x];
-                const int dx = einfo[x] & 255, rx = einfo[x] >> 8, px = epar[x];
-                for (int yi = sub; yi < MK; yi += 4) {
-                    const int y = ekept[yi];
-                    const long long ky = ekey[y];
-                    int add = ky > kx ? 1 : 0;
-                    if (ky == kx && y != x) {
-                        const int iy = einfo[y], dy = iy & 255;
-                        if (dy < dx) {
-                            add = 1;
-                        } else if (dy == dx) {
-                            const int py = epar[y];
-                            if (py == px) {
-                                add = (iy >> 8) < rx ? 1 : 0;
-                            } else {  // both at depth >= 2: walk up to the first difference
-                                int cx = x, cy = y, ax = px, ay = py, before = -1;
-                                for (int up = 0; up < kMaxDepth && before < 0; ++up) {
-                                    if (ax == ay) {
-                                        before = (einfo[cy] >> 8) < (einfo[cx] >> 8) ? 1 : 0;
-                                    } else if (ekey[ax] != ekey[ay]) {
-                                        before = ekey[ay] > ekey[ax] ? 1 : 0;
-                                    } else {
-                                        cx = ax;
-                                        cy = ay;
-                                        ax = epar[ax];
-                                        ay = epar[ay];
-                                    }
-                                }
-                                add = before > 0 ? 1 : 0;
-                            }
-                        }
-                    }
-                    n += add;
+            if (threadIdx.x == 0) ss.nkept = 0;
+            __syncthreads();
+            for (int x = threadIdx.x; x < M; x += kHeapThreads) {
+                epos[x] = -1;
+                if (ekey[x] >= t) {
+                    const int p = atomicAdd(&ss.nkept, 1);
+                    if (in_bounds(p, cap, a.status)) ekept[p] = x;
                 }
             }
-            __syncwarp();  // after the lanes' ancestor walks
-            n += __shfl_xor_sync(kFull, n, 1);
-            n += __shfl_xor_sync(kFull, n, 2);
-            if (xi < MK && sub == 0) epos[x] = n;
+            __syncthreads();
+            MK = min(ss.nkept, cap);
         }
+        if (compact)
+            count_positions<true>(ekey, einfo, epar, ekept, MK, epos);
+        else
+            count_positions<false>(ekey, einfo, epar, ekept, MK, epos);
         __syncthreads();
         bool bad = false;
         for (int x = threadIdx.x; x < M; x += kHeapThreads) {
