@@ -55,7 +55,7 @@ cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t s
 //   B*(N+1) x 32 bytes             per-(tree, node) scalars: block verification's per-position
 //                                  values, or the verifier pre-pass's log-normalisers
 //   B x 1024 bytes                 per tree, the recursive-rejection pre-pass's partial
-//                                  normalisers (8 chain nodes x 8 row parts x 16 bytes)
+//                                  normalisers (up to 8 chain nodes x 8 row parts x 16 bytes)
 //   B*L float2, B*L*K floats,      per-draft-row log-normaliser (float-float) and top-K
 //   B*L*K int32                    (x, id) of the first pass
 constexpr size_t kWsStatusBytes = 256;
