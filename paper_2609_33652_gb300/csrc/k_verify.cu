@@ -26,11 +26,13 @@
 // with the two-level Gumbel-max of the randomness contract: chunk keys log(chunk mass) + G
 // over chunks of 256 tokens, then the best token of the winning chunk.
 //
-// Scheduling. A pre-pass kernel (all SMs) computes the target log-normalisers of the nodes a
-// walk is most likely to visit, the first kPreChain internal nodes of the first-child chain
-// from the root (slot 0 is accepted at most visits), and the q rows' log-normalisers (per
-// depth, or per internal node for per-node rows). The walk kernel copies the tree's topology,
-// the children's target and q logits and their acceptance uniforms to shared memory once. At
+// Scheduling. A pre-pass (k_pre_split before the walk, or its CTAs inside the replay's grid in
+// k_replay_pre) computes the target log-normalisers of the nodes a walk is most likely to
+// visit, the first kPreChain internal nodes of the first-child chain from the root (slot 0 is
+// accepted at most visits), as kPreSplit partials per row that the walk merges in order, and
+// the q rows' log-normalisers (per depth, or per internal node for per-node rows). The walk
+// kernel copies the tree's topology, the children's target and q logits and their acceptance
+// uniforms to shared memory once. At
 // a node with a known normaliser it needs no staging and no cluster round: every CTA takes
 // the same decisions from the same inputs, and the slices are staged only if a rejection needs
 // the residual. At any other node the walk runs a staging round over that node and up to two
@@ -40,9 +42,10 @@
 // partial per CTA through distributed shared memory. 12 warps per CTA: 160 registers a thread
 // without spills (16 warps at 128 spilled in the walk's hot paths and ran slower). Element passes give lane l the elements 4l..4l+3 and
 // 128+4l..128+4l+3 of each 256-token chunk, so every shared-memory access is a conflict-free
-// 16-byte vector. Every normaliser comes from the same two functions over the row's chunk
-// statistics, whichever kernel computes it, and which nodes are pre-computed depends only on
-// the topology, so results do not depend on timing.
+// 16-byte vector. Each normaliser is computed by a fixed procedure chosen by the node alone
+// (pre-computed chain node, staged node), and which nodes are pre-computed depends only on the
+// topology, so results do not depend on timing or on which call (tsb_verify alone or
+// tsb_replay_verify) ran the pre-pass.
 #include <cooperative_groups.h>
 
 #include <mutex>
